@@ -1,0 +1,206 @@
+/*
+ * olive.h -- C ABI of libolive.so, the GB300 (sm_103a) implementation of the
+ * per-token scoring path of OLIVE ("Learning from Teacher Continuations at
+ * Student States").
+ *
+ * The path: a student prefix (prompt x and student tokens y_{1:k}) is cut at a
+ * student state and followed by a teacher continuation y~_{1:l}; the student
+ * is trained with the masked cross-entropy of Eq. (osd-ce) (Section 3.1) on the
+ * continuation tokens only.  The OPD baseline (Section 1) scores tokens with a
+ * per-token reverse KL against the teacher instead.  Four calls cover it:
+ *
+ *   olive_splice_pack        packs the spliced sequences and builds the loss mask
+ *   olive_token_logprob_fwd  LM-head projection + online log-sum-exp + masked
+ *                            target log-prob and loss (the [T,V] logits are
+ *                            never stored)
+ *   olive_token_loss_bwd     d loss / d hidden and d loss / d W
+ *   olive_token_divergence   full-vocabulary per-token KL (+ d KL / d h_s)
+ *
+ * Conventions shared by every call
+ *   - Every pointer argument is a DEVICE pointer unless stated otherwise.  The
+ *     caller owns every buffer; the library allocates no device memory and
+ *     keeps no state between calls.  Scratch memory comes from the caller's
+ *     `workspace` (size from olive_workspace_size, 256-byte aligned).
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  All calls
+ *     are asynchronous on it; none synchronises the host.
+ *   - The returned olive_status covers what the host can check before any
+ *     launch (null pointers, shapes, alignment, device).  On any non-OK
+ *     return nothing was launched.
+ *   - Errors in device data (a token id outside [0,V), offsets that do not
+ *     describe the batch, an internal wait that ran out of time) are OR-ed
+ *     into *dev_status as bits (1u << code), code from olive_status.  The
+ *     caller zeroes *dev_status and reads it whenever it synchronises.
+ *   - Row counts such as N_mask stay on the device (`n_rows`), so the three
+ *     compute calls can follow olive_splice_pack without a host round trip;
+ *     grids are sized from the host-side upper bound T.
+ *   - Tensors are row-major and contiguous.  bf16 is IEEE bfloat16.  Base
+ *     pointers of hidden, W, d_hidden and d_W must be 16-byte aligned, and
+ *     d (every hidden width) must be a multiple of 8.
+ *   - The library runs only on compute capability 10.3 (sm_103a).
+ */
+#ifndef OLIVE_H_
+#define OLIVE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define OLIVE_API __attribute__((visibility("default")))
+#else
+#define OLIVE_API
+#endif
+
+#define OLIVE_ABI_VERSION 1
+
+typedef enum {
+  OLIVE_OK = 0,
+  OLIVE_ERR_INVALID_ARG = 1,       /* null pointer, bad enum value            */
+  OLIVE_ERR_SHAPE = 2,             /* non-positive or too large size          */
+  OLIVE_ERR_ALIGNMENT = 3,         /* pointer or width breaks the 16-B rule   */
+  OLIVE_ERR_TOKEN_RANGE = 4,       /* (device) an id or target outside [0,V)  */
+  OLIVE_ERR_OFFSETS = 5,           /* (device) offsets / row list malformed   */
+  OLIVE_ERR_TIMEOUT = 6,           /* (device) an internal wait ran out       */
+  OLIVE_ERR_UNSUPPORTED_DEVICE = 7,/* current device is not sm_103           */
+  OLIVE_ERR_CUDA = 8,              /* a CUDA runtime/driver call failed       */
+  OLIVE_ERR_WORKSPACE = 9          /* workspace null, misaligned or too small */
+} olive_status;
+
+enum { OLIVE_REDUCE_SUM = 0, OLIVE_REDUCE_MEAN = 1 };
+enum { OLIVE_KL_REVERSE = 0, OLIVE_KL_FORWARD = 1 };
+enum { OLIVE_DTYPE_BF16 = 0, OLIVE_DTYPE_F32 = 1 };
+enum { OLIVE_OP_LOGPROB_FWD = 0, OLIVE_OP_LOSS_BWD = 1, OLIVE_OP_DIVERGENCE = 2 };
+
+/* ABI version of the loaded library (OLIVE_ABI_VERSION). */
+OLIVE_API int olive_abi_version(void);
+
+/* Static text for a status code. Never NULL. */
+OLIVE_API const char* olive_status_string(olive_status s);
+
+/*
+ * Workspace bytes a compute call needs for host-side upper bound T rows.
+ *   op  OLIVE_OP_LOGPROB_FWD / OLIVE_OP_LOSS_BWD: d = hidden width, d_t ignored.
+ *   op  OLIVE_OP_DIVERGENCE: d = student width d_s, d_t = teacher width.
+ *   `grad` (bwd / divergence): non-zero when gradients are requested
+ *   (OLIVE_OP_LOSS_BWD always computes them); `grad_dtype` is the dtype of
+ *   d_W for OLIVE_OP_LOSS_BWD (bf16 output needs an fp32 accumulator).
+ * Returns 0 for invalid arguments.
+ */
+OLIVE_API size_t olive_workspace_size(int op, int32_t T, int32_t d, int32_t d_t, int32_t V,
+                            int grad, int grad_dtype);
+
+/*
+ * olive_splice_pack -- builds the packed student-update batch of Section 3.1:
+ * for each sequence s the spliced sequence (x, y_{1:k}, y~_{1:l}) =
+ * prefix_s || continuation_s, laid back to back, with the loss of Eq. (osd-ce)
+ * on the continuation tokens only ("the prompt and student prefix remain in
+ * the conditioning context but are masked out of the loss").
+ *
+ * Inputs (device, int32):
+ *   prefix_ids  all prefixes (prompt + student prefix) back to back;
+ *   prefix_off  [S+1] CSR offsets, prefix_off[0] = 0, non-decreasing;
+ *               every prefix holds >= 1 id;
+ *   cont_ids    all continuations (already in student tokens) back to back;
+ *   cont_off    [S+1] CSR offsets, cont_off[0] = 0, non-decreasing (a
+ *               continuation may be empty);
+ *   S >= 1 sequences, V >= 1 vocabulary size, T_cap >= 1 capacity of the
+ *   packed outputs.
+ * Outputs (device), with T = sum_s (P_s + C_s) packed tokens:
+ *   ids[T_cap]        packed ids; positions >= T are set to 0;
+ *   targets[T_cap]    ids[t+1] when t+1 belongs to the same sequence, else -1
+ *                     (row t of the hidden states predicts token t+1);
+ *   loss_mask[T_cap]  1 where targets[t] is a continuation token y~_j, else 0;
+ *   cu_seqlens[S+1]   packed start of every sequence, cu_seqlens[S] = T;
+ *   cut_offsets[S]    packed index of y~_1 (= cu_seqlens[s] + P_s);
+ *   rows[T_cap]       the masked rows in ascending order (first n_rows valid);
+ *   n_rows[1]         N_mask = sum_s C_s.
+ * Device errors: OFFSETS (malformed offsets, empty prefix, T > T_cap: then
+ * n_rows = 0 and the outputs are cleared), TOKEN_RANGE (an id outside [0,V);
+ * the ids are still copied).
+ */
+OLIVE_API olive_status olive_splice_pack(const int32_t* prefix_ids, const int32_t* prefix_off,
+                               const int32_t* cont_ids, const int32_t* cont_off,
+                               int32_t S, int32_t V, int32_t T_cap,
+                               int32_t* ids, int32_t* targets, uint8_t* loss_mask,
+                               int32_t* cu_seqlens, int32_t* cut_offsets,
+                               int32_t* rows, int32_t* n_rows,
+                               int32_t* dev_status, void* stream);
+
+/*
+ * olive_token_logprob_fwd -- Eq. (osd-ce): for every masked row r (t = rows[r],
+ * r < *n_rows) with target y = targets[t],
+ *   z_v    = inv_tau * <hidden[t,:], W[v,:]>          (v = 0..V-1, fp32 accumulate)
+ *   lse[t] = log sum_v exp(z_v)
+ *   logp[t]= z_y - lse[t]
+ *   loss   = -sum_r logp[rows[r]]            (OLIVE_REDUCE_SUM, Eq. (osd-ce))
+ *          = that / N_mask                   (OLIVE_REDUCE_MEAN; 0 if N_mask = 0)
+ * inv_tau is the inverse sampling temperature (1.0 in Appendix A).
+ *   hidden  bf16 [T, d]     W bf16 [V, d]     targets int32 [T]
+ *   rows    int32 [>= *n_rows] ascending or not, each in [0,T)
+ *   logp, lse  fp32 [T]: written on every row, 0 on rows not in `rows`
+ *   loss    fp32 [1]
+ * The [T,V] logits are never stored: vocabulary tiles are reduced on chip.
+ * Device errors: TOKEN_RANGE (target outside [0,V); that row's logp is NaN),
+ * OFFSETS (*n_rows > T or a row outside [0,T)), TIMEOUT.
+ */
+OLIVE_API olive_status olive_token_logprob_fwd(const void* hidden, const void* W,
+                                     const int32_t* targets, const int32_t* rows,
+                                     const int32_t* n_rows, int32_t T, int32_t d, int32_t V,
+                                     float inv_tau, int reduction,
+                                     float* logp, float* lse, float* loss,
+                                     void* workspace, size_t ws_bytes,
+                                     int32_t* dev_status, void* stream);
+
+/*
+ * olive_token_loss_bwd -- gradients of the Eq. (osd-ce) loss through the LM
+ * head (the sampled sequences are fixed, Section 3.1, so ids get none):
+ *   G[r,v]    = g * inv_tau * (exp(z_v - lse[t]) - [v == y])
+ *               with g = *grad_loss, divided by N_mask for OLIVE_REDUCE_MEAN
+ *   d_hidden[t,:] = sum_v G[r,v] W[v,:]   on masked rows, 0 on all other rows
+ *   d_W[v,:]      = sum_r G[r,v] hidden[t,:]
+ * Arguments as in olive_token_logprob_fwd; lse fp32 [T] is the forward's
+ * output; grad_loss fp32 [1] (device); d_hidden [T,d] and d_W [V,d] of
+ * grad_dtype (OLIVE_DTYPE_BF16: fp32 accumulation, round-to-nearest-even
+ * store; OLIVE_DTYPE_F32).  Logits are recomputed tile by tile; G exists only
+ * as a bf16 slab of at most a fixed number of rows inside the workspace.
+ */
+OLIVE_API olive_status olive_token_loss_bwd(const void* hidden, const void* W,
+                                  const int32_t* targets, const int32_t* rows,
+                                  const int32_t* n_rows, int32_t T, int32_t d, int32_t V,
+                                  float inv_tau, int reduction,
+                                  const float* lse, const float* grad_loss,
+                                  void* d_hidden, void* d_W, int grad_dtype,
+                                  void* workspace, size_t ws_bytes,
+                                  int32_t* dev_status, void* stream);
+
+/*
+ * olive_token_divergence -- OPD's per-token divergence between the student
+ * pi_theta and the teacher pi_T over the full vocabulary (Section 1; the
+ * paper's top-16 approximation is not used): on masked row t,
+ *   p_s = softmax(inv_tau * h_s[t] W_s^T)   (width d_s)
+ *   p_t = softmax(inv_tau * h_t[t] W_t^T)   (width d_t, same V)
+ *   OLIVE_KL_REVERSE: kl[t] = sum_v p_s (log p_s - log p_t)
+ *   OLIVE_KL_FORWARD: kl[t] = sum_v p_t (log p_t - log p_s)
+ * kl fp32 [T] (0 on rows not in `rows`).  If grad_kl (fp32 [T], weights g_t)
+ * and d_h_s ([T, d_s] of grad_dtype) are both non-NULL, also writes the
+ * gradient of sum_t g_t kl[t] with respect to h_s:
+ *   reverse: d_h_s[t] = g_t inv_tau sum_v p_s (log p_s - log p_t - kl[t]) W_s[v]
+ *   forward: d_h_s[t] = g_t inv_tau sum_v (p_s - p_t) W_s[v]
+ * (0 on rows not in `rows`; the teacher receives no gradient).
+ */
+OLIVE_API olive_status olive_token_divergence(const void* h_s, const void* W_s, int32_t d_s,
+                                    const void* h_t, const void* W_t, int32_t d_t,
+                                    const int32_t* rows, const int32_t* n_rows,
+                                    int32_t T, int32_t V, float inv_tau, int direction,
+                                    float* kl, const float* grad_kl, void* d_h_s,
+                                    int grad_dtype, void* workspace, size_t ws_bytes,
+                                    int32_t* dev_status, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* OLIVE_H_ */

@@ -1,0 +1,266 @@
+"""Thin ctypes binding over libolive.so (include/olive.h), same entry names.
+
+Every function here only marshals torch tensors into pointers and sizes and
+calls the C ABI on the current torch CUDA stream; all computation happens in
+the library's CUDA kernels.  There is no fallback: if libolive.so is missing
+or fails to load, every call raises.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+
+import torch
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libolive.so")
+HEADER = os.path.join(os.path.dirname(HERE), "include", "olive.h")
+
+OLIVE_OK = 0
+STATUS_NAMES = {
+    0: "OLIVE_OK", 1: "OLIVE_ERR_INVALID_ARG", 2: "OLIVE_ERR_SHAPE", 3: "OLIVE_ERR_ALIGNMENT",
+    4: "OLIVE_ERR_TOKEN_RANGE", 5: "OLIVE_ERR_OFFSETS", 6: "OLIVE_ERR_TIMEOUT",
+    7: "OLIVE_ERR_UNSUPPORTED_DEVICE", 8: "OLIVE_ERR_CUDA", 9: "OLIVE_ERR_WORKSPACE",
+}
+REDUCE = {"sum": 0, "mean": 1}
+DIRECTION = {"reverse": 0, "forward": 1}
+DTYPE = {torch.bfloat16: 0, torch.float32: 1}
+OP = {"logprob_fwd": 0, "loss_bwd": 1, "divergence": 2}
+
+
+class OliveError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {STATUS_NAMES.get(status, status)}")
+
+
+_lib = None
+_P = ctypes.c_void_p
+_I = ctypes.c_int32
+_F = ctypes.c_float
+_S = ctypes.c_size_t
+
+
+def lib() -> ctypes.CDLL:
+    """Loads libolive.so (raises if it is not built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise OliveError(8, f"libolive.so not found at {LIB_PATH}; build it with "
+                            "paper_2609_36246_gb300.build.build()")
+    L = ctypes.CDLL(LIB_PATH)
+    L.olive_abi_version.restype = ctypes.c_int
+    L.olive_abi_version.argtypes = []
+    L.olive_status_string.restype = ctypes.c_char_p
+    L.olive_status_string.argtypes = [ctypes.c_int]
+    L.olive_workspace_size.restype = _S
+    L.olive_workspace_size.argtypes = [ctypes.c_int, _I, _I, _I, _I, ctypes.c_int, ctypes.c_int]
+    L.olive_splice_pack.restype = ctypes.c_int
+    L.olive_splice_pack.argtypes = [_P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P]
+    L.olive_token_logprob_fwd.restype = ctypes.c_int
+    L.olive_token_logprob_fwd.argtypes = [_P, _P, _P, _P, _P, _I, _I, _I, _F, ctypes.c_int,
+                                          _P, _P, _P, _P, _S, _P, _P]
+    L.olive_token_loss_bwd.restype = ctypes.c_int
+    L.olive_token_loss_bwd.argtypes = [_P, _P, _P, _P, _P, _I, _I, _I, _F, ctypes.c_int, _P, _P,
+                                       _P, _P, ctypes.c_int, _P, _S, _P, _P]
+    L.olive_token_divergence.restype = ctypes.c_int
+    L.olive_token_divergence.argtypes = [_P, _P, _I, _P, _P, _I, _P, _P, _I, _I, _F, ctypes.c_int,
+                                         _P, _P, _P, ctypes.c_int, _P, _S, _P, _P]
+    _lib = L
+    return L
+
+
+def declared_symbols() -> list[str]:
+    """Entry points declared with OLIVE_API in include/olive.h."""
+    with open(HEADER) as f:
+        text = f.read()
+    return re.findall(r"OLIVE_API\s+[\w\s\*]*?\b(olive_\w+)\s*\(", text)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream():
+    return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+
+
+def _check(st: int, where: str):
+    if st != OLIVE_OK:
+        raise OliveError(st, where)
+
+
+def _need(t, dtype, name):
+    if not isinstance(t, torch.Tensor) or not t.is_cuda or t.dtype != dtype or not t.is_contiguous():
+        raise TypeError(f"{name} must be a contiguous CUDA {dtype} tensor")
+
+
+def new_status(device=None) -> torch.Tensor:
+    return torch.zeros(1, dtype=torch.int32, device=device or "cuda")
+
+
+def status_bits(dev_status: torch.Tensor) -> list[str]:
+    """Names of the error bits set in a device status word (synchronises)."""
+    v = int(dev_status.item())
+    return [STATUS_NAMES[c] for c in range(1, 10) if v & (1 << c)]
+
+
+def olive_abi_version() -> int:
+    return lib().olive_abi_version()
+
+
+def olive_status_string(status: int) -> str:
+    return lib().olive_status_string(status).decode()
+
+
+def olive_workspace_size(op: str, T: int, d: int, V: int, d_t: int = 0, grad: bool = True,
+                         grad_dtype=torch.bfloat16) -> int:
+    return int(lib().olive_workspace_size(OP[op], T, d, d_t, V, int(grad), DTYPE[grad_dtype]))
+
+
+def workspace(nbytes: int, device=None) -> torch.Tensor:
+    return torch.empty(max(int(nbytes), 1), dtype=torch.uint8, device=device or "cuda")
+
+
+def olive_splice_pack(prefix_ids, prefix_off, cont_ids, cont_off, V: int, T_cap: int,
+                      dev_status=None) -> dict:
+    """Packs the spliced sequences; returns the device outputs of olive.h."""
+    for t, n in ((prefix_ids, "prefix_ids"), (prefix_off, "prefix_off"), (cont_ids, "cont_ids"),
+                 (cont_off, "cont_off")):
+        _need(t, torch.int32, n)
+    S = prefix_off.numel() - 1
+    dev = prefix_off.device
+    out = {
+        "ids": torch.empty(T_cap, dtype=torch.int32, device=dev),
+        "targets": torch.empty(T_cap, dtype=torch.int32, device=dev),
+        "loss_mask": torch.empty(T_cap, dtype=torch.uint8, device=dev),
+        "cu_seqlens": torch.empty(S + 1, dtype=torch.int32, device=dev),
+        "cut_offsets": torch.empty(max(S, 1), dtype=torch.int32, device=dev),
+        "rows": torch.empty(T_cap, dtype=torch.int32, device=dev),
+        "n_rows": torch.empty(1, dtype=torch.int32, device=dev),
+    }
+    out["dev_status"] = dev_status if dev_status is not None else new_status(dev)
+    # empty id arrays still need a valid device address
+    pid = prefix_ids if prefix_ids.numel() else torch.zeros(1, dtype=torch.int32, device=dev)
+    cid = cont_ids if cont_ids.numel() else torch.zeros(1, dtype=torch.int32, device=dev)
+    st = lib().olive_splice_pack(_ptr(pid), _ptr(prefix_off), _ptr(cid), _ptr(cont_off), S, V, T_cap,
+                                 _ptr(out["ids"]), _ptr(out["targets"]), _ptr(out["loss_mask"]),
+                                 _ptr(out["cu_seqlens"]), _ptr(out["cut_offsets"]),
+                                 _ptr(out["rows"]), _ptr(out["n_rows"]), _ptr(out["dev_status"]),
+                                 _stream())
+    _check(st, "olive_splice_pack")
+    return out
+
+
+def olive_token_logprob_fwd(hidden, W, targets, rows, n_rows, inv_tau: float = 1.0,
+                            reduction: str = "sum", ws=None, dev_status=None, out=None):
+    """Per-token log-probs, lse and the Eq. (osd-ce) loss. Returns (logp, lse, loss)."""
+    _need(hidden, torch.bfloat16, "hidden")
+    _need(W, torch.bfloat16, "W")
+    _need(targets, torch.int32, "targets")
+    _need(rows, torch.int32, "rows")
+    _need(n_rows, torch.int32, "n_rows")
+    T, d = hidden.shape
+    V = W.shape[0]
+    if W.shape[1] != d:
+        raise ValueError("hidden and W widths differ")
+    dev = hidden.device
+    if out is None:
+        out = (torch.empty(T, dtype=torch.float32, device=dev),
+               torch.empty(T, dtype=torch.float32, device=dev),
+               torch.empty(1, dtype=torch.float32, device=dev))
+    logp, lse, loss = out
+    need = olive_workspace_size("logprob_fwd", T, d, V)
+    if ws is None:
+        ws = workspace(need, dev)
+    ds = dev_status if dev_status is not None else new_status(dev)
+    st = lib().olive_token_logprob_fwd(_ptr(hidden), _ptr(W), _ptr(targets), _ptr(rows), _ptr(n_rows),
+                                       T, d, V, float(inv_tau), REDUCE[reduction], _ptr(logp),
+                                       _ptr(lse), _ptr(loss), _ptr(ws), ws.numel(), _ptr(ds),
+                                       _stream())
+    _check(st, "olive_token_logprob_fwd")
+    return logp, lse, loss
+
+
+def olive_token_loss_bwd(hidden, W, targets, rows, n_rows, lse, grad_loss, inv_tau: float = 1.0,
+                         reduction: str = "sum", grad_dtype=torch.bfloat16, ws=None,
+                         dev_status=None, out=None):
+    """d loss/d hidden and d loss/d W. grad_loss is a 1-element fp32 CUDA tensor."""
+    _need(hidden, torch.bfloat16, "hidden")
+    _need(W, torch.bfloat16, "W")
+    _need(lse, torch.float32, "lse")
+    _need(grad_loss, torch.float32, "grad_loss")
+    T, d = hidden.shape
+    V = W.shape[0]
+    dev = hidden.device
+    if out is None:
+        out = (torch.empty(T, d, dtype=grad_dtype, device=dev),
+               torch.empty(V, d, dtype=grad_dtype, device=dev))
+    dh, dw = out
+    need = olive_workspace_size("loss_bwd", T, d, V, grad_dtype=grad_dtype)
+    if ws is None:
+        ws = workspace(need, dev)
+    ds = dev_status if dev_status is not None else new_status(dev)
+    st = lib().olive_token_loss_bwd(_ptr(hidden), _ptr(W), _ptr(targets), _ptr(rows), _ptr(n_rows),
+                                    T, d, V, float(inv_tau), REDUCE[reduction], _ptr(lse),
+                                    _ptr(grad_loss), _ptr(dh), _ptr(dw), DTYPE[grad_dtype],
+                                    _ptr(ws), ws.numel(), _ptr(ds), _stream())
+    _check(st, "olive_token_loss_bwd")
+    return dh, dw
+
+
+def olive_token_divergence(h_s, W_s, h_t, W_t, rows, n_rows, inv_tau: float = 1.0,
+                           direction: str = "reverse", grad_kl=None, grad_dtype=torch.bfloat16,
+                           ws=None, dev_status=None):
+    """Per-token full-vocabulary KL; with grad_kl also d(sum g_t KL_t)/d h_s.
+
+    Returns (kl [T] fp32, d_h_s or None)."""
+    for t, n in ((h_s, "h_s"), (W_s, "W_s"), (h_t, "h_t"), (W_t, "W_t")):
+        _need(t, torch.bfloat16, n)
+    T, d_s = h_s.shape
+    d_t = h_t.shape[1]
+    V = W_s.shape[0]
+    if W_t.shape[0] != V or h_t.shape[0] != T:
+        raise ValueError("student and teacher shapes disagree")
+    dev = h_s.device
+    kl = torch.empty(T, dtype=torch.float32, device=dev)
+    dhs = None
+    if grad_kl is not None:
+        _need(grad_kl, torch.float32, "grad_kl")
+        dhs = torch.empty(T, d_s, dtype=grad_dtype, device=dev)
+    need = olive_workspace_size("divergence", T, d_s, V, d_t=d_t, grad=grad_kl is not None)
+    if ws is None:
+        ws = workspace(need, dev)
+    ds = dev_status if dev_status is not None else new_status(dev)
+    st = lib().olive_token_divergence(_ptr(h_s), _ptr(W_s), d_s, _ptr(h_t), _ptr(W_t), d_t,
+                                      _ptr(rows), _ptr(n_rows), T, V, float(inv_tau),
+                                      DIRECTION[direction], _ptr(kl), _ptr(grad_kl), _ptr(dhs),
+                                      DTYPE[grad_dtype], _ptr(ws), ws.numel(), _ptr(ds), _stream())
+    _check(st, "olive_token_divergence")
+    return kl, dhs
+
+
+class FusedLMHeadCE(torch.autograd.Function):
+    """Eq. (osd-ce) loss over the masked rows as an autograd op (bf16 grads)."""
+
+    @staticmethod
+    def forward(ctx, hidden, W, targets, rows, n_rows, inv_tau=1.0, reduction="sum"):
+        logp, lse, loss = olive_token_logprob_fwd(hidden, W, targets, rows, n_rows, inv_tau, reduction)
+        ctx.save_for_backward(hidden, W, targets, rows, n_rows, lse)
+        ctx.inv_tau, ctx.reduction = inv_tau, reduction
+        return loss[0]
+
+    @staticmethod
+    def backward(ctx, g):
+        hidden, W, targets, rows, n_rows, lse = ctx.saved_tensors
+        gl = g.reshape(1).to(torch.float32).contiguous()
+        dh, dw = olive_token_loss_bwd(hidden, W, targets, rows, n_rows, lse, gl, ctx.inv_tau,
+                                      ctx.reduction, grad_dtype=hidden.dtype)
+        return dh, dw, None, None, None, None, None
+
+
+def fused_lmhead_ce(hidden, W, targets, rows, n_rows, inv_tau=1.0, reduction="sum"):
+    return FusedLMHeadCE.apply(hidden, W, targets, rows, n_rows, inv_tau, reduction)

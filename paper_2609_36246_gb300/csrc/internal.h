@@ -1,0 +1,111 @@
+// internal.h -- host-side declarations shared by the translation units of
+// libolive.so.  Not part of the public ABI (include/olive.h is).
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "../../include/olive.h"
+
+namespace olive {
+
+constexpr int kSvMax = 64;        // most vocabulary segments per row tile
+constexpr int kRowAlign = 128;    // row tiles of the compacted hidden copy
+constexpr size_t kWsAlign = 256;  // alignment of every workspace region
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+// Launch context gathered once per API call.
+struct Ctx {
+  cudaStream_t stream;
+  int device;
+  int num_sms;
+  uint64_t wait_limit_ns;
+};
+
+// Fills ctx for the current device; checks compute capability 10.3.
+olive_status make_ctx(void* stream, Ctx* ctx);
+
+// Encodes a 2-D bf16 tensor map (row-major [outer, inner], row pitch in
+// bytes) with 128-byte swizzle and the given box.  Returns false on failure.
+bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+                    uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer);
+
+// Rows of the G slab used by the backward passes for vocabulary size V.
+int64_t slab_rows(int64_t Tpad, int64_t V);
+inline int64_t vpad(int64_t V) { return align_up(static_cast<size_t>(V), 8); }
+
+// ---- workspace carving (sizes in bytes; every region 256-byte aligned) ----
+struct FwdWs {
+  void* hc;       // bf16 [Tpad, d] compacted hidden rows
+  float* part_m;  // [kSvMax, Tpad]
+  float* part_s;  // [kSvMax, Tpad]
+  float* zy;      // [Tpad]
+  float* nll;     // [Tpad]
+};
+size_t fwd_ws_bytes(int64_t T, int64_t d);
+FwdWs carve_fwd(void* ws, int64_t T, int64_t d);
+
+struct BwdWs {
+  void* hc;       // bf16 [Tpad, d]
+  void* g;        // bf16 [Tc, Vpad]
+  float* dw_acc;  // fp32 [V, d] (bf16 output only)
+  int64_t tc;     // slab rows
+};
+size_t bwd_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype);
+BwdWs carve_bwd(void* ws, int64_t T, int64_t d, int64_t V, int grad_dtype);
+
+struct KlWs {
+  void* hcs;      // bf16 [Tpad, d_s]
+  void* hct;      // bf16 [Tpad, d_t]
+  float* part;    // [5, kSvMax, Tpad]
+  float* stats;   // [3, Tpad]: lse_s, lse_t, kl per compacted row
+  void* g;        // bf16 [Tc, Vpad] (gradient only)
+  int64_t tc;
+};
+size_t kl_ws_bytes(int64_t T, int64_t ds, int64_t dt, int64_t V, int grad);
+KlWs carve_kl(void* ws, int64_t T, int64_t ds, int64_t dt, int64_t V, int grad);
+
+// ---- launchers (validated arguments; return OLIVE_OK or OLIVE_ERR_CUDA) ----
+olive_status launch_splice_pack(const Ctx& c, const int32_t* prefix_ids, const int32_t* prefix_off,
+                                const int32_t* cont_ids, const int32_t* cont_off, int32_t S,
+                                int32_t V, int32_t T_cap, int32_t* ids, int32_t* targets,
+                                uint8_t* loss_mask, int32_t* cu_seqlens, int32_t* cut_offsets,
+                                int32_t* rows, int32_t* n_rows, int32_t* dev_status);
+
+// Copies hidden[rows[r]] to hc[r] for r < n_rows and zero-fills the rest of
+// the last 128-row tile.
+olive_status launch_gather_rows(const Ctx& c, const void* hidden, const int32_t* rows,
+                                const int32_t* n_rows, int32_t T, int32_t d, void* hc,
+                                int32_t* dev_status);
+
+olive_status launch_logprob_fwd(const Ctx& c, const void* hidden, const void* W,
+                                const int32_t* targets, const int32_t* rows, const int32_t* n_rows,
+                                int32_t T, int32_t d, int32_t V, float inv_tau, int reduction,
+                                float* logp, float* lse, float* loss, void* ws,
+                                int32_t* dev_status);
+
+olive_status launch_loss_bwd(const Ctx& c, const void* hidden, const void* W,
+                             const int32_t* targets, const int32_t* rows, const int32_t* n_rows,
+                             int32_t T, int32_t d, int32_t V, float inv_tau, int reduction,
+                             const float* lse, const float* grad_loss, void* d_hidden, void* d_W,
+                             int grad_dtype, void* ws, int32_t* dev_status);
+
+olive_status launch_divergence(const Ctx& c, const void* h_s, const void* W_s, int32_t d_s,
+                               const void* h_t, const void* W_t, int32_t d_t, const int32_t* rows,
+                               const int32_t* n_rows, int32_t T, int32_t V, float inv_tau,
+                               int direction, float* kl, const float* grad_kl, void* d_h_s,
+                               int grad_dtype, void* ws, int32_t* dev_status);
+
+// dH = G . W for one slab of G (shared by the CE and KL backward passes):
+// rows [slab_start, slab_start + Tc) of the compacted row list, scattered to
+// out[rows[r], :] in out_dtype.
+olive_status launch_dh_slab(const Ctx& c, const void* g, int64_t ldg, int64_t tc, const void* W,
+                            int32_t d, int32_t V, const int32_t* rows, const int32_t* n_rows,
+                            int32_t T, int64_t slab_start, void* out, int out_dtype,
+                            int32_t* dev_status);
+
+}  // namespace olive

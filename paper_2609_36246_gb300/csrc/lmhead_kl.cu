@@ -1,0 +1,393 @@
+// lmhead_kl.cu -- OPD's per-token divergence between student and teacher over
+// the full vocabulary (Section 1: OPD scores each rollout token with a reverse
+// KL against the teacher), and the gradient of sum_t g_t KL_t with respect to
+// the student hidden states.
+//
+// Forward (one pass over the vocabulary, nothing [T, V] is stored): every
+// 128 x 128 tile runs two tcgen05 products into two TMEM accumulators,
+// z_s = hs . W_s^T (K = d_s) and z_t = ht . W_t^T (K = d_t).  With the
+// "primary" distribution p (the student for the reverse KL, the teacher for
+// the forward KL) and the other one q, each epilogue thread keeps, in base-2
+// units x = z log2(e),
+//   m_p, s_p = sum 2^(x_p - m_p), A = sum 2^(x_p - m_p) (x_p - x_q),
+//   m_q, s_q = sum 2^(x_q - m_q)
+// so that KL = ln2 * A / s_p - lse_p + lse_q.  Per-segment partials are
+// merged by the finalize kernel.
+//
+// Gradient: the logits are recomputed per tile and turned into
+//   reverse: G = g_t inv_tau p_s (log p_s - log p_t - KL_t)
+//   forward: G = g_t inv_tau (p_s - p_t)
+// stored as a bf16 slab, then d_h_s = G . W_s by the shared dh GEMM.
+#include <cmath>
+
+#include "gemm_core.cuh"
+#include "sched.cuh"
+
+namespace olive {
+namespace {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr int kKlBN = 128;
+
+struct KlFwdKern {
+  static constexpr int kBN = kKlBN;
+  static constexpr bool kAMn = false;
+  static constexpr bool kBMn = false;
+  static constexpr bool kDual = true;
+  static constexpr int kStages = 6;
+
+  struct Params {
+    int32_t* dev_status;
+    uint64_t wait_limit_ns;
+    const int32_t* n_rows;
+    int32_t T, V, d_s, d_t;
+    int32_t ctas, group_rows, ld, reverse;
+    float scale2;
+    float* part;  // [5][kSvMax][ld]: m_p, s_p, m_q, s_q, A
+  };
+  struct Sched {
+    Split sp;
+  };
+  static __device__ Sched make_sched(const Params& p) {
+    Sched s;
+    s.sp = choose_split(read_n_rows(p.n_rows, p.T, p.dev_status), (p.V + kBN - 1) / kBN, p.ctas);
+    return s;
+  }
+  static __device__ int num_units(const Params&, const Sched& s) { return s.sp.units; }
+  static __device__ void unit_pos(const Params& p, const Sched& s, int u, int& i, int& sg) {
+    const Raster r{s.sp.rt, s.sp.sv, p.group_rows};
+    r.tile(u, i, sg);
+  }
+  static __device__ int unit_len(const Params& p, const Sched& s, int u) {
+    int i, sg;
+    unit_pos(p, s, u, i, sg);
+    return min(s.sp.seg, s.sp.vt - sg * s.sp.seg);
+  }
+  static __device__ TileC tile(const Params& p, const Sched& s, int u, int t) {
+    int i, sg;
+    unit_pos(p, s, u, i, sg);
+    TileC c;
+    c.m0 = i * kBM;
+    c.n0 = (sg * s.sp.seg + t) * kBN;
+    c.ka0 = 0;
+    c.kb0 = 0;
+    c.nk = (p.d_s + kBK - 1) / kBK;
+    c.nk2 = (p.d_t + kBK - 1) / kBK;
+    return c;
+  }
+  struct Epi {
+    int r, sg;
+    float mp, sp, mq, sq, A;
+    __device__ void begin(const Params& p, const Sched& s, int u, int row) {
+      int i;
+      unit_pos(p, s, u, i, sg);
+      r = i * kBM + row;
+      mp = mq = -INFINITY;
+      sp = sq = A = 0.f;
+    }
+    __device__ void chunk(const Params& p, const uint32_t (&a)[32], const uint32_t (&b)[32], int col0) {
+      const int nvalid = p.V - col0;
+      float xp[32], xq[32];
+      float cp = -INFINITY, cq = -INFINITY;
+#pragma unroll
+      for (int k = 0; k < 32; ++k) {
+        const float xs = __uint_as_float(a[k]) * p.scale2;
+        const float xt = __uint_as_float(b[k]) * p.scale2;
+        const bool ok = k < nvalid;
+        xp[k] = ok ? (p.reverse ? xs : xt) : -INFINITY;
+        xq[k] = ok ? (p.reverse ? xt : xs) : -INFINITY;
+        cp = fmaxf(cp, xp[k]);
+        cq = fmaxf(cq, xq[k]);
+      }
+      const float mpn = fmaxf(mp, cp);
+      const float mqn = fmaxf(mq, cq);
+      const float rp = fast_exp2(mp - mpn);
+      float es = 0.f, ea = 0.f, eq = 0.f;
+#pragma unroll
+      for (int k = 0; k < 32; ++k) {
+        const bool ok = k < nvalid;
+        const float e = fast_exp2(xp[k] - mpn);
+        es += e;
+        ea += ok ? e * (xp[k] - xq[k]) : 0.f;
+        eq += fast_exp2(xq[k] - mqn);
+      }
+      sp = sp * rp + es;
+      A = A * rp + ea;
+      sq = sq * fast_exp2(mq - mqn) + eq;
+      mp = mpn;
+      mq = mqn;
+    }
+    __device__ void tile(const Params& p, const Sched&, int, int, const TileC& tc, uint32_t taddr) {
+#pragma unroll 1
+      for (int c = 0; c < kBN; c += 32) {
+        const int col0 = tc.n0 + c;
+        if (col0 >= p.V) break;
+        uint32_t a[32], b[32];
+        tmem_ld_32x32b_x32(taddr + c, a);
+        tmem_ld_32x32b_x32(taddr + kBN + c, b);
+        tmem_ld_wait();
+        chunk(p, a, b, col0);
+      }
+    }
+    __device__ void end(const Params& p, const Sched& s, int) {
+      if (r >= s.sp.n) return;
+      const size_t plane = static_cast<size_t>(kSvMax) * p.ld;
+      const size_t o = static_cast<size_t>(sg) * p.ld + r;
+      p.part[0 * plane + o] = mp;
+      p.part[1 * plane + o] = sp;
+      p.part[2 * plane + o] = mq;
+      p.part[3 * plane + o] = sq;
+      p.part[4 * plane + o] = A;
+    }
+  };
+};
+
+__global__ void kl_finalize_kernel(const int32_t* __restrict__ n_rows, const int32_t* __restrict__ rows,
+                                   int T, int vt, int ctas, int ld, int reverse,
+                                   const float* __restrict__ part, float* __restrict__ kl,
+                                   float* __restrict__ stats, int32_t* dev_status) {
+  __shared__ int sh_sv;
+  const int n = read_n_rows(n_rows, T, nullptr);
+  if (threadIdx.x == 0) sh_sv = choose_split(n, vt, ctas).sv;
+  __syncthreads();
+  const int sv = sh_sv;
+  const size_t plane = static_cast<size_t>(kSvMax) * ld;
+  for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < n; r += gridDim.x * blockDim.x) {
+    float Mp = -INFINITY, Mq = -INFINITY;
+    for (int s = 0; s < sv; ++s) {
+      Mp = fmaxf(Mp, part[0 * plane + static_cast<size_t>(s) * ld + r]);
+      Mq = fmaxf(Mq, part[2 * plane + static_cast<size_t>(s) * ld + r]);
+    }
+    float Sp = 0.f, Sq = 0.f, A = 0.f;
+    for (int s = 0; s < sv; ++s) {
+      const size_t o = static_cast<size_t>(s) * ld + r;
+      const float wp = exp2f(part[0 * plane + o] - Mp);
+      Sp += part[1 * plane + o] * wp;
+      A += part[4 * plane + o] * wp;
+      Sq += part[3 * plane + o] * exp2f(part[2 * plane + o] - Mq);
+    }
+    const float lse_p = (Mp + log2f(Sp)) * kLn2;
+    const float lse_q = (Mq + log2f(Sq)) * kLn2;
+    const float k = kLn2 * (A / Sp) - lse_p + lse_q;
+    stats[0 * static_cast<size_t>(ld) + r] = reverse ? lse_p : lse_q;  // lse_s
+    stats[1 * static_cast<size_t>(ld) + r] = reverse ? lse_q : lse_p;  // lse_t
+    stats[2 * static_cast<size_t>(ld) + r] = k;
+    const int t = rows[r];
+    if (t >= 0 && t < T) kl[t] = k;
+  }
+}
+
+struct KlGradKern {
+  static constexpr int kBN = kKlBN;
+  static constexpr bool kAMn = false;
+  static constexpr bool kBMn = false;
+  static constexpr bool kDual = true;
+  static constexpr int kStages = 6;
+
+  struct Params {
+    int32_t* dev_status;
+    uint64_t wait_limit_ns;
+    const int32_t* n_rows;
+    const int32_t* rows;
+    const float* grad_kl;
+    const float* stats;
+    int32_t T, V, d_s, d_t, ld, reverse, group_rows;
+    int64_t slab_start, tc, ldg;
+    float inv_tau, scale2;
+    __nv_bfloat16* g;
+  };
+  struct Sched {
+    int n, in_slab, mt, vt, units;
+  };
+  static __device__ Sched make_sched(const Params& p) {
+    Sched s;
+    s.n = read_n_rows(p.n_rows, p.T, p.dev_status);
+    long long k = s.n - p.slab_start;
+    if (k < 0) k = 0;
+    if (k > p.tc) k = p.tc;
+    s.in_slab = static_cast<int>(k);
+    s.mt = (s.in_slab + kBM - 1) / kBM;
+    s.vt = (p.V + kBN - 1) / kBN;
+    s.units = s.mt * s.vt;
+    return s;
+  }
+  static __device__ int num_units(const Params&, const Sched& s) { return s.units; }
+  static __device__ int unit_len(const Params&, const Sched&, int) { return 1; }
+  static __device__ void pos(const Params& p, const Sched& s, int u, int& i, int& j) {
+    const Raster r{s.mt, s.vt, p.group_rows};
+    r.tile(u, i, j);
+  }
+  static __device__ TileC tile(const Params& p, const Sched& s, int u, int) {
+    int i, j;
+    pos(p, s, u, i, j);
+    TileC c;
+    c.m0 = static_cast<int>(p.slab_start) + i * kBM;
+    c.n0 = j * kBN;
+    c.ka0 = 0;
+    c.kb0 = 0;
+    c.nk = (p.d_s + kBK - 1) / kBK;
+    c.nk2 = (p.d_t + kBK - 1) / kBK;
+    return c;
+  }
+  struct Epi {
+    int r_local;
+    bool valid;
+    float ls2, lt2, kl, coef;
+    __device__ void begin(const Params& p, const Sched& s, int u, int row) {
+      int i, j;
+      pos(p, s, u, i, j);
+      r_local = i * kBM + row;
+      const long long r = p.slab_start + r_local;
+      valid = r < s.n;
+      ls2 = lt2 = kl = coef = 0.f;
+      if (valid) {
+        const int t = p.rows[r];
+        if (t >= 0 && t < p.T) {
+          ls2 = p.stats[0 * static_cast<size_t>(p.ld) + r] * kLog2e;
+          lt2 = p.stats[1 * static_cast<size_t>(p.ld) + r] * kLog2e;
+          kl = p.stats[2 * static_cast<size_t>(p.ld) + r];
+          coef = p.grad_kl[t] * p.inv_tau;
+        } else {
+          valid = false;
+        }
+      }
+    }
+    __device__ void tile(const Params& p, const Sched&, int, int, const TileC& tc, uint32_t taddr) {
+      __nv_bfloat16* grow = p.g + static_cast<size_t>(r_local) * p.ldg;
+#pragma unroll 1
+      for (int c = 0; c < kBN; c += 32) {
+        const int col0 = tc.n0 + c;
+        if (col0 >= p.V) break;
+        uint32_t a[32], b[32];
+        tmem_ld_32x32b_x32(taddr + c, a);
+        tmem_ld_32x32b_x32(taddr + kBN + c, b);
+        tmem_ld_wait();
+        float g[32];
+#pragma unroll
+        for (int k = 0; k < 32; ++k) {
+          const float ys = __uint_as_float(a[k]) * p.scale2 - ls2;  // log2 p_s
+          const float yt = __uint_as_float(b[k]) * p.scale2 - lt2;  // log2 p_t
+          const float ps = fast_exp2(ys);
+          float v;
+          if (p.reverse) v = ps * ((ys - yt) * kLn2 - kl);
+          else v = ps - fast_exp2(yt);
+          g[k] = valid ? coef * v : 0.f;
+        }
+        if (col0 + 32 <= p.V) {
+          store_bf16x32_kl(grow + col0, g);
+        } else {
+          const int nv = p.V - col0;
+#pragma unroll
+          for (int k = 0; k < 32; ++k)
+            if (k < nv) grow[col0 + k] = __float2bfloat16_rn(g[k]);
+        }
+      }
+    }
+    __device__ void end(const Params&, const Sched&, int) {}
+
+    __device__ static void store_bf16x32_kl(__nv_bfloat16* dst, const float (&g)[32]) {
+      uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        uint4 v;
+        v.x = pack_bf16x2(g[8 * q + 0], g[8 * q + 1]);
+        v.y = pack_bf16x2(g[8 * q + 2], g[8 * q + 3]);
+        v.z = pack_bf16x2(g[8 * q + 4], g[8 * q + 5]);
+        v.w = pack_bf16x2(g[8 * q + 6], g[8 * q + 7]);
+        d4[q] = v;
+      }
+    }
+  };
+};
+
+template <class K>
+olive_status launch_dual(const Ctx& c, const CUtensorMap& a, const CUtensorMap& b,
+                         const CUtensorMap& a2, const CUtensorMap& b2, const typename K::Params& p) {
+  const int smem = core_smem_bytes<K>();
+  if (cudaFuncSetAttribute(gemm_persistent<K>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+      cudaSuccess)
+    return OLIVE_ERR_CUDA;
+  gemm_persistent<K><<<c.num_sms, kThreads, smem, c.stream>>>(a, b, a2, b2, p);
+  return cudaGetLastError() == cudaSuccess ? OLIVE_OK : OLIVE_ERR_CUDA;
+}
+
+}  // namespace
+
+olive_status launch_divergence(const Ctx& c, const void* h_s, const void* W_s, int32_t d_s,
+                               const void* h_t, const void* W_t, int32_t d_t, const int32_t* rows,
+                               const int32_t* n_rows, int32_t T, int32_t V, float inv_tau,
+                               int direction, float* kl, const float* grad_kl, void* d_h_s,
+                               int grad_dtype, void* ws, int32_t* dev_status) {
+  const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
+  const int grad = d_h_s != nullptr;
+  const KlWs w = carve_kl(ws, T, d_s, d_t, V, grad);
+  const int reverse = direction == OLIVE_KL_REVERSE;
+  olive_status st;
+  if ((st = launch_gather_rows(c, h_s, rows, n_rows, T, d_s, w.hcs, dev_status)) != OLIVE_OK) return st;
+  if ((st = launch_gather_rows(c, h_t, rows, n_rows, T, d_t, w.hct, dev_status)) != OLIVE_OK) return st;
+  if (cudaMemsetAsync(kl, 0, sizeof(float) * T, c.stream) != cudaSuccess) return OLIVE_ERR_CUDA;
+
+  CUtensorMap mHs, mWs, mHt, mWt;
+  if (!encode_bf16_2d(&mHs, w.hcs, d_s, Tpad, 2ull * d_s, 64, 128)) return OLIVE_ERR_CUDA;
+  if (!encode_bf16_2d(&mWs, W_s, d_s, V, 2ull * d_s, 64, kKlBN)) return OLIVE_ERR_CUDA;
+  if (!encode_bf16_2d(&mHt, w.hct, d_t, Tpad, 2ull * d_t, 64, 128)) return OLIVE_ERR_CUDA;
+  if (!encode_bf16_2d(&mWt, W_t, d_t, V, 2ull * d_t, 64, kKlBN)) return OLIVE_ERR_CUDA;
+
+  KlFwdKern::Params p;
+  p.dev_status = dev_status;
+  p.wait_limit_ns = c.wait_limit_ns;
+  p.n_rows = n_rows;
+  p.T = T;
+  p.V = V;
+  p.d_s = d_s;
+  p.d_t = d_t;
+  p.ctas = c.num_sms;
+  p.group_rows = 16;
+  p.ld = static_cast<int32_t>(Tpad);
+  p.reverse = reverse;
+  p.scale2 = inv_tau * kLog2e;
+  p.part = w.part;
+  if ((st = launch_dual<KlFwdKern>(c, mHs, mWs, mHt, mWt, p)) != OLIVE_OK) return st;
+
+  const int vt = (V + kKlBN - 1) / kKlBN;
+  kl_finalize_kernel<<<c.num_sms * 4, 256, 0, c.stream>>>(n_rows, rows, T, vt, c.num_sms, p.ld,
+                                                           reverse, w.part, kl, w.stats, dev_status);
+  if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;
+  if (!grad) return OLIVE_OK;
+
+  const size_t elt = grad_dtype == OLIVE_DTYPE_BF16 ? 2 : 4;
+  if (cudaMemsetAsync(d_h_s, 0, elt * T * static_cast<size_t>(d_s), c.stream) != cudaSuccess)
+    return OLIVE_ERR_CUDA;
+  const int64_t ldg = vpad(V);
+  const int64_t n_slabs = ceil_div(Tpad, w.tc);
+  for (int64_t sl = 0; sl < n_slabs; ++sl) {
+    KlGradKern::Params gp;
+    gp.dev_status = dev_status;
+    gp.wait_limit_ns = c.wait_limit_ns;
+    gp.n_rows = n_rows;
+    gp.rows = rows;
+    gp.grad_kl = grad_kl;
+    gp.stats = w.stats;
+    gp.T = T;
+    gp.V = V;
+    gp.d_s = d_s;
+    gp.d_t = d_t;
+    gp.ld = p.ld;
+    gp.reverse = reverse;
+    gp.group_rows = 16;
+    gp.slab_start = sl * w.tc;
+    gp.tc = w.tc;
+    gp.ldg = ldg;
+    gp.inv_tau = inv_tau;
+    gp.scale2 = inv_tau * kLog2e;
+    gp.g = static_cast<__nv_bfloat16*>(w.g);
+    if ((st = launch_dual<KlGradKern>(c, mHs, mWs, mHt, mWt, gp)) != OLIVE_OK) return st;
+    if ((st = launch_dh_slab(c, w.g, ldg, w.tc, W_s, d_s, V, rows, n_rows, T, sl * w.tc, d_h_s,
+                             grad_dtype, dev_status)) != OLIVE_OK)
+      return st;
+  }
+  return OLIVE_OK;
+}
+
+}  // namespace olive

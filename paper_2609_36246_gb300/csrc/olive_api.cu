@@ -1,0 +1,308 @@
+// olive_api.cu -- the extern "C" entry points of libolive.so (include/olive.h):
+// host-side argument checks, workspace layout, device checks and the
+// tensor-map encoder.  All compute is in the kernels of the other files.
+#include <cudaTypedefs.h>
+
+#include <cstdlib>
+#include <mutex>
+
+#include "internal.h"
+
+namespace olive {
+
+namespace {
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  });
+  return fn;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+uint64_t wait_limit_from_env() {
+  // OLIVE_WAIT_LIMIT_MS bounds every internal wait of the GEMM kernels
+  // (default 1000 ms; 0 makes the first unsatisfied wait give up, which the
+  // tests use to exercise the timeout path).
+  const char* s = std::getenv("OLIVE_WAIT_LIMIT_MS");
+  if (!s || !*s) return 1000ull * 1000ull * 1000ull;
+  char* end = nullptr;
+  const unsigned long long ms = std::strtoull(s, &end, 10);
+  if (end == s) return 1000ull * 1000ull * 1000ull;
+  return static_cast<uint64_t>(ms) * 1000ull * 1000ull;
+}
+
+}  // namespace
+
+olive_status make_ctx(void* stream, Ctx* ctx) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return OLIVE_ERR_CUDA;
+  }
+  int major = 0, minor = 0, sms = 0;
+  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+    cudaGetLastError();
+    return OLIVE_ERR_CUDA;
+  }
+  if (major != 10 || minor != 3) return OLIVE_ERR_UNSUPPORTED_DEVICE;
+  if (!encode_fn()) return OLIVE_ERR_CUDA;
+  ctx->stream = static_cast<cudaStream_t>(stream);
+  ctx->device = dev;
+  ctx->num_sms = sms;
+  ctx->wait_limit_ns = wait_limit_from_env();
+  return OLIVE_OK;
+}
+
+bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+                    uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {row_bytes};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
+                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+int64_t slab_rows(int64_t Tpad, int64_t V) {
+  // G slab of at most ~2.5 GB (bf16), in whole 128-row tiles, <= 16384 rows
+  const int64_t budget = 2500ll * 1000 * 1000;
+  int64_t tc = budget / (2 * vpad(V)) / kRowAlign * kRowAlign;
+  if (tc < kRowAlign) tc = kRowAlign;
+  if (tc > 16384) tc = 16384;
+  if (tc > Tpad) tc = Tpad;
+  return tc;
+}
+
+// ------------------------------------------------------------- workspace ---
+namespace {
+struct Carver {
+  char* base;
+  size_t off = 0;
+  void* take(size_t bytes) {
+    void* p = base ? base + off : nullptr;
+    off = align_up(off + bytes, kWsAlign);
+    return p;
+  }
+};
+}  // namespace
+
+static FwdWs carve_fwd_impl(void* ws, int64_t T, int64_t d, size_t* total) {
+  const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
+  Carver c{static_cast<char*>(ws)};
+  FwdWs w;
+  w.hc = c.take(2ull * Tpad * d);
+  w.part_m = static_cast<float*>(c.take(4ull * kSvMax * Tpad));
+  w.part_s = static_cast<float*>(c.take(4ull * kSvMax * Tpad));
+  w.zy = static_cast<float*>(c.take(4ull * Tpad));
+  w.nll = static_cast<float*>(c.take(4ull * Tpad));
+  if (total) *total = c.off;
+  return w;
+}
+size_t fwd_ws_bytes(int64_t T, int64_t d) {
+  size_t n = 0;
+  carve_fwd_impl(nullptr, T, d, &n);
+  return n;
+}
+FwdWs carve_fwd(void* ws, int64_t T, int64_t d) { return carve_fwd_impl(ws, T, d, nullptr); }
+
+static BwdWs carve_bwd_impl(void* ws, int64_t T, int64_t d, int64_t V, int grad_dtype,
+                            size_t* total) {
+  const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
+  Carver c{static_cast<char*>(ws)};
+  BwdWs w;
+  w.tc = slab_rows(Tpad, V);
+  w.hc = c.take(2ull * Tpad * d);
+  w.g = c.take(2ull * w.tc * vpad(V));
+  w.dw_acc = grad_dtype == OLIVE_DTYPE_BF16 ? static_cast<float*>(c.take(4ull * V * d)) : nullptr;
+  if (total) *total = c.off;
+  return w;
+}
+size_t bwd_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype) {
+  size_t n = 0;
+  carve_bwd_impl(nullptr, T, d, V, grad_dtype, &n);
+  return n;
+}
+BwdWs carve_bwd(void* ws, int64_t T, int64_t d, int64_t V, int grad_dtype) {
+  return carve_bwd_impl(ws, T, d, V, grad_dtype, nullptr);
+}
+
+static KlWs carve_kl_impl(void* ws, int64_t T, int64_t ds, int64_t dt, int64_t V, int grad,
+                          size_t* total) {
+  const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
+  Carver c{static_cast<char*>(ws)};
+  KlWs w;
+  w.tc = slab_rows(Tpad, V);
+  w.hcs = c.take(2ull * Tpad * ds);
+  w.hct = c.take(2ull * Tpad * dt);
+  w.part = static_cast<float*>(c.take(4ull * 5 * kSvMax * Tpad));
+  w.stats = static_cast<float*>(c.take(4ull * 3 * Tpad));
+  w.g = grad ? c.take(2ull * w.tc * vpad(V)) : nullptr;
+  if (total) *total = c.off;
+  return w;
+}
+size_t kl_ws_bytes(int64_t T, int64_t ds, int64_t dt, int64_t V, int grad) {
+  size_t n = 0;
+  carve_kl_impl(nullptr, T, ds, dt, V, grad, &n);
+  return n;
+}
+KlWs carve_kl(void* ws, int64_t T, int64_t ds, int64_t dt, int64_t V, int grad) {
+  return carve_kl_impl(ws, T, ds, dt, V, grad, nullptr);
+}
+
+}  // namespace olive
+
+using namespace olive;
+
+namespace {
+
+constexpr int32_t kMaxDim = 1 << 20;  // widths above this are rejected
+
+olive_status check_ws(void* ws, size_t have, size_t need) {
+  if (need == 0) return OLIVE_ERR_SHAPE;
+  if (!ws || have < need || (reinterpret_cast<uintptr_t>(ws) & (kWsAlign - 1)) != 0)
+    return OLIVE_ERR_WORKSPACE;
+  return OLIVE_OK;
+}
+
+bool width_ok(int32_t d) { return d >= 8 && d <= kMaxDim && (d % 8) == 0; }
+
+}  // namespace
+
+extern "C" {
+
+int olive_abi_version(void) { return OLIVE_ABI_VERSION; }
+
+const char* olive_status_string(olive_status s) {
+  switch (s) {
+    case OLIVE_OK: return "ok";
+    case OLIVE_ERR_INVALID_ARG: return "invalid argument (null pointer or bad enum)";
+    case OLIVE_ERR_SHAPE: return "invalid shape";
+    case OLIVE_ERR_ALIGNMENT: return "pointer or width breaks the 16-byte rule";
+    case OLIVE_ERR_TOKEN_RANGE: return "token id or target outside [0, V)";
+    case OLIVE_ERR_OFFSETS: return "malformed offsets or row list";
+    case OLIVE_ERR_TIMEOUT: return "an internal wait ran out of time";
+    case OLIVE_ERR_UNSUPPORTED_DEVICE: return "device is not compute capability 10.3";
+    case OLIVE_ERR_CUDA: return "CUDA call failed";
+    case OLIVE_ERR_WORKSPACE: return "workspace null, misaligned or too small";
+  }
+  return "unknown status";
+}
+
+size_t olive_workspace_size(int op, int32_t T, int32_t d, int32_t d_t, int32_t V, int grad,
+                            int grad_dtype) {
+  if (T < 1 || V < 1 || !width_ok(d)) return 0;
+  switch (op) {
+    case OLIVE_OP_LOGPROB_FWD: return fwd_ws_bytes(T, d);
+    case OLIVE_OP_LOSS_BWD:
+      if (grad_dtype != OLIVE_DTYPE_BF16 && grad_dtype != OLIVE_DTYPE_F32) return 0;
+      return bwd_ws_bytes(T, d, V, grad_dtype);
+    case OLIVE_OP_DIVERGENCE:
+      if (!width_ok(d_t)) return 0;
+      return kl_ws_bytes(T, d, d_t, V, grad);
+    default: return 0;
+  }
+}
+
+olive_status olive_splice_pack(const int32_t* prefix_ids, const int32_t* prefix_off,
+                               const int32_t* cont_ids, const int32_t* cont_off, int32_t S,
+                               int32_t V, int32_t T_cap, int32_t* ids, int32_t* targets,
+                               uint8_t* loss_mask, int32_t* cu_seqlens, int32_t* cut_offsets,
+                               int32_t* rows, int32_t* n_rows, int32_t* dev_status, void* stream) {
+  if (!prefix_ids || !prefix_off || !cont_ids || !cont_off || !ids || !targets || !loss_mask ||
+      !cu_seqlens || !cut_offsets || !rows || !n_rows || !dev_status)
+    return OLIVE_ERR_INVALID_ARG;
+  if (S < 1 || V < 1 || T_cap < 1) return OLIVE_ERR_SHAPE;
+  Ctx c;
+  olive_status st = make_ctx(stream, &c);
+  if (st != OLIVE_OK) return st;
+  return launch_splice_pack(c, prefix_ids, prefix_off, cont_ids, cont_off, S, V, T_cap, ids,
+                            targets, loss_mask, cu_seqlens, cut_offsets, rows, n_rows, dev_status);
+}
+
+olive_status olive_token_logprob_fwd(const void* hidden, const void* W, const int32_t* targets,
+                                     const int32_t* rows, const int32_t* n_rows, int32_t T,
+                                     int32_t d, int32_t V, float inv_tau, int reduction,
+                                     float* logp, float* lse, float* loss, void* workspace,
+                                     size_t ws_bytes, int32_t* dev_status, void* stream) {
+  if (!hidden || !W || !targets || !rows || !n_rows || !logp || !lse || !loss || !dev_status)
+    return OLIVE_ERR_INVALID_ARG;
+  if (reduction != OLIVE_REDUCE_SUM && reduction != OLIVE_REDUCE_MEAN) return OLIVE_ERR_INVALID_ARG;
+  if (T < 1 || V < 1 || d < 1 || d > kMaxDim) return OLIVE_ERR_SHAPE;
+  if (!(inv_tau > 0.f) || !std::isfinite(inv_tau)) return OLIVE_ERR_INVALID_ARG;
+  if (d % 8 != 0 || !aligned16(hidden) || !aligned16(W)) return OLIVE_ERR_ALIGNMENT;
+  olive_status st = check_ws(workspace, ws_bytes, fwd_ws_bytes(T, d));
+  if (st != OLIVE_OK) return st;
+  Ctx c;
+  st = make_ctx(stream, &c);
+  if (st != OLIVE_OK) return st;
+  return launch_logprob_fwd(c, hidden, W, targets, rows, n_rows, T, d, V, inv_tau, reduction, logp,
+                            lse, loss, workspace, dev_status);
+}
+
+olive_status olive_token_loss_bwd(const void* hidden, const void* W, const int32_t* targets,
+                                  const int32_t* rows, const int32_t* n_rows, int32_t T, int32_t d,
+                                  int32_t V, float inv_tau, int reduction, const float* lse,
+                                  const float* grad_loss, void* d_hidden, void* d_W,
+                                  int grad_dtype, void* workspace, size_t ws_bytes,
+                                  int32_t* dev_status, void* stream) {
+  if (!hidden || !W || !targets || !rows || !n_rows || !lse || !grad_loss || !d_hidden || !d_W ||
+      !dev_status)
+    return OLIVE_ERR_INVALID_ARG;
+  if (reduction != OLIVE_REDUCE_SUM && reduction != OLIVE_REDUCE_MEAN) return OLIVE_ERR_INVALID_ARG;
+  if (grad_dtype != OLIVE_DTYPE_BF16 && grad_dtype != OLIVE_DTYPE_F32) return OLIVE_ERR_INVALID_ARG;
+  if (T < 1 || V < 1 || d < 1 || d > kMaxDim) return OLIVE_ERR_SHAPE;
+  if (!(inv_tau > 0.f) || !std::isfinite(inv_tau)) return OLIVE_ERR_INVALID_ARG;
+  if (d % 8 != 0 || !aligned16(hidden) || !aligned16(W) || !aligned16(d_hidden) || !aligned16(d_W))
+    return OLIVE_ERR_ALIGNMENT;
+  olive_status st = check_ws(workspace, ws_bytes, bwd_ws_bytes(T, d, V, grad_dtype));
+  if (st != OLIVE_OK) return st;
+  Ctx c;
+  st = make_ctx(stream, &c);
+  if (st != OLIVE_OK) return st;
+  return launch_loss_bwd(c, hidden, W, targets, rows, n_rows, T, d, V, inv_tau, reduction, lse,
+                         grad_loss, d_hidden, d_W, grad_dtype, workspace, dev_status);
+}
+
+olive_status olive_token_divergence(const void* h_s, const void* W_s, int32_t d_s, const void* h_t,
+                                    const void* W_t, int32_t d_t, const int32_t* rows,
+                                    const int32_t* n_rows, int32_t T, int32_t V, float inv_tau,
+                                    int direction, float* kl, const float* grad_kl, void* d_h_s,
+                                    int grad_dtype, void* workspace, size_t ws_bytes,
+                                    int32_t* dev_status, void* stream) {
+  if (!h_s || !W_s || !h_t || !W_t || !rows || !n_rows || !kl || !dev_status)
+    return OLIVE_ERR_INVALID_ARG;
+  if ((grad_kl == nullptr) != (d_h_s == nullptr)) return OLIVE_ERR_INVALID_ARG;
+  if (direction != OLIVE_KL_REVERSE && direction != OLIVE_KL_FORWARD) return OLIVE_ERR_INVALID_ARG;
+  if (grad_dtype != OLIVE_DTYPE_BF16 && grad_dtype != OLIVE_DTYPE_F32) return OLIVE_ERR_INVALID_ARG;
+  if (T < 1 || V < 1 || d_s < 1 || d_t < 1 || d_s > kMaxDim || d_t > kMaxDim) return OLIVE_ERR_SHAPE;
+  if (!(inv_tau > 0.f) || !std::isfinite(inv_tau)) return OLIVE_ERR_INVALID_ARG;
+  if (d_s % 8 != 0 || d_t % 8 != 0 || !aligned16(h_s) || !aligned16(W_s) || !aligned16(h_t) ||
+      !aligned16(W_t) || (d_h_s && !aligned16(d_h_s)))
+    return OLIVE_ERR_ALIGNMENT;
+  const int grad = d_h_s != nullptr;
+  olive_status st = check_ws(workspace, ws_bytes, kl_ws_bytes(T, d_s, d_t, V, grad));
+  if (st != OLIVE_OK) return st;
+  Ctx c;
+  st = make_ctx(stream, &c);
+  if (st != OLIVE_OK) return st;
+  return launch_divergence(c, h_s, W_s, d_s, h_t, W_t, d_t, rows, n_rows, T, V, inv_tau, direction,
+                           kl, grad_kl, d_h_s, grad_dtype, workspace, dev_status);
+}
+
+}  // extern "C"

@@ -1,0 +1,62 @@
+// sched.cuh -- device-side work decomposition shared by the kernels that
+// reduce a row over vocabulary tiles (forward log-sum-exp, divergence).
+//
+// The row count N_mask lives on the device, so every CTA (and the finalize
+// kernels) derive the same decomposition from it: rt row tiles of 128 rows,
+// vt vocabulary tiles, split into sv contiguous segments of seg tiles.  A
+// unit is one (row tile, segment); its partial (max, sum) per row is merged by
+// the finalize kernel.  sv is chosen to minimise the critical path
+// ceil(units / ctas) * seg, which removes most of the wave-quantisation loss
+// when rt is small compared with the SM count.
+#pragma once
+
+#include "internal.h"
+
+namespace olive {
+
+struct Split {
+  int n;     // valid rows
+  int rt;    // row tiles
+  int vt;    // vocabulary tiles
+  int sv;    // segments
+  int seg;   // tiles per segment
+  int units; // rt * sv
+};
+
+__host__ __device__ inline Split choose_split(int n, int vt, int ctas) {
+  Split s;
+  s.n = n;
+  s.rt = (n + 127) / 128;
+  s.vt = vt;
+  int best_sv = 1;
+  long long best_cost = -1;
+  const int max_sv = vt < kSvMax ? vt : kSvMax;
+  for (int sv = 1; sv <= max_sv; ++sv) {
+    const int seg = (vt + sv - 1) / sv;
+    const int sv_eff = (vt + seg - 1) / seg;
+    if (sv_eff != sv) continue;
+    const long long units = static_cast<long long>(s.rt) * sv;
+    const long long waves = (units + ctas - 1) / ctas;
+    // a unit also pays a pipeline fill and a partial write: ~1/8 tile
+    const long long cost = waves * (8LL * seg + 1);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best_sv = sv;
+    }
+  }
+  s.sv = best_sv;
+  s.seg = (vt + best_sv - 1) / best_sv;
+  s.units = s.rt * s.sv;
+  return s;
+}
+
+__device__ inline int read_n_rows(const int32_t* n_rows, int T, int32_t* dev_status) {
+  int n = *n_rows;
+  if (n < 0 || n > T) {
+    if (dev_status) atomicOr(dev_status, 1 << OLIVE_ERR_OFFSETS);
+    n = n < 0 ? 0 : T;
+  }
+  return n;
+}
+
+}  // namespace olive

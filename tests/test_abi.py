@@ -1,0 +1,127 @@
+"""Host-side checks of libolive.so that need no GPU.
+
+The library is (re)built with nvcc for sm_103a, loaded, and every entry point
+declared in include/olive.h must be exported.  Argument validation happens
+before any CUDA call, so bad pointers, shapes, alignment and workspace sizes
+are rejected here with the documented status codes; a call that passes
+validation on a machine without a usable device ends in OLIVE_ERR_CUDA (or
+OLIVE_ERR_UNSUPPORTED_DEVICE) without launching anything.
+"""
+
+import ctypes
+
+import pytest
+import torch
+
+from paper_2609_36246_gb300 import binding as B
+from paper_2609_36246_gb300 import build
+
+
+@pytest.fixture(scope="module")
+def L():
+    build.build()
+    return B.lib()
+
+
+def test_exports_every_declared_symbol(L):
+    names = B.declared_symbols()
+    assert set(names) >= {"olive_splice_pack", "olive_token_logprob_fwd", "olive_token_loss_bwd",
+                          "olive_token_divergence", "olive_workspace_size", "olive_status_string",
+                          "olive_abi_version"}
+    for n in names:
+        assert hasattr(L, n), n
+
+
+def test_abi_version_and_status_strings(L):
+    assert B.olive_abi_version() == 1
+    for code in range(10):
+        s = B.olive_status_string(code)
+        assert s and s != "unknown status"
+    assert B.olive_status_string(42) == "unknown status"
+
+
+def test_workspace_sizes(L):
+    T, d, V = 32768, 4096, 151936
+    fwd = B.olive_workspace_size("logprob_fwd", T, d, V)
+    bwd16 = B.olive_workspace_size("loss_bwd", T, d, V, grad_dtype=torch.bfloat16)
+    bwd32 = B.olive_workspace_size("loss_bwd", T, d, V, grad_dtype=torch.float32)
+    kl = B.olive_workspace_size("divergence", 16384, 4096, V, d_t=5120, grad=True)
+    assert fwd >= 2 * T * d and fwd % 256 == 0
+    # bf16 dW needs the fp32 accumulator on top
+    assert bwd16 - bwd32 >= 4 * V * d
+    assert kl > B.olive_workspace_size("divergence", 16384, 4096, V, d_t=5120, grad=False)
+    # invalid requests give 0
+    assert B.olive_workspace_size("logprob_fwd", 0, d, V) == 0
+    assert B.olive_workspace_size("logprob_fwd", T, 12, V) == 0
+    assert L.olive_workspace_size(7, T, d, 0, V, 1, 0) == 0
+
+
+def _fake(n=1 << 20):
+    # host buffer used only for its (16-byte aligned) address: validation
+    # never dereferences it
+    buf = ctypes.create_string_buffer(n + 256)
+    base = (ctypes.addressof(buf) + 255) // 256 * 256
+    return buf, base
+
+
+def test_fwd_argument_validation(L):
+    keep, p = _fake()
+    P = ctypes.c_void_p
+    args = dict(hidden=P(p), W=P(p), targets=P(p), rows=P(p), n_rows=P(p), T=64, d=64, V=100,
+                inv_tau=1.0, red=0, logp=P(p), lse=P(p), loss=P(p), ws=P(p), ws_bytes=1 << 20,
+                st=P(p), stream=None)
+
+    def call(**kw):
+        a = dict(args, **kw)
+        return L.olive_token_logprob_fwd(a["hidden"], a["W"], a["targets"], a["rows"], a["n_rows"],
+                                         a["T"], a["d"], a["V"], a["inv_tau"], a["red"], a["logp"],
+                                         a["lse"], a["loss"], a["ws"], a["ws_bytes"], a["st"],
+                                         a["stream"])
+
+    assert call(hidden=None) == 1
+    assert call(red=5) == 1
+    assert call(inv_tau=0.0) == 1
+    assert call(inv_tau=float("nan")) == 1
+    assert call(T=0) == 2
+    assert call(V=0) == 2
+    assert call(d=60) == 3
+    assert call(hidden=P(p + 2)) == 3
+    assert call(ws_bytes=16) == 9
+    assert call(ws=P(p + 8)) == 9
+    assert call(ws=None) == 1 or call(ws=None) == 9
+    # valid arguments: without a usable sm_103 device nothing launches
+    if not torch.cuda.is_available():
+        assert call() in (7, 8)
+
+
+def test_bwd_and_divergence_validation(L):
+    keep, p = _fake()
+    P = ctypes.c_void_p
+    # bwd: bad grad dtype, misaligned d_W
+    st = L.olive_token_loss_bwd(P(p), P(p), P(p), P(p), P(p), 64, 64, 100, 1.0, 0, P(p), P(p),
+                                P(p), P(p), 3, P(p), 1 << 20, P(p), None)
+    assert st == 1
+    st = L.olive_token_loss_bwd(P(p), P(p), P(p), P(p), P(p), 64, 64, 100, 1.0, 0, P(p), P(p),
+                                P(p), P(p + 4), 0, P(p), 1 << 20, P(p), None)
+    assert st == 3
+    # divergence: grad_kl without d_h_s
+    st = L.olive_token_divergence(P(p), P(p), 64, P(p), P(p), 64, P(p), P(p), 64, 100, 1.0, 0,
+                                  P(p), P(p), None, 0, P(p), 1 << 20, P(p), None)
+    assert st == 1
+    st = L.olive_token_divergence(P(p), P(p), 64, P(p), P(p), 64, P(p), P(p), 64, 100, 1.0, 9,
+                                  P(p), None, None, 0, P(p), 1 << 20, P(p), None)
+    assert st == 1
+    # splice/pack: empty batch, null output
+    st = L.olive_splice_pack(P(p), P(p), P(p), P(p), 0, 10, 10, P(p), P(p), P(p), P(p), P(p), P(p),
+                             P(p), P(p), None)
+    assert st == 2
+    st = L.olive_splice_pack(P(p), P(p), P(p), P(p), 1, 10, 10, None, P(p), P(p), P(p), P(p), P(p),
+                             P(p), P(p), None)
+    assert st == 1
+
+
+def test_binding_rejects_cpu_tensors(L):
+    h = torch.zeros(8, 64, dtype=torch.bfloat16)
+    with pytest.raises(TypeError):
+        B.olive_token_logprob_fwd(h, h, torch.zeros(8, dtype=torch.int32),
+                                  torch.zeros(8, dtype=torch.int32), torch.zeros(1, dtype=torch.int32))
