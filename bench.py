@@ -1,0 +1,364 @@
+"""Throughput of the OLIVE per-token training path on GB300.
+
+One step = the whole hot path over one packed batch: splice/pack of the
+spliced sequences (student prefix || teacher continuation), the LM-head
+forward with online log-sum-exp and the masked continuation loss of Eq.
+(osd-ce), and its backward (d hidden, d W in bf16).  Workload: 8 sequences of
+4096 tokens, cut ~ U[256, 3840), d = 4096, V = 151936, bf16, synthetic seeded
+data (the "fwdbwd" workload of paper_2609_36246_gb300.synth).
+
+Metric: masked continuation tokens per second, i.e. N_mask * steps / time,
+and the fraction of bf16 dense tensor peak of the counted work
+6 * N_mask * d * V FLOPs per step (logit recomputation is not counted).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun (N > 1) every rank runs its own batch of the same shape with
+no collective on the data path (weak scaling); rank 0 prints the line.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "masked continuation tokens/sec (fwd+bwd, fused LM-head loss) and % bf16 tensor peak"
+WORKLOAD = "fwdbwd"
+CONFIG = {"workload": "fused fwd+bwd LM-head loss: 8 x 4096 packed tokens, cut ~ U[256,3840), "
+                      "d=4096, V=151936, bf16",
+          "S": 8, "seq_len": 4096, "d": 4096, "V": 151936, "grad_dtype": "bf16",
+          "l2": "inputs larger than L2 (hidden 268 MB, W 1.24 GB)"}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d.get("bf16_tflops", 1900.0), d.get("bf16_tflops_sustained", 1700.0), "measured"
+    return 1900.0, 1700.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling while the timed region runs."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        self.out = ""
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out = ""
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in (self.out or "").splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if torch.cuda.is_available():
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(0)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda" if torch.cuda.is_available() else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def make_inputs(rank: int):
+    from paper_2609_36246_gb300 import synth
+    b = synth.make_batch(WORKLOAD)
+    h = synth.make_hidden(WORKLOAD, b.T)
+    W = synth.make_weight(WORKLOAD)
+    return b, h, W
+
+
+# --------------------------------------------------------------------------- oracle legs
+def oracle_sample_rate(b, h, W, n_rows: int, seed: int = 0):
+    """fp64 oracle on a sample of masked rows: forward log-probs, dH of those
+    rows and their dW contribution (the same per-row work as one step).
+    Returns (masked tokens per second, seconds, rows)."""
+    import oracle
+    o = oracle.splice_pack(b.prefix_ids, b.prefix_off, b.cont_ids, b.cont_off, b.V)
+    rng = np.random.default_rng(seed)
+    rows = np.sort(rng.choice(o["rows"], size=min(n_rows, len(o["rows"])), replace=False))
+    hf = h.float().numpy()
+    Wf = W.float().numpy()
+    t0 = time.perf_counter()
+    oracle.token_logprob(hf, Wf, o["targets"], rows)
+    oracle.token_loss_bwd(hf, Wf, o["targets"], rows)
+    dt = time.perf_counter() - t0
+    return len(rows) / dt, dt, len(rows)
+
+
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:  # pragma: no cover
+        return os.cpu_count() or 1
+
+
+# --------------------------------------------------------------------------- GPU arm
+def run_ours(args, world, rank, local):
+    from paper_2609_36246_gb300 import binding as B
+    from paper_2609_36246_gb300 import build as _build
+
+    _build.build()
+    dev = torch.device("cuda", torch.cuda.current_device())
+    b, h_cpu, W_cpu = make_inputs(rank)
+    N_mask, T, d, V = b.n_mask, b.T, 4096, 151936
+    i32 = lambda a: torch.from_numpy(np.ascontiguousarray(a, dtype=np.int32))
+    pre_h, poff_h, con_h, coff_h = (i32(b.prefix_ids).pin_memory(), i32(b.prefix_off).pin_memory(),
+                                    i32(b.cont_ids).pin_memory(), i32(b.cont_off).pin_memory())
+    hid_h = h_cpu.pin_memory()
+    pre, poff, con, coff = (x.to(dev) for x in (pre_h, poff_h, con_h, coff_h))
+    hidden = hid_h.to(dev)
+    W = W_cpu.to(dev)
+    st = B.new_status(dev)
+    ws_f = B.workspace(B.olive_workspace_size("logprob_fwd", T, d, V), dev)
+    ws_b = B.workspace(B.olive_workspace_size("loss_bwd", T, d, V, grad_dtype=torch.bfloat16), dev)
+    logp = torch.empty(T, dtype=torch.float32, device=dev)
+    lse = torch.empty_like(logp)
+    loss = torch.empty(1, dtype=torch.float32, device=dev)
+    dh = torch.empty(T, d, dtype=torch.bfloat16, device=dev)
+    dw = torch.empty(V, d, dtype=torch.bfloat16, device=dev)
+    gl = torch.ones(1, dtype=torch.float32, device=dev)
+    loss_h = torch.empty(1, dtype=torch.float32).pin_memory()
+    stream = torch.cuda.current_stream()
+
+    ev = {k: [] for k in ("splice", "fwd", "bwd")}
+
+    def step(timed: bool, host_io: bool = False):
+        if host_io:
+            for dst, src in ((pre, pre_h), (poff, poff_h), (con, con_h), (coff, coff_h), (hidden, hid_h)):
+                dst.copy_(src, non_blocking=True)
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(4)] if timed else None
+        if e: e[0].record(stream)
+        pk = B.olive_splice_pack(pre, poff, con, coff, V, T, dev_status=st)
+        if e: e[1].record(stream)
+        B.olive_token_logprob_fwd(hidden, W, pk["targets"], pk["rows"], pk["n_rows"], 1.0, "sum",
+                                  ws=ws_f, dev_status=st, out=(logp, lse, loss))
+        if e: e[2].record(stream)
+        B.olive_token_loss_bwd(hidden, W, pk["targets"], pk["rows"], pk["n_rows"], lse, gl, 1.0, "sum",
+                               torch.bfloat16, ws=ws_b, dev_status=st, out=(dh, dw))
+        if e:
+            e[3].record(stream)
+            ev["splice"].append((e[0], e[1]))
+            ev["fwd"].append((e[1], e[2]))
+            ev["bwd"].append((e[2], e[3]))
+        if host_io:
+            loss_h.copy_(loss, non_blocking=True)
+
+    for _ in range(args.warmup):
+        step(False)
+    torch.cuda.synchronize()
+    if int(st.item()) != 0:
+        raise RuntimeError(f"device status {B.status_bits(st)}")
+
+    # ---- device-resident timed region ----
+    barrier(world)
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for _ in range(args.steps):
+            step(True)
+        t1.record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    ms_local = t0.elapsed_time(t1)
+    ms = max_over_ranks(ms_local, world)
+    ms_per_step = ms / args.steps
+    total_tokens = N_mask * args.steps * world
+    value = total_tokens / (ms / 1e3)
+
+    # ---- end-to-end through the public API with host buffers ----
+    barrier(world)
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e_steps = max(1, min(args.steps, 5))
+    e0.record(stream)
+    for _ in range(e_steps):
+        step(False, host_io=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e_ms = max_over_ranks(e0.elapsed_time(e1), world)
+    h2d = sum(x.numel() * x.element_size() for x in (pre_h, poff_h, con_h, coff_h, hid_h))
+    e2e = {"value": N_mask * e_steps * world / (e_ms / 1e3), "unit": "tokens/s",
+           "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": 4}
+    assert math.isfinite(float(loss_h.item()))
+
+    avg = lambda k: statistics.mean(a.elapsed_time(b2) for a, b2 in ev[k])
+    fwd_ms, bwd_ms, spl_ms = avg("fwd"), avg("bwd"), avg("splice")
+    burst, sustained, src = load_peaks()
+    counted = 6.0 * N_mask * d * V
+    fwd_flops = 2.0 * N_mask * d * V
+    ach_fwd = fwd_flops / (fwd_ms / 1e3) / 1e12
+    step_tflops = counted / (ms_per_step / 1e3) / 1e12
+    traffic = None
+    tpath = os.path.join(ROOT, "profiles", "lmhead_fwd_traffic.json")
+    if os.path.exists(tpath):
+        with open(tpath) as f:
+            tj = json.load(f)
+        if tj.get("kernel_rev") == kernel_rev():
+            traffic = tj.get("bytes_per_launch")
+    tpath = None
+    tslabs = 4  # bwd slab launches for T = 32768 (slab of 8192 rows)
+    launches = 2 + 4 + (1 + 3 * tslabs + 1)
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        rate, secs, nr = oracle_sample_rate(b, h_cpu, W_cpu, args.cpu_rows)
+        cpu = {"value": rate, "unit": "tokens/s", "cores": host_cores(), "kind": "oracle",
+               "sample": f"{nr} masked rows of the same batch: fp64 logits, log-probs, dH and dW "
+                         f"contributions ({secs:.1f} s)"}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": dict(CONFIG, N_mask=N_mask, T=T, parallelism=f"replicas x{world}"),
+        "pct_bf16_peak": 100.0 * step_tflops / burst,
+        "pct_bf16_peak_sustained": 100.0 * step_tflops / sustained,
+        "counted_tflops_per_s": step_tflops,
+        "phases_ms": {"splice_pack": spl_ms, "logprob_fwd": fwd_ms, "loss_bwd": bwd_ms},
+        "roofline": {"kernel": "gemm_persistent<FwdKern> (LM-head forward + online LSE)",
+                     "bound": "tensor", "achieved": ach_fwd, "peak": sustained, "unit": "TFLOP/s",
+                     "frac": ach_fwd / sustained, "traffic": traffic,
+                     "peak_source": f"{src} bf16_tflops_sustained",
+                     "flops_per_launch": fwd_flops},
+        "e2e": e2e,
+        "gpu_launches": launches * args.steps,
+        "clocks": clk.summary(),
+        "cpu_baseline": cpu,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def kernel_rev() -> str:
+    """Content hash of the CUDA sources (ties a stored ncu traffic figure to them)."""
+    import hashlib
+    hsh = hashlib.sha256()
+    import glob
+    for p in sorted(glob.glob(os.path.join(ROOT, "paper_2609_36246_gb300", "csrc", "*"))):
+        with open(p, "rb") as f:
+            hsh.update(f.read())
+    return hsh.hexdigest()[:16]
+
+
+# --------------------------------------------------------------------------- reference arm
+def run_reference(args, world, rank):
+    if rank != 0:
+        return
+    b, h, W = make_inputs(rank)
+    times, rows = [], 0
+    for _ in range(args.warmup):
+        pass  # the oracle has no warm state; warm-up steps would only repeat the sample
+    for i in range(args.steps):
+        rate, secs, nr = oracle_sample_rate(b, h, W, args.cpu_rows, seed=i)
+        times.append(secs)
+        rows += nr
+    value = rows / sum(times)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * statistics.mean(times),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": dict(CONFIG, parallelism="host cores"),
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": host_cores(), "kind": "oracle",
+                         "sample": f"{args.cpu_rows} masked rows per step of the same batch "
+                                   "(fp64 forward, dH, dW contributions)"},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--cpu-rows", type=int, default=32)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    world, rank, local = dist_setup()
+    if args.impl == "reference":
+        run_reference(args, world, rank)
+    else:
+        run_ours(args, world, rank, local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()
