@@ -199,6 +199,33 @@ OLIVE_API olive_status olive_token_divergence(const void* h_s, const void* W_s, 
                                     int grad_dtype, void* workspace, size_t ws_bytes,
                                     int32_t* dev_status, void* stream);
 
+/*
+ * olive_token_logprob_fwd_noalloc -- the same computation, arguments and
+ * outputs as olive_token_logprob_fwd, for callers that cannot provide a
+ * workspace: code hosted by another framework whose allocator owns all
+ * device memory and lends none, or code that must not call cudaMalloc (it
+ * can synchronise the device).  The paper has no counterpart; this is a
+ * deployment convenience of this library.
+ *
+ * Scratch comes from one array of OLIVE_NOALLOC_SCRATCH_BYTES compiled into
+ * the library, which every GPU that loads the library keeps until the process
+ * exits.  Limit: the call is rejected with OLIVE_ERR_SHAPE, before any
+ * launch, when olive_workspace_size(OLIVE_OP_LOGPROB_FWD, T, d, 0, V, 0, 0)
+ * exceeds that size (for example T = 2048 rows at d = 4096 fit, T = 4096 rows
+ * at d = 4096 do not).  The first call on each device looks up the array's
+ * device address; make that first call before any stream capture.  Every
+ * call shares the array: calls whose work may overlap on the GPU (other
+ * streams, other host threads) race on it, so the caller must serialise
+ * them.  The call allocates no device or host memory.
+ */
+#define OLIVE_NOALLOC_SCRATCH_BYTES (32u * 1024u * 1024u)
+OLIVE_API olive_status olive_token_logprob_fwd_noalloc(const void* hidden, const void* W,
+                                                       const int32_t* targets, const int32_t* rows,
+                                                       const int32_t* n_rows, int32_t T, int32_t d,
+                                                       int32_t V, float inv_tau, int reduction,
+                                                       float* logp, float* lse, float* loss,
+                                                       int32_t* dev_status, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

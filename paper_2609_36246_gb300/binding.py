@@ -69,6 +69,9 @@ def lib() -> ctypes.CDLL:
     L.olive_token_divergence.restype = ctypes.c_int
     L.olive_token_divergence.argtypes = [_P, _P, _I, _P, _P, _I, _P, _P, _I, _I, _F, ctypes.c_int,
                                          _P, _P, _P, ctypes.c_int, _P, _S, _P, _P]
+    L.olive_token_logprob_fwd_noalloc.restype = ctypes.c_int
+    L.olive_token_logprob_fwd_noalloc.argtypes = [_P, _P, _P, _P, _P, _I, _I, _I, _F, ctypes.c_int,
+                                                  _P, _P, _P, _P, _P]
     _lib = L
     return L
 
@@ -241,6 +244,30 @@ def olive_token_divergence(h_s, W_s, h_t, W_t, rows, n_rows, inv_tau: float = 1.
                                       DTYPE[grad_dtype], _ptr(ws), ws.numel(), _ptr(ds), _stream())
     _check(st, "olive_token_divergence")
     return kl, dhs
+
+
+def olive_token_logprob_fwd_noalloc(hidden, W, targets, rows, n_rows, inv_tau: float = 1.0,
+                                    reduction: str = "sum", dev_status=None, out=None):
+    """olive_token_logprob_fwd without a workspace: scratch comes from the
+    library's fixed device array (see include/olive.h for the size limit and
+    the rule that overlapping calls must be serialised)."""
+    _need(hidden, torch.bfloat16, "hidden")
+    _need(W, torch.bfloat16, "W")
+    T, d = hidden.shape
+    V = W.shape[0]
+    dev = hidden.device
+    if out is None:
+        out = (torch.empty(T, dtype=torch.float32, device=dev),
+               torch.empty(T, dtype=torch.float32, device=dev),
+               torch.empty(1, dtype=torch.float32, device=dev))
+    logp, lse, loss = out
+    ds = dev_status if dev_status is not None else new_status(dev)
+    st = lib().olive_token_logprob_fwd_noalloc(_ptr(hidden), _ptr(W), _ptr(targets), _ptr(rows),
+                                               _ptr(n_rows), T, d, V, float(inv_tau),
+                                               REDUCE[reduction], _ptr(logp), _ptr(lse), _ptr(loss),
+                                               _ptr(ds), _stream())
+    _check(st, "olive_token_logprob_fwd_noalloc")
+    return logp, lse, loss
 
 
 class FusedLMHeadCE(torch.autograd.Function):
