@@ -260,19 +260,17 @@ def run_ours(args, world, rank, local):
     fwd_ms, bwd_ms, spl_ms = avg("fwd"), avg("bwd"), avg("splice")
     burst, sustained, src = load_peaks()
     counted = 6.0 * N_mask * d * V
+    step_tflops = counted / (ms_per_step / 1e3) / 1e12
+    # dominant kernel: the fused backward (one launch per olive_token_loss_bwd
+    # call, bracketed together with its row gather); algorithmic work per
+    # launch = dH + dW = 4 N_mask d V (the logit recomputation is not counted)
+    bwd_flops = 4.0 * N_mask * d * V
+    ach_bwd = bwd_flops / (bwd_ms / 1e3) / 1e12
     fwd_flops = 2.0 * N_mask * d * V
     ach_fwd = fwd_flops / (fwd_ms / 1e3) / 1e12
-    step_tflops = counted / (ms_per_step / 1e3) / 1e12
-    traffic = None
-    tpath = os.path.join(ROOT, "profiles", "lmhead_fwd_traffic.json")
-    if os.path.exists(tpath):
-        with open(tpath) as f:
-            tj = json.load(f)
-        if tj.get("kernel_rev") == kernel_rev():
-            traffic = tj.get("bytes_per_launch")
-    tpath = None
-    tslabs = 4  # bwd slab launches for T = 32768 (slab of 8192 rows)
-    launches = 2 + 4 + (1 + 3 * tslabs + 1)
+    rev = kernel_rev()
+    traffic = profile_traffic("bwd_fused_kernel", rev)
+    launches = 2 + 4 + 2  # splice (scan, fill), forward (gather, GEMM, finalize, loss), backward (gather, fused)
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
@@ -290,11 +288,16 @@ def run_ours(args, world, rank, local):
         "pct_bf16_peak_sustained": 100.0 * step_tflops / sustained,
         "counted_tflops_per_s": step_tflops,
         "phases_ms": {"splice_pack": spl_ms, "logprob_fwd": fwd_ms, "loss_bwd": bwd_ms},
-        "roofline": {"kernel": "gemm_persistent<FwdKern> (LM-head forward + online LSE)",
-                     "bound": "tensor", "achieved": ach_fwd, "peak": sustained, "unit": "TFLOP/s",
-                     "frac": ach_fwd / sustained, "traffic": traffic,
+        "roofline": {"kernel": "bwd_fused_kernel (recompute + G, dH, dW tiles)", "bound": "tensor",
+                     "achieved": ach_bwd, "peak": sustained, "unit": "TFLOP/s",
+                     "frac": ach_bwd / sustained, "traffic": traffic,
                      "peak_source": f"{src} bf16_tflops_sustained",
-                     "flops_per_launch": fwd_flops},
+                     "flops_per_launch": bwd_flops, "kernel_rev": rev,
+                     "note": "algorithmic FLOPs exclude the logit recomputation (1/3 of executed)"},
+        "roofline_fwd": {"kernel": "gemm_persistent<FwdKern> (LM-head forward + online LSE)",
+                         "bound": "tensor", "achieved": ach_fwd, "peak": sustained,
+                         "unit": "TFLOP/s", "frac": ach_fwd / sustained,
+                         "traffic": profile_traffic("FwdKern", rev), "flops_per_launch": fwd_flops},
         "e2e": e2e,
         "gpu_launches": launches * args.steps,
         "clocks": clk.summary(),
@@ -304,12 +307,27 @@ def run_ours(args, world, rank, local):
         print(json.dumps(line), flush=True)
 
 
+def profile_traffic(kernel: str, rev: str):
+    """DRAM bytes per launch of `kernel` recorded from an ncu capture of the
+    current sources (a `traffic: <kernel> <rev> <bytes>` line in a profiles/
+    summary), else None."""
+    import glob
+    for path in sorted(glob.glob(os.path.join(ROOT, "profiles", "*"))):
+        with open(path) as f:
+            for line in f:
+                parts = line.strip().split()
+                if len(parts) == 4 and parts[0] == "traffic:" and parts[1] == kernel and parts[2] == rev:
+                    return float(parts[3])
+    return None
+
+
 def kernel_rev() -> str:
     """Content hash of the CUDA sources (ties a stored ncu traffic figure to them)."""
     import hashlib
     hsh = hashlib.sha256()
     import glob
-    for p in sorted(glob.glob(os.path.join(ROOT, "paper_2609_36246_gb300", "csrc", "*"))):
+    for p in sorted(glob.glob(os.path.join(ROOT, "paper_2609_36246_gb300", "csrc", "*.cu*"))) + \
+            sorted(glob.glob(os.path.join(ROOT, "paper_2609_36246_gb300", "csrc", "*.h"))):
         with open(p, "rb") as f:
             hsh.update(f.read())
     return hsh.hexdigest()[:16]

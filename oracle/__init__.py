@@ -13,4 +13,5 @@ from .olive_oracle import (  # noqa: F401
     token_logprob,
     token_loss_bwd,
     token_loss_bwd_rows,
+    token_loss_bwd_vocab,
 )

@@ -25,7 +25,7 @@ Section 1; temperature, Appendix A, Table opd-config):
                           forward direction as an option, and the gradient of
                           sum_t g_t KL_t with respect to the student hidden.
 
-Readings where the paper is silent (each is listed in the design doc):
+Readings where the paper is silent:
   - causal shift: row t of ``hidden`` predicts packed token t+1 of the same
     sequence, so y~_1 is scored from the last prefix row and the last row of
     every sequence has no target;
@@ -268,6 +268,34 @@ def token_loss_bwd_rows(hidden, W, targets, rows, inv_tau: float = 1.0,
         for v0 in range(0, W.shape[0], _VOCAB_CHUNK):
             v1 = min(W.shape[0], v0 + _VOCAB_CHUNK)
             out[r0:r0 + len(rr)] += G[:, v0:v1] @ W[v0:v1].astype(np.float64)
+    return out
+
+
+def token_loss_bwd_vocab(hidden, W, targets, rows, vocab, inv_tau: float = 1.0,
+                         reduction: str = "sum", grad_loss: float = 1.0):
+    """dW for a subset ``vocab`` of vocabulary rows only (sampled checks).
+
+    Same definition as ``token_loss_bwd``: every masked row's full softmax is
+    formed (its lse needs all V logits), then
+    dW[v] = sum_t g inv_tau (p[t, v] - [v == y_t]) h[t] for v in ``vocab``.
+    Returns dW_vocab [len(vocab), d].
+    """
+    _check_reduction(reduction)
+    rows = np.asarray(rows, dtype=np.int64)
+    vocab = np.asarray(vocab, dtype=np.int64)
+    targets = np.asarray(targets, dtype=np.int64)
+    g = float(grad_loss)
+    if reduction == "mean" and len(rows):
+        g = g / len(rows)
+    out = np.zeros((len(vocab), np.asarray(W).shape[1]), dtype=np.float64)
+    for r0 in range(0, len(rows), _ROW_CHUNK):
+        rr = rows[r0:r0 + _ROW_CHUNK]
+        h = _as_f64_rows(hidden, rr)
+        lp, _ = log_softmax_rows(logits(h, W, inv_tau))
+        G = np.exp(lp[:, vocab])
+        G -= (targets[rr][:, None] == vocab[None, :])
+        G *= g * float(inv_tau)
+        out += G.T @ h
     return out
 
 

@@ -215,7 +215,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       // ignores the abort flag: it only waits for work already in flight)
       umma_commit(drain_bar);
       volatile int keep_waiting = 0;
-      const WaitCtl own{&keep_waiting, p.wait_limit_ns};
+      const uint64_t floor_ns = 200ull * 1000 * 1000;  // in-flight MMAs finish in microseconds
+      const WaitCtl own{&keep_waiting, p.wait_limit_ns > floor_ns ? p.wait_limit_ns : floor_ns};
       mbar_wait(drain_bar, 0, own);
     }
     __syncwarp();
@@ -232,9 +233,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       epi.begin(p, sched, u, row);
       for (int t = 0; t < nt; ++t) {
         const TileC tc = Kern::tile(p, sched, u, t);
-        if (!mbar_wait(tfull_bar(buf), aphase, ctl)) { ok = false; break; }
+        // warp-uniform decision: tcgen05.ld below is a warp-collective
+        if (!__all_sync(0xffffffffu, mbar_wait(tfull_bar(buf), aphase, ctl))) { ok = false; break; }
         tc_fence_after();
-        __syncwarp();
         epi.tile(p, sched, u, t, tc, lane_addr + static_cast<uint32_t>(buf * L::ACC_COLS));
         tc_fence_before();
         mbar_arrive(tempty_bar(buf));

@@ -53,6 +53,7 @@ struct BwdWs {
   void* hc;       // bf16 [Tpad, d]
   void* g;        // bf16 [Tc, Vpad]
   float* dw_acc;  // fp32 [V, d] (bf16 output only)
+  uint32_t* counters;  // tile-scheduler counters of the fused backward
   int64_t tc;     // slab rows
 };
 size_t bwd_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype);
@@ -64,6 +65,7 @@ struct KlWs {
   float* part;    // [5, kSvMax, Tpad]
   float* stats;   // [3, Tpad]: lse_s, lse_t, kl per compacted row
   void* g;        // bf16 [Tc, Vpad] (gradient only)
+  uint32_t* counters;  // tile-scheduler counters (gradient only)
   int64_t tc;
 };
 size_t kl_ws_bytes(int64_t T, int64_t ds, int64_t dt, int64_t V, int grad);
@@ -100,12 +102,16 @@ olive_status launch_divergence(const Ctx& c, const void* h_s, const void* W_s, i
                                int direction, float* kl, const float* grad_kl, void* d_h_s,
                                int grad_dtype, void* ws, int32_t* dev_status);
 
-// dH = G . W for one slab of G (shared by the CE and KL backward passes):
-// rows [slab_start, slab_start + Tc) of the compacted row list, scattered to
-// out[rows[r], :] in out_dtype.
-olive_status launch_dh_slab(const Ctx& c, const void* g, int64_t ldg, int64_t tc, const void* W,
-                            int32_t d, int32_t V, const int32_t* rows, const int32_t* n_rows,
-                            int32_t T, int64_t slab_start, void* out, int out_dtype,
-                            int32_t* dev_status);
+// Words of tile-scheduler counters the fused backward needs.
+size_t bwd_counter_words(int64_t Tpad, int64_t tc);
+
+// Divergence backward (fused kernel): d_h_s from the compacted student and
+// teacher rows, the per-row statistics of the forward and a G buffer of tc rows.
+olive_status launch_kl_bwd(const Ctx& c, const void* hcs, const void* hct, const void* W_s,
+                           int32_t d_s, const void* W_t, int32_t d_t, const int32_t* rows,
+                           const int32_t* n_rows, int32_t T, int32_t V, float inv_tau, int reverse,
+                           const float* grad_kl, const float* stats, int32_t ld_stats, void* g,
+                           int64_t tc, uint32_t* counters, void* d_h_s, int grad_dtype,
+                           int32_t* dev_status);
 
 }  // namespace olive

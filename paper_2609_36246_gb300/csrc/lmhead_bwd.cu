@@ -1,20 +1,37 @@
-// lmhead_bwd.cu -- gradients of the Eq. (osd-ce) loss through the LM head
-// (Section 3.1: the sampled sequences are fixed, so only hidden and W get
-// gradients).  With p = softmax(z) from the forward's lse,
-//   G[r, v] = g * inv_tau * (p[r, v] - [v == y_r]),
+// lmhead_bwd.cu -- backward passes of the LM-head losses in one persistent,
+// cooperatively launched kernel with a dynamic tile scheduler.
+//
+// Cross-entropy (Eq. (osd-ce), Section 3.1; the sampled sequences are fixed,
+// so only hidden and W get gradients).  With p = softmax(z) from the
+// forward's lse and G[r, v] = g inv_tau (p[r, v] - [v == y_r]):
 //   dH = G . W        (M = rows, N = d, K = V)
 //   dW = G^T . hc     (M = V,    N = d, K = rows)
+// Divergence (OPD's per-token KL, Section 1): G = g_t inv_tau p_s
+// (log p_s - log p_t - KL_t) (reverse) or g_t inv_tau (p_s - p_t) (forward),
+// and dH_s = G . W_s.
 //
-// The logits are recomputed tile by tile; the G tiles they produce go to a
-// bf16 slab of at most Tc rows in the workspace, which the two gradient GEMMs
-// then stream.  Per slab of Tc compacted rows:
-//   grad   tcgen05 GEMM hc . W^T (128 x 256 tiles) whose epilogue turns each
-//          logit into G (softmax - onehot, scaled) and stores it as bf16
-//   dh     tcgen05 GEMM G . W with W read MN-major; epilogue scatters rows
-//          to d_hidden[rows[r]]
-//   dw     tcgen05 GEMM G^T . hc with both operands MN-major; epilogue
-//          accumulates into an fp32 [V, d] buffer (first slab stores)
-// then one pass rounds the fp32 dW to bf16 when bf16 output was asked for.
+// The logits are recomputed tile by tile and turned into G in the epilogue;
+// G exists only as a bf16 slab of at most tc_max compacted rows in the
+// workspace.  The masked rows are split into equal slabs of <= tc_max rows;
+// per slab the work is a list of tiles of three kinds, all 128 x 256 fp32
+// accumulators in TMEM:
+//   GRAD    z = hc . W^T (K = d; KL: two products, student and teacher, into
+//           two 128-column halves) -> G tile (bf16) in the slab
+//   DH      G . W  (A = G K-major, B = W MN-major, K = V) -> d_hidden rows
+//   DW      G^T . hc (A = G MN-major, B = hc MN-major, K = slab rows) -> dW
+//           (CE only; stored directly in the output dtype when there is one
+//           slab, otherwise through an fp32 accumulator)
+// The tiles of all slabs form one list in dependency order and CTA c takes
+// tiles c, c+G, c+2G, ... (a static round robin: tiles that share an operand
+// run at the same time on neighbouring CTAs, which an atomic work queue was
+// measured to lose).  Before loading a tile the producer warp waits (bounded)
+// until the tiles it reads have been published through release counters: DH
+// of row tile i needs every GRAD tile of row tile i, DW needs every GRAD tile
+// of its slab, and GRAD of slab s+1 needs every DH/DW tile of slab s (they
+// share the G buffer).  Each CTA walks its tiles in increasing order and a
+// tile only waits on tiles with smaller indices, so the lowest unfinished
+// tile never waits and all waits end; the cooperative launch keeps every CTA
+// resident.
 #include <cmath>
 
 #include "gemm_core.cuh"
@@ -24,6 +41,154 @@ namespace olive {
 namespace {
 
 constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr int kBN = 256;
+constexpr int kStages = 4;
+
+enum Kind : int { K_NONE = -1, K_GRAD = 0, K_KLGRAD = 1, K_DH = 2, K_DW = 3 };
+
+// CE maps: 0 hc K-major 64x128, 1 W K-major 64x256, 2 G K-major 64x128,
+//          3 W MN-major 64x64, 4 G MN-major 64x64, 5 hc MN-major 64x64
+// KL maps: 0 hs K-major 64x128, 1 W_s K-major 64x128, 2 G K-major 64x128,
+//          3 W_s MN-major 64x64, 4 ht K-major 64x128, 5 W_t K-major 64x128
+struct BwdMaps {
+  CUtensorMap m[6];
+};
+
+struct BwdParams {
+  int32_t* dev_status;
+  uint64_t wait_limit_ns;
+  const int32_t* n_rows;
+  const int32_t* rows;
+  const int32_t* targets;    // CE
+  const float* lse;          // CE, indexed by packed row
+  const float* grad_loss;    // CE, device scalar
+  const float* grad_kl;      // KL, [T]
+  const float* stats;        // KL, [3][ld_stats]: lse_s, lse_t, kl per compacted row
+  int32_t ld_stats;
+  int32_t kl;                // 0: cross-entropy, 1: divergence
+  int32_t reverse;           // KL direction
+  int32_t T, d, d2, V, reduction, out_dtype, group_rows;
+  int32_t tc_max;            // rows of the G buffer (multiple of 128)
+  int32_t max_slabs, max_rt; // counter array dimensions
+  int64_t ldg;               // G row stride in elements
+  float inv_tau, scale2;
+  __nv_bfloat16* g;
+  void* dh_out;              // [T, d] out_dtype
+  void* dw_out;              // [V, d] out_dtype (CE)
+  float* dw_acc;             // [V, d] fp32 accumulator used when there are several slabs
+  uint32_t* counters;        // [2 max_slabs + max_slabs * max_rt], zeroed before launch
+};
+
+struct Plan {
+  int n, n_slabs, rps, vt, ntd, mtv, bn_grad;
+  float coef;  // CE: g * inv_tau (/ N_mask for the mean)
+};
+
+struct Unit {
+  int kind, s, i, j, in_s, row0, mt;
+};
+
+__device__ __forceinline__ uint32_t* ctr_grad(const BwdParams& p, int s) { return p.counters + s; }
+__device__ __forceinline__ uint32_t* ctr_dhdw(const BwdParams& p, int s) {
+  return p.counters + p.max_slabs + s;
+}
+__device__ __forceinline__ uint32_t* ctr_row(const BwdParams& p, int s, int i) {
+  return p.counters + 2 * p.max_slabs + static_cast<size_t>(s) * p.max_rt + i;
+}
+
+__device__ Plan make_plan(const BwdParams& p) {
+  Plan pl;
+  pl.n = read_n_rows(p.n_rows, p.T, p.dev_status);
+  pl.n_slabs = pl.n > 0 ? (pl.n + p.tc_max - 1) / p.tc_max : 1;
+  if (pl.n_slabs > p.max_slabs) pl.n_slabs = p.max_slabs;  // cannot happen for n <= T
+  const int per = (pl.n + pl.n_slabs - 1) / pl.n_slabs;
+  pl.rps = (per + 127) / 128 * 128;
+  pl.bn_grad = p.kl ? 128 : 256;
+  pl.vt = (p.V + pl.bn_grad - 1) / pl.bn_grad;
+  pl.ntd = (p.d + kBN - 1) / kBN;
+  pl.mtv = (p.V + kBM - 1) / kBM;
+  pl.coef = 0.f;
+  if (!p.kl) {
+    float g = *p.grad_loss;
+    if (p.reduction == OLIVE_REDUCE_MEAN && pl.n > 0) g = g / static_cast<float>(pl.n);
+    pl.coef = g * p.inv_tau;
+  }
+  return pl;
+}
+
+__device__ __forceinline__ int slab_in(const Plan& pl, int s) {
+  const int r = pl.n - s * pl.rps;
+  return r < 0 ? 0 : (r > pl.rps ? pl.rps : r);
+}
+__device__ __forceinline__ int units_grad(const Plan& pl, int mt) { return mt * pl.vt; }
+__device__ __forceinline__ int units_dh(const Plan& pl, int mt) { return mt * pl.ntd; }
+__device__ __forceinline__ int units_dw(const BwdParams& p, const Plan& pl, int s, int in_s) {
+  return (!p.kl && (s == 0 || in_s > 0)) ? pl.mtv * pl.ntd : 0;
+}
+
+__device__ int total_units(const BwdParams& p, const Plan& pl) {
+  int t = 0;
+  for (int s = 0; s < pl.n_slabs; ++s) {
+    const int in_s = slab_in(pl, s);
+    const int mt = (in_s + 127) / 128;
+    t += units_grad(pl, mt) + units_dh(pl, mt) + units_dw(p, pl, s, in_s);
+  }
+  return t;
+}
+
+__device__ Unit decode(const BwdParams& p, const Plan& pl, int u) {
+  Unit x;
+  x.kind = K_NONE;
+  for (int s = 0; s < pl.n_slabs; ++s) {
+    const int in_s = slab_in(pl, s);
+    const int mt = (in_s + 127) / 128;
+    x.s = s;
+    x.in_s = in_s;
+    x.row0 = s * pl.rps;
+    x.mt = mt;
+    const int ug = units_grad(pl, mt);
+    if (u < ug) {
+      const Raster r{mt, pl.vt, p.group_rows};
+      r.tile(u, x.i, x.j);
+      x.kind = p.kl ? K_KLGRAD : K_GRAD;
+      return x;
+    }
+    u -= ug;
+    const int uh = units_dh(pl, mt);
+    if (u < uh) {
+      x.i = u / pl.ntd;
+      x.j = u % pl.ntd;
+      x.kind = K_DH;
+      return x;
+    }
+    u -= uh;
+    const int uw = units_dw(p, pl, s, in_s);
+    if (u < uw) {
+      x.i = u / pl.ntd;
+      x.j = u % pl.ntd;
+      x.kind = K_DW;
+      return x;
+    }
+    u -= uw;
+  }
+  return x;
+}
+
+// K steps of each product of a unit
+__device__ __forceinline__ void unit_ksteps(const BwdParams& p, const Unit& x, int& nk, int& nk2) {
+  nk2 = 0;
+  switch (x.kind) {
+    case K_GRAD: nk = (p.d + kBK - 1) / kBK; break;
+    case K_KLGRAD:
+      nk = (p.d + kBK - 1) / kBK;
+      nk2 = (p.d2 + kBK - 1) / kBK;
+      break;
+    case K_DH: nk = (p.V + kBK - 1) / kBK; break;
+    case K_DW: nk = (x.in_s + kBK - 1) / kBK; break;
+    default: nk = 0;
+  }
+}
 
 __device__ __forceinline__ void store_bf16x32(__nv_bfloat16* dst, const float (&g)[32]) {
   uint4* d4 = reinterpret_cast<uint4*>(dst);
@@ -44,336 +209,460 @@ __device__ __forceinline__ void store_f32x32(float* dst, const float (&g)[32]) {
   for (int q = 0; q < 8; ++q) d4[q] = make_float4(g[4 * q], g[4 * q + 1], g[4 * q + 2], g[4 * q + 3]);
 }
 
-// ------------------------------------------------------------------ grad ---
-struct GradKern {
-  static constexpr int kBN = 256;
-  static constexpr bool kAMn = false;
-  static constexpr bool kBMn = false;
-  static constexpr bool kDual = false;
-  static constexpr int kStages = 4;
-
-  struct Params {
-    int32_t* dev_status;
-    uint64_t wait_limit_ns;
-    const int32_t* n_rows;
-    const int32_t* rows;
-    const int32_t* targets;
-    const float* lse;
-    const float* grad_loss;
-    int32_t T, d, V, reduction;
-    int32_t group_rows;
-    int64_t slab_start, tc, ldg;
-    float inv_tau, scale2;
-    __nv_bfloat16* g;
-  };
-  struct Sched {
-    int n, in_slab, mt, vt, units;
-    float coef;
-  };
-  static __device__ Sched make_sched(const Params& p) {
-    Sched s;
-    s.n = read_n_rows(p.n_rows, p.T, p.dev_status);
-    long long k = s.n - p.slab_start;
-    if (k < 0) k = 0;
-    if (k > p.tc) k = p.tc;
-    s.in_slab = static_cast<int>(k);
-    s.mt = (s.in_slab + kBM - 1) / kBM;
-    s.vt = (p.V + kBN - 1) / kBN;
-    s.units = s.mt * s.vt;
-    float g = *p.grad_loss;
-    if (p.reduction == OLIVE_REDUCE_MEAN && s.n > 0) g = g / static_cast<float>(s.n);
-    s.coef = g * p.inv_tau;
-    return s;
-  }
-  static __device__ int num_units(const Params&, const Sched& s) { return s.units; }
-  static __device__ int unit_len(const Params&, const Sched&, int) { return 1; }
-  static __device__ void pos(const Params& p, const Sched& s, int u, int& i, int& j) {
-    const Raster r{s.mt, s.vt, p.group_rows};
-    r.tile(u, i, j);
-  }
-  static __device__ TileC tile(const Params& p, const Sched& s, int u, int) {
-    int i, j;
-    pos(p, s, u, i, j);
-    TileC c;
-    c.m0 = static_cast<int>(p.slab_start) + i * kBM;
-    c.n0 = j * kBN;
-    c.ka0 = 0;
-    c.kb0 = 0;
-    c.nk = (p.d + kBK - 1) / kBK;
-    c.nk2 = 0;
-    return c;
-  }
-  struct Epi {
-    int r_local, y;
-    bool valid;
-    float lse2;
-    __device__ void begin(const Params& p, const Sched& s, int u, int row) {
-      int i, j;
-      pos(p, s, u, i, j);
-      r_local = i * kBM + row;
-      const long long r = p.slab_start + r_local;
-      valid = r < s.n;
-      y = -1;
-      lse2 = 0.f;
-      if (valid) {
-        const int t = p.rows[r];
-        if (t >= 0 && t < p.T) {
-          y = p.targets[t];
-          lse2 = p.lse[t] * kLog2e;
-        } else {
-          valid = false;
-        }
-      }
+// 32 values -> row segment of `n_valid` (<= 32) elements, bf16 or fp32
+__device__ __forceinline__ void store_row32(void* base, size_t off, int dtype, int n_valid,
+                                            const float (&g)[32]) {
+  if (dtype == OLIVE_DTYPE_BF16) {
+    __nv_bfloat16* o = static_cast<__nv_bfloat16*>(base) + off;
+    if (n_valid >= 32) {
+      store_bf16x32(o, g);
+    } else {
+#pragma unroll
+      for (int k = 0; k < 32; ++k)
+        if (k < n_valid) o[k] = __float2bfloat16_rn(g[k]);
     }
-    __device__ void tile(const Params& p, const Sched& s, int, int, const TileC& tc, uint32_t taddr) {
-      __nv_bfloat16* grow = p.g + static_cast<size_t>(r_local) * p.ldg;
-#pragma unroll 1
-      for (int c = 0; c < kBN; c += 32) {
-        const int col0 = tc.n0 + c;
-        if (col0 >= p.V) break;
-        uint32_t a[32];
-        tmem_ld_32x32b_x32(taddr + c, a);
-        tmem_ld_wait();
-        float g[32];
+  } else {
+    float* o = static_cast<float*>(base) + off;
+    if (n_valid >= 32) {
+      store_f32x32(o, g);
+    } else {
 #pragma unroll
-        for (int k = 0; k < 32; ++k) {
-          const float pr = fast_exp2(__uint_as_float(a[k]) * p.scale2 - lse2);
-          g[k] = valid ? s.coef * (pr - (col0 + k == y ? 1.f : 0.f)) : 0.f;
-        }
-        if (col0 + 32 <= p.V) {
-          store_bf16x32(grow + col0, g);
-        } else {
-          const int nv = p.V - col0;
-#pragma unroll
-          for (int k = 0; k < 32; ++k)
-            if (k < nv) grow[col0 + k] = __float2bfloat16_rn(g[k]);
-        }
-      }
+      for (int k = 0; k < 32; ++k)
+        if (k < n_valid) o[k] = g[k];
     }
-    __device__ void end(const Params&, const Sched&, int) {}
-  };
-};
-
-// -------------------------------------------------------------------- dh ---
-struct DhKern {
-  static constexpr int kBN = 256;
-  static constexpr bool kAMn = false;  // G slab [rows, V]: K = V contiguous
-  static constexpr bool kBMn = true;   // W [V, d]: N = d contiguous
-  static constexpr bool kDual = false;
-  static constexpr int kStages = 4;
-
-  struct Params {
-    int32_t* dev_status;
-    uint64_t wait_limit_ns;
-    const int32_t* n_rows;
-    const int32_t* rows;
-    int32_t T, d, V, out_dtype;
-    int64_t slab_start, tc;
-    void* out;
-  };
-  struct Sched {
-    int n, in_slab, mt, nt, units;
-  };
-  static __device__ Sched make_sched(const Params& p) {
-    Sched s;
-    s.n = read_n_rows(p.n_rows, p.T, p.dev_status);
-    long long k = s.n - p.slab_start;
-    if (k < 0) k = 0;
-    if (k > p.tc) k = p.tc;
-    s.in_slab = static_cast<int>(k);
-    s.mt = (s.in_slab + kBM - 1) / kBM;
-    s.nt = (p.d + kBN - 1) / kBN;
-    s.units = s.mt * s.nt;
-    return s;
-  }
-  static __device__ int num_units(const Params&, const Sched& s) { return s.units; }
-  static __device__ int unit_len(const Params&, const Sched&, int) { return 1; }
-  static __device__ TileC tile(const Params& p, const Sched& s, int u, int) {
-    TileC c;
-    c.m0 = (u / s.nt) * kBM;
-    c.n0 = (u % s.nt) * kBN;
-    c.ka0 = 0;
-    c.kb0 = 0;
-    c.nk = (p.V + kBK - 1) / kBK;
-    c.nk2 = 0;
-    return c;
-  }
-  struct Epi {
-    int t;
-    __device__ void begin(const Params& p, const Sched& s, int u, int row) {
-      const long long r = p.slab_start + (u / s.nt) * kBM + row;
-      t = -1;
-      if (r < s.n) {
-        const int tt = p.rows[r];
-        if (tt >= 0 && tt < p.T) t = tt;
-      }
-    }
-    __device__ void tile(const Params& p, const Sched&, int, int, const TileC& tc, uint32_t taddr) {
-#pragma unroll 1
-      for (int c = 0; c < kBN; c += 32) {
-        const int col0 = tc.n0 + c;
-        if (col0 >= p.d) break;
-        uint32_t a[32];
-        tmem_ld_32x32b_x32(taddr + c, a);
-        tmem_ld_wait();
-        if (t < 0) continue;
-        float g[32];
-#pragma unroll
-        for (int k = 0; k < 32; ++k) g[k] = __uint_as_float(a[k]);
-        const size_t off = static_cast<size_t>(t) * p.d + col0;
-        if (p.out_dtype == OLIVE_DTYPE_BF16) {
-          __nv_bfloat16* o = static_cast<__nv_bfloat16*>(p.out) + off;
-          if (col0 + 32 <= p.d) store_bf16x32(o, g);
-          else {
-#pragma unroll
-            for (int k = 0; k < 32; ++k)
-              if (k < p.d - col0) o[k] = __float2bfloat16_rn(g[k]);
-          }
-        } else {
-          float* o = static_cast<float*>(p.out) + off;
-          if (col0 + 32 <= p.d) store_f32x32(o, g);
-          else {
-#pragma unroll
-            for (int k = 0; k < 32; ++k)
-              if (k < p.d - col0) o[k] = g[k];
-          }
-        }
-      }
-    }
-    __device__ void end(const Params&, const Sched&, int) {}
-  };
-};
-
-// -------------------------------------------------------------------- dw ---
-struct DwKern {
-  static constexpr int kBN = 256;
-  static constexpr bool kAMn = true;   // A = G^T: G slab [rows, V], M = V contiguous
-  static constexpr bool kBMn = true;   // B = hc [rows, d]: N = d contiguous
-  static constexpr bool kDual = false;
-  static constexpr int kStages = 4;
-
-  struct Params {
-    int32_t* dev_status;
-    uint64_t wait_limit_ns;
-    const int32_t* n_rows;
-    int32_t T, d, V, first;
-    int64_t slab_start, tc;
-    float* out;  // fp32 [V, d]
-  };
-  struct Sched {
-    int n, in_slab, nk, mt, nt, units;
-  };
-  static __device__ Sched make_sched(const Params& p) {
-    Sched s;
-    s.n = read_n_rows(p.n_rows, p.T, p.dev_status);
-    long long k = s.n - p.slab_start;
-    if (k < 0) k = 0;
-    if (k > p.tc) k = p.tc;
-    s.in_slab = static_cast<int>(k);
-    s.nk = (s.in_slab + kBK - 1) / kBK;
-    s.mt = (p.V + kBM - 1) / kBM;
-    s.nt = (p.d + kBN - 1) / kBN;
-    s.units = (p.first || s.in_slab > 0) ? s.mt * s.nt : 0;
-    return s;
-  }
-  static __device__ int num_units(const Params&, const Sched& s) { return s.units; }
-  static __device__ int unit_len(const Params&, const Sched&, int) { return 1; }
-  static __device__ TileC tile(const Params& p, const Sched& s, int u, int) {
-    TileC c;
-    c.m0 = (u / s.nt) * kBM;
-    c.n0 = (u % s.nt) * kBN;
-    c.ka0 = 0;
-    c.kb0 = static_cast<int>(p.slab_start);
-    c.nk = s.nk;
-    c.nk2 = 0;
-    return c;
-  }
-  struct Epi {
-    int v;
-    __device__ void begin(const Params&, const Sched& s, int u, int row) { v = (u / s.nt) * kBM + row; }
-    __device__ void tile(const Params& p, const Sched&, int, int, const TileC& tc, uint32_t taddr) {
-#pragma unroll 1
-      for (int c = 0; c < kBN; c += 32) {
-        const int col0 = tc.n0 + c;
-        if (col0 >= p.d) break;
-        float g[32];
-        if (tc.nk > 0) {
-          uint32_t a[32];
-          tmem_ld_32x32b_x32(taddr + c, a);
-          tmem_ld_wait();
-#pragma unroll
-          for (int k = 0; k < 32; ++k) g[k] = __uint_as_float(a[k]);
-        } else {
-#pragma unroll
-          for (int k = 0; k < 32; ++k) g[k] = 0.f;
-        }
-        if (v >= p.V) continue;
-        float* o = p.out + static_cast<size_t>(v) * p.d + col0;
-        if (col0 + 32 <= p.d) {
-          if (!p.first) {
-            const float4* o4 = reinterpret_cast<const float4*>(o);
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {
-              const float4 x = o4[q];
-              g[4 * q] += x.x;
-              g[4 * q + 1] += x.y;
-              g[4 * q + 2] += x.z;
-              g[4 * q + 3] += x.w;
-            }
-          }
-          store_f32x32(o, g);
-        } else {
-#pragma unroll
-          for (int k = 0; k < 32; ++k)
-            if (k < p.d - col0) o[k] = p.first ? g[k] : o[k] + g[k];
-        }
-      }
-    }
-    __device__ void end(const Params&, const Sched&, int) {}
-  };
-};
-
-__global__ void f32_to_bf16_kernel(const float4* __restrict__ in, uint2* __restrict__ out, size_t n4) {
-  for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n4;
-       i += static_cast<size_t>(gridDim.x) * blockDim.x) {
-    const float4 x = in[i];
-    out[i] = make_uint2(pack_bf16x2(x.x, x.y), pack_bf16x2(x.z, x.w));
   }
 }
 
-template <class K>
-olive_status launch_core(const Ctx& c, const CUtensorMap& a, const CUtensorMap& b,
-                         const typename K::Params& p) {
-  const int smem = core_smem_bytes<K>();
-  if (cudaFuncSetAttribute(gemm_persistent<K>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+// ------------------------------------------------------------- epilogues ---
+__device__ void epi_grad(const BwdParams& p, const Plan& pl, const Unit& x, int row, uint32_t taddr) {
+  const int r_local = x.i * kBM + row;
+  const int r = x.row0 + r_local;
+  bool valid = r_local < x.in_s;
+  int y = -1;
+  float lse2 = 0.f;
+  if (valid) {
+    const int t = p.rows[r];
+    if (t >= 0 && t < p.T) {
+      y = p.targets[t];
+      lse2 = p.lse[t] * kLog2e;
+    } else {
+      valid = false;
+    }
+  }
+  __nv_bfloat16* grow = p.g + static_cast<size_t>(r_local) * p.ldg;
+  const int n0 = x.j * kBN;
+#pragma unroll 1
+  for (int c = 0; c < kBN; c += 32) {
+    const int col0 = n0 + c;
+    if (col0 >= p.V) break;
+    uint32_t a[32];
+    tmem_ld_32x32b_x32(taddr + c, a);
+    tmem_ld_wait();
+    float g[32];
+#pragma unroll
+    for (int k = 0; k < 32; ++k) {
+      const float pr = fast_exp2(__uint_as_float(a[k]) * p.scale2 - lse2);
+      g[k] = valid ? pl.coef * (pr - (col0 + k == y ? 1.f : 0.f)) : 0.f;
+    }
+    store_row32(grow, col0, OLIVE_DTYPE_BF16, p.V - col0, g);
+  }
+}
+
+__device__ void epi_klgrad(const BwdParams& p, const Unit& x, int row, uint32_t taddr) {
+  const int r_local = x.i * kBM + row;
+  const int r = x.row0 + r_local;
+  bool valid = r_local < x.in_s;
+  float ls2 = 0.f, lt2 = 0.f, kl = 0.f, coef = 0.f;
+  if (valid) {
+    const int t = p.rows[r];
+    if (t >= 0 && t < p.T) {
+      ls2 = p.stats[0 * static_cast<size_t>(p.ld_stats) + r] * kLog2e;
+      lt2 = p.stats[1 * static_cast<size_t>(p.ld_stats) + r] * kLog2e;
+      kl = p.stats[2 * static_cast<size_t>(p.ld_stats) + r];
+      coef = p.grad_kl[t] * p.inv_tau;
+    } else {
+      valid = false;
+    }
+  }
+  __nv_bfloat16* grow = p.g + static_cast<size_t>(r_local) * p.ldg;
+  const int n0 = x.j * 128;
+#pragma unroll 1
+  for (int c = 0; c < 128; c += 32) {
+    const int col0 = n0 + c;
+    if (col0 >= p.V) break;
+    uint32_t a[32], b[32];
+    tmem_ld_32x32b_x32(taddr + c, a);
+    tmem_ld_32x32b_x32(taddr + 128 + c, b);
+    tmem_ld_wait();
+    float g[32];
+#pragma unroll
+    for (int k = 0; k < 32; ++k) {
+      const float ys = __uint_as_float(a[k]) * p.scale2 - ls2;  // log2 p_s
+      const float yt = __uint_as_float(b[k]) * p.scale2 - lt2;  // log2 p_t
+      const float ps = fast_exp2(ys);
+      const float v = p.reverse ? ps * ((ys - yt) * kLn2 - kl) : ps - fast_exp2(yt);
+      g[k] = valid ? coef * v : 0.f;
+    }
+    store_row32(grow, col0, OLIVE_DTYPE_BF16, p.V - col0, g);
+  }
+}
+
+__device__ void epi_dh(const BwdParams& p, const Unit& x, int row, uint32_t taddr) {
+  const int r_local = x.i * kBM + row;
+  int t = -1;
+  if (r_local < x.in_s) {
+    const int tt = p.rows[x.row0 + r_local];
+    if (tt >= 0 && tt < p.T) t = tt;
+  }
+  const int n0 = x.j * kBN;
+#pragma unroll 1
+  for (int c = 0; c < kBN; c += 32) {
+    const int col0 = n0 + c;
+    if (col0 >= p.d) break;
+    uint32_t a[32];
+    tmem_ld_32x32b_x32(taddr + c, a);
+    tmem_ld_wait();
+    if (t < 0) continue;
+    float g[32];
+#pragma unroll
+    for (int k = 0; k < 32; ++k) g[k] = __uint_as_float(a[k]);
+    store_row32(p.dh_out, static_cast<size_t>(t) * p.d + col0, p.out_dtype, p.d - col0, g);
+  }
+}
+
+__device__ void epi_dw(const BwdParams& p, const Plan& pl, const Unit& x, int row, uint32_t taddr,
+                       int nk) {
+  const int v = x.i * kBM + row;
+  const bool first = x.s == 0;
+  const bool last = x.s == pl.n_slabs - 1;
+  const int n0 = x.j * kBN;
+#pragma unroll 1
+  for (int c = 0; c < kBN; c += 32) {
+    const int col0 = n0 + c;
+    if (col0 >= p.d) break;
+    float g[32];
+    if (nk > 0) {
+      uint32_t a[32];
+      tmem_ld_32x32b_x32(taddr + c, a);
+      tmem_ld_wait();
+#pragma unroll
+      for (int k = 0; k < 32; ++k) g[k] = __uint_as_float(a[k]);
+    } else {
+#pragma unroll
+      for (int k = 0; k < 32; ++k) g[k] = 0.f;
+    }
+    if (v >= p.V) continue;
+    const size_t off = static_cast<size_t>(v) * p.d + col0;
+    const int nv = p.d - col0;
+    if (!first) {
+      const float* acc = p.dw_acc + off;
+      if (nv >= 32) {
+        const float4* a4 = reinterpret_cast<const float4*>(acc);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const float4 z = a4[q];
+          g[4 * q] += z.x;
+          g[4 * q + 1] += z.y;
+          g[4 * q + 2] += z.z;
+          g[4 * q + 3] += z.w;
+        }
+      } else {
+#pragma unroll
+        for (int k = 0; k < 32; ++k)
+          if (k < nv) g[k] += acc[k];
+      }
+    }
+    if (last) store_row32(p.dw_out, off, p.out_dtype, nv, g);
+    else store_row32(p.dw_acc, off, OLIVE_DTYPE_F32, nv, g);
+  }
+}
+
+// ---------------------------------------------------------------- kernel ---
+struct BwdLayout {
+  static constexpr int A_BYTES = kBM * kBK * 2;      // 16 KB
+  static constexpr int B_BYTES = kBN * kBK * 2;      // 32 KB
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int RING_BYTES = STAGE_BYTES * kStages;
+  // full[S], empty[S], tfull[2], tempty[2], drain
+  static constexpr int NBARS = 2 * kStages + 5;
+  static constexpr int BAR_BYTES = 8 * NBARS;
+  static constexpr int MISC_BYTES = 128;
+  static constexpr int SMEM_BYTES = 1024 + RING_BYTES + BAR_BYTES + MISC_BYTES;
+  static constexpr uint32_t TMEM_COLS = 512;
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+    bwd_fused_kernel(const __grid_constant__ BwdMaps maps, const BwdParams p) {
+  using L = BwdLayout;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+  const uint32_t ring = base;
+  const uint32_t bar0 = base + L::RING_BYTES;
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (kStages + s); };
+  auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * kStages + b); };
+  auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * kStages + 2 + b); };
+  const uint32_t drain_bar = bar0 + 8u * (2 * kStages + 4);
+  uint8_t* misc = gbase + L::RING_BYTES + L::BAR_BYTES;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(misc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 4);
+  Plan* plan_smem = reinterpret_cast<Plan*>(misc + 64);
+  static_assert(sizeof(Plan) <= 64, "Plan too large");
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(tfull_bar(b), 1);
+      mbar_init(tempty_bar(b), kEpiThreads);
+    }
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    *plan_smem = make_plan(p);
+    fence_mbar_init();
+  }
+  if (warp == kProducerWarp && lane == 0) {
+#pragma unroll
+    for (int m = 0; m < 6; ++m) tma_prefetch_desc(&maps.m[m]);
+  }
+  if (warp == kMmaWarp) {
+    tmem_alloc(smem_u32(tmem_slot), L::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+
+  const uint32_t tmem_base = *tmem_slot;
+  const Plan pl = *plan_smem;
+  const WaitCtl ctl{abort_flag, p.wait_limit_ns};
+
+  const int total = total_units(p, pl);
+
+  if (warp == kProducerWarp) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; ok && u < total; u += gridDim.x) {
+        const Unit x = decode(p, pl, u);
+        // wait until the tiles this one reads are published
+        bool dep = true;
+        if ((x.kind == K_GRAD || x.kind == K_KLGRAD) && x.s > 0) {
+          const int pin = slab_in(pl, x.s - 1);
+          const int pmt = (pin + 127) / 128;
+          dep = wait_counter(ctr_dhdw(p, x.s - 1),
+                             units_dh(pl, pmt) + units_dw(p, pl, x.s - 1, pin), ctl);
+        } else if (x.kind == K_DH) {
+          dep = wait_counter(ctr_row(p, x.s, x.i), pl.vt, ctl);
+        } else if (x.kind == K_DW) {
+          dep = wait_counter(ctr_grad(p, x.s), units_grad(pl, x.mt), ctl);
+        }
+        if (!dep) { ok = false; break; }
+        fence_proxy_async_global();
+        int nk, nk2;
+        unit_ksteps(p, x, nk, nk2);
+        const uint32_t bytes = x.kind == K_KLGRAD ? L::A_BYTES + 128 * kBK * 2 : L::STAGE_BYTES;
+        for (int k = 0; k < nk + nk2; ++k) {
+          if (!mbar_wait(empty_bar(stage), phase ^ 1u, ctl)) { ok = false; break; }
+          const uint32_t sA = ring + stage * L::STAGE_BYTES;
+          const uint32_t sB = sA + L::A_BYTES;
+          const uint32_t fb = full_bar(stage);
+          mbar_arrive_expect_tx(fb, bytes);
+          switch (x.kind) {
+            case K_GRAD:
+              tma_load_2d(sA, &maps.m[0], fb, k * kBK, x.row0 + x.i * kBM);
+              tma_load_2d(sB, &maps.m[1], fb, k * kBK, x.j * kBN);
+              break;
+            case K_KLGRAD: {
+              const bool second = k >= nk;
+              const int kk = (second ? k - nk : k) * kBK;
+              tma_load_2d(sA, &maps.m[second ? 4 : 0], fb, kk, x.row0 + x.i * kBM);
+              tma_load_2d(sB, &maps.m[second ? 5 : 1], fb, kk, x.j * 128);
+              break;
+            }
+            case K_DH:
+              tma_load_2d(sA, &maps.m[2], fb, k * kBK, x.i * kBM);
+#pragma unroll
+              for (int b = 0; b < 4; ++b) tma_load_2d(sB + b * 8192, &maps.m[3], fb, x.j * kBN + 64 * b, k * kBK);
+              break;
+            case K_DW:
+#pragma unroll
+              for (int b = 0; b < 2; ++b) tma_load_2d(sA + b * 8192, &maps.m[4], fb, x.i * kBM + 64 * b, k * kBK);
+#pragma unroll
+              for (int b = 0; b < 4; ++b)
+                tma_load_2d(sB + b * 8192, &maps.m[5], fb, x.j * kBN + 64 * b, x.row0 + k * kBK);
+              break;
+            default: break;
+          }
+          if (++stage == kStages) { stage = 0; phase ^= 1u; }
+        }
+      }
+      if (!ok) {
+        const uint64_t t0 = global_timer_ns();
+        while (global_timer_ns() - t0 < 50000) nanosleep_ns(1000);
+      }
+    }
+    __syncwarp();
+  } else if (warp == kMmaWarp) {
+    if (lane == 0) {
+      int stage = 0, buf = 0;
+      uint32_t phase = 0, aphase = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; ok && u < total; u += gridDim.x) {
+        const Unit x = decode(p, pl, u);
+        int nk, nk2;
+        unit_ksteps(p, x, nk, nk2);
+        uint32_t idesc;
+        bool a_mn = false, b_mn = false;
+        switch (x.kind) {
+          case K_KLGRAD: idesc = idesc_bf16(kBM, 128, false, false); break;
+          case K_DH: idesc = idesc_bf16(kBM, kBN, false, true); b_mn = true; break;
+          case K_DW: idesc = idesc_bf16(kBM, kBN, true, true); a_mn = b_mn = true; break;
+          default: idesc = idesc_bf16(kBM, kBN, false, false); break;
+        }
+        if (!mbar_wait(tempty_bar(buf), aphase ^ 1u, ctl)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t acc = tmem_base + static_cast<uint32_t>(buf * kBN);
+        for (int k = 0; k < nk + nk2; ++k) {
+          if (!mbar_wait(full_bar(stage), phase, ctl)) { ok = false; break; }
+          tc_fence_after();
+          const bool second = k >= nk;
+          const uint32_t dt = second ? acc + 128 : acc;
+          const int kl = second ? k - nk : k;
+          const uint32_t sA = ring + stage * L::STAGE_BYTES;
+          const uint32_t sB = sA + L::A_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < kBK / 16; ++kk) {
+            const uint64_t ad = a_mn ? sdesc_sw128(sA + kk * 2048, 8192, 1024)
+                                     : sdesc_sw128(sA + kk * 32, 16, 1024);
+            const uint64_t bd = b_mn ? sdesc_sw128(sB + kk * 2048, 8192, 1024)
+                                     : sdesc_sw128(sB + kk * 32, 16, 1024);
+            umma_bf16(dt, ad, bd, idesc, (kl > 0 || kk > 0) ? 1u : 0u);
+          }
+          umma_commit(empty_bar(stage));
+          if (++stage == kStages) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+        umma_commit(tfull_bar(buf));
+        if (++buf == 2) { buf = 0; aphase ^= 1u; }
+      }
+      umma_commit(drain_bar);
+      volatile int keep_waiting = 0;
+      const uint64_t floor_ns = 200ull * 1000 * 1000;  // in-flight MMAs finish in microseconds
+      const WaitCtl own{&keep_waiting, p.wait_limit_ns > floor_ns ? p.wait_limit_ns : floor_ns};
+      mbar_wait(drain_bar, 0, own);
+    }
+    __syncwarp();
+  } else {
+    const int row = threadIdx.x;
+    const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
+    int buf = 0;
+    uint32_t aphase = 0;
+    // every wait below ends in one group decision (bar.red.and), so the 128
+    // epilogue threads always leave the loop together
+    for (int u = blockIdx.x; u < total; u += gridDim.x) {
+      const Unit x = decode(p, pl, u);
+      int nk, nk2;
+      unit_ksteps(p, x, nk, nk2);
+      if (!named_bar_and(1, kEpiThreads, mbar_wait(tfull_bar(buf), aphase, ctl))) break;
+      tc_fence_after();
+      __syncwarp();
+      const uint32_t taddr = lane_addr + static_cast<uint32_t>(buf * kBN);
+      if (x.kind == K_DW && x.s > 0) {
+        // the fp32 partial of the previous slab must be visible before it is read
+        const bool seen = row == 0 ? wait_counter(ctr_grad(p, x.s), units_grad(pl, x.mt), ctl) : true;
+        if (!named_bar_and(1, kEpiThreads, seen)) break;
+      }
+      switch (x.kind) {
+        case K_GRAD: epi_grad(p, pl, x, row, taddr); break;
+        case K_KLGRAD: epi_klgrad(p, x, row, taddr); break;
+        case K_DH: epi_dh(p, x, row, taddr); break;
+        case K_DW: epi_dw(p, pl, x, row, taddr, nk); break;
+        default: break;
+      }
+      tc_fence_before();
+      mbar_arrive(tempty_bar(buf));
+      if (++buf == 2) { buf = 0; aphase ^= 1u; }
+      // publish: every epilogue thread's stores, then one release increment
+      fence_proxy_async_global();
+      __threadfence();
+      named_bar_sync(1, kEpiThreads);
+      if (row == 0) {
+        if (x.kind == K_GRAD || x.kind == K_KLGRAD) {
+          red_release_add(ctr_row(p, x.s, x.i), 1u);
+          red_release_add(ctr_grad(p, x.s), 1u);
+        } else {
+          red_release_add(ctr_dhdw(p, x.s), 1u);
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x == 0 && *abort_flag) atomicOr(p.dev_status, kStatusTimeoutBit);
+  if (warp == kMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, L::TMEM_COLS);
+  }
+}
+
+olive_status launch_bwd_fused(const Ctx& c, const BwdMaps& maps, const BwdParams& p) {
+  const int smem = BwdLayout::SMEM_BYTES;
+  if (cudaFuncSetAttribute(bwd_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
       cudaSuccess)
     return OLIVE_ERR_CUDA;
-  gemm_persistent<K><<<c.num_sms, kThreads, smem, c.stream>>>(a, b, a, b, p);
-  return cudaGetLastError() == cudaSuccess ? OLIVE_OK : OLIVE_ERR_CUDA;
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, bwd_fused_kernel, kThreads, smem) !=
+          cudaSuccess ||
+      per_sm < 1)
+    return OLIVE_ERR_CUDA;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(c.num_sms);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = c.stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (cudaLaunchKernelEx(&cfg, bwd_fused_kernel, maps, p) != cudaSuccess) {
+    cudaGetLastError();
+    return OLIVE_ERR_CUDA;
+  }
+  return OLIVE_OK;
 }
 
-}  // namespace
-
-olive_status launch_dh_slab(const Ctx& c, const void* g, int64_t ldg, int64_t tc, const void* W,
-                            int32_t d, int32_t V, const int32_t* rows, const int32_t* n_rows,
-                            int32_t T, int64_t slab_start, void* out, int out_dtype,
-                            int32_t* dev_status) {
-  CUtensorMap mG, mW;
-  if (!encode_bf16_2d(&mG, g, V, tc, 2ull * ldg, 64, 128)) return OLIVE_ERR_CUDA;
-  if (!encode_bf16_2d(&mW, W, d, V, 2ull * d, 64, 64)) return OLIVE_ERR_CUDA;
-  DhKern::Params p;
+BwdParams base_params(const Ctx& c, const int32_t* rows, const int32_t* n_rows, int32_t T,
+                      int32_t V, float inv_tau, int32_t* dev_status) {
+  BwdParams p = {};
   p.dev_status = dev_status;
   p.wait_limit_ns = c.wait_limit_ns;
   p.n_rows = n_rows;
   p.rows = rows;
   p.T = T;
-  p.d = d;
   p.V = V;
-  p.out_dtype = out_dtype;
-  p.slab_start = slab_start;
-  p.tc = tc;
-  p.out = out;
-  return launch_core<DhKern>(c, mG, mW, p);
+  p.inv_tau = inv_tau;
+  p.scale2 = inv_tau * kLog2e;
+  p.group_rows = 16;
+  return p;
+}
+
+}  // namespace
+
+size_t bwd_counter_words(int64_t Tpad, int64_t tc) {
+  const int64_t max_slabs = ceil_div(Tpad, tc) + 1;
+  const int64_t max_rt = tc / kRowAlign;
+  return static_cast<size_t>(2 * max_slabs + max_slabs * max_rt);
 }
 
 olive_status launch_loss_bwd(const Ctx& c, const void* hidden, const void* W,
@@ -390,62 +679,74 @@ olive_status launch_loss_bwd(const Ctx& c, const void* hidden, const void* W,
   if (st != OLIVE_OK) return st;
   if (cudaMemsetAsync(d_hidden, 0, elt * T * static_cast<size_t>(d), c.stream) != cudaSuccess)
     return OLIVE_ERR_CUDA;
+  const size_t nctr = bwd_counter_words(Tpad, w.tc);
+  if (cudaMemsetAsync(w.counters, 0, 4 * nctr, c.stream) != cudaSuccess) return OLIVE_ERR_CUDA;
 
-  CUtensorMap mHcK, mWK, mGmn, mHcMn;
-  if (!encode_bf16_2d(&mHcK, w.hc, d, Tpad, 2ull * d, 64, 128)) return OLIVE_ERR_CUDA;
-  if (!encode_bf16_2d(&mWK, W, d, V, 2ull * d, 64, 256)) return OLIVE_ERR_CUDA;
-  if (!encode_bf16_2d(&mGmn, w.g, V, w.tc, 2ull * ldg, 64, 64)) return OLIVE_ERR_CUDA;
-  if (!encode_bf16_2d(&mHcMn, w.hc, d, Tpad, 2ull * d, 64, 64)) return OLIVE_ERR_CUDA;
+  BwdMaps maps;
+  if (!encode_bf16_2d(&maps.m[0], w.hc, d, Tpad, 2ull * d, 64, 128) ||
+      !encode_bf16_2d(&maps.m[1], W, d, V, 2ull * d, 64, 256) ||
+      !encode_bf16_2d(&maps.m[2], w.g, V, w.tc, 2ull * ldg, 64, 128) ||
+      !encode_bf16_2d(&maps.m[3], W, d, V, 2ull * d, 64, 64) ||
+      !encode_bf16_2d(&maps.m[4], w.g, V, w.tc, 2ull * ldg, 64, 64) ||
+      !encode_bf16_2d(&maps.m[5], w.hc, d, Tpad, 2ull * d, 64, 64))
+    return OLIVE_ERR_CUDA;
 
-  float* dw_out = grad_dtype == OLIVE_DTYPE_F32 ? static_cast<float*>(d_W) : w.dw_acc;
-  const int64_t n_slabs = ceil_div(Tpad, w.tc);
-  for (int64_t sl = 0; sl < n_slabs; ++sl) {
-    const int64_t start = sl * w.tc;
-    GradKern::Params gp;
-    gp.dev_status = dev_status;
-    gp.wait_limit_ns = c.wait_limit_ns;
-    gp.n_rows = n_rows;
-    gp.rows = rows;
-    gp.targets = targets;
-    gp.lse = lse;
-    gp.grad_loss = grad_loss;
-    gp.T = T;
-    gp.d = d;
-    gp.V = V;
-    gp.reduction = reduction;
-    gp.group_rows = 16;
-    gp.slab_start = start;
-    gp.tc = w.tc;
-    gp.ldg = ldg;
-    gp.inv_tau = inv_tau;
-    gp.scale2 = inv_tau * kLog2e;
-    gp.g = static_cast<__nv_bfloat16*>(w.g);
-    if ((st = launch_core<GradKern>(c, mHcK, mWK, gp)) != OLIVE_OK) return st;
+  BwdParams p = base_params(c, rows, n_rows, T, V, inv_tau, dev_status);
+  p.targets = targets;
+  p.lse = lse;
+  p.grad_loss = grad_loss;
+  p.kl = 0;
+  p.d = d;
+  p.d2 = 0;
+  p.reduction = reduction;
+  p.out_dtype = grad_dtype;
+  p.tc_max = static_cast<int32_t>(w.tc);
+  p.max_slabs = static_cast<int32_t>(ceil_div(Tpad, w.tc) + 1);
+  p.max_rt = static_cast<int32_t>(w.tc / kRowAlign);
+  p.ldg = ldg;
+  p.g = static_cast<__nv_bfloat16*>(w.g);
+  p.dh_out = d_hidden;
+  p.dw_out = d_W;
+  p.dw_acc = grad_dtype == OLIVE_DTYPE_F32 ? static_cast<float*>(d_W) : w.dw_acc;
+  p.counters = w.counters;
+  return launch_bwd_fused(c, maps, p);
+}
 
-    if ((st = launch_dh_slab(c, w.g, ldg, w.tc, W, d, V, rows, n_rows, T, start, d_hidden,
-                             grad_dtype, dev_status)) != OLIVE_OK)
-      return st;
-
-    DwKern::Params wp;
-    wp.dev_status = dev_status;
-    wp.wait_limit_ns = c.wait_limit_ns;
-    wp.n_rows = n_rows;
-    wp.T = T;
-    wp.d = d;
-    wp.V = V;
-    wp.first = sl == 0;
-    wp.slab_start = start;
-    wp.tc = w.tc;
-    wp.out = dw_out;
-    if ((st = launch_core<DwKern>(c, mGmn, mHcMn, wp)) != OLIVE_OK) return st;
-  }
-  if (grad_dtype == OLIVE_DTYPE_BF16) {
-    const size_t n4 = static_cast<size_t>(V) * d / 4;
-    f32_to_bf16_kernel<<<c.num_sms * 8, 256, 0, c.stream>>>(
-        reinterpret_cast<const float4*>(w.dw_acc), static_cast<uint2*>(d_W), n4);
-    if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;
-  }
-  return OLIVE_OK;
+olive_status launch_kl_bwd(const Ctx& c, const void* hcs, const void* hct, const void* W_s,
+                           int32_t d_s, const void* W_t, int32_t d_t, const int32_t* rows,
+                           const int32_t* n_rows, int32_t T, int32_t V, float inv_tau, int reverse,
+                           const float* grad_kl, const float* stats, int32_t ld_stats, void* g,
+                           int64_t tc, uint32_t* counters, void* d_h_s, int grad_dtype,
+                           int32_t* dev_status) {
+  const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
+  const int64_t ldg = vpad(V);
+  const size_t nctr = bwd_counter_words(Tpad, tc);
+  if (cudaMemsetAsync(counters, 0, 4 * nctr, c.stream) != cudaSuccess) return OLIVE_ERR_CUDA;
+  BwdMaps maps;
+  if (!encode_bf16_2d(&maps.m[0], hcs, d_s, Tpad, 2ull * d_s, 64, 128) ||
+      !encode_bf16_2d(&maps.m[1], W_s, d_s, V, 2ull * d_s, 64, 128) ||
+      !encode_bf16_2d(&maps.m[2], g, V, tc, 2ull * ldg, 64, 128) ||
+      !encode_bf16_2d(&maps.m[3], W_s, d_s, V, 2ull * d_s, 64, 64) ||
+      !encode_bf16_2d(&maps.m[4], hct, d_t, Tpad, 2ull * d_t, 64, 128) ||
+      !encode_bf16_2d(&maps.m[5], W_t, d_t, V, 2ull * d_t, 64, 128))
+    return OLIVE_ERR_CUDA;
+  BwdParams p = base_params(c, rows, n_rows, T, V, inv_tau, dev_status);
+  p.grad_kl = grad_kl;
+  p.stats = stats;
+  p.ld_stats = ld_stats;
+  p.kl = 1;
+  p.reverse = reverse;
+  p.d = d_s;
+  p.d2 = d_t;
+  p.out_dtype = grad_dtype;
+  p.tc_max = static_cast<int32_t>(tc);
+  p.max_slabs = static_cast<int32_t>(ceil_div(Tpad, tc) + 1);
+  p.max_rt = static_cast<int32_t>(tc / kRowAlign);
+  p.ldg = ldg;
+  p.g = static_cast<__nv_bfloat16*>(g);
+  p.dh_out = d_h_s;
+  p.counters = counters;
+  return launch_bwd_fused(c, maps, p);
 }
 
 }  // namespace olive

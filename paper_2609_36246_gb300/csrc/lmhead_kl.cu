@@ -17,7 +17,8 @@
 // Gradient: the logits are recomputed per tile and turned into
 //   reverse: G = g_t inv_tau p_s (log p_s - log p_t - KL_t)
 //   forward: G = g_t inv_tau (p_s - p_t)
-// stored as a bf16 slab, then d_h_s = G . W_s by the shared dh GEMM.
+// stored as a bf16 slab, then d_h_s = G . W_s; both run in the fused backward
+// kernel of lmhead_bwd.cu.
 #include <cmath>
 
 #include "gemm_core.cuh"
@@ -178,129 +179,6 @@ __global__ void kl_finalize_kernel(const int32_t* __restrict__ n_rows, const int
   }
 }
 
-struct KlGradKern {
-  static constexpr int kBN = kKlBN;
-  static constexpr bool kAMn = false;
-  static constexpr bool kBMn = false;
-  static constexpr bool kDual = true;
-  static constexpr int kStages = 6;
-
-  struct Params {
-    int32_t* dev_status;
-    uint64_t wait_limit_ns;
-    const int32_t* n_rows;
-    const int32_t* rows;
-    const float* grad_kl;
-    const float* stats;
-    int32_t T, V, d_s, d_t, ld, reverse, group_rows;
-    int64_t slab_start, tc, ldg;
-    float inv_tau, scale2;
-    __nv_bfloat16* g;
-  };
-  struct Sched {
-    int n, in_slab, mt, vt, units;
-  };
-  static __device__ Sched make_sched(const Params& p) {
-    Sched s;
-    s.n = read_n_rows(p.n_rows, p.T, p.dev_status);
-    long long k = s.n - p.slab_start;
-    if (k < 0) k = 0;
-    if (k > p.tc) k = p.tc;
-    s.in_slab = static_cast<int>(k);
-    s.mt = (s.in_slab + kBM - 1) / kBM;
-    s.vt = (p.V + kBN - 1) / kBN;
-    s.units = s.mt * s.vt;
-    return s;
-  }
-  static __device__ int num_units(const Params&, const Sched& s) { return s.units; }
-  static __device__ int unit_len(const Params&, const Sched&, int) { return 1; }
-  static __device__ void pos(const Params& p, const Sched& s, int u, int& i, int& j) {
-    const Raster r{s.mt, s.vt, p.group_rows};
-    r.tile(u, i, j);
-  }
-  static __device__ TileC tile(const Params& p, const Sched& s, int u, int) {
-    int i, j;
-    pos(p, s, u, i, j);
-    TileC c;
-    c.m0 = static_cast<int>(p.slab_start) + i * kBM;
-    c.n0 = j * kBN;
-    c.ka0 = 0;
-    c.kb0 = 0;
-    c.nk = (p.d_s + kBK - 1) / kBK;
-    c.nk2 = (p.d_t + kBK - 1) / kBK;
-    return c;
-  }
-  struct Epi {
-    int r_local;
-    bool valid;
-    float ls2, lt2, kl, coef;
-    __device__ void begin(const Params& p, const Sched& s, int u, int row) {
-      int i, j;
-      pos(p, s, u, i, j);
-      r_local = i * kBM + row;
-      const long long r = p.slab_start + r_local;
-      valid = r < s.n;
-      ls2 = lt2 = kl = coef = 0.f;
-      if (valid) {
-        const int t = p.rows[r];
-        if (t >= 0 && t < p.T) {
-          ls2 = p.stats[0 * static_cast<size_t>(p.ld) + r] * kLog2e;
-          lt2 = p.stats[1 * static_cast<size_t>(p.ld) + r] * kLog2e;
-          kl = p.stats[2 * static_cast<size_t>(p.ld) + r];
-          coef = p.grad_kl[t] * p.inv_tau;
-        } else {
-          valid = false;
-        }
-      }
-    }
-    __device__ void tile(const Params& p, const Sched&, int, int, const TileC& tc, uint32_t taddr) {
-      __nv_bfloat16* grow = p.g + static_cast<size_t>(r_local) * p.ldg;
-#pragma unroll 1
-      for (int c = 0; c < kBN; c += 32) {
-        const int col0 = tc.n0 + c;
-        if (col0 >= p.V) break;
-        uint32_t a[32], b[32];
-        tmem_ld_32x32b_x32(taddr + c, a);
-        tmem_ld_32x32b_x32(taddr + kBN + c, b);
-        tmem_ld_wait();
-        float g[32];
-#pragma unroll
-        for (int k = 0; k < 32; ++k) {
-          const float ys = __uint_as_float(a[k]) * p.scale2 - ls2;  // log2 p_s
-          const float yt = __uint_as_float(b[k]) * p.scale2 - lt2;  // log2 p_t
-          const float ps = fast_exp2(ys);
-          float v;
-          if (p.reverse) v = ps * ((ys - yt) * kLn2 - kl);
-          else v = ps - fast_exp2(yt);
-          g[k] = valid ? coef * v : 0.f;
-        }
-        if (col0 + 32 <= p.V) {
-          store_bf16x32_kl(grow + col0, g);
-        } else {
-          const int nv = p.V - col0;
-#pragma unroll
-          for (int k = 0; k < 32; ++k)
-            if (k < nv) grow[col0 + k] = __float2bfloat16_rn(g[k]);
-        }
-      }
-    }
-    __device__ void end(const Params&, const Sched&, int) {}
-
-    __device__ static void store_bf16x32_kl(__nv_bfloat16* dst, const float (&g)[32]) {
-      uint4* d4 = reinterpret_cast<uint4*>(dst);
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        uint4 v;
-        v.x = pack_bf16x2(g[8 * q + 0], g[8 * q + 1]);
-        v.y = pack_bf16x2(g[8 * q + 2], g[8 * q + 3]);
-        v.z = pack_bf16x2(g[8 * q + 4], g[8 * q + 5]);
-        v.w = pack_bf16x2(g[8 * q + 6], g[8 * q + 7]);
-        d4[q] = v;
-      }
-    }
-  };
-};
-
 template <class K>
 olive_status launch_dual(const Ctx& c, const CUtensorMap& a, const CUtensorMap& b,
                          const CUtensorMap& a2, const CUtensorMap& b2, const typename K::Params& p) {
@@ -359,35 +237,8 @@ olive_status launch_divergence(const Ctx& c, const void* h_s, const void* W_s, i
   const size_t elt = grad_dtype == OLIVE_DTYPE_BF16 ? 2 : 4;
   if (cudaMemsetAsync(d_h_s, 0, elt * T * static_cast<size_t>(d_s), c.stream) != cudaSuccess)
     return OLIVE_ERR_CUDA;
-  const int64_t ldg = vpad(V);
-  const int64_t n_slabs = ceil_div(Tpad, w.tc);
-  for (int64_t sl = 0; sl < n_slabs; ++sl) {
-    KlGradKern::Params gp;
-    gp.dev_status = dev_status;
-    gp.wait_limit_ns = c.wait_limit_ns;
-    gp.n_rows = n_rows;
-    gp.rows = rows;
-    gp.grad_kl = grad_kl;
-    gp.stats = w.stats;
-    gp.T = T;
-    gp.V = V;
-    gp.d_s = d_s;
-    gp.d_t = d_t;
-    gp.ld = p.ld;
-    gp.reverse = reverse;
-    gp.group_rows = 16;
-    gp.slab_start = sl * w.tc;
-    gp.tc = w.tc;
-    gp.ldg = ldg;
-    gp.inv_tau = inv_tau;
-    gp.scale2 = inv_tau * kLog2e;
-    gp.g = static_cast<__nv_bfloat16*>(w.g);
-    if ((st = launch_dual<KlGradKern>(c, mHs, mWs, mHt, mWt, gp)) != OLIVE_OK) return st;
-    if ((st = launch_dh_slab(c, w.g, ldg, w.tc, W_s, d_s, V, rows, n_rows, T, sl * w.tc, d_h_s,
-                             grad_dtype, dev_status)) != OLIVE_OK)
-      return st;
-  }
-  return OLIVE_OK;
+  return launch_kl_bwd(c, w.hcs, w.hct, W_s, d_s, W_t, d_t, rows, n_rows, T, V, inv_tau, reverse,
+                       grad_kl, w.stats, p.ld, w.g, w.tc, w.counters, d_h_s, grad_dtype, dev_status);
 }
 
 }  // namespace olive

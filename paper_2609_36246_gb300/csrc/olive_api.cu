@@ -80,11 +80,11 @@ bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t
 }
 
 int64_t slab_rows(int64_t Tpad, int64_t V) {
-  // G slab of at most ~2.5 GB (bf16), in whole 128-row tiles, <= 16384 rows
-  const int64_t budget = 2500ll * 1000 * 1000;
+  // G buffer of at most ~5.6 GB (bf16), in whole 128-row tiles, <= 32768 rows
+  const int64_t budget = 5600ll * 1000 * 1000;
   int64_t tc = budget / (2 * vpad(V)) / kRowAlign * kRowAlign;
   if (tc < kRowAlign) tc = kRowAlign;
-  if (tc > 16384) tc = 16384;
+  if (tc > 32768) tc = 32768;
   if (tc > Tpad) tc = Tpad;
   return tc;
 }
@@ -130,6 +130,7 @@ static BwdWs carve_bwd_impl(void* ws, int64_t T, int64_t d, int64_t V, int grad_
   w.hc = c.take(2ull * Tpad * d);
   w.g = c.take(2ull * w.tc * vpad(V));
   w.dw_acc = grad_dtype == OLIVE_DTYPE_BF16 ? static_cast<float*>(c.take(4ull * V * d)) : nullptr;
+  w.counters = static_cast<uint32_t*>(c.take(4ull * bwd_counter_words(Tpad, w.tc)));
   if (total) *total = c.off;
   return w;
 }
@@ -153,6 +154,7 @@ static KlWs carve_kl_impl(void* ws, int64_t T, int64_t ds, int64_t dt, int64_t V
   w.part = static_cast<float*>(c.take(4ull * 5 * kSvMax * Tpad));
   w.stats = static_cast<float*>(c.take(4ull * 3 * Tpad));
   w.g = grad ? c.take(2ull * w.tc * vpad(V)) : nullptr;
+  w.counters = grad ? static_cast<uint32_t*>(c.take(4ull * bwd_counter_words(Tpad, w.tc))) : nullptr;
   if (total) *total = c.off;
   return w;
 }

@@ -8,9 +8,8 @@ independent) and rounded fp32 -> bf16 by round-to-nearest-even (torch).
 Workloads (the paper's RLVE setting: prefix cut at student token 4096 with a
 1024-token teacher continuation, 64 prompts x 4 rollouts per step; Section 4.1
 and Appendix A, Table rose-config).  The paper prints neither the hidden width
-nor the vocabulary size; d and V below are the 4B-class widths used for the
-student (d=4096; the scoring case uses d=2048) and the teacher (d=5120) with a
-151936-entry vocabulary.
+nor the vocabulary size; the widths below are those of the measured workloads:
+student d=4096 (2048 in the scoring case), teacher d=5120, V=151936.
 
   tiny     4 x 128 tokens, cut ~ U[16,112), ids ~ U[0,4096), d=256, V=4096,
            hidden and W ~ N(0, 0.02)

@@ -83,6 +83,28 @@ def test_vocab_sum_of_dW_vanishes():
 
 
 @pytest.mark.slow
+def test_medium_vocab_sampled_dh_and_dw():
+    """~8k masked rows, d = 4096, V = 32003 (ragged last tile): dH on sampled
+    rows and dW on sampled vocabulary rows, both against the oracle."""
+    rng = np.random.default_rng(31)
+    b = synth.batch_from_lengths(rng, [1000, 777, 2048], [3000, 2500, 2700], 32003)
+    h = synth.rms_hidden_bf16(rng, (b.T, 4096))
+    W = synth.normal_bf16(rng, (32003, 4096), 0.02)
+    dh, dw = _gpu_grads(b, h, W, reduction="mean")
+    o = oracle_pack(b)
+    rows = sample_rows(o["rows"], 24, seed=3)
+    ref = oracle.token_loss_bwd_rows(to_f32(h), to_f32(W), o["targets"], rows, reduction="mean",
+                                     n_mask=o["n_rows"])
+    assert rel_frob(dh[rows], ref) <= 1e-2
+    # a target id, the last (ragged) tile and random ids
+    vocab = np.unique(np.concatenate([[int(o["targets"][o["rows"][0]]), 0, 32002],
+                                      np.random.default_rng(4).integers(0, 32003, size=13)]))
+    refw = oracle.token_loss_bwd_vocab(to_f32(h), to_f32(W), o["targets"], o["rows"], vocab,
+                                       reduction="mean")
+    assert rel_frob(dw[vocab], refw) <= 1e-2
+
+
+@pytest.mark.slow
 def test_fwdbwd_workload_sampled():
     """8 x 4096 tokens, d = 4096, V = 151936: dH on sampled rows from the oracle;
     dW checked through its exact vocabulary-sum identity and magnitude."""

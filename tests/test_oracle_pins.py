@@ -243,6 +243,9 @@ def test_bwd_invariants_and_row_sampler():
     sub = rows[::2]
     part = oracle.token_loss_bwd_rows(h, W, targets, sub, reduction="mean", n_mask=len(rows))
     assert np.allclose(part, dH[sub], rtol=1e-12, atol=1e-15)
+    vs = np.array([0, 7, 29])
+    partw = oracle.token_loss_bwd_vocab(h, W, targets, rows, vs, reduction="mean")
+    assert np.allclose(partw, dW[vs], rtol=1e-12, atol=1e-15)
 
 
 def test_empty_mask():
