@@ -272,6 +272,15 @@ def run_ours(args, world, rank, local):
     traffic = profile_traffic("bwd_fused_kernel", rev)
     launches = 2 + 4 + 2  # splice (scan, fill), forward (gather, GEMM, finalize, loss), backward (gather, fused)
 
+    extra = {}
+    if not args.no_extra:
+        del ws_f, ws_b, dh, dw
+        torch.cuda.empty_cache()
+        extra["kl_divergence"] = measure_kl(dev, burst)
+        torch.cuda.empty_cache()
+        extra["varlen"] = measure_varlen(dev, burst)
+        torch.cuda.empty_cache()
+
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         rate, secs, nr = oracle_sample_rate(b, h_cpu, W_cpu, args.cpu_rows)
@@ -302,6 +311,7 @@ def run_ours(args, world, rank, local):
         "gpu_launches": launches * args.steps,
         "clocks": clk.summary(),
         "cpu_baseline": cpu,
+        "other_workloads": extra,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -319,6 +329,89 @@ def profile_traffic(kernel: str, rev: str):
                 if len(parts) == 4 and parts[0] == "traffic:" and parts[1] == kernel and parts[2] == rev:
                     return float(parts[3])
     return None
+
+
+def gpu_inputs(seed: int, T: int, d: int, V: int, dev):
+    """Seeded bf16 hidden rows (RMS-normalised N(0,1)) and W ~ N(0, 0.02),
+    drawn on the device (timing-only workloads; parity runs use synth)."""
+    g = torch.Generator(device=dev).manual_seed(seed)
+    h = torch.randn(T, d, generator=g, device=dev, dtype=torch.float32)
+    h = (h * torch.rsqrt(h.square().mean(dim=1, keepdim=True) + 1e-6)).to(torch.bfloat16)
+    W = (torch.randn(V, d, generator=g, device=dev, dtype=torch.float32) * 0.02).to(torch.bfloat16)
+    return h, W
+
+
+def time_calls(fn, steps: int, warmup: int) -> float:
+    """Mean ms per call of fn() on the current stream (CUDA events)."""
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(steps):
+        fn()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / steps
+
+
+def measure_kl(dev, burst: float, steps: int = 3):
+    """OPD per-token full-vocabulary KL forward + d/dh_s (16384 rows,
+    student d = 4096, teacher d = 5120, V = 151936)."""
+    from paper_2609_36246_gb300 import binding as B
+    N, ds, dt, V = 16384, 4096, 5120, 151936
+    hs, Ws = gpu_inputs(21, N, ds, V, dev)
+    ht, Wt = gpu_inputs(22, N, dt, V, dev)
+    rows = torch.arange(N, dtype=torch.int32, device=dev)
+    n = torch.tensor([N], dtype=torch.int32, device=dev)
+    gk = torch.ones(N, dtype=torch.float32, device=dev)
+    ws = B.workspace(B.olive_workspace_size("divergence", N, ds, V, d_t=dt, grad=True), dev)
+    st = B.new_status(dev)
+    ms = time_calls(lambda: B.olive_token_divergence(hs, Ws, ht, Wt, rows, n, 1.0, "reverse", gk,
+                                                     torch.bfloat16, ws=ws, dev_status=st),
+                    steps, 1)
+    if int(st.item()) != 0:
+        raise RuntimeError(f"divergence status {B.status_bits(st)}")
+    flops = 2.0 * N * V * (ds + dt) + 2.0 * N * V * ds
+    return {"workload": "per-token reverse KL + d/dh_s: 16384 rows, d_s=4096, d_t=5120, V=151936",
+            "value": N / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
+            "pct_bf16_peak": 100.0 * flops / (ms / 1e3) / 1e12 / burst, "steps": steps}
+
+
+def measure_varlen(dev, burst: float, steps: int = 2):
+    """splice/pack + forward + backward on the variable-length batch
+    (64 sequences, lengths U[1024,16384], ~557k packed tokens)."""
+    from paper_2609_36246_gb300 import binding as B
+    from paper_2609_36246_gb300 import synth
+    b = synth.make_batch("varlen")
+    d, V, T = 4096, 151936, b.T
+    h, W = gpu_inputs(23, T, d, V, dev)
+    i32 = lambda a: torch.from_numpy(np.ascontiguousarray(a, dtype=np.int32)).to(dev)
+    pre, poff, con, coff = i32(b.prefix_ids), i32(b.prefix_off), i32(b.cont_ids), i32(b.cont_off)
+    ws_f = B.workspace(B.olive_workspace_size("logprob_fwd", T, d, V), dev)
+    ws_b = B.workspace(B.olive_workspace_size("loss_bwd", T, d, V), dev)
+    st = B.new_status(dev)
+    gl = torch.ones(1, dtype=torch.float32, device=dev)
+    out_f = (torch.empty(T, device=dev), torch.empty(T, device=dev), torch.empty(1, device=dev))
+    out_b = (torch.empty(T, d, dtype=torch.bfloat16, device=dev),
+             torch.empty(V, d, dtype=torch.bfloat16, device=dev))
+
+    def step():
+        pk = B.olive_splice_pack(pre, poff, con, coff, V, T, dev_status=st)
+        _, lse, _ = B.olive_token_logprob_fwd(h, W, pk["targets"], pk["rows"], pk["n_rows"], 1.0,
+                                              "mean", ws=ws_f, dev_status=st, out=out_f)
+        B.olive_token_loss_bwd(h, W, pk["targets"], pk["rows"], pk["n_rows"], lse, gl, 1.0, "mean",
+                               torch.bfloat16, ws=ws_b, dev_status=st, out=out_b)
+
+    ms = time_calls(step, steps, 1)
+    if int(st.item()) != 0:
+        raise RuntimeError(f"varlen status {B.status_bits(st)}")
+    n = b.n_mask
+    return {"workload": f"variable-length batch: 64 sequences, {T} packed tokens, N_mask={n}, "
+                        "d=4096, V=151936", "value": n / (ms / 1e3), "unit": "tokens/s",
+            "ms_per_step": ms, "pct_bf16_peak": 100.0 * 6.0 * n * d * V / (ms / 1e3) / 1e12 / burst,
+            "steps": steps}
 
 
 def kernel_rev() -> str:
@@ -367,6 +460,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-rows", type=int, default=32)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extra", action="store_true",
+                    help="skip the divergence and variable-length measurements")
     args = ap.parse_args()
     world, rank, local = dist_setup()
     if args.impl == "reference":
