@@ -1,0 +1,153 @@
+"""The oracle's pins catch plausible mistakes.
+
+Each mutant is a copy of oracle/olive_oracle.py with one planted mistake (an
+off-by-one mask, a dropped term, a wrong sign, a missing factor, swapped
+directions, a wrong denominator).  The pin checks below restate the pins of
+test_oracle_pins.py as functions of the oracle module; all of them must hold
+for the real oracle and at least one must fail for every mutant.  Everything
+runs on the CPU.
+"""
+
+import importlib.util
+import json
+import math
+import os
+import types
+
+import numpy as np
+import pytest
+import scipy.special
+import torch
+import torch.nn.functional as F
+
+import oracle.olive_oracle as real
+
+SRC = real.__file__
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "splice_pack_small.json")
+
+MUTANTS = {
+    "mask_includes_prefix_target": ("mask.append(1 if i + 1 >= P else 0)",
+                                    "mask.append(1 if i + 1 >= P - 1 else 0)"),
+    "target_not_shifted": ("targets.append(seq[i + 1])", "targets.append(seq[i])"),
+    "cut_at_prefix_start": ("cut.append(cu[-1] + P)", "cut.append(cu[-1])"),
+    "lse_drops_log_sum": ("lse = m + np.log(np.exp(z - m[:, None]).sum(axis=1))", "lse = m"),
+    "logits_skip_temperature": ("    z *= float(inv_tau)\n", "    z *= 1.0\n"),
+    "grad_drops_onehot": ("        G[np.arange(len(rr)), targets[rr]] -= 1.0\n        G *= g * float(inv_tau)\n        dH[rr] = G @ W64",
+                          "        G *= g * float(inv_tau)\n        dH[rr] = G @ W64"),
+    "grad_wrong_sign": ("        G *= g * float(inv_tau)\n        dH[rr] = G @ W64",
+                        "        G *= -g * float(inv_tau)\n        dH[rr] = G @ W64"),
+    "grad_drops_inv_tau": ("        G *= g * float(inv_tau)\n        dH[rr] = G @ W64",
+                           "        G *= g\n        dH[rr] = G @ W64"),
+    "dW_transposed_pairing": ("        dW += G.T @ h", "        dW += G.T @ h[::-1]"),
+    "mean_over_all_rows": ("        loss = loss / len(rows) if len(rows) else 0.0",
+                           "        loss = loss / len(targets) if len(rows) else 0.0"),
+    "kl_directions_swapped": ("            k = (ps * (lps - lpt)).sum(axis=1)",
+                              "            k = (pt * (lpt - lps)).sum(axis=1)"),
+    "kl_grad_drops_kl_term": ("                dz = ps * (lps - lpt - k[:, None])",
+                              "                dz = ps * (lps - lpt)"),
+    "kl_grad_forward_sign": ("                dz = ps - pt", "                dz = pt - ps"),
+}
+
+
+def load_variant(name=None):
+    with open(SRC) as f:
+        text = f.read()
+    if name is not None:
+        old, new = MUTANTS[name]
+        assert text.count(old) == 1, f"mutation site for {name} not unique"
+        text = text.replace(old, new)
+    mod = types.ModuleType(f"oracle_variant_{name}")
+    exec(compile(text, SRC, "exec"), mod.__dict__)
+    return mod
+
+
+def _case(seed, T=10, d=12, V=41):
+    rng = np.random.default_rng(seed)
+    h = rng.standard_normal((T, d))
+    W = rng.standard_normal((V, d)) * 0.3
+    targets = rng.integers(0, V, size=T)
+    rows = np.sort(rng.choice(T, size=T // 2, replace=False))
+    return h, W, targets, rows
+
+
+# ----------------------------------------------------------------- pin checks
+def pin_golden_splice(O):
+    with open(GOLDEN) as f:
+        g = json.load(f)
+    out = O.splice_pack(g["prefix_ids"], g["prefix_off"], g["cont_ids"], g["cont_off"], g["V"])
+    return all(list(map(int, np.atleast_1d(out[k]))) == (v if isinstance(v, list) else [v])
+               for k, v in g["expect"].items())
+
+
+def pin_uniform(O):
+    h = np.random.default_rng(0).standard_normal((5, 8))
+    logp, _, loss = O.token_logprob(h, np.zeros((64, 8)), np.arange(5), np.arange(5))
+    return np.allclose(logp, -math.log(64), atol=1e-12) and abs(loss - 5 * math.log(64)) < 1e-9
+
+
+def pin_scipy(O):
+    h, W, t, r = _case(1)
+    logp, lse, _ = O.token_logprob(h, W, t, r, inv_tau=1.3)
+    z = 1.3 * h @ W.T
+    ref = scipy.special.log_softmax(z, axis=1)
+    return (np.allclose(logp[r], ref[r, t[r]], atol=1e-10)
+            and np.allclose(lse[r], scipy.special.logsumexp(z, axis=1)[r], atol=1e-10))
+
+
+def pin_torch_ce_and_autograd(O):
+    ok = True
+    for red in ("sum", "mean"):
+        h, W, t, r = _case(2)
+        _, _, loss = O.token_logprob(h, W, t, r, inv_tau=1.5, reduction=red)
+        dH, dW = O.token_loss_bwd(h, W, t, r, inv_tau=1.5, reduction=red, grad_loss=0.7)
+        ht = torch.from_numpy(h).requires_grad_(True)
+        Wt = torch.from_numpy(W).requires_grad_(True)
+        z = 1.5 * (ht[torch.from_numpy(r)] @ Wt.T)
+        ref = F.cross_entropy(z, torch.from_numpy(t[r]), reduction=red)
+        (0.7 * ref).backward()
+        ok &= abs(loss - ref.item()) < 1e-9 * max(1.0, abs(ref.item()))
+        ok &= np.allclose(dH, ht.grad.numpy(), atol=1e-12) and np.allclose(dW, Wt.grad.numpy(), atol=1e-12)
+    return bool(ok)
+
+
+def pin_kl(O):
+    ok = True
+    rng = np.random.default_rng(3)
+    hs, Ws = rng.standard_normal((6, 7)), rng.standard_normal((30, 7)) * 0.5
+    ht, Wt = rng.standard_normal((6, 9)), rng.standard_normal((30, 9)) * 0.5
+    r = np.array([0, 2, 5])
+    for direction in ("reverse", "forward"):
+        kl, dHs = O.token_divergence(hs, Ws, ht, Wt, r, 1.1, direction, grad_kl=np.ones(6))
+        hs_t = torch.from_numpy(hs).requires_grad_(True)
+        lps = F.log_softmax(1.1 * (hs_t[torch.from_numpy(r)] @ torch.from_numpy(Ws).T), 1)
+        lpt = F.log_softmax(1.1 * (torch.from_numpy(ht)[torch.from_numpy(r)] @ torch.from_numpy(Wt).T), 1)
+        if direction == "reverse":
+            ref = F.kl_div(lpt, lps, log_target=True, reduction="none").sum(1)
+        else:
+            ref = F.kl_div(lps, lpt, log_target=True, reduction="none").sum(1)
+        ref.sum().backward()
+        ok &= np.allclose(kl[r], ref.detach().numpy(), atol=1e-12)
+        ok &= np.allclose(dHs, hs_t.grad.numpy(), atol=1e-12)
+    return bool(ok)
+
+
+PINS = [pin_golden_splice, pin_uniform, pin_scipy, pin_torch_ce_and_autograd, pin_kl]
+
+
+def test_real_oracle_passes_every_pin():
+    O = load_variant(None)
+    assert all(pin(O) for pin in PINS)
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_every_mutant_is_caught(name):
+    O = load_variant(name)
+    failed = []
+    for pin in PINS:
+        try:
+            ok = pin(O)
+        except Exception:  # a crash also counts as caught
+            ok = False
+        if not ok:
+            failed.append(pin.__name__)
+    assert failed, f"mutant {name} passed every pin"
