@@ -278,6 +278,8 @@ def run_ours(args, world, rank, local):
         torch.cuda.empty_cache()
         extra["kl_divergence"] = measure_kl(dev, burst)
         torch.cuda.empty_cache()
+        extra["scoring_fwd"], extra["topk_entropy"] = measure_scoring(dev, burst)
+        torch.cuda.empty_cache()
         extra["varlen"] = measure_varlen(dev, burst)
         torch.cuda.empty_cache()
 
@@ -377,6 +379,39 @@ def measure_kl(dev, burst: float, steps: int = 3):
     return {"workload": "per-token reverse KL + d/dh_s: 16384 rows, d_s=4096, d_t=5120, V=151936",
             "value": N / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
             "pct_bf16_peak": 100.0 * flops / (ms / 1e3) / 1e12 / burst, "steps": steps}
+
+
+def measure_scoring(dev, burst: float, steps: int = 5):
+    """Forward scoring (log-probs + loss, no backward) and the entropy / top-16
+    sweep on 2 x (4096 prefix + 4096 continuation) tokens, d = 2048, V = 151936."""
+    from paper_2609_36246_gb300 import binding as B
+    from paper_2609_36246_gb300 import synth
+    b = synth.make_batch("scoring")
+    d, V, T = 2048, 151936, b.T
+    h, W = gpu_inputs(24, T, d, V, dev)
+    i32 = lambda a: torch.from_numpy(np.ascontiguousarray(a, dtype=np.int32)).to(dev)
+    st = B.new_status(dev)
+    pk = B.olive_splice_pack(i32(b.prefix_ids), i32(b.prefix_off), i32(b.cont_ids),
+                             i32(b.cont_off), V, T, dev_status=st)
+    ws_f = B.workspace(B.olive_workspace_size("logprob_fwd", T, d, V), dev)
+    ws_k = B.workspace(B.olive_workspace_size("topk_fwd", T, d, V), dev)
+    out = (torch.empty(T, device=dev), torch.empty(T, device=dev), torch.empty(1, device=dev))
+    ms_f = time_calls(lambda: B.olive_token_logprob_fwd(h, W, pk["targets"], pk["rows"],
+                                                        pk["n_rows"], ws=ws_f, dev_status=st,
+                                                        out=out), steps, 1)
+    ms_k = time_calls(lambda: B.olive_token_topk_fwd(h, W, pk["rows"], pk["n_rows"], 16, ws=ws_k,
+                                                     dev_status=st), steps, 1)
+    if int(st.item()) != 0:
+        raise RuntimeError(f"scoring status {B.status_bits(st)}")
+    n = b.n_mask
+    flops = 2.0 * n * d * V
+    res = {"workload": "forward scoring: 2 x (4096 + 4096) tokens, N_mask=8192, d=2048, V=151936",
+           "value": n / (ms_f / 1e3), "unit": "tokens/s", "ms_per_step": ms_f,
+           "pct_bf16_peak": 100.0 * flops / (ms_f / 1e3) / 1e12 / burst, "steps": steps}
+    top = {"workload": "entropy + top-16 log-probs, same batch", "value": n / (ms_k / 1e3),
+           "unit": "tokens/s", "ms_per_step": ms_k,
+           "pct_bf16_peak": 100.0 * flops / (ms_k / 1e3) / 1e12 / burst, "steps": steps}
+    return res, top
 
 
 def measure_varlen(dev, burst: float, steps: int = 2):

@@ -72,7 +72,8 @@ typedef enum {
 enum { OLIVE_REDUCE_SUM = 0, OLIVE_REDUCE_MEAN = 1 };
 enum { OLIVE_KL_REVERSE = 0, OLIVE_KL_FORWARD = 1 };
 enum { OLIVE_DTYPE_BF16 = 0, OLIVE_DTYPE_F32 = 1 };
-enum { OLIVE_OP_LOGPROB_FWD = 0, OLIVE_OP_LOSS_BWD = 1, OLIVE_OP_DIVERGENCE = 2 };
+enum { OLIVE_OP_LOGPROB_FWD = 0, OLIVE_OP_LOSS_BWD = 1, OLIVE_OP_DIVERGENCE = 2,
+       OLIVE_OP_TOPK_FWD = 3 };
 
 /* ABI version of the loaded library (OLIVE_ABI_VERSION). */
 OLIVE_API int olive_abi_version(void);
@@ -84,6 +85,7 @@ OLIVE_API const char* olive_status_string(olive_status s);
  * Workspace bytes a compute call needs for host-side upper bound T rows.
  *   op  OLIVE_OP_LOGPROB_FWD / OLIVE_OP_LOSS_BWD: d = hidden width, d_t ignored.
  *   op  OLIVE_OP_DIVERGENCE: d = student width d_s, d_t = teacher width.
+ *   op  OLIVE_OP_TOPK_FWD: d = hidden width, d_t ignored.
  *   `grad` (bwd / divergence): non-zero when gradients are requested
  *   (OLIVE_OP_LOSS_BWD always computes them); `grad_dtype` is the dtype of
  *   d_W for OLIVE_OP_LOSS_BWD (bf16 output needs an fp32 accumulator).
@@ -153,6 +155,27 @@ OLIVE_API olive_status olive_token_logprob_fwd(const void* hidden, const void* W
                                      float* logp, float* lse, float* loss,
                                      void* workspace, size_t ws_bytes,
                                      int32_t* dev_status, void* stream);
+
+/*
+ * olive_token_topk_fwd -- per-token entropy and the K largest log-probs of
+ * the student, from the same LM-head sweep as olive_token_logprob_fwd.  OPD
+ * consumes the student's top-16 log-probs per token (Appendix A, Table
+ * opd-config, "LogProb top-K 16"); the entropy is -sum_v p_v log p_v.  On
+ * every masked row r (t = rows[r], r < *n_rows), with z = inv_tau h[t] W^T:
+ *   lse[t]           = log sum_v exp(z_v)
+ *   entropy[t]       = lse[t] - sum_v p_v z_v
+ *   topk_logp[t, j]  = z_(j) - lse[t], the j-th largest, j = 0..K-1
+ *   topk_ids[t, j]   = its vocabulary id (equal log-probs: smaller id first)
+ * 1 <= K <= 16.  Rows not in `rows` get 0 (ids -1).  lse, entropy fp32 [T];
+ * topk_logp fp32 [T, K]; topk_ids int32 [T, K].  The logits are not stored.
+ */
+OLIVE_API olive_status olive_token_topk_fwd(const void* hidden, const void* W,
+                                            const int32_t* rows, const int32_t* n_rows,
+                                            int32_t T, int32_t d, int32_t V, float inv_tau,
+                                            int32_t K, float* lse, float* entropy,
+                                            float* topk_logp, int32_t* topk_ids,
+                                            void* workspace, size_t ws_bytes,
+                                            int32_t* dev_status, void* stream);
 
 /*
  * olive_token_loss_bwd -- gradients of the Eq. (osd-ce) loss through the LM

@@ -11,6 +11,7 @@ from .olive_oracle import (  # noqa: F401
     splice_pack,
     token_divergence,
     token_logprob,
+    token_topk,
     token_loss_bwd,
     token_loss_bwd_rows,
     token_loss_bwd_vocab,

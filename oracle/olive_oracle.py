@@ -20,6 +20,8 @@ Section 1; temperature, Appendix A, Table opd-config):
 * ``token_loss_bwd``   -- d loss / d hidden and d loss / d W of Eq. (osd-ce)
                           through the LM head (sequences held fixed,
                           Section 3.1, so no gradient flows through the ids).
+* ``token_topk``       -- per-token entropy and the student's K largest
+                          log-probs (Appendix A: OPD reads the top-16).
 * ``token_divergence`` -- OPD's per-token reverse KL between student and
                           teacher over the full vocabulary (Section 1), the
                           forward direction as an option, and the gradient of
@@ -297,6 +299,38 @@ def token_loss_bwd_vocab(hidden, W, targets, rows, vocab, inv_tau: float = 1.0,
         G *= g * float(inv_tau)
         out += G.T @ h
     return out
+
+
+# --------------------------------------------------------------------------
+# Per-token entropy and top-K log-probs of the student (Appendix A, Table
+# opd-config: OPD consumes the student's top-16 log-probs per token)
+# --------------------------------------------------------------------------
+def token_topk(hidden, W, rows, K: int, inv_tau: float = 1.0):
+    """Entropy and the K largest log-probabilities of pi_theta per masked row.
+
+    For each row in ``rows``: lse, H = -sum_v p_v log p_v, and the K largest
+    log p_v in descending order with their vocabulary ids; equal log-probs are
+    ordered by ascending id.  Returns (lse [T], H [T], topk_logp [T, K],
+    topk_ids [T, K]) with 0 / -1 off ``rows``.
+    """
+    hidden = np.asarray(hidden)
+    T = hidden.shape[0]
+    rows = np.asarray(rows, dtype=np.int64)
+    lse = np.zeros(T, dtype=np.float64)
+    H = np.zeros(T, dtype=np.float64)
+    tv = np.zeros((T, K), dtype=np.float64)
+    ti = np.full((T, K), -1, dtype=np.int64)
+    for r0 in range(0, len(rows), _ROW_CHUNK):
+        rr = rows[r0:r0 + _ROW_CHUNK]
+        lp, l = log_softmax_rows(logits(_as_f64_rows(hidden, rr), W, inv_tau))
+        lse[rr] = l
+        H[rr] = -(np.exp(lp) * lp).sum(axis=1)
+        ids = np.arange(lp.shape[1])
+        for k, r in enumerate(rr):
+            order = np.lexsort((ids, -lp[k]))[:K]
+            tv[r] = lp[k, order]
+            ti[r] = order
+    return lse, H, tv, ti
 
 
 # --------------------------------------------------------------------------

@@ -27,7 +27,7 @@ STATUS_NAMES = {
 REDUCE = {"sum": 0, "mean": 1}
 DIRECTION = {"reverse": 0, "forward": 1}
 DTYPE = {torch.bfloat16: 0, torch.float32: 1}
-OP = {"logprob_fwd": 0, "loss_bwd": 1, "divergence": 2}
+OP = {"logprob_fwd": 0, "loss_bwd": 1, "divergence": 2, "topk_fwd": 3}
 
 
 class OliveError(RuntimeError):
@@ -69,6 +69,9 @@ def lib() -> ctypes.CDLL:
     L.olive_token_divergence.restype = ctypes.c_int
     L.olive_token_divergence.argtypes = [_P, _P, _I, _P, _P, _I, _P, _P, _I, _I, _F, ctypes.c_int,
                                          _P, _P, _P, ctypes.c_int, _P, _S, _P, _P]
+    L.olive_token_topk_fwd.restype = ctypes.c_int
+    L.olive_token_topk_fwd.argtypes = [_P, _P, _P, _P, _I, _I, _I, _F, _I, _P, _P, _P, _P, _P, _S,
+                                       _P, _P]
     L.olive_token_logprob_fwd_noalloc.restype = ctypes.c_int
     L.olive_token_logprob_fwd_noalloc.argtypes = [_P, _P, _P, _P, _P, _I, _I, _I, _F, ctypes.c_int,
                                                   _P, _P, _P, _P, _P]
@@ -186,6 +189,32 @@ def olive_token_logprob_fwd(hidden, W, targets, rows, n_rows, inv_tau: float = 1
                                        _stream())
     _check(st, "olive_token_logprob_fwd")
     return logp, lse, loss
+
+
+def olive_token_topk_fwd(hidden, W, rows, n_rows, K: int = 16, inv_tau: float = 1.0, ws=None,
+                         dev_status=None):
+    """Per-token lse, entropy and the K largest log-probs with their ids.
+
+    Returns (lse [T], entropy [T], topk_logp [T, K], topk_ids [T, K])."""
+    _need(hidden, torch.bfloat16, "hidden")
+    _need(W, torch.bfloat16, "W")
+    _need(rows, torch.int32, "rows")
+    _need(n_rows, torch.int32, "n_rows")
+    T, d = hidden.shape
+    V = W.shape[0]
+    dev = hidden.device
+    lse = torch.empty(T, dtype=torch.float32, device=dev)
+    ent = torch.empty(T, dtype=torch.float32, device=dev)
+    tv = torch.empty(T, K, dtype=torch.float32, device=dev)
+    ti = torch.empty(T, K, dtype=torch.int32, device=dev)
+    if ws is None:
+        ws = workspace(olive_workspace_size("topk_fwd", T, d, V), dev)
+    ds = dev_status if dev_status is not None else new_status(dev)
+    st = lib().olive_token_topk_fwd(_ptr(hidden), _ptr(W), _ptr(rows), _ptr(n_rows), T, d, V,
+                                    float(inv_tau), int(K), _ptr(lse), _ptr(ent), _ptr(tv), _ptr(ti),
+                                    _ptr(ws), ws.numel(), _ptr(ds), _stream())
+    _check(st, "olive_token_topk_fwd")
+    return lse, ent, tv, ti
 
 
 def olive_token_loss_bwd(hidden, W, targets, rows, n_rows, lse, grad_loss, inv_tau: float = 1.0,

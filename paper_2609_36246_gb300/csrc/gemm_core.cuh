@@ -20,8 +20,9 @@
 // A Kern policy supplies:
 //   Params (with int32_t* dev_status and uint64_t wait_limit_ns), kBN, kAMn,
 //   kBMn, kDual, kStages, Sched, make_sched(p) (thread 0; may read device
-//   counters such as n_rows), num_units(p,s), unit_len(p,s,u), tile(p,s,u,t)
-//   and Epi with begin(p,s,u,row), tile(p,s,u,t,tc,taddr), end(p,s,u).
+//   counters such as n_rows), num_units(p,s), unit_len(p,s,u), tile(p,s,u,t),
+//   kEpiSmem (bytes of shared-memory scratch for the epilogue) and Epi with
+//   init(smem), begin(p,s,u,row), tile(p,s,u,t,tc,taddr), end(p,s,u).
 #pragma once
 
 #include "sm103.cuh"
@@ -54,7 +55,9 @@ struct CoreLayout {
   // barriers: full[S], empty[S], tfull[2], tempty[2], drain
   static constexpr int BAR_BYTES = 8 * (2 * Kern::kStages + 5);
   static constexpr int MISC_BYTES = 64;
-  static constexpr int SMEM_BYTES = 1024 /*alignment slack*/ + RING_BYTES + BAR_BYTES + MISC_BYTES;
+  static constexpr int EPI_BYTES = Kern::kEpiSmem;  // scratch for the epilogue policy
+  static constexpr int SMEM_BYTES =
+      1024 /*alignment slack*/ + RING_BYTES + BAR_BYTES + MISC_BYTES + EPI_BYTES;
   static constexpr int ACC_COLS = Kern::kDual ? 2 * Kern::kBN : Kern::kBN;
   static constexpr uint32_t TMEM_COLS = 2 * ACC_COLS;
   static_assert(TMEM_COLS <= 512, "two accumulators must fit in TMEM");
@@ -228,6 +231,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t aphase = 0;
     bool ok = true;
     typename Kern::Epi epi;
+    epi.init(misc + L::MISC_BYTES);
     for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
       const int nt = Kern::unit_len(p, sched, u);
       epi.begin(p, sched, u, row);

@@ -49,6 +49,17 @@ struct FwdWs {
 size_t fwd_ws_bytes(int64_t T, int64_t d);
 FwdWs carve_fwd(void* ws, int64_t T, int64_t d);
 
+struct TopkWs {
+  void* hc;          // bf16 [Tpad, d]
+  float* part_m;     // [kSvMax, Tpad]
+  float* part_s;     // [kSvMax, Tpad]
+  float* part_a;     // [kSvMax, Tpad] entropy numerators
+  float* part_tv;    // [kSvMax, Tpad, 16] per-segment top logits
+  int32_t* part_ti;  // [kSvMax, Tpad, 16] their vocabulary ids
+};
+size_t topk_ws_bytes(int64_t T, int64_t d);
+TopkWs carve_topk(void* ws, int64_t T, int64_t d);
+
 struct BwdWs {
   void* hc;       // bf16 [Tpad, d]
   void* g;        // bf16 [Tc, Vpad]
@@ -89,6 +100,11 @@ olive_status launch_logprob_fwd(const Ctx& c, const void* hidden, const void* W,
                                 int32_t T, int32_t d, int32_t V, float inv_tau, int reduction,
                                 float* logp, float* lse, float* loss, void* ws,
                                 int32_t* dev_status);
+
+olive_status launch_topk_fwd(const Ctx& c, const void* hidden, const void* W, const int32_t* rows,
+                             const int32_t* n_rows, int32_t T, int32_t d, int32_t V, float inv_tau,
+                             int32_t K, float* lse, float* entropy, float* topk_logp,
+                             int32_t* topk_ids, void* ws, int32_t* dev_status);
 
 olive_status launch_loss_bwd(const Ctx& c, const void* hidden, const void* W,
                              const int32_t* targets, const int32_t* rows, const int32_t* n_rows,

@@ -37,6 +37,7 @@ struct KlFwdKern {
   static constexpr bool kBMn = false;
   static constexpr bool kDual = true;
   static constexpr int kStages = 6;
+  static constexpr int kEpiSmem = 0;
 
   struct Params {
     int32_t* dev_status;
@@ -80,6 +81,7 @@ struct KlFwdKern {
   struct Epi {
     int r, sg;
     float mp, sp, mq, sq, A;
+    __device__ void init(uint8_t*) {}
     __device__ void begin(const Params& p, const Sched& s, int u, int row) {
       int i;
       unit_pos(p, s, u, i, sg);

@@ -121,6 +121,26 @@ size_t fwd_ws_bytes(int64_t T, int64_t d) {
 }
 FwdWs carve_fwd(void* ws, int64_t T, int64_t d) { return carve_fwd_impl(ws, T, d, nullptr); }
 
+static TopkWs carve_topk_impl(void* ws, int64_t T, int64_t d, size_t* total) {
+  const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
+  Carver c{static_cast<char*>(ws)};
+  TopkWs w;
+  w.hc = c.take(2ull * Tpad * d);
+  w.part_m = static_cast<float*>(c.take(4ull * kSvMax * Tpad));
+  w.part_s = static_cast<float*>(c.take(4ull * kSvMax * Tpad));
+  w.part_a = static_cast<float*>(c.take(4ull * kSvMax * Tpad));
+  w.part_tv = static_cast<float*>(c.take(4ull * 16 * kSvMax * Tpad));
+  w.part_ti = static_cast<int32_t*>(c.take(4ull * 16 * kSvMax * Tpad));
+  if (total) *total = c.off;
+  return w;
+}
+size_t topk_ws_bytes(int64_t T, int64_t d) {
+  size_t n = 0;
+  carve_topk_impl(nullptr, T, d, &n);
+  return n;
+}
+TopkWs carve_topk(void* ws, int64_t T, int64_t d) { return carve_topk_impl(ws, T, d, nullptr); }
+
 static BwdWs carve_bwd_impl(void* ws, int64_t T, int64_t d, int64_t V, int grad_dtype,
                             size_t* total) {
   const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
@@ -217,6 +237,7 @@ size_t olive_workspace_size(int op, int32_t T, int32_t d, int32_t d_t, int32_t V
     case OLIVE_OP_DIVERGENCE:
       if (!width_ok(d_t)) return 0;
       return kl_ws_bytes(T, d, d_t, V, grad);
+    case OLIVE_OP_TOPK_FWD: return topk_ws_bytes(T, d);
     default: return 0;
   }
 }
@@ -255,6 +276,26 @@ olive_status olive_token_logprob_fwd(const void* hidden, const void* W, const in
   if (st != OLIVE_OK) return st;
   return launch_logprob_fwd(c, hidden, W, targets, rows, n_rows, T, d, V, inv_tau, reduction, logp,
                             lse, loss, workspace, dev_status);
+}
+
+olive_status olive_token_topk_fwd(const void* hidden, const void* W, const int32_t* rows,
+                                  const int32_t* n_rows, int32_t T, int32_t d, int32_t V,
+                                  float inv_tau, int32_t K, float* lse, float* entropy,
+                                  float* topk_logp, int32_t* topk_ids, void* workspace,
+                                  size_t ws_bytes, int32_t* dev_status, void* stream) {
+  if (!hidden || !W || !rows || !n_rows || !lse || !entropy || !topk_logp || !topk_ids ||
+      !dev_status)
+    return OLIVE_ERR_INVALID_ARG;
+  if (T < 1 || V < 1 || d < 1 || d > kMaxDim || K < 1 || K > 16 || K > V) return OLIVE_ERR_SHAPE;
+  if (!(inv_tau > 0.f) || !std::isfinite(inv_tau)) return OLIVE_ERR_INVALID_ARG;
+  if (d % 8 != 0 || !aligned16(hidden) || !aligned16(W)) return OLIVE_ERR_ALIGNMENT;
+  olive_status st = check_ws(workspace, ws_bytes, topk_ws_bytes(T, d));
+  if (st != OLIVE_OK) return st;
+  Ctx c;
+  st = make_ctx(stream, &c);
+  if (st != OLIVE_OK) return st;
+  return launch_topk_fwd(c, hidden, W, rows, n_rows, T, d, V, inv_tau, K, lse, entropy, topk_logp,
+                         topk_ids, workspace, dev_status);
 }
 
 olive_status olive_token_loss_bwd(const void* hidden, const void* W, const int32_t* targets,

@@ -318,3 +318,42 @@ def test_bf16_widening_exact():
     x = torch.randn(1000, generator=torch.Generator().manual_seed(0)).to(torch.bfloat16)
     bits = x.view(torch.int16).numpy().view(np.uint16)
     assert np.array_equal(oracle.bf16_bits_to_f64(bits), x.double().numpy())
+
+
+# --------------------------------------------------------------------------
+# entropy and top-K
+# --------------------------------------------------------------------------
+def test_topk_matches_torch_and_entropy_matches_scipy():
+    import scipy.stats
+    h, W, targets, rows = _case(17, T=15, d=10, V=90)
+    lse, H, tv, ti = oracle.token_topk(h, W, rows, 16, inv_tau=0.9)
+    z = torch.from_numpy(0.9 * h @ W.T)
+    lp = torch.log_softmax(z, dim=1)
+    ref_v, ref_i = torch.topk(lp, 16, dim=1)
+    assert np.allclose(tv[rows], ref_v.numpy()[rows], atol=1e-12)
+    assert np.array_equal(ti[rows], ref_i.numpy()[rows])
+    p = np.exp(lp.numpy())
+    assert np.allclose(H[rows], scipy.stats.entropy(p[rows], axis=1), atol=1e-12)
+    off = np.setdiff1d(np.arange(len(h)), rows)
+    assert np.all(ti[off] == -1) and not tv[off].any() and not H[off].any()
+
+
+def test_topk_closed_forms():
+    V, d = 100, 4
+    h = np.random.default_rng(0).standard_normal((3, d))
+    lse, H, tv, ti = oracle.token_topk(h, np.zeros((V, d)), [0, 1, 2], 5)
+    # uniform: H = ln V, every log-prob = -ln V, ties ordered by ascending id
+    assert np.allclose(H, math.log(V), atol=1e-12)
+    assert np.allclose(tv, -math.log(V), atol=1e-12)
+    assert np.array_equal(ti, np.tile(np.arange(5), (3, 1)))
+    # a dominant entry: entropy -> 0, top-1 is that id with log-prob -> 0
+    W = np.zeros((V, d))
+    W[37, 0] = 40.0
+    h1 = np.zeros((1, d))
+    h1[0, 0] = 1.0
+    _, H1, tv1, ti1 = oracle.token_topk(h1, W, [0], 3)
+    a = (V - 1) * math.exp(-40.0)
+    # H = ln Z - 40 e^40 / Z with Z = e^40 + V - 1, i.e. a + 40 a / (1 + a)
+    assert ti1[0, 0] == 37 and abs(tv1[0, 0]) < 1e-15
+    assert H1[0] == pytest.approx(a + 40 * a / (1 + a), rel=1e-3)
+    assert np.array_equal(ti1[0, 1:], [0, 1])

@@ -1,0 +1,112 @@
+"""olive_token_topk_fwd (CUDA): per-token entropy and the K largest log-probs
+against the oracle.
+
+Values are compared within the log-prob tolerance.  The order of two
+log-probs closer than the tolerance is not unique (fp32 GPU logits against
+fp64 oracle ones), so ids are checked for validity: every returned id must
+carry, in the oracle, a log-prob within tolerance of the returned value and
+no smaller than the oracle's K-th largest minus the tolerance; where the
+oracle's neighbours are separated by more than the tolerance the id must be
+the oracle's exactly.
+"""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_36246_gb300 import binding as B
+from paper_2609_36246_gb300 import synth
+from tests.parity import LOGP_ATOL, LOGP_RTOL, assert_close_logp, sample_rows, to_f32, to_f64
+
+pytestmark = pytest.mark.gpu
+
+
+def _gpu(h, W, rows, K, inv_tau=1.0):
+    r = torch.from_numpy(np.asarray(rows, dtype=np.int32)).cuda()
+    n = torch.tensor([len(rows)], dtype=torch.int32, device="cuda")
+    st = B.new_status()
+    out = B.olive_token_topk_fwd(h.cuda(), W.cuda(), r, n, K, inv_tau, dev_status=st)
+    torch.cuda.synchronize()
+    assert B.status_bits(st) == []
+    return [t.cpu().numpy() for t in out]
+
+
+def _check_rows(rows, K, gpu, ref_lse, ref_H, ref_lp_full):
+    lse, H, tv, ti = gpu
+    assert_close_logp(lse[rows], ref_lse, "lse")
+    assert_close_logp(H[rows], ref_H, "entropy")
+    for k, t in enumerate(rows):
+        lp = ref_lp_full[k]
+        order = np.lexsort((np.arange(len(lp)), -lp))[:K + 1]
+        tol = LOGP_ATOL + LOGP_RTOL * np.abs(lp[order[:K]])
+        assert_close_logp(tv[t], lp[order[:K]], f"top-K values row {t}")
+        assert np.all(np.diff(tv[t]) <= 1e-6), "values must be descending"
+        assert len(set(ti[t].tolist())) == K
+        kth = lp[order[K - 1]]
+        for j in range(K):
+            g = int(ti[t, j])
+            assert 0 <= g < len(lp)
+            assert abs(lp[g] - tv[t, j]) <= tol[j] + 1e-6, (t, j, g)
+            assert lp[g] >= kth - tol[-1]
+            gap_lo = lp[order[j]] - lp[order[j + 1]]
+            gap_hi = lp[order[j - 1]] - lp[order[j]] if j > 0 else np.inf
+            if min(gap_lo, gap_hi) > 4 * tol[j]:
+                assert g == order[j], (t, j, g, order[j])
+
+
+def _oracle_full(h, W, rows, inv_tau):
+    lp, lse = oracle.log_softmax_rows(oracle.logits(to_f64(h)[rows], to_f64(W), inv_tau))
+    H = -(np.exp(lp) * lp).sum(axis=1)
+    return lse, H, lp
+
+
+@pytest.mark.parametrize("T,V,d,K,inv_tau", [
+    (300, 4097, 64, 16, 1.0),
+    (200, 300, 72, 5, 0.7),
+    (130, 1000, 128, 1, 1.0),
+    (260, 20000, 256, 16, 1.2),
+])
+def test_small_shapes(T, V, d, K, inv_tau):
+    rng = np.random.default_rng(T + V)
+    h = synth.normal_bf16(rng, (T, d), 1.0)
+    W = synth.normal_bf16(rng, (V, d), 0.3)
+    rows = np.sort(rng.choice(T, size=T * 3 // 4, replace=False))
+    gpu = _gpu(h, W, rows, K, inv_tau)
+    lse, H, lp = _oracle_full(h, W, rows, inv_tau)
+    _check_rows(rows, K, gpu, lse, H, lp)
+    # the oracle's own top-K agrees on the sampled statistics
+    rl, rH, rv, ri = oracle.token_topk(to_f64(h), to_f64(W), rows[:3], K, inv_tau)
+    assert np.allclose(rl[rows[:3]], lse[:3]) and np.allclose(rH[rows[:3]], H[:3])
+    off = np.setdiff1d(np.arange(T), rows)
+    assert not gpu[0][off].any() and not gpu[1][off].any()
+    assert not gpu[2][off].any() and np.all(gpu[3][off] == -1)
+
+
+def test_uniform_logits_ties_take_smallest_ids():
+    T, V, d, K = 140, 3000, 64, 16
+    h = synth.normal_bf16(np.random.default_rng(1), (T, d), 1.0)
+    W = torch.zeros(V, d, dtype=torch.bfloat16)
+    lse, H, tv, ti = _gpu(h, W, np.arange(T), K)
+    assert np.allclose(lse, math.log(V), atol=1e-5) and np.allclose(H, math.log(V), atol=1e-4)
+    assert np.allclose(tv, -math.log(V), atol=1e-5)
+    assert np.array_equal(ti, np.tile(np.arange(K), (T, 1)))
+
+
+@pytest.mark.slow
+def test_scoring_workload_sampled_rows():
+    """2 x (4096 + 4096) tokens, d = 2048, V = 151936, K = 16: sampled rows."""
+    b = synth.make_batch("scoring")
+    h = synth.make_hidden("scoring", b.T)
+    W = synth.make_weight("scoring")
+    o = oracle.splice_pack(b.prefix_ids, b.prefix_off, b.cont_ids, b.cont_off, b.V)
+    gpu = _gpu(h, W, o["rows"], 16)
+    pick = sample_rows(o["rows"], 16, seed=6)
+    lp, lse = oracle.log_softmax_rows(oracle.logits(to_f32(h[torch.from_numpy(pick)]).astype(np.float64), to_f32(W), 1.0))
+    H = -(np.exp(lp) * lp).sum(axis=1)
+    _check_rows(pick, 16, gpu, lse, H, lp)
+    # entropy at this scale sits near ln V - sigma^2 / 2 (sanity band)
+    ent = gpu[1][o["rows"]]
+    assert abs(ent.mean() - (math.log(151936) - 0.02 ** 2 * 2048 / 2)) < 0.1
