@@ -59,8 +59,10 @@ struct CoreLayout {
   static constexpr int SMEM_BYTES =
       1024 /*alignment slack*/ + RING_BYTES + BAR_BYTES + MISC_BYTES + EPI_BYTES;
   static constexpr int ACC_COLS = Kern::kDual ? 2 * Kern::kBN : Kern::kBN;
-  static constexpr uint32_t TMEM_COLS = 2 * ACC_COLS;
-  static_assert(TMEM_COLS <= 512, "two accumulators must fit in TMEM");
+  static constexpr int ACC_BUFS = Kern::kAccBufs;  // 2: epilogue overlaps the next tile's MMAs
+  static constexpr uint32_t TMEM_COLS = ACC_BUFS * ACC_COLS;
+  static_assert(ACC_BUFS == 1 || ACC_BUFS == 2, "one or two accumulators");
+  static_assert(TMEM_COLS <= 512, "the accumulators must fit in TMEM");
   static_assert(SMEM_BYTES <= 227 * 1024, "shared memory budget");
 };
 
@@ -211,7 +213,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if (!ok) break;
           umma_commit(tfull_bar(buf));
-          if (++buf == 2) { buf = 0; aphase ^= 1u; }
+          if (++buf == L::ACC_BUFS) { buf = 0; aphase ^= 1u; }
         }
       }
       // arrives once every MMA issued above has completed (bounded wait that
@@ -243,7 +245,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         epi.tile(p, sched, u, t, tc, lane_addr + static_cast<uint32_t>(buf * L::ACC_COLS));
         tc_fence_before();
         mbar_arrive(tempty_bar(buf));
-        if (++buf == 2) { buf = 0; aphase ^= 1u; }
+        if (++buf == L::ACC_BUFS) { buf = 0; aphase ^= 1u; }
       }
       if (!ok) break;
       epi.end(p, sched, u);

@@ -16,7 +16,7 @@
 // per slab the work is a list of tiles of three kinds, all 128 x 256 fp32
 // accumulators in TMEM:
 //   GRAD    z = hc . W^T (K = d; KL: two products, student and teacher, into
-//           two 128-column halves) -> G tile (bf16) in the slab
+//           the two 256-column halves of TMEM) -> G tile (bf16) in the slab
 //   DH      G . W  (A = G K-major, B = W MN-major, K = V) -> d_hidden rows
 //   DW      G^T . hc (A = G MN-major, B = hc MN-major, K = slab rows) -> dW
 //           (CE only; stored directly in the output dtype when there is one
@@ -49,8 +49,8 @@ enum Kind : int { K_NONE = -1, K_GRAD = 0, K_KLGRAD = 1, K_DH = 2, K_DW = 3 };
 
 // CE maps: 0 hc K-major 64x128, 1 W K-major 64x256, 2 G K-major 64x128,
 //          3 W MN-major 64x64, 4 G MN-major 64x64, 5 hc MN-major 64x64
-// KL maps: 0 hs K-major 64x128, 1 W_s K-major 64x128, 2 G K-major 64x128,
-//          3 W_s MN-major 64x64, 4 ht K-major 64x128, 5 W_t K-major 64x128
+// KL maps: 0 hs K-major 64x128, 1 W_s K-major 64x256, 2 G K-major 64x128,
+//          3 W_s MN-major 64x64, 4 ht K-major 64x128, 5 W_t K-major 64x256
 struct BwdMaps {
   CUtensorMap m[6];
 };
@@ -104,7 +104,7 @@ __device__ Plan make_plan(const BwdParams& p) {
   if (pl.n_slabs > p.max_slabs) pl.n_slabs = p.max_slabs;  // cannot happen for n <= T
   const int per = (pl.n + pl.n_slabs - 1) / pl.n_slabs;
   pl.rps = (per + 127) / 128 * 128;
-  pl.bn_grad = p.kl ? 128 : 256;
+  pl.bn_grad = 256;
   pl.vt = (p.V + pl.bn_grad - 1) / pl.bn_grad;
   pl.ntd = (p.d + kBN - 1) / kBN;
   pl.mtv = (p.V + kBM - 1) / kBM;
@@ -285,14 +285,14 @@ __device__ void epi_klgrad(const BwdParams& p, const Unit& x, int row, uint32_t 
     }
   }
   __nv_bfloat16* grow = p.g + static_cast<size_t>(r_local) * p.ldg;
-  const int n0 = x.j * 128;
+  const int n0 = x.j * kBN;
 #pragma unroll 1
-  for (int c = 0; c < 128; c += 32) {
+  for (int c = 0; c < kBN; c += 32) {
     const int col0 = n0 + c;
     if (col0 >= p.V) break;
     uint32_t a[32], b[32];
     tmem_ld_32x32b_x32(taddr + c, a);
-    tmem_ld_32x32b_x32(taddr + 128 + c, b);
+    tmem_ld_32x32b_x32(taddr + kBN + c, b);
     tmem_ld_wait();
     float g[32];
 #pragma unroll
@@ -442,6 +442,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const uint32_t tmem_base = *tmem_slot;
   const Plan pl = *plan_smem;
+  // cross-entropy: two 256-column accumulators (the epilogue of one tile
+  // overlaps the next tile's MMAs); divergence: one 512-column accumulator
+  // holding the student and teacher products of a 128 x 256 tile
+  const int nbufs = p.kl ? 1 : 2;
   const WaitCtl ctl{abort_flag, p.wait_limit_ns};
 
   const int total = total_units(p, pl);
@@ -469,13 +473,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         fence_proxy_async_global();
         int nk, nk2;
         unit_ksteps(p, x, nk, nk2);
-        const uint32_t bytes = x.kind == K_KLGRAD ? L::A_BYTES + 128 * kBK * 2 : L::STAGE_BYTES;
         for (int k = 0; k < nk + nk2; ++k) {
           if (!mbar_wait(empty_bar(stage), phase ^ 1u, ctl)) { ok = false; break; }
           const uint32_t sA = ring + stage * L::STAGE_BYTES;
           const uint32_t sB = sA + L::A_BYTES;
           const uint32_t fb = full_bar(stage);
-          mbar_arrive_expect_tx(fb, bytes);
+          mbar_arrive_expect_tx(fb, L::STAGE_BYTES);
           switch (x.kind) {
             case K_GRAD:
               tma_load_2d(sA, &maps.m[0], fb, k * kBK, x.row0 + x.i * kBM);
@@ -485,7 +488,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               const bool second = k >= nk;
               const int kk = (second ? k - nk : k) * kBK;
               tma_load_2d(sA, &maps.m[second ? 4 : 0], fb, kk, x.row0 + x.i * kBM);
-              tma_load_2d(sB, &maps.m[second ? 5 : 1], fb, kk, x.j * 128);
+              tma_load_2d(sB, &maps.m[second ? 5 : 1], fb, kk, x.j * kBN);
               break;
             }
             case K_DH:
@@ -523,7 +526,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t idesc;
         bool a_mn = false, b_mn = false;
         switch (x.kind) {
-          case K_KLGRAD: idesc = idesc_bf16(kBM, 128, false, false); break;
+          case K_KLGRAD: idesc = idesc_bf16(kBM, kBN, false, false); break;
           case K_DH: idesc = idesc_bf16(kBM, kBN, false, true); b_mn = true; break;
           case K_DW: idesc = idesc_bf16(kBM, kBN, true, true); a_mn = b_mn = true; break;
           default: idesc = idesc_bf16(kBM, kBN, false, false); break;
@@ -535,7 +538,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!mbar_wait(full_bar(stage), phase, ctl)) { ok = false; break; }
           tc_fence_after();
           const bool second = k >= nk;
-          const uint32_t dt = second ? acc + 128 : acc;
+          const uint32_t dt = second ? acc + kBN : acc;
           const int kl = second ? k - nk : k;
           const uint32_t sA = ring + stage * L::STAGE_BYTES;
           const uint32_t sB = sA + L::A_BYTES;
@@ -552,7 +555,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (!ok) break;
         umma_commit(tfull_bar(buf));
-        if (++buf == 2) { buf = 0; aphase ^= 1u; }
+        if (++buf == nbufs) { buf = 0; aphase ^= 1u; }
       }
       umma_commit(drain_bar);
       volatile int keep_waiting = 0;
@@ -590,7 +593,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       tc_fence_before();
       mbar_arrive(tempty_bar(buf));
-      if (++buf == 2) { buf = 0; aphase ^= 1u; }
+      if (++buf == nbufs) { buf = 0; aphase ^= 1u; }
       // publish: every epilogue thread's stores, then one release increment
       fence_proxy_async_global();
       __threadfence();
@@ -724,11 +727,11 @@ olive_status launch_kl_bwd(const Ctx& c, const void* hcs, const void* hct, const
   if (cudaMemsetAsync(counters, 0, 4 * nctr, c.stream) != cudaSuccess) return OLIVE_ERR_CUDA;
   BwdMaps maps;
   if (!encode_bf16_2d(&maps.m[0], hcs, d_s, Tpad, 2ull * d_s, 64, 128) ||
-      !encode_bf16_2d(&maps.m[1], W_s, d_s, V, 2ull * d_s, 64, 128) ||
+      !encode_bf16_2d(&maps.m[1], W_s, d_s, V, 2ull * d_s, 64, 256) ||
       !encode_bf16_2d(&maps.m[2], g, V, tc, 2ull * ldg, 64, 128) ||
       !encode_bf16_2d(&maps.m[3], W_s, d_s, V, 2ull * d_s, 64, 64) ||
       !encode_bf16_2d(&maps.m[4], hct, d_t, Tpad, 2ull * d_t, 64, 128) ||
-      !encode_bf16_2d(&maps.m[5], W_t, d_t, V, 2ull * d_t, 64, 128))
+      !encode_bf16_2d(&maps.m[5], W_t, d_t, V, 2ull * d_t, 64, 256))
     return OLIVE_ERR_CUDA;
   BwdParams p = base_params(c, rows, n_rows, T, V, inv_tau, dev_status);
   p.grad_kl = grad_kl;

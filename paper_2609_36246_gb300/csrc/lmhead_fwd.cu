@@ -53,6 +53,7 @@ struct FwdKernT {
   static constexpr bool kBMn = false;
   static constexpr bool kDual = false;
   static constexpr int kStages = 4;
+  static constexpr int kAccBufs = 2;
   // stats: per-thread candidate buffer of 32 (value, id) pairs, slot-major
   static constexpr int kEpiSmem = kStats ? 32 * kEpiThreads * 8 : 0;
 
