@@ -73,7 +73,7 @@ enum { OLIVE_REDUCE_SUM = 0, OLIVE_REDUCE_MEAN = 1 };
 enum { OLIVE_KL_REVERSE = 0, OLIVE_KL_FORWARD = 1 };
 enum { OLIVE_DTYPE_BF16 = 0, OLIVE_DTYPE_F32 = 1 };
 enum { OLIVE_OP_LOGPROB_FWD = 0, OLIVE_OP_LOSS_BWD = 1, OLIVE_OP_DIVERGENCE = 2,
-       OLIVE_OP_TOPK_FWD = 3 };
+       OLIVE_OP_TOPK_FWD = 3, OLIVE_OP_SPLICE_MASKED = 4 };
 
 /* ABI version of the loaded library (OLIVE_ABI_VERSION). */
 OLIVE_API int olive_abi_version(void);
@@ -86,6 +86,7 @@ OLIVE_API const char* olive_status_string(olive_status s);
  *   op  OLIVE_OP_LOGPROB_FWD / OLIVE_OP_LOSS_BWD: d = hidden width, d_t ignored.
  *   op  OLIVE_OP_DIVERGENCE: d = student width d_s, d_t = teacher width.
  *   op  OLIVE_OP_TOPK_FWD: d = hidden width, d_t ignored.
+ *   op  OLIVE_OP_SPLICE_MASKED: T = T_cap; d, d_t, V ignored.
  *   `grad` (bwd / divergence): non-zero when gradients are requested
  *   (OLIVE_OP_LOSS_BWD always computes them); `grad_dtype` is the dtype of
  *   d_W for OLIVE_OP_LOSS_BWD (bf16 output needs an fp32 accumulator).
@@ -130,6 +131,27 @@ OLIVE_API olive_status olive_splice_pack(const int32_t* prefix_ids, const int32_
                                int32_t* cu_seqlens, int32_t* cut_offsets,
                                int32_t* rows, int32_t* n_rows,
                                int32_t* dev_status, void* stream);
+
+/*
+ * olive_splice_pack_masked -- olive_splice_pack for multi-turn OLIVE
+ * (Section 3.2): the whole interaction (student turns, environment
+ * observations, teacher turns) is kept as context, and the loss applies only
+ * to the teacher's actions.  cont_loss (device, uint8, one flag per
+ * continuation id, same CSR as cont_ids) marks the continuation tokens that
+ * are teacher actions; row t is masked when targets[t] is such a token.
+ * Outputs and device errors as in olive_splice_pack, with
+ * n_rows = number of flagged continuation tokens and rows ascending.
+ * workspace: olive_workspace_size(OLIVE_OP_SPLICE_MASKED, T_cap, ...) bytes.
+ */
+OLIVE_API olive_status olive_splice_pack_masked(const int32_t* prefix_ids,
+                                                const int32_t* prefix_off, const int32_t* cont_ids,
+                                                const int32_t* cont_off, const uint8_t* cont_loss,
+                                                int32_t S, int32_t V, int32_t T_cap, int32_t* ids,
+                                                int32_t* targets, uint8_t* loss_mask,
+                                                int32_t* cu_seqlens, int32_t* cut_offsets,
+                                                int32_t* rows, int32_t* n_rows, void* workspace,
+                                                size_t ws_bytes, int32_t* dev_status,
+                                                void* stream);
 
 /*
  * olive_token_logprob_fwd -- Eq. (osd-ce): for every masked row r (t = rows[r],

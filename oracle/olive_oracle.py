@@ -75,7 +75,7 @@ def bf16_bits_to_f64(bits) -> np.ndarray:
 # --------------------------------------------------------------------------
 # Splice / pack  (Section 3.1, Eq. (osd-ce) and the masking sentence after it)
 # --------------------------------------------------------------------------
-def splice_pack(prefix_ids, prefix_off, cont_ids, cont_off, V: int) -> dict:
+def splice_pack(prefix_ids, prefix_off, cont_ids, cont_off, V: int, cont_loss=None) -> dict:
     """Pack S spliced sequences prefix_s || continuation_s back to back.
 
     prefix_s is x || y_{1:k} (prompt and student prefix), continuation_s is
@@ -91,6 +91,11 @@ def splice_pack(prefix_ids, prefix_off, cont_ids, cont_off, V: int) -> dict:
       cu_seqlens[S+1], cut_offsets[S] (packed index of y~_1),
       rows[N_mask]   the masked t in ascending order, n_rows = N_mask,
       token_range_ok whether every id lies in [0, V).
+    Multi-turn OLIVE (Section 3.2) keeps the whole interaction as context but
+    applies the loss only to the teacher's actions: ``cont_loss`` (optional,
+    one flag per continuation id) marks the continuation tokens that are
+    teacher actions; a row is then masked only when its target is such a
+    token (environment observations inside the continuation stay unmasked).
     Raises OracleError for offsets that do not describe S sequences with a
     non-empty prefix.
     """
@@ -105,6 +110,10 @@ def splice_pack(prefix_ids, prefix_off, cont_ids, cont_off, V: int) -> dict:
         raise OracleError("offsets must start at 0")
     if prefix_off[-1] != len(prefix_ids) or cont_off[-1] != len(cont_ids):
         raise OracleError("last offset must equal the number of ids")
+    if cont_loss is not None:
+        cont_loss = np.asarray(cont_loss).astype(bool)
+        if len(cont_loss) != len(cont_ids):
+            raise OracleError("cont_loss needs one flag per continuation id")
 
     ids, targets, mask, cu, cut = [], [], [], [0], []
     for s in range(S):
@@ -122,8 +131,12 @@ def splice_pack(prefix_ids, prefix_off, cont_ids, cont_off, V: int) -> dict:
             if i + 1 < L:
                 targets.append(seq[i + 1])
                 # the target of row i is seq[i+1]; it is a teacher token
-                # y~_j exactly when i+1 >= P.
-                mask.append(1 if i + 1 >= P else 0)
+                # y~_j exactly when i+1 >= P (and, with cont_loss, a
+                # teacher action rather than an observation)
+                in_loss = i + 1 >= P
+                if in_loss and cont_loss is not None:
+                    in_loss = bool(cont_loss[cont_off[s] + (i + 1 - P)])
+                mask.append(1 if in_loss else 0)
             else:
                 targets.append(-1)
                 mask.append(0)

@@ -27,7 +27,7 @@ STATUS_NAMES = {
 REDUCE = {"sum": 0, "mean": 1}
 DIRECTION = {"reverse": 0, "forward": 1}
 DTYPE = {torch.bfloat16: 0, torch.float32: 1}
-OP = {"logprob_fwd": 0, "loss_bwd": 1, "divergence": 2, "topk_fwd": 3}
+OP = {"logprob_fwd": 0, "loss_bwd": 1, "divergence": 2, "topk_fwd": 3, "splice_masked": 4}
 
 
 class OliveError(RuntimeError):
@@ -69,6 +69,9 @@ def lib() -> ctypes.CDLL:
     L.olive_token_divergence.restype = ctypes.c_int
     L.olive_token_divergence.argtypes = [_P, _P, _I, _P, _P, _I, _P, _P, _I, _I, _F, ctypes.c_int,
                                          _P, _P, _P, ctypes.c_int, _P, _S, _P, _P]
+    L.olive_splice_pack_masked.restype = ctypes.c_int
+    L.olive_splice_pack_masked.argtypes = [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P, _P,
+                                           _P, _P, _S, _P, _P]
     L.olive_token_topk_fwd.restype = ctypes.c_int
     L.olive_token_topk_fwd.argtypes = [_P, _P, _P, _P, _I, _I, _I, _F, _I, _P, _P, _P, _P, _P, _S,
                                        _P, _P]
@@ -131,14 +134,7 @@ def workspace(nbytes: int, device=None) -> torch.Tensor:
     return torch.empty(max(int(nbytes), 1), dtype=torch.uint8, device=device or "cuda")
 
 
-def olive_splice_pack(prefix_ids, prefix_off, cont_ids, cont_off, V: int, T_cap: int,
-                      dev_status=None) -> dict:
-    """Packs the spliced sequences; returns the device outputs of olive.h."""
-    for t, n in ((prefix_ids, "prefix_ids"), (prefix_off, "prefix_off"), (cont_ids, "cont_ids"),
-                 (cont_off, "cont_off")):
-        _need(t, torch.int32, n)
-    S = prefix_off.numel() - 1
-    dev = prefix_off.device
+def _pack_outputs(S: int, T_cap: int, dev, dev_status):
     out = {
         "ids": torch.empty(T_cap, dtype=torch.int32, device=dev),
         "targets": torch.empty(T_cap, dtype=torch.int32, device=dev),
@@ -149,6 +145,18 @@ def olive_splice_pack(prefix_ids, prefix_off, cont_ids, cont_off, V: int, T_cap:
         "n_rows": torch.empty(1, dtype=torch.int32, device=dev),
     }
     out["dev_status"] = dev_status if dev_status is not None else new_status(dev)
+    return out
+
+
+def olive_splice_pack(prefix_ids, prefix_off, cont_ids, cont_off, V: int, T_cap: int,
+                      dev_status=None) -> dict:
+    """Packs the spliced sequences; returns the device outputs of olive.h."""
+    for t, n in ((prefix_ids, "prefix_ids"), (prefix_off, "prefix_off"), (cont_ids, "cont_ids"),
+                 (cont_off, "cont_off")):
+        _need(t, torch.int32, n)
+    S = prefix_off.numel() - 1
+    dev = prefix_off.device
+    out = _pack_outputs(S, T_cap, dev, dev_status)
     # empty id arrays still need a valid device address
     pid = prefix_ids if prefix_ids.numel() else torch.zeros(1, dtype=torch.int32, device=dev)
     cid = cont_ids if cont_ids.numel() else torch.zeros(1, dtype=torch.int32, device=dev)
@@ -158,6 +166,31 @@ def olive_splice_pack(prefix_ids, prefix_off, cont_ids, cont_off, V: int, T_cap:
                                  _ptr(out["rows"]), _ptr(out["n_rows"]), _ptr(out["dev_status"]),
                                  _stream())
     _check(st, "olive_splice_pack")
+    return out
+
+
+def olive_splice_pack_masked(prefix_ids, prefix_off, cont_ids, cont_off, cont_loss, V: int,
+                             T_cap: int, dev_status=None) -> dict:
+    """Multi-turn packing: cont_loss (uint8, one flag per continuation id)
+    selects the teacher-action tokens that carry the loss."""
+    for t, n in ((prefix_ids, "prefix_ids"), (prefix_off, "prefix_off"), (cont_ids, "cont_ids"),
+                 (cont_off, "cont_off")):
+        _need(t, torch.int32, n)
+    _need(cont_loss, torch.uint8, "cont_loss")
+    S = prefix_off.numel() - 1
+    dev = prefix_off.device
+    out = _pack_outputs(S, T_cap, dev, dev_status)
+    pid = prefix_ids if prefix_ids.numel() else torch.zeros(1, dtype=torch.int32, device=dev)
+    cid = cont_ids if cont_ids.numel() else torch.zeros(1, dtype=torch.int32, device=dev)
+    cfl = cont_loss if cont_loss.numel() else torch.zeros(1, dtype=torch.uint8, device=dev)
+    ws = workspace(olive_workspace_size("splice_masked", T_cap, 8, 1), dev)
+    st = lib().olive_splice_pack_masked(_ptr(pid), _ptr(prefix_off), _ptr(cid), _ptr(cont_off),
+                                        _ptr(cfl), S, V, T_cap, _ptr(out["ids"]),
+                                        _ptr(out["targets"]), _ptr(out["loss_mask"]),
+                                        _ptr(out["cu_seqlens"]), _ptr(out["cut_offsets"]),
+                                        _ptr(out["rows"]), _ptr(out["n_rows"]), _ptr(ws), ws.numel(),
+                                        _ptr(out["dev_status"]), _stream())
+    _check(st, "olive_splice_pack_masked")
     return out
 
 

@@ -89,6 +89,17 @@ olive_status launch_splice_pack(const Ctx& c, const int32_t* prefix_ids, const i
                                 uint8_t* loss_mask, int32_t* cu_seqlens, int32_t* cut_offsets,
                                 int32_t* rows, int32_t* n_rows, int32_t* dev_status);
 
+// Multi-turn variant: the loss flag of every continuation token selects the
+// rows; ws holds one int per 2048 packed positions.
+size_t splice_masked_ws_bytes(int64_t T_cap);
+olive_status launch_splice_pack_masked(const Ctx& c, const int32_t* prefix_ids,
+                                       const int32_t* prefix_off, const int32_t* cont_ids,
+                                       const int32_t* cont_off, const uint8_t* cont_loss, int32_t S,
+                                       int32_t V, int32_t T_cap, int32_t* ids, int32_t* targets,
+                                       uint8_t* loss_mask, int32_t* cu_seqlens,
+                                       int32_t* cut_offsets, int32_t* rows, int32_t* n_rows,
+                                       void* ws, int32_t* dev_status);
+
 // Copies hidden[rows[r]] to hc[r] for r < n_rows and zero-fills the rest of
 // the last 128-row tile.
 olive_status launch_gather_rows(const Ctx& c, const void* hidden, const int32_t* rows,

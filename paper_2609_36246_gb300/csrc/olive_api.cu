@@ -228,6 +228,7 @@ const char* olive_status_string(olive_status s) {
 
 size_t olive_workspace_size(int op, int32_t T, int32_t d, int32_t d_t, int32_t V, int grad,
                             int grad_dtype) {
+  if (op == OLIVE_OP_SPLICE_MASKED) return T < 1 ? 0 : splice_masked_ws_bytes(T);
   if (T < 1 || V < 1 || !width_ok(d)) return 0;
   switch (op) {
     case OLIVE_OP_LOGPROB_FWD: return fwd_ws_bytes(T, d);
@@ -256,6 +257,27 @@ olive_status olive_splice_pack(const int32_t* prefix_ids, const int32_t* prefix_
   if (st != OLIVE_OK) return st;
   return launch_splice_pack(c, prefix_ids, prefix_off, cont_ids, cont_off, S, V, T_cap, ids,
                             targets, loss_mask, cu_seqlens, cut_offsets, rows, n_rows, dev_status);
+}
+
+olive_status olive_splice_pack_masked(const int32_t* prefix_ids, const int32_t* prefix_off,
+                                      const int32_t* cont_ids, const int32_t* cont_off,
+                                      const uint8_t* cont_loss, int32_t S, int32_t V, int32_t T_cap,
+                                      int32_t* ids, int32_t* targets, uint8_t* loss_mask,
+                                      int32_t* cu_seqlens, int32_t* cut_offsets, int32_t* rows,
+                                      int32_t* n_rows, void* workspace, size_t ws_bytes,
+                                      int32_t* dev_status, void* stream) {
+  if (!prefix_ids || !prefix_off || !cont_ids || !cont_off || !cont_loss || !ids || !targets ||
+      !loss_mask || !cu_seqlens || !cut_offsets || !rows || !n_rows || !dev_status)
+    return OLIVE_ERR_INVALID_ARG;
+  if (S < 1 || V < 1 || T_cap < 1) return OLIVE_ERR_SHAPE;
+  olive_status st = check_ws(workspace, ws_bytes, splice_masked_ws_bytes(T_cap));
+  if (st != OLIVE_OK) return st;
+  Ctx c;
+  st = make_ctx(stream, &c);
+  if (st != OLIVE_OK) return st;
+  return launch_splice_pack_masked(c, prefix_ids, prefix_off, cont_ids, cont_off, cont_loss, S, V,
+                                   T_cap, ids, targets, loss_mask, cu_seqlens, cut_offsets, rows,
+                                   n_rows, workspace, dev_status);
 }
 
 olive_status olive_token_logprob_fwd(const void* hidden, const void* W, const int32_t* targets,

@@ -24,10 +24,12 @@ import oracle.olive_oracle as real
 
 SRC = real.__file__
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "splice_pack_small.json")
+GOLDEN_TURNS = os.path.join(os.path.dirname(__file__), "golden", "splice_pack_turns.json")
 
 MUTANTS = {
-    "mask_includes_prefix_target": ("mask.append(1 if i + 1 >= P else 0)",
-                                    "mask.append(1 if i + 1 >= P - 1 else 0)"),
+    "mask_includes_prefix_target": ("in_loss = i + 1 >= P\n", "in_loss = i + 1 >= P - 1\n"),
+    "turn_flag_off_by_one": ("in_loss = bool(cont_loss[cont_off[s] + (i + 1 - P)])",
+                             "in_loss = bool(cont_loss[cont_off[s] + (i - P)])"),
     "target_not_shifted": ("targets.append(seq[i + 1])", "targets.append(seq[i])"),
     "cut_at_prefix_start": ("cut.append(cu[-1] + P)", "cut.append(cu[-1])"),
     "lse_drops_log_sum": ("lse = m + np.log(np.exp(z - m[:, None]).sum(axis=1))", "lse = m"),
@@ -75,6 +77,15 @@ def pin_golden_splice(O):
     with open(GOLDEN) as f:
         g = json.load(f)
     out = O.splice_pack(g["prefix_ids"], g["prefix_off"], g["cont_ids"], g["cont_off"], g["V"])
+    return all(list(map(int, np.atleast_1d(out[k]))) == (v if isinstance(v, list) else [v])
+               for k, v in g["expect"].items())
+
+
+def pin_turns_golden(O):
+    with open(GOLDEN_TURNS) as f:
+        g = json.load(f)
+    out = O.splice_pack(g["prefix_ids"], g["prefix_off"], g["cont_ids"], g["cont_off"], g["V"],
+                        cont_loss=g["cont_loss"])
     return all(list(map(int, np.atleast_1d(out[k]))) == (v if isinstance(v, list) else [v])
                for k, v in g["expect"].items())
 
@@ -131,7 +142,7 @@ def pin_kl(O):
     return bool(ok)
 
 
-PINS = [pin_golden_splice, pin_uniform, pin_scipy, pin_torch_ce_and_autograd, pin_kl]
+PINS = [pin_golden_splice, pin_turns_golden, pin_uniform, pin_scipy, pin_torch_ce_and_autograd, pin_kl]
 
 
 def test_real_oracle_passes_every_pin():

@@ -72,6 +72,33 @@ def test_splice_pack_invariants(seed):
         assert o["targets"][o["cu_seqlens"][s + 1] - 1] == -1
 
 
+def test_splice_pack_turns_golden():
+    with open(os.path.join(GOLDEN, "splice_pack_turns.json")) as f:
+        g = json.load(f)
+    out = oracle.splice_pack(g["prefix_ids"], g["prefix_off"], g["cont_ids"], g["cont_off"], g["V"],
+                             cont_loss=g["cont_loss"])
+    for k, v in g["expect"].items():
+        got = out[k]
+        assert (list(map(int, got)) if isinstance(v, list) else int(got)) == v, k
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_splice_pack_turn_flags_invariants(seed):
+    rng = np.random.default_rng(50 + seed)
+    S = int(rng.integers(1, 7))
+    b = synth.batch_from_lengths(rng, rng.integers(1, 20, size=S), rng.integers(0, 20, size=S), 500)
+    flags = rng.integers(0, 2, size=len(b.cont_ids))
+    o = oracle.splice_pack(b.prefix_ids, b.prefix_off, b.cont_ids, b.cont_off, b.V, cont_loss=flags)
+    plain = oracle.splice_pack(b.prefix_ids, b.prefix_off, b.cont_ids, b.cont_off, b.V)
+    assert o["n_rows"] == int(flags.sum())
+    # the masked rows are a subset of the plain ones whose targets are flagged actions
+    assert set(o["rows"]).issubset(set(plain["rows"]))
+    assert np.array_equal(o["targets"][o["rows"]], b.cont_ids[flags.astype(bool)])
+    ones = oracle.splice_pack(b.prefix_ids, b.prefix_off, b.cont_ids, b.cont_off, b.V,
+                              cont_loss=np.ones(len(b.cont_ids)))
+    assert np.array_equal(ones["rows"], plain["rows"])
+
+
 def test_splice_pack_rejects_empty_prefix_and_flags_range():
     with pytest.raises(oracle.OracleError):
         oracle.splice_pack([], [0, 0], [1, 2], [0, 2], 10)
