@@ -200,6 +200,31 @@ OLIVE_API olive_status olive_token_topk_fwd(const void* hidden, const void* W,
                                             int32_t* dev_status, void* stream);
 
 /*
+ * olive_topk_compare -- student/teacher agreement on each masked row's top-K
+ * tokens, from two olive_token_topk_fwd outputs (student: s_ids, s_logp;
+ * teacher: t_ids, t_lse) and the teacher's LM head (h_t [T, d_t], W_t
+ * [V, d_t], bf16):
+ *   overlap[t] = |top_K(p_s) intersect top_K(p_t)| / K  (the top-K overlap
+ *                ratio tracked during OPD, Section 4.1)
+ *   kl_topk[t] = sum_{j<K} p_s(v_j) (log p_s(v_j) - log p_t(v_j)) over the
+ *                student's top-K ids v_j, with log p_t(v) = inv_tau
+ *                h_t[t] . W_t[v] - t_lse[t]: the reverse KL of Section 1
+ *                truncated to the student's K most probable tokens (the
+ *                paper's "top-16 KL approximation" is not printed in full;
+ *                this is the reading implemented, no renormalisation).
+ * 1 <= K <= 16; s_ids, t_ids int32 [T, K]; s_logp fp32 [T, K]; t_lse fp32
+ * [T]; overlap, kl_topk fp32 [T] (0 on rows not in `rows`).  An id outside
+ * [0, V) gives NaN and OLIVE_ERR_TOKEN_RANGE.
+ */
+OLIVE_API olive_status olive_topk_compare(const void* h_t, const void* W_t, int32_t d_t,
+                                          const int32_t* rows, const int32_t* n_rows, int32_t T,
+                                          int32_t V, float inv_tau, int32_t K,
+                                          const int32_t* s_ids, const float* s_logp,
+                                          const int32_t* t_ids, const float* t_lse,
+                                          float* overlap, float* kl_topk, int32_t* dev_status,
+                                          void* stream);
+
+/*
  * olive_token_loss_bwd -- gradients of the Eq. (osd-ce) loss through the LM
  * head (the sampled sequences are fixed, Section 3.1, so ids get none):
  *   G[r,v]    = g * inv_tau * (exp(z_v - lse[t]) - [v == y])

@@ -22,6 +22,8 @@ Section 1; temperature, Appendix A, Table opd-config):
                           Section 3.1, so no gradient flows through the ids).
 * ``token_topk``       -- per-token entropy and the student's K largest
                           log-probs (Appendix A: OPD reads the top-16).
+* ``token_topk_compare`` -- student/teacher top-K overlap and the top-K
+                          truncation of the reverse KL.
 * ``token_divergence`` -- OPD's per-token reverse KL between student and
                           teacher over the full vocabulary (Section 1), the
                           forward direction as an option, and the gradient of
@@ -344,6 +346,44 @@ def token_topk(hidden, W, rows, K: int, inv_tau: float = 1.0):
             tv[r] = lp[k, order]
             ti[r] = order
     return lse, H, tv, ti
+
+
+def token_topk_compare(h_s, W_s, h_t, W_t, rows, K: int, inv_tau: float = 1.0):
+    """Top-K agreement between student and teacher per masked row.
+
+    overlap[t]  = |top_K(p_s) intersect top_K(p_t)| / K   (the student/teacher
+                  top-K overlap ratio tracked during OPD, Section 4.1)
+    kl_topk[t]  = sum over the student's K most probable tokens v of
+                  p_s(v) (log p_s(v) - log p_t(v)), both log-probs over the
+                  full vocabulary: the reverse KL of Section 1 truncated to
+                  the top-K terms (the paper's "top-16 KL approximation",
+                  whose exact form it does not print; this is the reading
+                  used here).
+    Also returns the gaps between the K-th and (K+1)-th largest log-probs of
+    the student and of the teacher (0 / inf off ``rows``), which tell a test
+    where top-K membership is decided by more than rounding.
+    """
+    T = np.asarray(h_s).shape[0]
+    rows = np.asarray(rows, dtype=np.int64)
+    overlap = np.zeros(T)
+    kl = np.zeros(T)
+    gap_s = np.full(T, np.inf)
+    gap_t = np.full(T, np.inf)
+    for r0 in range(0, len(rows), _ROW_CHUNK):
+        rr = rows[r0:r0 + _ROW_CHUNK]
+        lps, _ = log_softmax_rows(logits(_as_f64_rows(h_s, rr), W_s, inv_tau))
+        lpt, _ = log_softmax_rows(logits(_as_f64_rows(h_t, rr), W_t, inv_tau))
+        ids = np.arange(lps.shape[1])
+        for k, r in enumerate(rr):
+            os_ = np.lexsort((ids, -lps[k]))
+            ot_ = np.lexsort((ids, -lpt[k]))
+            S, Tk = os_[:K], ot_[:K]
+            overlap[r] = len(set(S.tolist()) & set(Tk.tolist())) / K
+            kl[r] = float((np.exp(lps[k, S]) * (lps[k, S] - lpt[k, S])).sum())
+            if len(ids) > K:
+                gap_s[r] = lps[k, os_[K - 1]] - lps[k, os_[K]]
+                gap_t[r] = lpt[k, ot_[K - 1]] - lpt[k, ot_[K]]
+    return overlap, kl, gap_s, gap_t
 
 
 # --------------------------------------------------------------------------

@@ -72,6 +72,9 @@ def lib() -> ctypes.CDLL:
     L.olive_splice_pack_masked.restype = ctypes.c_int
     L.olive_splice_pack_masked.argtypes = [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P, _P,
                                            _P, _P, _S, _P, _P]
+    L.olive_topk_compare.restype = ctypes.c_int
+    L.olive_topk_compare.argtypes = [_P, _P, _I, _P, _P, _I, _I, _F, _I, _P, _P, _P, _P, _P, _P, _P,
+                                     _P]
     L.olive_token_topk_fwd.restype = ctypes.c_int
     L.olive_token_topk_fwd.argtypes = [_P, _P, _P, _P, _I, _I, _I, _F, _I, _P, _P, _P, _P, _P, _S,
                                        _P, _P]
@@ -248,6 +251,31 @@ def olive_token_topk_fwd(hidden, W, rows, n_rows, K: int = 16, inv_tau: float = 
                                     _ptr(ws), ws.numel(), _ptr(ds), _stream())
     _check(st, "olive_token_topk_fwd")
     return lse, ent, tv, ti
+
+
+def olive_topk_compare(h_t, W_t, rows, n_rows, s_ids, s_logp, t_ids, t_lse, inv_tau: float = 1.0,
+                       dev_status=None):
+    """Top-K overlap ratio and top-K truncated reverse KL per masked row.
+
+    Returns (overlap [T], kl_topk [T])."""
+    _need(h_t, torch.bfloat16, "h_t")
+    _need(W_t, torch.bfloat16, "W_t")
+    _need(s_ids, torch.int32, "s_ids")
+    _need(t_ids, torch.int32, "t_ids")
+    _need(s_logp, torch.float32, "s_logp")
+    _need(t_lse, torch.float32, "t_lse")
+    T, d_t = h_t.shape
+    V = W_t.shape[0]
+    K = s_ids.shape[1]
+    dev = h_t.device
+    ov = torch.empty(T, dtype=torch.float32, device=dev)
+    kl = torch.empty(T, dtype=torch.float32, device=dev)
+    ds = dev_status if dev_status is not None else new_status(dev)
+    st = lib().olive_topk_compare(_ptr(h_t), _ptr(W_t), d_t, _ptr(rows), _ptr(n_rows), T, V,
+                                  float(inv_tau), K, _ptr(s_ids), _ptr(s_logp), _ptr(t_ids),
+                                  _ptr(t_lse), _ptr(ov), _ptr(kl), _ptr(ds), _stream())
+    _check(st, "olive_topk_compare")
+    return ov, kl
 
 
 def olive_token_loss_bwd(hidden, W, targets, rows, n_rows, lse, grad_loss, inv_tau: float = 1.0,

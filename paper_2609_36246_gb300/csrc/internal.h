@@ -117,6 +117,12 @@ olive_status launch_topk_fwd(const Ctx& c, const void* hidden, const void* W, co
                              int32_t K, float* lse, float* entropy, float* topk_logp,
                              int32_t* topk_ids, void* ws, int32_t* dev_status);
 
+olive_status launch_topk_compare(const Ctx& c, const void* h_t, const void* W_t, int32_t d_t,
+                                 const int32_t* rows, const int32_t* n_rows, int32_t T, int32_t V,
+                                 float inv_tau, int32_t K, const int32_t* s_ids,
+                                 const float* s_logp, const int32_t* t_ids, const float* t_lse,
+                                 float* overlap, float* kl_topk, int32_t* dev_status);
+
 olive_status launch_loss_bwd(const Ctx& c, const void* hidden, const void* W,
                              const int32_t* targets, const int32_t* rows, const int32_t* n_rows,
                              int32_t T, int32_t d, int32_t V, float inv_tau, int reduction,

@@ -320,6 +320,25 @@ olive_status olive_token_topk_fwd(const void* hidden, const void* W, const int32
                          topk_ids, workspace, dev_status);
 }
 
+olive_status olive_topk_compare(const void* h_t, const void* W_t, int32_t d_t,
+                                const int32_t* rows, const int32_t* n_rows, int32_t T, int32_t V,
+                                float inv_tau, int32_t K, const int32_t* s_ids,
+                                const float* s_logp, const int32_t* t_ids, const float* t_lse,
+                                float* overlap, float* kl_topk, int32_t* dev_status,
+                                void* stream) {
+  if (!h_t || !W_t || !rows || !n_rows || !s_ids || !s_logp || !t_ids || !t_lse || !overlap ||
+      !kl_topk || !dev_status)
+    return OLIVE_ERR_INVALID_ARG;
+  if (T < 1 || V < 1 || d_t < 1 || d_t > kMaxDim || K < 1 || K > 16 || K > V) return OLIVE_ERR_SHAPE;
+  if (!(inv_tau > 0.f) || !std::isfinite(inv_tau)) return OLIVE_ERR_INVALID_ARG;
+  if (d_t % 8 != 0 || !aligned16(h_t) || !aligned16(W_t)) return OLIVE_ERR_ALIGNMENT;
+  Ctx c;
+  olive_status st = make_ctx(stream, &c);
+  if (st != OLIVE_OK) return st;
+  return launch_topk_compare(c, h_t, W_t, d_t, rows, n_rows, T, V, inv_tau, K, s_ids, s_logp,
+                             t_ids, t_lse, overlap, kl_topk, dev_status);
+}
+
 olive_status olive_token_loss_bwd(const void* hidden, const void* W, const int32_t* targets,
                                   const int32_t* rows, const int32_t* n_rows, int32_t T, int32_t d,
                                   int32_t V, float inv_tau, int reduction, const float* lse,

@@ -10,6 +10,8 @@
 // when rt is small compared with the SM count.
 #pragma once
 
+#include <cuda_bf16.h>
+
 #include "internal.h"
 
 namespace olive {

@@ -1,0 +1,98 @@
+// topk_compare.cu -- student/teacher agreement on the top-K tokens of each
+// masked row, from the top-K lists of olive_token_topk_fwd:
+//   overlap[t] = |top_K(student) intersect top_K(teacher)| / K  (the top-K
+//                overlap ratio the paper tracks during OPD, Section 4.1)
+//   kl_topk[t] = sum over the student's K most probable tokens v of
+//                p_s(v) (log p_s(v) - log p_t(v)), log-probs over the full
+//                vocabulary: the reverse KL of Section 1 truncated to its
+//                top-K terms (the paper's "top-16 KL approximation"; its exact
+//                form is not printed, this is the reading implemented)
+// One warp per masked row; the teacher's log-probs at the student's K ids
+// need K dot products h_t[t] . W_t[v] (d_t each), which the warp computes with
+// 16-byte loads split across lanes and a shuffle reduction.
+#include <cmath>
+
+#include "sched.cuh"
+
+namespace olive {
+namespace {
+
+__device__ __forceinline__ float dot_bf16x8(uint4 a, uint4 b) {
+  const __nv_bfloat162* pa = reinterpret_cast<const __nv_bfloat162*>(&a);
+  const __nv_bfloat162* pb = reinterpret_cast<const __nv_bfloat162*>(&b);
+  float s = 0.f;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const float2 x = __bfloat1622float2(pa[q]);
+    const float2 y = __bfloat1622float2(pb[q]);
+    s = fmaf(x.x, y.x, s);
+    s = fmaf(x.y, y.y, s);
+  }
+  return s;
+}
+
+__global__ void topk_compare_kernel(const uint4* __restrict__ h_t, const uint4* __restrict__ W_t,
+                                    int d8, const int32_t* __restrict__ rows,
+                                    const int32_t* __restrict__ n_rows, int T, int V, float inv_tau,
+                                    int K, const int32_t* __restrict__ s_ids,
+                                    const float* __restrict__ s_logp,
+                                    const int32_t* __restrict__ t_ids,
+                                    const float* __restrict__ t_lse, float* __restrict__ overlap,
+                                    float* __restrict__ kl_topk, int32_t* dev_status) {
+  const int n = read_n_rows(n_rows, T, dev_status);
+  const int lane = threadIdx.x & 31;
+  const int warps = (gridDim.x * blockDim.x) >> 5;
+  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < n; r += warps) {
+    const int t = rows[r];
+    if (t < 0 || t >= T) continue;  // reported by the callers' gathers
+    const bool in_k = lane < K;
+    const int sid = in_k ? s_ids[static_cast<size_t>(t) * K + lane] : -1;
+    const float slp = in_k ? s_logp[static_cast<size_t>(t) * K + lane] : 0.f;
+    const int tid = in_k ? t_ids[static_cast<size_t>(t) * K + lane] : -2;
+    bool found = false;
+    for (int k = 0; k < K; ++k) found |= __shfl_sync(0xffffffffu, tid, k) == sid;
+    const int common = __popc(__ballot_sync(0xffffffffu, in_k && found));
+    const float lse_t = t_lse[t];
+    const uint4* hrow = h_t + static_cast<size_t>(t) * d8;
+    float kl = 0.f;
+    bool bad = false;
+    for (int j = 0; j < K; ++j) {
+      const int v = __shfl_sync(0xffffffffu, sid, j);
+      const float lps = __shfl_sync(0xffffffffu, slp, j);
+      if (v < 0 || v >= V) {
+        bad = true;
+        continue;
+      }
+      const uint4* wrow = W_t + static_cast<size_t>(v) * d8;
+      float part = 0.f;
+      for (int c = lane; c < d8; c += 32) part += dot_bf16x8(__ldg(hrow + c), __ldg(wrow + c));
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+      const float lpt = part * inv_tau - lse_t;
+      kl += expf(lps) * (lps - lpt);
+    }
+    if (lane == 0) {
+      overlap[t] = static_cast<float>(common) / static_cast<float>(K);
+      kl_topk[t] = bad ? NAN : kl;
+      if (bad) atomicOr(dev_status, 1 << OLIVE_ERR_TOKEN_RANGE);
+    }
+  }
+}
+
+}  // namespace
+
+olive_status launch_topk_compare(const Ctx& c, const void* h_t, const void* W_t, int32_t d_t,
+                                 const int32_t* rows, const int32_t* n_rows, int32_t T, int32_t V,
+                                 float inv_tau, int32_t K, const int32_t* s_ids,
+                                 const float* s_logp, const int32_t* t_ids, const float* t_lse,
+                                 float* overlap, float* kl_topk, int32_t* dev_status) {
+  if (cudaMemsetAsync(overlap, 0, sizeof(float) * T, c.stream) != cudaSuccess ||
+      cudaMemsetAsync(kl_topk, 0, sizeof(float) * T, c.stream) != cudaSuccess)
+    return OLIVE_ERR_CUDA;
+  topk_compare_kernel<<<c.num_sms * 8, 256, 0, c.stream>>>(
+      static_cast<const uint4*>(h_t), static_cast<const uint4*>(W_t), d_t / 8, rows, n_rows, T, V,
+      inv_tau, K, s_ids, s_logp, t_ids, t_lse, overlap, kl_topk, dev_status);
+  return cudaGetLastError() == cudaSuccess ? OLIVE_OK : OLIVE_ERR_CUDA;
+}
+
+}  // namespace olive

@@ -384,3 +384,29 @@ def test_topk_closed_forms():
     assert ti1[0, 0] == 37 and abs(tv1[0, 0]) < 1e-15
     assert H1[0] == pytest.approx(a + 40 * a / (1 + a), rel=1e-3)
     assert np.array_equal(ti1[0, 1:], [0, 1])
+
+
+def test_topk_compare_pins():
+    rng = np.random.default_rng(18)
+    T, d, V, K = 6, 9, 60, 8
+    hs, Ws = rng.standard_normal((T, d)), rng.standard_normal((V, d)) * 0.8
+    ht, Wt = rng.standard_normal((T, d + 3)), rng.standard_normal((V, d + 3)) * 0.8
+    rows = np.array([0, 2, 3, 5])
+    # identical models: full overlap, zero truncated KL
+    ov, kl, _, _ = oracle.token_topk_compare(hs, Ws, hs, Ws, rows, K)
+    assert np.all(ov[rows] == 1.0) and np.allclose(kl[rows], 0, atol=1e-14)
+    # K = V: the truncation is the full reverse KL, and the overlap is 1
+    ovV, klV, _, _ = oracle.token_topk_compare(hs, Ws, ht, Wt, rows, V)
+    full, _ = oracle.token_divergence(hs, Ws, ht, Wt, rows)
+    assert np.allclose(klV[rows], full[rows], rtol=1e-12, atol=1e-14) and np.all(ovV[rows] == 1.0)
+    # against torch.topk on independently formed log-probs
+    ov, kl, gs, gt = oracle.token_topk_compare(hs, Ws, ht, Wt, rows, K)
+    lps = torch.log_softmax(torch.from_numpy(hs @ Ws.T), 1)
+    lpt = torch.log_softmax(torch.from_numpy(ht @ Wt.T), 1)
+    for r in rows:
+        S = torch.topk(lps[r], K).indices
+        Tk = torch.topk(lpt[r], K).indices
+        assert ov[r] == len(set(S.tolist()) & set(Tk.tolist())) / K
+        ref = (lps[r, S].exp() * (lps[r, S] - lpt[r, S])).sum().item()
+        assert kl[r] == pytest.approx(ref, rel=1e-12, abs=1e-14)
+        assert gs[r] > 0 and gt[r] > 0
