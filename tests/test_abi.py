@@ -120,6 +120,39 @@ def test_bwd_and_divergence_validation(L):
     assert st == 1
 
 
+def test_new_entry_points_validation(L):
+    keep, p = _fake()
+    P = ctypes.c_void_p
+    # top-K: K outside [1, 16] or above V, misaligned width
+    for K, V, want in ((0, 100, 2), (17, 100, 2), (8, 4, 2)):
+        st = L.olive_token_topk_fwd(P(p), P(p), P(p), P(p), 64, 64, V, 1.0, K, P(p), P(p), P(p),
+                                    P(p), P(p), 1 << 20, P(p), None)
+        assert st == want, (K, V)
+    st = L.olive_token_topk_fwd(P(p), P(p), P(p), P(p), 64, 60, 100, 1.0, 4, P(p), P(p), P(p),
+                                P(p), P(p), 1 << 20, P(p), None)
+    assert st == 3
+    st = L.olive_token_topk_fwd(P(p), P(p), P(p), P(p), 64, 64, 100, 1.0, 4, None, P(p), P(p),
+                                P(p), P(p), 1 << 20, P(p), None)
+    assert st == 1
+    # top-K compare: null list, bad K
+    st = L.olive_topk_compare(P(p), P(p), 64, P(p), P(p), 64, 100, 1.0, 4, None, P(p), P(p), P(p),
+                              P(p), P(p), P(p), None)
+    assert st == 1
+    st = L.olive_topk_compare(P(p), P(p), 64, P(p), P(p), 64, 100, 1.0, 20, P(p), P(p), P(p), P(p),
+                              P(p), P(p), P(p), None)
+    assert st == 2
+    # multi-turn splice: null flags, workspace too small
+    st = L.olive_splice_pack_masked(P(p), P(p), P(p), P(p), None, 1, 10, 10, P(p), P(p), P(p), P(p),
+                                    P(p), P(p), P(p), P(p), 1 << 20, P(p), None)
+    assert st == 1
+    st = L.olive_splice_pack_masked(P(p), P(p), P(p), P(p), P(p), 1, 10, 100000, P(p), P(p), P(p),
+                                    P(p), P(p), P(p), P(p), P(p), 8, P(p), None)
+    assert st == 9
+    assert B.olive_workspace_size("splice_masked", 100000, 8, 1) >= 4 * 49
+    assert B.olive_workspace_size("topk_fwd", 4096, 4096, 151936) > B.olive_workspace_size(
+        "logprob_fwd", 4096, 4096, 151936)
+
+
 def test_binding_rejects_cpu_tensors(L):
     h = torch.zeros(8, 64, dtype=torch.bfloat16)
     with pytest.raises(TypeError):
