@@ -13,6 +13,7 @@ from .olive_oracle import (  # noqa: F401
     token_logprob,
     token_topk,
     token_topk_compare,
+    token_topk_kl_bwd,
     token_loss_bwd,
     token_loss_bwd_rows,
     token_loss_bwd_vocab,

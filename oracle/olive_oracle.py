@@ -24,6 +24,8 @@ Section 1; temperature, Appendix A, Table opd-config):
                           log-probs (Appendix A: OPD reads the top-16).
 * ``token_topk_compare`` -- student/teacher top-K overlap and the top-K
                           truncation of the reverse KL.
+* ``token_topk_kl_bwd`` -- gradients of the top-K truncated KL (top-K set
+                          held fixed).
 * ``token_divergence`` -- OPD's per-token reverse KL between student and
                           teacher over the full vocabulary (Section 1), the
                           forward direction as an option, and the gradient of
@@ -384,6 +386,43 @@ def token_topk_compare(h_s, W_s, h_t, W_t, rows, K: int, inv_tau: float = 1.0):
                 gap_s[r] = lps[k, os_[K - 1]] - lps[k, os_[K]]
                 gap_t[r] = lpt[k, ot_[K - 1]] - lpt[k, ot_[K]]
     return overlap, kl, gap_s, gap_t
+
+
+def token_topk_kl_bwd(h_s, W_s, h_t, W_t, rows, K: int, inv_tau: float = 1.0, grad=None):
+    """Gradient of sum_t g_t kl_topk[t] (see ``token_topk_compare``) with
+    respect to the student's hidden rows and LM head, the top-K set S_t of
+    the student held fixed (it is selected, not differentiated):
+      with l = log p_s, q = log p_t, P_S = sum_{v in S} p_s(v) and
+      KL_K = sum_{v in S} p_s(v) (l_v - q_v),
+      dz_u = p_s(u) ([u in S] (l_u - q_u + 1) - KL_K - P_S)
+      G[t, u] = g_t inv_tau dz_u,  dH_s[t] = G[t] W_s,  dW_s = G^T h_s.
+    Returns (dH_s [T, d_s], dW_s [V, d_s]).
+    """
+    h_s = np.asarray(h_s)
+    T = h_s.shape[0]
+    rows = np.asarray(rows, dtype=np.int64)
+    g = np.ones(T) if grad is None else np.asarray(grad, dtype=np.float64)
+    W64 = np.asarray(W_s).astype(np.float64)
+    dH = np.zeros((T, h_s.shape[1]))
+    dW = np.zeros_like(W64)
+    for r0 in range(0, len(rows), _ROW_CHUNK):
+        rr = rows[r0:r0 + _ROW_CHUNK]
+        hs = _as_f64_rows(h_s, rr)
+        lps, _ = log_softmax_rows(logits(hs, W_s, inv_tau))
+        lpt, _ = log_softmax_rows(logits(_as_f64_rows(h_t, rr), W_t, inv_tau))
+        ps = np.exp(lps)
+        ids = np.arange(lps.shape[1])
+        G = np.zeros_like(lps)
+        for k in range(len(rr)):
+            S = np.lexsort((ids, -lps[k]))[:K]
+            kl = float((ps[k, S] * (lps[k, S] - lpt[k, S])).sum())
+            P_S = float(ps[k, S].sum())
+            G[k] = -ps[k] * (kl + P_S)
+            G[k, S] += ps[k, S] * (lps[k, S] - lpt[k, S] + 1.0)
+        G *= (g[rr] * float(inv_tau))[:, None]
+        dH[rr] = G @ W64
+        dW += G.T @ hs
+    return dH, dW
 
 
 # --------------------------------------------------------------------------

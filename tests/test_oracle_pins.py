@@ -410,3 +410,28 @@ def test_topk_compare_pins():
         ref = (lps[r, S].exp() * (lps[r, S] - lpt[r, S])).sum().item()
         assert kl[r] == pytest.approx(ref, rel=1e-12, abs=1e-14)
         assert gs[r] > 0 and gt[r] > 0
+
+
+def test_topk_kl_bwd_matches_autograd_with_fixed_set():
+    rng = np.random.default_rng(19)
+    T, ds, dt, V, K = 5, 7, 9, 40, 6
+    hs, Ws = rng.standard_normal((T, ds)), rng.standard_normal((V, ds)) * 0.7
+    ht, Wt = rng.standard_normal((T, dt)), rng.standard_normal((V, dt)) * 0.7
+    rows = np.array([0, 1, 3, 4])
+    g = rng.uniform(0.5, 2.0, size=T)
+    dH, dW = oracle.token_topk_kl_bwd(hs, Ws, ht, Wt, rows, K, inv_tau=1.2, grad=g)
+    hs_t = torch.from_numpy(hs).requires_grad_(True)
+    Ws_t = torch.from_numpy(Ws).requires_grad_(True)
+    r = torch.from_numpy(rows)
+    lps = torch.log_softmax(1.2 * (hs_t[r] @ Ws_t.T), 1)
+    lpt = torch.log_softmax(1.2 * (torch.from_numpy(ht)[r] @ torch.from_numpy(Wt).T), 1)
+    S = torch.topk(lps.detach(), K, dim=1).indices          # the set is selected, not differentiated
+    ls, lt = lps.gather(1, S), lpt.gather(1, S)
+    kl = (ls.exp() * (ls - lt)).sum(1)
+    (kl * torch.from_numpy(g)[r]).sum().backward()
+    assert np.allclose(dH, hs_t.grad.numpy(), rtol=1e-10, atol=1e-13)
+    assert np.allclose(dW, Ws_t.grad.numpy(), rtol=1e-10, atol=1e-13)
+    # K = V: the gradient of the full reverse KL
+    dHV, _ = oracle.token_topk_kl_bwd(hs, Ws, ht, Wt, rows, V, inv_tau=1.2, grad=g)
+    _, full = oracle.token_divergence(hs, Ws, ht, Wt, rows, 1.2, "reverse", grad_kl=g)
+    assert np.allclose(dHV, full, rtol=1e-10, atol=1e-13)
