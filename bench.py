@@ -278,6 +278,8 @@ def run_ours(args, world, rank, local):
         torch.cuda.empty_cache()
         extra["kl_divergence"] = measure_kl(dev, burst)
         torch.cuda.empty_cache()
+        extra["topk_kl"] = measure_topk_kl(dev, burst)
+        torch.cuda.empty_cache()
         extra["scoring_fwd"], extra["topk_entropy"] = measure_scoring(dev, burst)
         torch.cuda.empty_cache()
         extra["varlen"] = measure_varlen(dev, burst)
@@ -377,6 +379,41 @@ def measure_kl(dev, burst: float, steps: int = 3):
         raise RuntimeError(f"divergence status {B.status_bits(st)}")
     flops = 2.0 * N * V * (ds + dt) + 2.0 * N * V * ds
     return {"workload": "per-token reverse KL + d/dh_s: 16384 rows, d_s=4096, d_t=5120, V=151936",
+            "value": N / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
+            "pct_bf16_peak": 100.0 * flops / (ms / 1e3) / 1e12 / burst, "steps": steps}
+
+
+def measure_topk_kl(dev, burst: float, steps: int = 3):
+    """OPD with the top-16 KL: student and teacher entropy/top-16 sweeps, the
+    top-16 compare (overlap, truncated KL, teacher log-probs at the student's
+    ids) and the gradient w.r.t. h_s and W_s (16384 rows, student d = 4096,
+    teacher d = 5120, V = 151936)."""
+    from paper_2609_36246_gb300 import binding as B
+    N, ds, dt, V, K = 16384, 4096, 5120, 151936, 16
+    hs, Ws = gpu_inputs(21, N, ds, V, dev)
+    ht, Wt = gpu_inputs(22, N, dt, V, dev)
+    rows = torch.arange(N, dtype=torch.int32, device=dev)
+    n = torch.tensor([N], dtype=torch.int32, device=dev)
+    gk = torch.ones(N, dtype=torch.float32, device=dev)
+    ws_k = B.workspace(B.olive_workspace_size("topk_fwd", N, dt, V), dev)
+    ws_b = B.workspace(B.olive_workspace_size("topk_kl_bwd", N, ds, V), dev)
+    out_b = (torch.empty(N, ds, dtype=torch.bfloat16, device=dev),
+             torch.empty(V, ds, dtype=torch.bfloat16, device=dev))
+    st = B.new_status(dev)
+
+    def step():
+        s_lse, _, s_lp, s_id = B.olive_token_topk_fwd(hs, Ws, rows, n, K, ws=ws_k, dev_status=st)
+        t_lse, _, _, t_id = B.olive_token_topk_fwd(ht, Wt, rows, n, K, ws=ws_k, dev_status=st)
+        _, kl, tlp = B.olive_topk_compare(ht, Wt, rows, n, s_id, s_lp, t_id, t_lse, dev_status=st,
+                                          want_t_logp=True)
+        B.olive_topk_kl_bwd(hs, Ws, rows, n, s_lse, s_id, s_lp, tlp, kl, gk, ws=ws_b,
+                            dev_status=st, out=out_b)
+
+    ms = time_calls(step, steps, 1)
+    if int(st.item()) != 0:
+        raise RuntimeError(f"top-K KL status {B.status_bits(st)}")
+    flops = 2.0 * N * V * (ds + dt) + 4.0 * N * V * ds
+    return {"workload": "top-16 KL + d/dh_s, d/dW_s: 16384 rows, d_s=4096, d_t=5120, V=151936",
             "value": N / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
             "pct_bf16_peak": 100.0 * flops / (ms / 1e3) / 1e12 / burst, "steps": steps}
 

@@ -16,6 +16,15 @@
  *   olive_token_loss_bwd     d loss / d hidden and d loss / d W
  *   olive_token_divergence   full-vocabulary per-token KL (+ d KL / d h_s)
  *
+ * and these extend it:
+ *
+ *   olive_splice_pack_masked multi-turn packing, loss only on teacher actions
+ *                            (Section 3.2)
+ *   olive_token_topk_fwd     per-token entropy and top-K log-probs
+ *   olive_topk_compare       student/teacher top-K overlap and top-K KL
+ *   olive_topk_kl_bwd        gradient of the top-K KL
+ *   olive_token_logprob_fwd_noalloc  the forward without a workspace
+ *
  * Conventions shared by every call
  *   - Every pointer argument is a DEVICE pointer unless stated otherwise.  The
  *     caller owns every buffer; the library allocates no device memory and
@@ -73,7 +82,7 @@ enum { OLIVE_REDUCE_SUM = 0, OLIVE_REDUCE_MEAN = 1 };
 enum { OLIVE_KL_REVERSE = 0, OLIVE_KL_FORWARD = 1 };
 enum { OLIVE_DTYPE_BF16 = 0, OLIVE_DTYPE_F32 = 1 };
 enum { OLIVE_OP_LOGPROB_FWD = 0, OLIVE_OP_LOSS_BWD = 1, OLIVE_OP_DIVERGENCE = 2,
-       OLIVE_OP_TOPK_FWD = 3, OLIVE_OP_SPLICE_MASKED = 4 };
+       OLIVE_OP_TOPK_FWD = 3, OLIVE_OP_SPLICE_MASKED = 4, OLIVE_OP_TOPK_KL_BWD = 5 };
 
 /* ABI version of the loaded library (OLIVE_ABI_VERSION). */
 OLIVE_API int olive_abi_version(void);
@@ -87,6 +96,8 @@ OLIVE_API const char* olive_status_string(olive_status s);
  *   op  OLIVE_OP_DIVERGENCE: d = student width d_s, d_t = teacher width.
  *   op  OLIVE_OP_TOPK_FWD: d = hidden width, d_t ignored.
  *   op  OLIVE_OP_SPLICE_MASKED: T = T_cap; d, d_t, V ignored.
+ *   op  OLIVE_OP_TOPK_KL_BWD: d = student width, grad_dtype as for
+ *       OLIVE_OP_LOSS_BWD, d_t ignored.
  *   `grad` (bwd / divergence): non-zero when gradients are requested
  *   (OLIVE_OP_LOSS_BWD always computes them); `grad_dtype` is the dtype of
  *   d_W for OLIVE_OP_LOSS_BWD (bf16 output needs an fp32 accumulator).
@@ -212,17 +223,47 @@ OLIVE_API olive_status olive_token_topk_fwd(const void* hidden, const void* W,
  *                truncated to the student's K most probable tokens (the
  *                paper's "top-16 KL approximation" is not printed in full;
  *                this is the reading implemented, no renormalisation).
+ *   t_logp_s[t, j] = log p_t(v_j), the teacher's log-prob at the student's
+ *                j-th id (optional: NULL skips it; the input of
+ *                olive_topk_kl_bwd)
  * 1 <= K <= 16; s_ids, t_ids int32 [T, K]; s_logp fp32 [T, K]; t_lse fp32
- * [T]; overlap, kl_topk fp32 [T] (0 on rows not in `rows`).  An id outside
- * [0, V) gives NaN and OLIVE_ERR_TOKEN_RANGE.
+ * [T]; overlap, kl_topk fp32 [T], t_logp_s fp32 [T, K] (0 on rows not in
+ * `rows`).  An id outside [0, V) gives NaN and OLIVE_ERR_TOKEN_RANGE.
  */
 OLIVE_API olive_status olive_topk_compare(const void* h_t, const void* W_t, int32_t d_t,
                                           const int32_t* rows, const int32_t* n_rows, int32_t T,
                                           int32_t V, float inv_tau, int32_t K,
                                           const int32_t* s_ids, const float* s_logp,
                                           const int32_t* t_ids, const float* t_lse,
-                                          float* overlap, float* kl_topk, int32_t* dev_status,
-                                          void* stream);
+                                          float* overlap, float* kl_topk, float* t_logp_s,
+                                          int32_t* dev_status, void* stream);
+
+/*
+ * olive_topk_kl_bwd -- gradient of sum_t g_t kl_topk[t] (the truncated
+ * reverse KL of olive_topk_compare) with respect to the student's hidden rows
+ * and LM head, the student's top-K set S_t held fixed (it is selected, not
+ * differentiated).  With l = log p_s, q = log p_t at the ids of S_t,
+ * P_S = sum_{v in S_t} p_s(v) and KL_K = kl_topk[t]:
+ *   G[t, u]  = g_t inv_tau p_s(u) ([u in S_t] (l_u - q_u + 1) - KL_K - P_S)
+ *   d_h_s[t] = sum_u G[t, u] W_s[u]     (0 on rows not in `rows`)
+ *   d_W_s[u] = sum_t G[t, u] h_s[t]
+ * Inputs: h_s [T, d], W_s [V, d] bf16; s_lse fp32 [T], s_ids int32 [T, K],
+ * s_logp fp32 [T, K] from olive_token_topk_fwd on the student; t_logp_s
+ * fp32 [T, K] and kl_topk fp32 [T] from olive_topk_compare; grad_kl fp32 [T]
+ * the weights g_t.  d_h_s [T, d] and d_W_s [V, d] of grad_dtype as in
+ * olive_token_loss_bwd.  The softmax term is recomputed tile by tile as in
+ * that backward; the K entries of S_t per row are written over it.  1 <= K
+ * <= 16; an id outside [0, V) sets OLIVE_ERR_TOKEN_RANGE.  workspace:
+ * olive_workspace_size(OLIVE_OP_TOPK_KL_BWD, T, d, 0, V, 1, grad_dtype) bytes.
+ */
+OLIVE_API olive_status olive_topk_kl_bwd(const void* h_s, const void* W_s, const int32_t* rows,
+                                         const int32_t* n_rows, int32_t T, int32_t d, int32_t V,
+                                         float inv_tau, int32_t K, const float* s_lse,
+                                         const int32_t* s_ids, const float* s_logp,
+                                         const float* t_logp_s, const float* kl_topk,
+                                         const float* grad_kl, void* d_h_s, void* d_W_s,
+                                         int grad_dtype, void* workspace, size_t ws_bytes,
+                                         int32_t* dev_status, void* stream);
 
 /*
  * olive_token_loss_bwd -- gradients of the Eq. (osd-ce) loss through the LM

@@ -388,7 +388,8 @@ def token_topk_compare(h_s, W_s, h_t, W_t, rows, K: int, inv_tau: float = 1.0):
     return overlap, kl, gap_s, gap_t
 
 
-def token_topk_kl_bwd(h_s, W_s, h_t, W_t, rows, K: int, inv_tau: float = 1.0, grad=None):
+def token_topk_kl_bwd(h_s, W_s, h_t, W_t, rows, K: int, inv_tau: float = 1.0, grad=None,
+                      with_dW: bool = True):
     """Gradient of sum_t g_t kl_topk[t] (see ``token_topk_compare``) with
     respect to the student's hidden rows and LM head, the top-K set S_t of
     the student held fixed (it is selected, not differentiated):
@@ -396,15 +397,15 @@ def token_topk_kl_bwd(h_s, W_s, h_t, W_t, rows, K: int, inv_tau: float = 1.0, gr
       KL_K = sum_{v in S} p_s(v) (l_v - q_v),
       dz_u = p_s(u) ([u in S] (l_u - q_u + 1) - KL_K - P_S)
       G[t, u] = g_t inv_tau dz_u,  dH_s[t] = G[t] W_s,  dW_s = G^T h_s.
-    Returns (dH_s [T, d_s], dW_s [V, d_s]).
+    Returns (dH_s [T, d_s], dW_s [V, d_s] or None without ``with_dW``).
     """
     h_s = np.asarray(h_s)
+    W_s = np.asarray(W_s)
     T = h_s.shape[0]
     rows = np.asarray(rows, dtype=np.int64)
     g = np.ones(T) if grad is None else np.asarray(grad, dtype=np.float64)
-    W64 = np.asarray(W_s).astype(np.float64)
     dH = np.zeros((T, h_s.shape[1]))
-    dW = np.zeros_like(W64)
+    dW = np.zeros(W_s.shape) if with_dW else None
     for r0 in range(0, len(rows), _ROW_CHUNK):
         rr = rows[r0:r0 + _ROW_CHUNK]
         hs = _as_f64_rows(h_s, rr)
@@ -420,8 +421,11 @@ def token_topk_kl_bwd(h_s, W_s, h_t, W_t, rows, K: int, inv_tau: float = 1.0, gr
             G[k] = -ps[k] * (kl + P_S)
             G[k, S] += ps[k, S] * (lps[k, S] - lpt[k, S] + 1.0)
         G *= (g[rr] * float(inv_tau))[:, None]
-        dH[rr] = G @ W64
-        dW += G.T @ hs
+        for v0 in range(0, W_s.shape[0], _VOCAB_CHUNK):
+            v1 = min(W_s.shape[0], v0 + _VOCAB_CHUNK)
+            dH[rr] += G[:, v0:v1] @ W_s[v0:v1].astype(np.float64)
+        if with_dW:
+            dW += G.T @ hs
     return dH, dW
 
 

@@ -27,7 +27,8 @@ STATUS_NAMES = {
 REDUCE = {"sum": 0, "mean": 1}
 DIRECTION = {"reverse": 0, "forward": 1}
 DTYPE = {torch.bfloat16: 0, torch.float32: 1}
-OP = {"logprob_fwd": 0, "loss_bwd": 1, "divergence": 2, "topk_fwd": 3, "splice_masked": 4}
+OP = {"logprob_fwd": 0, "loss_bwd": 1, "divergence": 2, "topk_fwd": 3, "splice_masked": 4,
+      "topk_kl_bwd": 5}
 
 
 class OliveError(RuntimeError):
@@ -74,7 +75,10 @@ def lib() -> ctypes.CDLL:
                                            _P, _P, _S, _P, _P]
     L.olive_topk_compare.restype = ctypes.c_int
     L.olive_topk_compare.argtypes = [_P, _P, _I, _P, _P, _I, _I, _F, _I, _P, _P, _P, _P, _P, _P, _P,
-                                     _P]
+                                     _P, _P]
+    L.olive_topk_kl_bwd.restype = ctypes.c_int
+    L.olive_topk_kl_bwd.argtypes = [_P, _P, _P, _P, _I, _I, _I, _F, _I, _P, _P, _P, _P, _P, _P, _P,
+                                    _P, ctypes.c_int, _P, _S, _P, _P]
     L.olive_token_topk_fwd.restype = ctypes.c_int
     L.olive_token_topk_fwd.argtypes = [_P, _P, _P, _P, _I, _I, _I, _F, _I, _P, _P, _P, _P, _P, _S,
                                        _P, _P]
@@ -254,10 +258,11 @@ def olive_token_topk_fwd(hidden, W, rows, n_rows, K: int = 16, inv_tau: float = 
 
 
 def olive_topk_compare(h_t, W_t, rows, n_rows, s_ids, s_logp, t_ids, t_lse, inv_tau: float = 1.0,
-                       dev_status=None):
+                       dev_status=None, want_t_logp=False):
     """Top-K overlap ratio and top-K truncated reverse KL per masked row.
 
-    Returns (overlap [T], kl_topk [T])."""
+    Returns (overlap [T], kl_topk [T]), plus the teacher's log-probs at the
+    student's top-K ids [T, K] when want_t_logp."""
     _need(h_t, torch.bfloat16, "h_t")
     _need(W_t, torch.bfloat16, "W_t")
     _need(s_ids, torch.int32, "s_ids")
@@ -270,12 +275,43 @@ def olive_topk_compare(h_t, W_t, rows, n_rows, s_ids, s_logp, t_ids, t_lse, inv_
     dev = h_t.device
     ov = torch.empty(T, dtype=torch.float32, device=dev)
     kl = torch.empty(T, dtype=torch.float32, device=dev)
+    tlp = torch.empty(T, K, dtype=torch.float32, device=dev) if want_t_logp else None
     ds = dev_status if dev_status is not None else new_status(dev)
     st = lib().olive_topk_compare(_ptr(h_t), _ptr(W_t), d_t, _ptr(rows), _ptr(n_rows), T, V,
                                   float(inv_tau), K, _ptr(s_ids), _ptr(s_logp), _ptr(t_ids),
-                                  _ptr(t_lse), _ptr(ov), _ptr(kl), _ptr(ds), _stream())
+                                  _ptr(t_lse), _ptr(ov), _ptr(kl), _ptr(tlp), _ptr(ds), _stream())
     _check(st, "olive_topk_compare")
-    return ov, kl
+    return (ov, kl, tlp) if want_t_logp else (ov, kl)
+
+
+def olive_topk_kl_bwd(h_s, W_s, rows, n_rows, s_lse, s_ids, s_logp, t_logp_s, kl_topk, grad_kl,
+                      inv_tau: float = 1.0, grad_dtype=torch.bfloat16, ws=None, dev_status=None,
+                      out=None):
+    """Gradient of sum_t grad_kl[t] kl_topk[t] with respect to h_s and W_s,
+    the student's top-K set held fixed.  Returns (d_h_s [T, d], d_W_s [V, d])."""
+    _need(h_s, torch.bfloat16, "h_s")
+    _need(W_s, torch.bfloat16, "W_s")
+    _need(s_ids, torch.int32, "s_ids")
+    for t, n in ((s_lse, "s_lse"), (s_logp, "s_logp"), (t_logp_s, "t_logp_s"), (kl_topk, "kl_topk"),
+                 (grad_kl, "grad_kl")):
+        _need(t, torch.float32, n)
+    T, d = h_s.shape
+    V = W_s.shape[0]
+    K = s_ids.shape[1]
+    dev = h_s.device
+    if out is None:
+        out = (torch.empty(T, d, dtype=grad_dtype, device=dev),
+               torch.empty(V, d, dtype=grad_dtype, device=dev))
+    dh, dw = out
+    if ws is None:
+        ws = workspace(olive_workspace_size("topk_kl_bwd", T, d, V, grad_dtype=grad_dtype), dev)
+    ds = dev_status if dev_status is not None else new_status(dev)
+    st = lib().olive_topk_kl_bwd(_ptr(h_s), _ptr(W_s), _ptr(rows), _ptr(n_rows), T, d, V,
+                                 float(inv_tau), K, _ptr(s_lse), _ptr(s_ids), _ptr(s_logp),
+                                 _ptr(t_logp_s), _ptr(kl_topk), _ptr(grad_kl), _ptr(dh), _ptr(dw),
+                                 DTYPE[grad_dtype], _ptr(ws), ws.numel(), _ptr(ds), _stream())
+    _check(st, "olive_topk_kl_bwd")
+    return dh, dw
 
 
 def olive_token_loss_bwd(hidden, W, targets, rows, n_rows, lse, grad_loss, inv_tau: float = 1.0,

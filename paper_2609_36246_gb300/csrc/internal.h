@@ -69,6 +69,7 @@ struct BwdWs {
 };
 size_t bwd_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype);
 BwdWs carve_bwd(void* ws, int64_t T, int64_t d, int64_t V, int grad_dtype);
+size_t topk_kl_bwd_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype);
 
 struct KlWs {
   void* hcs;      // bf16 [Tpad, d_s]
@@ -121,13 +122,38 @@ olive_status launch_topk_compare(const Ctx& c, const void* h_t, const void* W_t,
                                  const int32_t* rows, const int32_t* n_rows, int32_t T, int32_t V,
                                  float inv_tau, int32_t K, const int32_t* s_ids,
                                  const float* s_logp, const int32_t* t_ids, const float* t_lse,
-                                 float* overlap, float* kl_topk, int32_t* dev_status);
+                                 float* overlap, float* kl_topk, float* t_logp_s,
+                                 int32_t* dev_status);
 
+// Top-K KL gradient in place of the cross-entropy one: per masked row t the
+// softmax coefficient coef[t] and the full gradient values val[t, k] at the
+// ids[t, k] of the student's top-K set (K <= 16).
+struct SparseGrad {
+  const float* coef;
+  const float* val;
+  const int32_t* ids;
+  int32_t K;
+};
+
+// Cross-entropy backward (sg == nullptr: targets, grad_loss, reduction used)
+// or, with sg, the top-K KL backward (targets, grad_loss unused; lse is the
+// student's).
 olive_status launch_loss_bwd(const Ctx& c, const void* hidden, const void* W,
                              const int32_t* targets, const int32_t* rows, const int32_t* n_rows,
                              int32_t T, int32_t d, int32_t V, float inv_tau, int reduction,
                              const float* lse, const float* grad_loss, void* d_hidden, void* d_W,
-                             int grad_dtype, void* ws, int32_t* dev_status);
+                             int grad_dtype, void* ws, int32_t* dev_status,
+                             const SparseGrad* sg = nullptr);
+
+// Fills coef [T] and val [T, K] of the top-K KL gradient on the masked rows
+// from the forward's top-K lists, the teacher's log-probs at the student's
+// ids (t_logp_s), kl_topk and the weights grad_kl.
+olive_status launch_topk_kl_prep(const Ctx& c, const int32_t* rows, const int32_t* n_rows,
+                                 int32_t T, int32_t V, float inv_tau, int32_t K,
+                                 const int32_t* s_ids, const float* s_logp,
+                                 const float* t_logp_s, const float* kl_topk,
+                                 const float* grad_kl, float* coef, float* val,
+                                 int32_t* dev_status);
 
 olive_status launch_divergence(const Ctx& c, const void* h_s, const void* W_s, int32_t d_s,
                                const void* h_t, const void* W_t, int32_t d_t, const int32_t* rows,

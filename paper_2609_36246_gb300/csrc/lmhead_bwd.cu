@@ -9,6 +9,15 @@
 // Divergence (OPD's per-token KL, Section 1): G = g_t inv_tau p_s
 // (log p_s - log p_t - KL_t) (reverse) or g_t inv_tau (p_s - p_t) (forward),
 // and dH_s = G . W_s.
+// Top-K truncated reverse KL (OPD's top-16 approximation as read here, the
+// student's top-K set S held fixed): with l = log p_s, q = log p_t at the ids
+// of S, P_S = sum_S p_s and KL_K the forward value,
+//   G[r, u] = g_t inv_tau p_s(u) ([u in S] (l_u - q_u + 1) - KL_K - P_S),
+// i.e. a softmax term with the per-row coefficient -g_t inv_tau (KL_K + P_S)
+// plus K sparse entries whose full values a prologue kernel computes from the
+// forward's top-K lists; the GRAD epilogue writes the softmax term and then
+// overwrites the (at most K) entries of S that fall in its tile.  dH and dW
+// are then the cross-entropy tiles unchanged.
 //
 // The logits are recomputed tile by tile and turned into G in the epilogue;
 // G exists only as a bf16 slab of at most tc_max compacted rows in the
@@ -64,6 +73,10 @@ struct BwdParams {
   const float* lse;          // CE, indexed by packed row
   const float* grad_loss;    // CE, device scalar
   const float* grad_kl;      // KL, [T]
+  const float* sp_coef;      // top-K KL, [T]: softmax coefficient per row
+  const float* sp_val;       // top-K KL, [T, sp_k]: full G values at the ids of S
+  const int32_t* sp_ids;     // top-K KL, [T, sp_k]: the ids of S
+  int32_t sp_k;              // 0: cross-entropy targets; K: top-K KL
   const float* stats;        // KL, [3][ld_stats]: lse_s, lse_t, kl per compacted row
   int32_t ld_stats;
   int32_t kl;                // 0: cross-entropy, 1: divergence
@@ -109,7 +122,7 @@ __device__ Plan make_plan(const BwdParams& p) {
   pl.ntd = (p.d + kBN - 1) / kBN;
   pl.mtv = (p.V + kBM - 1) / kBM;
   pl.coef = 0.f;
-  if (!p.kl) {
+  if (!p.kl && p.sp_k == 0) {
     float g = *p.grad_loss;
     if (p.reduction == OLIVE_REDUCE_MEAN && pl.n > 0) g = g / static_cast<float>(pl.n);
     pl.coef = g * p.inv_tau;
@@ -238,12 +251,13 @@ __device__ void epi_grad(const BwdParams& p, const Plan& pl, const Unit& x, int 
   const int r_local = x.i * kBM + row;
   const int r = x.row0 + r_local;
   bool valid = r_local < x.in_s;
-  int y = -1;
-  float lse2 = 0.f;
+  int y = -1, t = -1;
+  float lse2 = 0.f, coef = pl.coef;
   if (valid) {
-    const int t = p.rows[r];
+    t = p.rows[r];
     if (t >= 0 && t < p.T) {
-      y = p.targets[t];
+      if (p.sp_k == 0) y = p.targets[t];
+      else coef = p.sp_coef[t];
       lse2 = p.lse[t] * kLog2e;
     } else {
       valid = false;
@@ -262,9 +276,20 @@ __device__ void epi_grad(const BwdParams& p, const Plan& pl, const Unit& x, int 
 #pragma unroll
     for (int k = 0; k < 32; ++k) {
       const float pr = fast_exp2(__uint_as_float(a[k]) * p.scale2 - lse2);
-      g[k] = valid ? pl.coef * (pr - (col0 + k == y ? 1.f : 0.f)) : 0.f;
+      g[k] = valid ? coef * (pr - (col0 + k == y ? 1.f : 0.f)) : 0.f;
     }
     store_row32(grow, col0, OLIVE_DTYPE_BF16, p.V - col0, g);
+  }
+  if (p.sp_k > 0 && valid) {
+    // the entries of S in this tile: same thread, same addresses, so these
+    // stores land after the softmax values written above
+    const int n1 = min(n0 + kBN, p.V);
+    const size_t o = static_cast<size_t>(t) * p.sp_k;
+#pragma unroll 1
+    for (int k = 0; k < p.sp_k; ++k) {
+      const int u = p.sp_ids[o + k];
+      if (u >= n0 && u < n1) grow[u] = __float2bfloat16_rn(p.sp_val[o + k]);
+    }
   }
 }
 
@@ -672,7 +697,8 @@ olive_status launch_loss_bwd(const Ctx& c, const void* hidden, const void* W,
                              const int32_t* targets, const int32_t* rows, const int32_t* n_rows,
                              int32_t T, int32_t d, int32_t V, float inv_tau, int reduction,
                              const float* lse, const float* grad_loss, void* d_hidden, void* d_W,
-                             int grad_dtype, void* ws, int32_t* dev_status) {
+                             int grad_dtype, void* ws, int32_t* dev_status,
+                             const SparseGrad* sg) {
   const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
   const BwdWs w = carve_bwd(ws, T, d, V, grad_dtype);
   const int64_t ldg = vpad(V);
@@ -698,6 +724,12 @@ olive_status launch_loss_bwd(const Ctx& c, const void* hidden, const void* W,
   p.targets = targets;
   p.lse = lse;
   p.grad_loss = grad_loss;
+  if (sg) {
+    p.sp_coef = sg->coef;
+    p.sp_val = sg->val;
+    p.sp_ids = sg->ids;
+    p.sp_k = sg->K;
+  }
   p.kl = 0;
   p.d = d;
   p.d2 = 0;

@@ -163,6 +163,12 @@ BwdWs carve_bwd(void* ws, int64_t T, int64_t d, int64_t V, int grad_dtype) {
   return carve_bwd_impl(ws, T, d, V, grad_dtype, nullptr);
 }
 
+// the backward's regions, then coef [T] and val [T, 16] of the top-K KL gradient
+size_t topk_kl_bwd_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype) {
+  return bwd_ws_bytes(T, d, V, grad_dtype) + align_up(4ull * T, kWsAlign) +
+         align_up(4ull * 16 * T, kWsAlign);
+}
+
 static KlWs carve_kl_impl(void* ws, int64_t T, int64_t ds, int64_t dt, int64_t V, int grad,
                           size_t* total) {
   const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
@@ -239,6 +245,9 @@ size_t olive_workspace_size(int op, int32_t T, int32_t d, int32_t d_t, int32_t V
       if (!width_ok(d_t)) return 0;
       return kl_ws_bytes(T, d, d_t, V, grad);
     case OLIVE_OP_TOPK_FWD: return topk_ws_bytes(T, d);
+    case OLIVE_OP_TOPK_KL_BWD:
+      if (grad_dtype != OLIVE_DTYPE_BF16 && grad_dtype != OLIVE_DTYPE_F32) return 0;
+      return topk_kl_bwd_ws_bytes(T, d, V, grad_dtype);
     default: return 0;
   }
 }
@@ -324,8 +333,8 @@ olive_status olive_topk_compare(const void* h_t, const void* W_t, int32_t d_t,
                                 const int32_t* rows, const int32_t* n_rows, int32_t T, int32_t V,
                                 float inv_tau, int32_t K, const int32_t* s_ids,
                                 const float* s_logp, const int32_t* t_ids, const float* t_lse,
-                                float* overlap, float* kl_topk, int32_t* dev_status,
-                                void* stream) {
+                                float* overlap, float* kl_topk, float* t_logp_s,
+                                int32_t* dev_status, void* stream) {
   if (!h_t || !W_t || !rows || !n_rows || !s_ids || !s_logp || !t_ids || !t_lse || !overlap ||
       !kl_topk || !dev_status)
     return OLIVE_ERR_INVALID_ARG;
@@ -336,7 +345,38 @@ olive_status olive_topk_compare(const void* h_t, const void* W_t, int32_t d_t,
   olive_status st = make_ctx(stream, &c);
   if (st != OLIVE_OK) return st;
   return launch_topk_compare(c, h_t, W_t, d_t, rows, n_rows, T, V, inv_tau, K, s_ids, s_logp,
-                             t_ids, t_lse, overlap, kl_topk, dev_status);
+                             t_ids, t_lse, overlap, kl_topk, t_logp_s, dev_status);
+}
+
+olive_status olive_topk_kl_bwd(const void* h_s, const void* W_s, const int32_t* rows,
+                               const int32_t* n_rows, int32_t T, int32_t d, int32_t V,
+                               float inv_tau, int32_t K, const float* s_lse, const int32_t* s_ids,
+                               const float* s_logp, const float* t_logp_s, const float* kl_topk,
+                               const float* grad_kl, void* d_h_s, void* d_W_s, int grad_dtype,
+                               void* workspace, size_t ws_bytes, int32_t* dev_status,
+                               void* stream) {
+  if (!h_s || !W_s || !rows || !n_rows || !s_lse || !s_ids || !s_logp || !t_logp_s || !kl_topk ||
+      !grad_kl || !d_h_s || !d_W_s || !dev_status)
+    return OLIVE_ERR_INVALID_ARG;
+  if (grad_dtype != OLIVE_DTYPE_BF16 && grad_dtype != OLIVE_DTYPE_F32) return OLIVE_ERR_INVALID_ARG;
+  if (T < 1 || V < 1 || d < 1 || d > kMaxDim || K < 1 || K > 16 || K > V) return OLIVE_ERR_SHAPE;
+  if (!(inv_tau > 0.f) || !std::isfinite(inv_tau)) return OLIVE_ERR_INVALID_ARG;
+  if (d % 8 != 0 || !aligned16(h_s) || !aligned16(W_s) || !aligned16(d_h_s) || !aligned16(d_W_s))
+    return OLIVE_ERR_ALIGNMENT;
+  olive_status st = check_ws(workspace, ws_bytes, topk_kl_bwd_ws_bytes(T, d, V, grad_dtype));
+  if (st != OLIVE_OK) return st;
+  Ctx c;
+  st = make_ctx(stream, &c);
+  if (st != OLIVE_OK) return st;
+  char* sparse = static_cast<char*>(workspace) + bwd_ws_bytes(T, d, V, grad_dtype);
+  float* coef = reinterpret_cast<float*>(sparse);
+  float* val = reinterpret_cast<float*>(sparse + align_up(4ull * T, kWsAlign));
+  st = launch_topk_kl_prep(c, rows, n_rows, T, V, inv_tau, K, s_ids, s_logp, t_logp_s, kl_topk,
+                           grad_kl, coef, val, dev_status);
+  if (st != OLIVE_OK) return st;
+  const SparseGrad sg{coef, val, s_ids, K};
+  return launch_loss_bwd(c, h_s, W_s, nullptr, rows, n_rows, T, d, V, inv_tau, OLIVE_REDUCE_SUM,
+                         s_lse, nullptr, d_h_s, d_W_s, grad_dtype, workspace, dev_status, &sg);
 }
 
 olive_status olive_token_loss_bwd(const void* hidden, const void* W, const int32_t* targets,

@@ -7,9 +7,17 @@
 //                vocabulary: the reverse KL of Section 1 truncated to its
 //                top-K terms (the paper's "top-16 KL approximation"; its exact
 //                form is not printed, this is the reading implemented)
+//   t_logp_s[t, j] = log p_t at the student's j-th id (optional output, the
+//                input of the top-K KL gradient)
 // One warp per masked row; the teacher's log-probs at the student's K ids
 // need K dot products h_t[t] . W_t[v] (d_t each), which the warp computes with
 // 16-byte loads split across lanes and a shuffle reduction.
+//
+// topk_kl_prep turns those lists into the sparse part of the top-K KL
+// gradient (see lmhead_bwd.cu): per masked row, with g = grad_kl[t] inv_tau,
+// P_S = sum_j exp(l_j) and A = kl_topk[t] + P_S,
+//   coef[t]   = -g A                       (multiplies p_s(u) for every u)
+//   val[t, j] = g exp(l_j) (l_j - q_j + 1 - A)   (G at the j-th id of S)
 #include <cmath>
 
 #include "sched.cuh"
@@ -38,7 +46,8 @@ __global__ void topk_compare_kernel(const uint4* __restrict__ h_t, const uint4* 
                                     const float* __restrict__ s_logp,
                                     const int32_t* __restrict__ t_ids,
                                     const float* __restrict__ t_lse, float* __restrict__ overlap,
-                                    float* __restrict__ kl_topk, int32_t* dev_status) {
+                                    float* __restrict__ kl_topk, float* __restrict__ t_logp_s,
+                                    int32_t* dev_status) {
   const int n = read_n_rows(n_rows, T, dev_status);
   const int lane = threadIdx.x & 31;
   const int warps = (gridDim.x * blockDim.x) >> 5;
@@ -61,6 +70,7 @@ __global__ void topk_compare_kernel(const uint4* __restrict__ h_t, const uint4* 
       const float lps = __shfl_sync(0xffffffffu, slp, j);
       if (v < 0 || v >= V) {
         bad = true;
+        if (t_logp_s && lane == 0) t_logp_s[static_cast<size_t>(t) * K + j] = NAN;
         continue;
       }
       const uint4* wrow = W_t + static_cast<size_t>(v) * d8;
@@ -70,6 +80,7 @@ __global__ void topk_compare_kernel(const uint4* __restrict__ h_t, const uint4* 
       for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
       const float lpt = part * inv_tau - lse_t;
       kl += expf(lps) * (lps - lpt);
+      if (t_logp_s && lane == 0) t_logp_s[static_cast<size_t>(t) * K + j] = lpt;
     }
     if (lane == 0) {
       overlap[t] = static_cast<float>(common) / static_cast<float>(K);
@@ -79,19 +90,69 @@ __global__ void topk_compare_kernel(const uint4* __restrict__ h_t, const uint4* 
   }
 }
 
+__global__ void topk_kl_prep_kernel(const int32_t* __restrict__ rows,
+                                    const int32_t* __restrict__ n_rows, int T, int V,
+                                    float inv_tau, int K, const int32_t* __restrict__ s_ids,
+                                    const float* __restrict__ s_logp,
+                                    const float* __restrict__ t_logp_s,
+                                    const float* __restrict__ kl_topk,
+                                    const float* __restrict__ grad_kl, float* __restrict__ coef,
+                                    float* __restrict__ val, int32_t* dev_status) {
+  const int n = read_n_rows(n_rows, T, dev_status);
+  for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < n; r += gridDim.x * blockDim.x) {
+    const int t = rows[r];
+    if (t < 0 || t >= T) continue;  // reported by the backward's gather
+    const size_t o = static_cast<size_t>(t) * K;
+    const float g = grad_kl[t] * inv_tau;
+    float P = 0.f;
+    bool bad = false;
+    for (int j = 0; j < K; ++j) {
+      P += expf(s_logp[o + j]);
+      const int v = s_ids[o + j];
+      bad |= v < 0 || v >= V;
+    }
+    const float A = kl_topk[t] + P;
+    coef[t] = -g * A;
+    for (int j = 0; j < K; ++j) {
+      const float l = s_logp[o + j];
+      val[o + j] = g * expf(l) * (l - t_logp_s[o + j] + 1.f - A);
+    }
+    if (bad) atomicOr(dev_status, 1 << OLIVE_ERR_TOKEN_RANGE);
+  }
+}
+
 }  // namespace
+
+olive_status launch_topk_kl_prep(const Ctx& c, const int32_t* rows, const int32_t* n_rows,
+                                 int32_t T, int32_t V, float inv_tau, int32_t K,
+                                 const int32_t* s_ids, const float* s_logp,
+                                 const float* t_logp_s, const float* kl_topk,
+                                 const float* grad_kl, float* coef, float* val,
+                                 int32_t* dev_status) {
+  const int threads = 256;
+  int blocks = static_cast<int>(ceil_div(T, threads));
+  if (blocks > c.num_sms * 4) blocks = c.num_sms * 4;
+  topk_kl_prep_kernel<<<blocks, threads, 0, c.stream>>>(rows, n_rows, T, V, inv_tau, K, s_ids,
+                                                        s_logp, t_logp_s, kl_topk, grad_kl, coef,
+                                                        val, dev_status);
+  return cudaGetLastError() == cudaSuccess ? OLIVE_OK : OLIVE_ERR_CUDA;
+}
 
 olive_status launch_topk_compare(const Ctx& c, const void* h_t, const void* W_t, int32_t d_t,
                                  const int32_t* rows, const int32_t* n_rows, int32_t T, int32_t V,
                                  float inv_tau, int32_t K, const int32_t* s_ids,
                                  const float* s_logp, const int32_t* t_ids, const float* t_lse,
-                                 float* overlap, float* kl_topk, int32_t* dev_status) {
+                                 float* overlap, float* kl_topk, float* t_logp_s,
+                                 int32_t* dev_status) {
   if (cudaMemsetAsync(overlap, 0, sizeof(float) * T, c.stream) != cudaSuccess ||
-      cudaMemsetAsync(kl_topk, 0, sizeof(float) * T, c.stream) != cudaSuccess)
+      cudaMemsetAsync(kl_topk, 0, sizeof(float) * T, c.stream) != cudaSuccess ||
+      (t_logp_s &&
+       cudaMemsetAsync(t_logp_s, 0, sizeof(float) * T * static_cast<size_t>(K), c.stream) !=
+           cudaSuccess))
     return OLIVE_ERR_CUDA;
   topk_compare_kernel<<<c.num_sms * 8, 256, 0, c.stream>>>(
       static_cast<const uint4*>(h_t), static_cast<const uint4*>(W_t), d_t / 8, rows, n_rows, T, V,
-      inv_tau, K, s_ids, s_logp, t_ids, t_lse, overlap, kl_topk, dev_status);
+      inv_tau, K, s_ids, s_logp, t_ids, t_lse, overlap, kl_topk, t_logp_s, dev_status);
   return cudaGetLastError() == cudaSuccess ? OLIVE_OK : OLIVE_ERR_CUDA;
 }
 

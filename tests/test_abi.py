@@ -136,11 +136,28 @@ def test_new_entry_points_validation(L):
     assert st == 1
     # top-K compare: null list, bad K
     st = L.olive_topk_compare(P(p), P(p), 64, P(p), P(p), 64, 100, 1.0, 4, None, P(p), P(p), P(p),
-                              P(p), P(p), P(p), None)
+                              P(p), P(p), None, P(p), None)
     assert st == 1
     st = L.olive_topk_compare(P(p), P(p), 64, P(p), P(p), 64, 100, 1.0, 20, P(p), P(p), P(p), P(p),
-                              P(p), P(p), P(p), None)
+                              P(p), P(p), None, P(p), None)
     assert st == 2
+    # top-K KL backward: missing t_logp_s, bad K, bad dtype, misaligned d_W_s, workspace
+    ws = B.olive_workspace_size("topk_kl_bwd", 64, 64, 100, grad_dtype=torch.float32)
+    assert ws > B.olive_workspace_size("loss_bwd", 64, 64, 100, grad_dtype=torch.float32)
+
+    def kl_bwd(**kw):
+        a = dict(tlp=P(p), K=4, dt=1, dw=P(p), ws_bytes=1 << 20)
+        a.update(kw)
+        return L.olive_topk_kl_bwd(P(p), P(p), P(p), P(p), 64, 64, 100, 1.0, a["K"], P(p), P(p),
+                                   P(p), a["tlp"], P(p), P(p), P(p), a["dw"], a["dt"], P(p),
+                                   a["ws_bytes"], P(p), None)
+    assert kl_bwd(tlp=None) == 1
+    assert kl_bwd(K=0) == 2 and kl_bwd(K=17) == 2
+    assert kl_bwd(dt=4) == 1
+    assert kl_bwd(dw=P(p + 4)) == 3
+    assert kl_bwd(ws_bytes=ws - 1) == 9
+    if not torch.cuda.is_available():
+        assert kl_bwd(ws_bytes=ws) in (7, 8)
     # multi-turn splice: null flags, workspace too small
     st = L.olive_splice_pack_masked(P(p), P(p), P(p), P(p), None, 1, 10, 10, P(p), P(p), P(p), P(p),
                                     P(p), P(p), P(p), P(p), 1 << 20, P(p), None)

@@ -40,7 +40,7 @@ MUTANTS = {
                         "        G *= -g * float(inv_tau)\n        dH[rr] = G @ W64"),
     "grad_drops_inv_tau": ("        G *= g * float(inv_tau)\n        dH[rr] = G @ W64",
                            "        G *= g\n        dH[rr] = G @ W64"),
-    "dW_transposed_pairing": ("        dW += G.T @ h", "        dW += G.T @ h[::-1]"),
+    "dW_transposed_pairing": ("        dW += G.T @ h\n", "        dW += G.T @ h[::-1]\n"),
     "mean_over_all_rows": ("        loss = loss / len(rows) if len(rows) else 0.0",
                            "        loss = loss / len(targets) if len(rows) else 0.0"),
     "kl_directions_swapped": ("            k = (ps * (lps - lpt)).sum(axis=1)",
@@ -48,6 +48,8 @@ MUTANTS = {
     "kl_grad_drops_kl_term": ("                dz = ps * (lps - lpt - k[:, None])",
                               "                dz = ps * (lps - lpt)"),
     "kl_grad_forward_sign": ("                dz = ps - pt", "                dz = pt - ps"),
+    "topk_grad_drops_mass_term": ("            G[k] = -ps[k] * (kl + P_S)", "            G[k] = -ps[k] * kl"),
+    "topk_grad_drops_plus_one": ("(lps[k, S] - lpt[k, S] + 1.0)", "(lps[k, S] - lpt[k, S])"),
 }
 
 
@@ -142,7 +144,26 @@ def pin_kl(O):
     return bool(ok)
 
 
-PINS = [pin_golden_splice, pin_turns_golden, pin_uniform, pin_scipy, pin_torch_ce_and_autograd, pin_kl]
+def pin_topk_kl_grad(O):
+    rng = np.random.default_rng(4)
+    hs, Ws = rng.standard_normal((5, 6)), rng.standard_normal((25, 6)) * 0.6
+    ht, Wt = rng.standard_normal((5, 8)), rng.standard_normal((25, 8)) * 0.6
+    r = np.array([1, 2, 4])
+    dH, dW = O.token_topk_kl_bwd(hs, Ws, ht, Wt, r, 5, inv_tau=0.9)
+    hs_t = torch.from_numpy(hs).requires_grad_(True)
+    Ws_t = torch.from_numpy(Ws).requires_grad_(True)
+    rr = torch.from_numpy(r)
+    lps = F.log_softmax(0.9 * (hs_t[rr] @ Ws_t.T), 1)
+    lpt = F.log_softmax(0.9 * (torch.from_numpy(ht)[rr] @ torch.from_numpy(Wt).T), 1)
+    S = torch.topk(lps.detach(), 5, dim=1).indices
+    ls, lt = lps.gather(1, S), lpt.gather(1, S)
+    (ls.exp() * (ls - lt)).sum().backward()
+    return bool(np.allclose(dH, hs_t.grad.numpy(), atol=1e-12)
+                and np.allclose(dW, Ws_t.grad.numpy(), atol=1e-12))
+
+
+PINS = [pin_golden_splice, pin_turns_golden, pin_uniform, pin_scipy, pin_torch_ce_and_autograd, pin_kl,
+        pin_topk_kl_grad]
 
 
 def test_real_oracle_passes_every_pin():
