@@ -18,6 +18,8 @@
  *
  * and these extend it:
  *
+ *   olive_token_loss_fwd_bwd the forward and backward of a training step in
+ *                            one pass over the logits (no recomputation)
  *   olive_splice_pack_masked multi-turn packing, loss only on teacher actions
  *                            (Section 3.2)
  *   olive_token_topk_fwd     per-token entropy and top-K log-probs
@@ -82,7 +84,8 @@ enum { OLIVE_REDUCE_SUM = 0, OLIVE_REDUCE_MEAN = 1 };
 enum { OLIVE_KL_REVERSE = 0, OLIVE_KL_FORWARD = 1 };
 enum { OLIVE_DTYPE_BF16 = 0, OLIVE_DTYPE_F32 = 1 };
 enum { OLIVE_OP_LOGPROB_FWD = 0, OLIVE_OP_LOSS_BWD = 1, OLIVE_OP_DIVERGENCE = 2,
-       OLIVE_OP_TOPK_FWD = 3, OLIVE_OP_SPLICE_MASKED = 4, OLIVE_OP_TOPK_KL_BWD = 5 };
+       OLIVE_OP_TOPK_FWD = 3, OLIVE_OP_SPLICE_MASKED = 4, OLIVE_OP_TOPK_KL_BWD = 5,
+       OLIVE_OP_LOSS_FWD_BWD = 6 };
 
 /* ABI version of the loaded library (OLIVE_ABI_VERSION). */
 OLIVE_API int olive_abi_version(void);
@@ -96,8 +99,8 @@ OLIVE_API const char* olive_status_string(olive_status s);
  *   op  OLIVE_OP_DIVERGENCE: d = student width d_s, d_t = teacher width.
  *   op  OLIVE_OP_TOPK_FWD: d = hidden width, d_t ignored.
  *   op  OLIVE_OP_SPLICE_MASKED: T = T_cap; d, d_t, V ignored.
- *   op  OLIVE_OP_TOPK_KL_BWD: d = student width, grad_dtype as for
- *       OLIVE_OP_LOSS_BWD, d_t ignored.
+ *   op  OLIVE_OP_TOPK_KL_BWD, OLIVE_OP_LOSS_FWD_BWD: d = (student) hidden
+ *       width, grad_dtype as for OLIVE_OP_LOSS_BWD, d_t ignored.
  *   `grad` (bwd / divergence): non-zero when gradients are requested
  *   (OLIVE_OP_LOSS_BWD always computes them); `grad_dtype` is the dtype of
  *   d_W for OLIVE_OP_LOSS_BWD (bf16 output needs an fp32 accumulator).
@@ -286,6 +289,30 @@ OLIVE_API olive_status olive_token_loss_bwd(const void* hidden, const void* W,
                                   void* d_hidden, void* d_W, int grad_dtype,
                                   void* workspace, size_t ws_bytes,
                                   int32_t* dev_status, void* stream);
+
+/*
+ * olive_token_loss_fwd_bwd -- olive_token_logprob_fwd and olive_token_loss_bwd
+ * of one training step in a single call, for callers that know the loss
+ * gradient before the forward runs (*grad_loss is read on the device, e.g. 1
+ * for a loss that is the objective itself).  Outputs and arguments as in
+ * those two calls: logp, lse fp32 [T], loss fp32 [1], d_hidden [T, d] and
+ * d_W [V, d] of grad_dtype.  Each logit tile is computed once: the forward
+ * product stores e = exp(z - tile max) in bf16 in the G slab of the workspace
+ * (one slab of at most a fixed number of rows at a time, never [T, V]), a
+ * bandwidth-bound pass turns it into G once the row's lse is known, and the
+ * dH and dW products follow.  Compared with olive_token_loss_bwd, G carries
+ * one more bf16 rounding of p (relative 2^-9 per entry; the target entry is
+ * formed from the fp32 logit).  workspace: olive_workspace_size(
+ * OLIVE_OP_LOSS_FWD_BWD, T, d, 0, V, 1, grad_dtype) bytes.
+ */
+OLIVE_API olive_status olive_token_loss_fwd_bwd(const void* hidden, const void* W,
+                                                const int32_t* targets, const int32_t* rows,
+                                                const int32_t* n_rows, int32_t T, int32_t d,
+                                                int32_t V, float inv_tau, int reduction,
+                                                const float* grad_loss, float* logp, float* lse,
+                                                float* loss, void* d_hidden, void* d_W,
+                                                int grad_dtype, void* workspace, size_t ws_bytes,
+                                                int32_t* dev_status, void* stream);
 
 /*
  * olive_token_divergence -- OPD's per-token divergence between the student

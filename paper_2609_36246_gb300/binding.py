@@ -28,7 +28,7 @@ REDUCE = {"sum": 0, "mean": 1}
 DIRECTION = {"reverse": 0, "forward": 1}
 DTYPE = {torch.bfloat16: 0, torch.float32: 1}
 OP = {"logprob_fwd": 0, "loss_bwd": 1, "divergence": 2, "topk_fwd": 3, "splice_masked": 4,
-      "topk_kl_bwd": 5}
+      "topk_kl_bwd": 5, "loss_fwd_bwd": 6}
 
 
 class OliveError(RuntimeError):
@@ -76,6 +76,9 @@ def lib() -> ctypes.CDLL:
     L.olive_topk_compare.restype = ctypes.c_int
     L.olive_topk_compare.argtypes = [_P, _P, _I, _P, _P, _I, _I, _F, _I, _P, _P, _P, _P, _P, _P, _P,
                                      _P, _P]
+    L.olive_token_loss_fwd_bwd.restype = ctypes.c_int
+    L.olive_token_loss_fwd_bwd.argtypes = [_P, _P, _P, _P, _P, _I, _I, _I, _F, ctypes.c_int, _P, _P,
+                                           _P, _P, _P, _P, ctypes.c_int, _P, _S, _P, _P]
     L.olive_topk_kl_bwd.restype = ctypes.c_int
     L.olive_topk_kl_bwd.argtypes = [_P, _P, _P, _P, _I, _I, _I, _F, _I, _P, _P, _P, _P, _P, _P, _P,
                                     _P, ctypes.c_int, _P, _S, _P, _P]
@@ -339,6 +342,38 @@ def olive_token_loss_bwd(hidden, W, targets, rows, n_rows, lse, grad_loss, inv_t
                                     _ptr(ws), ws.numel(), _ptr(ds), _stream())
     _check(st, "olive_token_loss_bwd")
     return dh, dw
+
+
+def olive_token_loss_fwd_bwd(hidden, W, targets, rows, n_rows, grad_loss, inv_tau: float = 1.0,
+                             reduction: str = "sum", grad_dtype=torch.bfloat16, ws=None,
+                             dev_status=None, out=None):
+    """Forward and backward of one training step in one pass over the logits.
+
+    grad_loss is a 1-element fp32 CUDA tensor (the loss gradient, known before
+    the call).  Returns (logp [T], lse [T], loss [1], d_hidden [T, d], d_W [V, d])."""
+    _need(hidden, torch.bfloat16, "hidden")
+    _need(W, torch.bfloat16, "W")
+    _need(grad_loss, torch.float32, "grad_loss")
+    T, d = hidden.shape
+    V = W.shape[0]
+    dev = hidden.device
+    if out is None:
+        out = (torch.empty(T, dtype=torch.float32, device=dev),
+               torch.empty(T, dtype=torch.float32, device=dev),
+               torch.empty(1, dtype=torch.float32, device=dev),
+               torch.empty(T, d, dtype=grad_dtype, device=dev),
+               torch.empty(V, d, dtype=grad_dtype, device=dev))
+    logp, lse, loss, dh, dw = out
+    if ws is None:
+        ws = workspace(olive_workspace_size("loss_fwd_bwd", T, d, V, grad_dtype=grad_dtype), dev)
+    ds = dev_status if dev_status is not None else new_status(dev)
+    st = lib().olive_token_loss_fwd_bwd(_ptr(hidden), _ptr(W), _ptr(targets), _ptr(rows),
+                                        _ptr(n_rows), T, d, V, float(inv_tau), REDUCE[reduction],
+                                        _ptr(grad_loss), _ptr(logp), _ptr(lse), _ptr(loss),
+                                        _ptr(dh), _ptr(dw), DTYPE[grad_dtype], _ptr(ws), ws.numel(),
+                                        _ptr(ds), _stream())
+    _check(st, "olive_token_loss_fwd_bwd")
+    return logp, lse, loss, dh, dw
 
 
 def olive_token_divergence(h_s, W_s, h_t, W_t, rows, n_rows, inv_tau: float = 1.0,

@@ -71,6 +71,20 @@ size_t bwd_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype);
 BwdWs carve_bwd(void* ws, int64_t T, int64_t d, int64_t V, int grad_dtype);
 size_t topk_kl_bwd_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype);
 
+// fused forward + backward: the backward's regions plus the ZSAVE partials
+struct FbWs {
+  void* hc;        // bf16 [Tpad, d]
+  void* g;         // bf16 [Tc, Vpad]: e = 2^(x - m_tile), then G
+  float* part_zm;  // [Tc, vt] tile max (base 2)
+  float* part_zs;  // [Tc, vt] tile sums
+  float* zy;       // [Tc] target logits of the slab
+  float* nll;      // [Tpad] per-row loss terms
+  float* dw_acc;   // fp32 [V, d] (bf16 output only)
+  int64_t tc;
+};
+size_t fb_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype);
+FbWs carve_fb(void* ws, int64_t T, int64_t d, int64_t V, int grad_dtype);
+
 struct KlWs {
   void* hcs;      // bf16 [Tpad, d_s]
   void* hct;      // bf16 [Tpad, d_t]
@@ -112,6 +126,19 @@ olive_status launch_logprob_fwd(const Ctx& c, const void* hidden, const void* W,
                                 int32_t T, int32_t d, int32_t V, float inv_tau, int reduction,
                                 float* logp, float* lse, float* loss, void* ws,
                                 int32_t* dev_status);
+
+// One block sums the per-row loss terms nll[0, n) in a fixed order (fp64).
+olive_status launch_loss_reduce(const Ctx& c, const int32_t* n_rows, int32_t T, const float* nll,
+                                int reduction, float* loss);
+
+// Forward and backward of the Eq. (osd-ce) loss in one pass over the logits
+// (grad_loss is read on the device before the gradients are formed).
+olive_status launch_loss_fwd_bwd(const Ctx& c, const void* hidden, const void* W,
+                                 const int32_t* targets, const int32_t* rows,
+                                 const int32_t* n_rows, int32_t T, int32_t d, int32_t V,
+                                 float inv_tau, int reduction, const float* grad_loss, float* logp,
+                                 float* lse, float* loss, void* d_hidden, void* d_W, int grad_dtype,
+                                 void* ws, int32_t* dev_status);
 
 olive_status launch_topk_fwd(const Ctx& c, const void* hidden, const void* W, const int32_t* rows,
                              const int32_t* n_rows, int32_t T, int32_t d, int32_t V, float inv_tau,

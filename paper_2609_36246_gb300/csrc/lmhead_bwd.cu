@@ -41,6 +41,15 @@
 // tile only waits on tiles with smaller indices, so the lowest unfinished
 // tile never waits and all waits end; the cooperative launch keeps every CTA
 // resident.
+//
+// Forward + backward in one call (olive_token_loss_fwd_bwd) avoids the logit
+// recomputation: per slab, a launch of ZSAVE tiles (the forward product) stores
+// e = 2^(x - m_tile) in bf16 in the G slab with the tile's (max, sum) per row;
+// conv_kernel merges the partials into lse, writes logp and the row's loss
+// term, and turns the slab into G in place (G = g inv_tau (e 2^(m_tile -
+// lse2) - [v == y]), the target entry from the exact fp32 z_y); a second
+// launch runs the DH and DW tiles of the slab.  The launches are stream
+// ordered, so these phases need no tile counters.
 #include <cmath>
 
 #include "gemm_core.cuh"
@@ -54,7 +63,10 @@ constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kBN = 256;
 constexpr int kStages = 4;
 
-enum Kind : int { K_NONE = -1, K_GRAD = 0, K_KLGRAD = 1, K_DH = 2, K_DW = 3 };
+enum Kind : int { K_NONE = -1, K_GRAD = 0, K_KLGRAD = 1, K_DH = 2, K_DW = 3, K_ZSAVE = 4 };
+// phases: one launch of every tile kind with dependency waits, or one slab's
+// forward (ZSAVE) tiles, or one slab's DH and DW tiles
+enum Phase : int { PH_ALL = 0, PH_Z = 1, PH_DHDW = 2 };
 
 // CE maps: 0 hc K-major 64x128, 1 W K-major 64x256, 2 G K-major 64x128,
 //          3 W MN-major 64x64, 4 G MN-major 64x64, 5 hc MN-major 64x64
@@ -77,6 +89,10 @@ struct BwdParams {
   const float* sp_val;       // top-K KL, [T, sp_k]: full G values at the ids of S
   const int32_t* sp_ids;     // top-K KL, [T, sp_k]: the ids of S
   int32_t sp_k;              // 0: cross-entropy targets; K: top-K KL
+  int32_t phase, slab;       // Phase; the slab of PH_Z / PH_DHDW
+  float* part_zm;            // PH_Z: [tc, vt] tile max (base 2) per slab row
+  float* part_zs;            // PH_Z: [tc, vt] tile sum of 2^(x - max)
+  float* zy_s;               // PH_Z: [tc] target logit (natural units)
   const float* stats;        // KL, [3][ld_stats]: lse_s, lse_t, kl per compacted row
   int32_t ld_stats;
   int32_t kl;                // 0: cross-entropy, 1: divergence
@@ -113,16 +129,16 @@ __device__ __forceinline__ uint32_t* ctr_row(const BwdParams& p, int s, int i) {
 __device__ Plan make_plan(const BwdParams& p) {
   Plan pl;
   pl.n = read_n_rows(p.n_rows, p.T, p.dev_status);
-  pl.n_slabs = pl.n > 0 ? (pl.n + p.tc_max - 1) / p.tc_max : 1;
+  const SlabPlan sp(pl.n, p.tc_max);
+  pl.n_slabs = sp.n_slabs;
   if (pl.n_slabs > p.max_slabs) pl.n_slabs = p.max_slabs;  // cannot happen for n <= T
-  const int per = (pl.n + pl.n_slabs - 1) / pl.n_slabs;
-  pl.rps = (per + 127) / 128 * 128;
+  pl.rps = sp.rps;
   pl.bn_grad = 256;
   pl.vt = (p.V + pl.bn_grad - 1) / pl.bn_grad;
   pl.ntd = (p.d + kBN - 1) / kBN;
   pl.mtv = (p.V + kBM - 1) / kBM;
   pl.coef = 0.f;
-  if (!p.kl && p.sp_k == 0) {
+  if (!p.kl && p.sp_k == 0 && p.phase == PH_ALL) {
     float g = *p.grad_loss;
     if (p.reduction == OLIVE_REDUCE_MEAN && pl.n > 0) g = g / static_cast<float>(pl.n);
     pl.coef = g * p.inv_tau;
@@ -140,12 +156,19 @@ __device__ __forceinline__ int units_dw(const BwdParams& p, const Plan& pl, int 
   return (!p.kl && (s == 0 || in_s > 0)) ? pl.mtv * pl.ntd : 0;
 }
 
+// slabs a launch covers
+__device__ __forceinline__ int slab_lo(const BwdParams& p) { return p.phase == PH_ALL ? 0 : p.slab; }
+__device__ __forceinline__ int slab_hi(const BwdParams& p, const Plan& pl) {
+  return p.phase == PH_ALL ? pl.n_slabs : (p.slab < pl.n_slabs ? p.slab + 1 : 0);
+}
+
 __device__ int total_units(const BwdParams& p, const Plan& pl) {
   int t = 0;
-  for (int s = 0; s < pl.n_slabs; ++s) {
+  for (int s = slab_lo(p); s < slab_hi(p, pl); ++s) {
     const int in_s = slab_in(pl, s);
     const int mt = (in_s + 127) / 128;
-    t += units_grad(pl, mt) + units_dh(pl, mt) + units_dw(p, pl, s, in_s);
+    if (p.phase != PH_DHDW) t += units_grad(pl, mt);
+    if (p.phase != PH_Z) t += units_dh(pl, mt) + units_dw(p, pl, s, in_s);
   }
   return t;
 }
@@ -153,21 +176,22 @@ __device__ int total_units(const BwdParams& p, const Plan& pl) {
 __device__ Unit decode(const BwdParams& p, const Plan& pl, int u) {
   Unit x;
   x.kind = K_NONE;
-  for (int s = 0; s < pl.n_slabs; ++s) {
+  for (int s = slab_lo(p); s < slab_hi(p, pl); ++s) {
     const int in_s = slab_in(pl, s);
     const int mt = (in_s + 127) / 128;
     x.s = s;
     x.in_s = in_s;
     x.row0 = s * pl.rps;
     x.mt = mt;
-    const int ug = units_grad(pl, mt);
+    const int ug = p.phase == PH_DHDW ? 0 : units_grad(pl, mt);
     if (u < ug) {
       const Raster r{mt, pl.vt, p.group_rows};
       r.tile(u, x.i, x.j);
-      x.kind = p.kl ? K_KLGRAD : K_GRAD;
+      x.kind = p.phase == PH_Z ? K_ZSAVE : (p.kl ? K_KLGRAD : K_GRAD);
       return x;
     }
     u -= ug;
+    if (p.phase == PH_Z) continue;
     const int uh = units_dh(pl, mt);
     if (u < uh) {
       x.i = u / pl.ntd;
@@ -192,7 +216,8 @@ __device__ Unit decode(const BwdParams& p, const Plan& pl, int u) {
 __device__ __forceinline__ void unit_ksteps(const BwdParams& p, const Unit& x, int& nk, int& nk2) {
   nk2 = 0;
   switch (x.kind) {
-    case K_GRAD: nk = (p.d + kBK - 1) / kBK; break;
+    case K_GRAD:
+    case K_ZSAVE: nk = (p.d + kBK - 1) / kBK; break;
     case K_KLGRAD:
       nk = (p.d + kBK - 1) / kBK;
       nk2 = (p.d2 + kBK - 1) / kBK;
@@ -329,6 +354,63 @@ __device__ void epi_klgrad(const BwdParams& p, const Unit& x, int row, uint32_t 
       g[k] = valid ? coef * v : 0.f;
     }
     store_row32(grow, col0, OLIVE_DTYPE_BF16, p.V - col0, g);
+  }
+}
+
+// forward tile of the fused forward + backward: per row the tile's max and
+// sum of 2^(x - max) in base-2 units, e = 2^(x - max) stored in bf16 at the
+// row's G slab columns (zeros on padding rows), and the exact target logit
+__device__ void epi_zsave(const BwdParams& p, const Plan& pl, const Unit& x, int row,
+                          uint32_t taddr) {
+  const int r_local = x.i * kBM + row;
+  bool valid = r_local < x.in_s;
+  int y = -1;
+  if (valid) {
+    const int t = p.rows[x.row0 + r_local];
+    if (t >= 0 && t < p.T) y = p.targets[t];
+    else valid = false;
+  }
+  const int n0 = x.j * kBN;
+  float tm = -INFINITY;
+#pragma unroll 1
+  for (int c = 0; c < kBN; c += 32) {
+    const int col0 = n0 + c;
+    if (col0 >= p.V) break;
+    uint32_t a[32];
+    tmem_ld_32x32b_x32(taddr + c, a);
+    tmem_ld_wait();
+    const int nv = p.V - col0;
+#pragma unroll
+    for (int k = 0; k < 32; ++k)
+      if (k < nv) tm = fmaxf(tm, __uint_as_float(a[k]) * p.scale2);
+    if (y >= col0 && y < col0 + 32) {
+#pragma unroll
+      for (int k = 0; k < 32; ++k)
+        if (col0 + k == y) p.zy_s[r_local] = __uint_as_float(a[k]) * p.inv_tau;
+    }
+  }
+  __nv_bfloat16* grow = p.g + static_cast<size_t>(r_local) * p.ldg;
+  float ts = 0.f;
+#pragma unroll 1
+  for (int c = 0; c < kBN; c += 32) {
+    const int col0 = n0 + c;
+    if (col0 >= p.V) break;
+    uint32_t a[32];
+    tmem_ld_32x32b_x32(taddr + c, a);
+    tmem_ld_wait();
+    const int nv = p.V - col0;
+    float e[32];
+#pragma unroll
+    for (int k = 0; k < 32; ++k) {
+      e[k] = (valid && k < nv) ? fast_exp2(__uint_as_float(a[k]) * p.scale2 - tm) : 0.f;
+      ts += e[k];
+    }
+    store_row32(grow, col0, OLIVE_DTYPE_BF16, nv, e);
+  }
+  if (valid) {
+    const size_t o = static_cast<size_t>(r_local) * pl.vt + x.j;
+    p.part_zm[o] = tm;
+    p.part_zs[o] = ts;
   }
 }
 
@@ -484,7 +566,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const Unit x = decode(p, pl, u);
         // wait until the tiles this one reads are published
         bool dep = true;
-        if ((x.kind == K_GRAD || x.kind == K_KLGRAD) && x.s > 0) {
+        if (p.phase != PH_ALL) {
+          // phases are separate launches in stream order: nothing to wait for
+        } else if ((x.kind == K_GRAD || x.kind == K_KLGRAD) && x.s > 0) {
           const int pin = slab_in(pl, x.s - 1);
           const int pmt = (pin + 127) / 128;
           dep = wait_counter(ctr_dhdw(p, x.s - 1),
@@ -506,6 +590,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           mbar_arrive_expect_tx(fb, L::STAGE_BYTES);
           switch (x.kind) {
             case K_GRAD:
+            case K_ZSAVE:
               tma_load_2d(sA, &maps.m[0], fb, k * kBK, x.row0 + x.i * kBM);
               tma_load_2d(sB, &maps.m[1], fb, k * kBK, x.j * kBN);
               break;
@@ -604,7 +689,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       __syncwarp();
       const uint32_t taddr = lane_addr + static_cast<uint32_t>(buf * kBN);
-      if (x.kind == K_DW && x.s > 0) {
+      if (x.kind == K_DW && x.s > 0 && p.phase == PH_ALL) {
         // the fp32 partial of the previous slab must be visible before it is read
         const bool seen = row == 0 ? wait_counter(ctr_grad(p, x.s), units_grad(pl, x.mt), ctl) : true;
         if (!named_bar_and(1, kEpiThreads, seen)) break;
@@ -612,6 +697,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       switch (x.kind) {
         case K_GRAD: epi_grad(p, pl, x, row, taddr); break;
         case K_KLGRAD: epi_klgrad(p, x, row, taddr); break;
+        case K_ZSAVE: epi_zsave(p, pl, x, row, taddr); break;
         case K_DH: epi_dh(p, x, row, taddr); break;
         case K_DW: epi_dw(p, pl, x, row, taddr, nk); break;
         default: break;
@@ -623,7 +709,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       fence_proxy_async_global();
       __threadfence();
       named_bar_sync(1, kEpiThreads);
-      if (row == 0) {
+      if (row == 0 && p.phase == PH_ALL) {
         if (x.kind == K_GRAD || x.kind == K_KLGRAD) {
           red_release_add(ctr_row(p, x.s, x.i), 1u);
           red_release_add(ctr_grad(p, x.s), 1u);
@@ -640,6 +726,101 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == kMmaWarp) {
     tc_fence_after();
     tmem_dealloc(tmem_base, L::TMEM_COLS);
+  }
+}
+
+// (max, sum) pairs in base 2; an empty side (max = -inf) contributes nothing
+__device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2) {
+  if (m2 == -INFINITY) return;
+  if (m == -INFINITY) {
+    m = m2;
+    s = s2;
+    return;
+  }
+  const float mn = fmaxf(m, m2);
+  s = s * fast_exp2(m - mn) + s2 * fast_exp2(m2 - mn);
+  m = mn;
+}
+
+// One warp per masked row of the slab: merges the ZSAVE partials into lse,
+// writes logp, lse and the row's loss term, then rewrites the row's slab
+// entries e = 2^(x - m_tile) as G = coef (e 2^(m_tile - lse2) - [v == y]) in
+// place (32 lanes x 8 columns cover one 256-wide tile per step, so the tile
+// max is one broadcast load).  The target entry uses the exact z_y.
+__global__ void __launch_bounds__(256)
+    conv_kernel(const int32_t* __restrict__ n_rows, const int32_t* __restrict__ rows,
+                const int32_t* __restrict__ targets, int T, int V, int tc, int slab, int vt,
+                int64_t ldg, float inv_tau, int reduction, const float* __restrict__ grad_loss,
+                const float* __restrict__ part_zm, const float* __restrict__ part_zs,
+                const float* __restrict__ zy_s, __nv_bfloat16* g, float* __restrict__ logp,
+                float* __restrict__ lse, float* __restrict__ nll, int32_t* dev_status) {
+  const int n = read_n_rows(n_rows, T, nullptr);
+  const SlabPlan sp(n, tc);
+  if (slab >= sp.n_slabs) return;
+  const int in_s = sp.rows_in(n, slab);
+  const int row0 = slab * sp.rps;
+  float gs = *grad_loss;
+  if (reduction == OLIVE_REDUCE_MEAN && n > 0) gs = gs / static_cast<float>(n);
+  const float coef = gs * inv_tau;
+  const int lane = threadIdx.x & 31;
+  const int warps = (gridDim.x * blockDim.x) >> 5;
+  const int nvec = (V + 7) / 8;
+  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < in_s; r += warps) {
+    const int t = rows[row0 + r];
+    if (t < 0 || t >= T) {
+      if (lane == 0) nll[row0 + r] = 0.f;  // reported by the gather; the G row is zero
+      continue;
+    }
+    const int y = targets[t];
+    const float* zm = part_zm + static_cast<size_t>(r) * vt;
+    const float* zs = part_zs + static_cast<size_t>(r) * vt;
+    float m = -INFINITY, sum = 0.f;
+    for (int j = lane; j < vt; j += 32) lse_merge(m, sum, zm[j], zs[j]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+      const float s2 = __shfl_xor_sync(0xffffffffu, sum, o);
+      lse_merge(m, sum, m2, s2);
+    }
+    const float lse2 = m + log2f(sum);
+    const float l = lse2 * kLn2;
+    const bool ybad = y < 0 || y >= V;
+    const float lp = ybad ? NAN : zy_s[r] - l;
+    if (lane == 0) {
+      logp[t] = lp;
+      lse[t] = l;
+      nll[row0 + r] = -lp;
+      if (ybad) atomicOr(dev_status, 1 << OLIVE_ERR_TOKEN_RANGE);
+    }
+    const float gy = coef * expm1f(lp);
+    uint4* grow = reinterpret_cast<uint4*>(g + static_cast<size_t>(r) * ldg);
+#pragma unroll 1
+    for (int base = 0; base < nvec; base += 128) {
+      uint4 v[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int idx = base + 32 * q + lane;
+        if (idx < nvec) v[q] = grow[idx];
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int idx = base + 32 * q + lane;
+        if (idx >= nvec) continue;
+        const float sc = coef * fast_exp2(zm[(base >> 5) + q] - lse2);
+        __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&v[q]);
+        const int col = idx * 8;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 u = __bfloat1622float2(h2[e]);
+          float a = col + 2 * e < V ? u.x * sc : 0.f;
+          float b = col + 2 * e + 1 < V ? u.y * sc : 0.f;
+          if (col + 2 * e == y) a = gy;
+          if (col + 2 * e + 1 == y) b = gy;
+          h2[e] = __floats2bfloat162_rn(a, b);
+        }
+        grow[idx] = v[q];
+      }
+    }
   }
 }
 
@@ -745,6 +926,70 @@ olive_status launch_loss_bwd(const Ctx& c, const void* hidden, const void* W,
   p.dw_acc = grad_dtype == OLIVE_DTYPE_F32 ? static_cast<float*>(d_W) : w.dw_acc;
   p.counters = w.counters;
   return launch_bwd_fused(c, maps, p);
+}
+
+olive_status launch_loss_fwd_bwd(const Ctx& c, const void* hidden, const void* W,
+                                 const int32_t* targets, const int32_t* rows,
+                                 const int32_t* n_rows, int32_t T, int32_t d, int32_t V,
+                                 float inv_tau, int reduction, const float* grad_loss, float* logp,
+                                 float* lse, float* loss, void* d_hidden, void* d_W, int grad_dtype,
+                                 void* ws, int32_t* dev_status) {
+  const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
+  const FbWs w = carve_fb(ws, T, d, V, grad_dtype);
+  const int64_t ldg = vpad(V);
+  const size_t elt = grad_dtype == OLIVE_DTYPE_BF16 ? 2 : 4;
+  const int vt = static_cast<int>(ceil_div(V, kBN));
+
+  olive_status st = launch_gather_rows(c, hidden, rows, n_rows, T, d, w.hc, dev_status);
+  if (st != OLIVE_OK) return st;
+  if (cudaMemsetAsync(d_hidden, 0, elt * T * static_cast<size_t>(d), c.stream) != cudaSuccess ||
+      cudaMemsetAsync(logp, 0, sizeof(float) * T, c.stream) != cudaSuccess ||
+      cudaMemsetAsync(lse, 0, sizeof(float) * T, c.stream) != cudaSuccess)
+    return OLIVE_ERR_CUDA;
+
+  BwdMaps maps;
+  if (!encode_bf16_2d(&maps.m[0], w.hc, d, Tpad, 2ull * d, 64, 128) ||
+      !encode_bf16_2d(&maps.m[1], W, d, V, 2ull * d, 64, 256) ||
+      !encode_bf16_2d(&maps.m[2], w.g, V, w.tc, 2ull * ldg, 64, 128) ||
+      !encode_bf16_2d(&maps.m[3], W, d, V, 2ull * d, 64, 64) ||
+      !encode_bf16_2d(&maps.m[4], w.g, V, w.tc, 2ull * ldg, 64, 64) ||
+      !encode_bf16_2d(&maps.m[5], w.hc, d, Tpad, 2ull * d, 64, 64))
+    return OLIVE_ERR_CUDA;
+
+  BwdParams p = base_params(c, rows, n_rows, T, V, inv_tau, dev_status);
+  p.targets = targets;
+  p.kl = 0;
+  p.d = d;
+  p.reduction = reduction;
+  p.out_dtype = grad_dtype;
+  p.tc_max = static_cast<int32_t>(w.tc);
+  const int64_t max_slabs = ceil_div(Tpad, w.tc);
+  p.max_slabs = static_cast<int32_t>(max_slabs + 1);
+  p.max_rt = static_cast<int32_t>(w.tc / kRowAlign);
+  p.ldg = ldg;
+  p.g = static_cast<__nv_bfloat16*>(w.g);
+  p.dh_out = d_hidden;
+  p.dw_out = d_W;
+  p.dw_acc = grad_dtype == OLIVE_DTYPE_F32 ? static_cast<float*>(d_W) : w.dw_acc;
+  p.part_zm = w.part_zm;
+  p.part_zs = w.part_zs;
+  p.zy_s = w.zy;
+
+  int conv_blocks = static_cast<int>(ceil_div(w.tc, 8));
+  if (conv_blocks > c.num_sms * 16) conv_blocks = c.num_sms * 16;
+  for (int s = 0; s < max_slabs; ++s) {
+    p.slab = s;
+    p.phase = PH_Z;
+    if ((st = launch_bwd_fused(c, maps, p)) != OLIVE_OK) return st;
+    conv_kernel<<<conv_blocks, 256, 0, c.stream>>>(
+        n_rows, rows, targets, T, V, static_cast<int>(w.tc), s, vt, ldg, inv_tau, reduction,
+        grad_loss, w.part_zm, w.part_zs, w.zy, static_cast<__nv_bfloat16*>(w.g), logp, lse, w.nll,
+        dev_status);
+    if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;
+    p.phase = PH_DHDW;
+    if ((st = launch_bwd_fused(c, maps, p)) != OLIVE_OK) return st;
+  }
+  return launch_loss_reduce(c, n_rows, T, w.nll, reduction, loss);
 }
 
 olive_status launch_kl_bwd(const Ctx& c, const void* hcs, const void* hct, const void* W_s,

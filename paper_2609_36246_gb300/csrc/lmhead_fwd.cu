@@ -411,6 +411,12 @@ olive_status launch_gather_rows(const Ctx& c, const void* hidden, const int32_t*
   return cudaGetLastError() == cudaSuccess ? OLIVE_OK : OLIVE_ERR_CUDA;
 }
 
+olive_status launch_loss_reduce(const Ctx& c, const int32_t* n_rows, int32_t T, const float* nll,
+                                int reduction, float* loss) {
+  loss_reduce_kernel<<<1, 1024, 0, c.stream>>>(n_rows, T, nll, reduction, loss);
+  return cudaGetLastError() == cudaSuccess ? OLIVE_OK : OLIVE_ERR_CUDA;
+}
+
 olive_status launch_logprob_fwd(const Ctx& c, const void* hidden, const void* W,
                                 const int32_t* targets, const int32_t* rows, const int32_t* n_rows,
                                 int32_t T, int32_t d, int32_t V, float inv_tau, int reduction,

@@ -80,11 +80,17 @@ bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t
 }
 
 int64_t slab_rows(int64_t Tpad, int64_t V) {
-  // G buffer of at most ~5.6 GB (bf16), in whole 128-row tiles, <= 32768 rows
+  // G buffer of at most ~5.6 GB (bf16), in whole 128-row tiles, <= 32768 rows;
+  // OLIVE_SLAB_ROWS (a multiple of 128) can lower the cap, e.g. to exercise
+  // several slabs on small inputs
   const int64_t budget = 5600ll * 1000 * 1000;
   int64_t tc = budget / (2 * vpad(V)) / kRowAlign * kRowAlign;
   if (tc < kRowAlign) tc = kRowAlign;
   if (tc > 32768) tc = 32768;
+  if (const char* e = std::getenv("OLIVE_SLAB_ROWS")) {
+    const long long cap = std::atoll(e);
+    if (cap >= kRowAlign && cap % kRowAlign == 0 && cap < tc) tc = cap;
+  }
   if (tc > Tpad) tc = Tpad;
   return tc;
 }
@@ -161,6 +167,32 @@ size_t bwd_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype) {
 }
 BwdWs carve_bwd(void* ws, int64_t T, int64_t d, int64_t V, int grad_dtype) {
   return carve_bwd_impl(ws, T, d, V, grad_dtype, nullptr);
+}
+
+static FbWs carve_fb_impl(void* ws, int64_t T, int64_t d, int64_t V, int grad_dtype,
+                          size_t* total) {
+  const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
+  const int64_t vt = ceil_div(V, 256);
+  Carver c{static_cast<char*>(ws)};
+  FbWs w;
+  w.tc = slab_rows(Tpad, V);
+  w.hc = c.take(2ull * Tpad * d);
+  w.g = c.take(2ull * w.tc * vpad(V));
+  w.part_zm = static_cast<float*>(c.take(4ull * w.tc * vt));
+  w.part_zs = static_cast<float*>(c.take(4ull * w.tc * vt));
+  w.zy = static_cast<float*>(c.take(4ull * w.tc));
+  w.nll = static_cast<float*>(c.take(4ull * Tpad));
+  w.dw_acc = grad_dtype == OLIVE_DTYPE_BF16 ? static_cast<float*>(c.take(4ull * V * d)) : nullptr;
+  if (total) *total = c.off;
+  return w;
+}
+size_t fb_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype) {
+  size_t n = 0;
+  carve_fb_impl(nullptr, T, d, V, grad_dtype, &n);
+  return n;
+}
+FbWs carve_fb(void* ws, int64_t T, int64_t d, int64_t V, int grad_dtype) {
+  return carve_fb_impl(ws, T, d, V, grad_dtype, nullptr);
 }
 
 // the backward's regions, then coef [T] and val [T, 16] of the top-K KL gradient
@@ -245,6 +277,9 @@ size_t olive_workspace_size(int op, int32_t T, int32_t d, int32_t d_t, int32_t V
       if (!width_ok(d_t)) return 0;
       return kl_ws_bytes(T, d, d_t, V, grad);
     case OLIVE_OP_TOPK_FWD: return topk_ws_bytes(T, d);
+    case OLIVE_OP_LOSS_FWD_BWD:
+      if (grad_dtype != OLIVE_DTYPE_BF16 && grad_dtype != OLIVE_DTYPE_F32) return 0;
+      return fb_ws_bytes(T, d, V, grad_dtype);
     case OLIVE_OP_TOPK_KL_BWD:
       if (grad_dtype != OLIVE_DTYPE_BF16 && grad_dtype != OLIVE_DTYPE_F32) return 0;
       return topk_kl_bwd_ws_bytes(T, d, V, grad_dtype);
@@ -401,6 +436,31 @@ olive_status olive_token_loss_bwd(const void* hidden, const void* W, const int32
   if (st != OLIVE_OK) return st;
   return launch_loss_bwd(c, hidden, W, targets, rows, n_rows, T, d, V, inv_tau, reduction, lse,
                          grad_loss, d_hidden, d_W, grad_dtype, workspace, dev_status);
+}
+
+olive_status olive_token_loss_fwd_bwd(const void* hidden, const void* W, const int32_t* targets,
+                                      const int32_t* rows, const int32_t* n_rows, int32_t T,
+                                      int32_t d, int32_t V, float inv_tau, int reduction,
+                                      const float* grad_loss, float* logp, float* lse, float* loss,
+                                      void* d_hidden, void* d_W, int grad_dtype, void* workspace,
+                                      size_t ws_bytes, int32_t* dev_status, void* stream) {
+  if (!hidden || !W || !targets || !rows || !n_rows || !grad_loss || !logp || !lse || !loss ||
+      !d_hidden || !d_W || !dev_status)
+    return OLIVE_ERR_INVALID_ARG;
+  if (reduction != OLIVE_REDUCE_SUM && reduction != OLIVE_REDUCE_MEAN) return OLIVE_ERR_INVALID_ARG;
+  if (grad_dtype != OLIVE_DTYPE_BF16 && grad_dtype != OLIVE_DTYPE_F32) return OLIVE_ERR_INVALID_ARG;
+  if (T < 1 || V < 1 || d < 1 || d > kMaxDim) return OLIVE_ERR_SHAPE;
+  if (!(inv_tau > 0.f) || !std::isfinite(inv_tau)) return OLIVE_ERR_INVALID_ARG;
+  if (d % 8 != 0 || !aligned16(hidden) || !aligned16(W) || !aligned16(d_hidden) || !aligned16(d_W))
+    return OLIVE_ERR_ALIGNMENT;
+  olive_status st = check_ws(workspace, ws_bytes, fb_ws_bytes(T, d, V, grad_dtype));
+  if (st != OLIVE_OK) return st;
+  Ctx c;
+  st = make_ctx(stream, &c);
+  if (st != OLIVE_OK) return st;
+  return launch_loss_fwd_bwd(c, hidden, W, targets, rows, n_rows, T, d, V, inv_tau, reduction,
+                             grad_loss, logp, lse, loss, d_hidden, d_W, grad_dtype, workspace,
+                             dev_status);
 }
 
 olive_status olive_token_divergence(const void* h_s, const void* W_s, int32_t d_s, const void* h_t,

@@ -52,6 +52,22 @@ __host__ __device__ inline Split choose_split(int n, int vt, int ctas) {
   return s;
 }
 
+// Slabs of the G buffer: n masked rows are cut into n_slabs equal slabs of
+// at most tc rows (rps rows each, a multiple of 128); slab s covers compacted
+// rows [row0, row0 + in_s).  Shared by every kernel that works on one slab.
+struct SlabPlan {
+  int n_slabs, rps;
+  __host__ __device__ SlabPlan(int n, int tc) {
+    n_slabs = n > 0 ? (n + tc - 1) / tc : 1;
+    const int per = (n + n_slabs - 1) / n_slabs;
+    rps = (per + 127) / 128 * 128;
+  }
+  __host__ __device__ int rows_in(int n, int s) const {
+    const int r = n - s * rps;
+    return r < 0 ? 0 : (r > rps ? rps : r);
+  }
+};
+
 __device__ inline int read_n_rows(const int32_t* n_rows, int T, int32_t* dev_status) {
   int n = *n_rows;
   if (n < 0 || n > T) {

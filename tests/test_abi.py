@@ -170,6 +170,26 @@ def test_new_entry_points_validation(L):
         "logprob_fwd", 4096, 4096, 151936)
 
 
+def test_fwd_bwd_validation(L):
+    keep, p = _fake()
+    P = ctypes.c_void_p
+    ws = B.olive_workspace_size("loss_fwd_bwd", 64, 64, 100, grad_dtype=torch.bfloat16)
+    assert ws >= B.olive_workspace_size("loss_bwd", 64, 64, 100, grad_dtype=torch.bfloat16) - 4096
+
+    def call(**kw):
+        a = dict(gl=P(p), red=0, dt=0, dh=P(p), d=64, ws_bytes=ws)
+        a.update(kw)
+        return L.olive_token_loss_fwd_bwd(P(p), P(p), P(p), P(p), P(p), 64, a["d"], 100, 1.0,
+                                          a["red"], a["gl"], P(p), P(p), P(p), a["dh"], P(p),
+                                          a["dt"], P(p), a["ws_bytes"], P(p), None)
+    assert call(gl=None) == 1
+    assert call(red=3) == 1 and call(dt=2) == 1
+    assert call(d=60) == 3 and call(dh=P(p + 2)) == 3
+    assert call(ws_bytes=ws - 1) == 9
+    if not torch.cuda.is_available():
+        assert call() in (7, 8)
+
+
 def test_binding_rejects_cpu_tensors(L):
     h = torch.zeros(8, 64, dtype=torch.bfloat16)
     with pytest.raises(TypeError):

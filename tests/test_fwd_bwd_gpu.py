@@ -1,0 +1,178 @@
+"""olive_token_loss_fwd_bwd (CUDA: forward and backward of Eq. (osd-ce) in one
+pass over the logits) against the oracle's token_logprob and token_loss_bwd."""
+
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_36246_gb300 import binding as B
+from paper_2609_36246_gb300 import synth
+from tests.parity import (assert_close_grad, assert_close_logp, assert_close_loss, gpu_pack,
+                          oracle_pack, rel_frob, sample_rows, to_f32, to_f64)
+
+pytestmark = pytest.mark.gpu
+
+
+def _gpu(b, h, W, inv_tau=1.0, reduction="sum", grad_loss=1.0, grad_dtype=torch.bfloat16):
+    g = gpu_pack(b)
+    hc, Wc = h.cuda(), W.cuda()
+    st = g["dev_status"]
+    gl = torch.tensor([grad_loss], dtype=torch.float32, device="cuda")
+    logp, lse, loss, dh, dw = B.olive_token_loss_fwd_bwd(hc, Wc, g["targets"], g["rows"], g["n_rows"],
+                                                         gl, inv_tau, reduction, grad_dtype,
+                                                         dev_status=st)
+    torch.cuda.synchronize()
+    assert B.status_bits(st) == []
+    return (logp.cpu().numpy(), lse.cpu().numpy(), float(loss.item()), dh.float().cpu().numpy(),
+            dw.float().cpu().numpy())
+
+
+def _full_check(b, h, W, **kw):
+    logp, lse, loss, dh, dw = _gpu(b, h, W, **kw)
+    o = oracle_pack(b)
+    tau, red = kw.get("inv_tau", 1.0), kw.get("reduction", "sum")
+    rl, rlse, rloss = oracle.token_logprob(to_f64(h), to_f64(W), o["targets"], o["rows"], tau, red)
+    assert_close_logp(logp, rl)
+    assert_close_logp(lse[o["rows"]], rlse[o["rows"]], "lse")
+    assert_close_loss(loss, rloss)
+    rdh, rdw = oracle.token_loss_bwd(to_f64(h), to_f64(W), o["targets"], o["rows"], tau, red,
+                                     kw.get("grad_loss", 1.0))
+    assert_close_grad(dh, rdh, "dH")
+    assert_close_grad(dw, rdw, "dW")
+    off = np.setdiff1d(np.arange(b.T), o["rows"])
+    assert not dh[off].any() and not logp[off].any()
+    return logp, dh, dw
+
+
+def test_tiny_workload_full():
+    b = synth.make_batch("tiny")
+    _full_check(b, synth.make_hidden("tiny", b.T), synth.make_weight("tiny"))
+
+
+@pytest.mark.parametrize("S,V,d,kw", [
+    (3, 4097, 64, dict()),
+    (5, 300, 72, dict(inv_tau=0.7, reduction="mean", grad_loss=2.5)),
+    (8, 1000, 128, dict(grad_dtype=torch.float32)),
+    (12, 5000, 256, dict(reduction="mean", grad_dtype=torch.float32)),
+    (4, 700, 320, dict(inv_tau=1.2)),  # d = 320: a partial 256-wide output tile
+    (7, 13, 24, dict()),               # V below one 8-wide vector group
+])
+def test_random_shapes(S, V, d, kw):
+    b, h, W = synth.random_case(S * 17 + V, S, V, d, max_prefix=30, max_cont=80, std_w=0.08)
+    _full_check(b, h, W, **kw)
+
+
+def test_single_entry_vocabulary():
+    rng = np.random.default_rng(4)
+    b = synth.batch_from_lengths(rng, [3, 5], [7, 4], 1)
+    h = synth.normal_bf16(rng, (b.T, 64), 1.0)
+    W = synth.normal_bf16(rng, (1, 64), 0.3)
+    logp, _, loss, dh, dw = _gpu(b, h, W, grad_dtype=torch.float32)
+    # log p = 0 and G = p - 1 = 0 in real arithmetic; fp32 leaves a few ulp
+    assert np.abs(logp).max() <= 1e-6 and abs(loss) <= 1e-5
+    assert np.abs(dh).max() <= 1e-5 and np.abs(dw).max() <= 1e-5
+
+
+def test_matches_the_two_call_path():
+    b, h, W = synth.random_case(77, 6, 3001, 128, max_prefix=40, max_cont=200, std_w=0.1)
+    logp, dh, dw = _full_check(b, h, W, grad_dtype=torch.float32)
+    g = gpu_pack(b)
+    hc, Wc = h.cuda(), W.cuda()
+    l2, lse2, _ = B.olive_token_logprob_fwd(hc, Wc, g["targets"], g["rows"], g["n_rows"])
+    gl = torch.ones(1, dtype=torch.float32, device="cuda")
+    dh2, dw2 = B.olive_token_loss_bwd(hc, Wc, g["targets"], g["rows"], g["n_rows"], lse2, gl,
+                                      grad_dtype=torch.float32)
+    assert np.abs(logp - l2.cpu().numpy()).max() <= 1e-4
+    assert rel_frob(dh, dh2.cpu().numpy()) <= 5e-3
+    assert rel_frob(dw, dw2.cpu().numpy()) <= 5e-3
+
+
+@pytest.mark.parametrize("slab_rows,grad_dtype", [(256, torch.float32), (384, torch.bfloat16)])
+def test_several_slabs(slab_rows, grad_dtype, monkeypatch):
+    """A lowered slab cap splits ~2.3k masked rows into many slabs: dW
+    accumulates across them (fp32 accumulator for a bf16 output)."""
+    monkeypatch.setenv("OLIVE_SLAB_ROWS", str(slab_rows))
+    rng = np.random.default_rng(slab_rows)
+    b = synth.batch_from_lengths(rng, [5, 40, 1], [900, 700, 750], 2000)
+    h = synth.normal_bf16(rng, (b.T, 64), 1.0)
+    W = synth.normal_bf16(rng, (2000, 64), 0.1)
+    assert b.n_mask > 6 * slab_rows
+    _full_check(b, h, W, reduction="mean", grad_dtype=grad_dtype)
+
+
+def test_empty_mask():
+    rng = np.random.default_rng(22)
+    b = synth.batch_from_lengths(rng, [9, 4], [0, 0], 300)
+    h = synth.normal_bf16(rng, (b.T, 64), 1.0)
+    W = synth.normal_bf16(rng, (300, 64), 0.1)
+    logp, _, loss, dh, dw = _gpu(b, h, W, reduction="mean")
+    assert loss == 0.0 and not logp.any() and not dh.any() and not dw.any()
+
+
+def test_confident_rows_keep_their_accuracy():
+    """Targets equal to a dominant logit (p_y close to 1): G_y = g (p_y - 1) is
+    small and formed from the fp32 target logit (a bf16-rounded p_y would be
+    off by up to 2^-9 p_y), so each such row's dH keeps the gradient tolerance
+    on its own.  Rows with 1 - p_y below ~1e-4 are left out: there fp32 itself
+    (an ulp of the logit against 1 - p_y) bounds every implementation."""
+    rng = np.random.default_rng(5)
+    P, C, V, d = 40, 300, 1000, 64
+    h = synth.normal_bf16(rng, (P + C, d), 1.0)
+    W = synth.normal_bf16(rng, (V, d), 1.2)
+    z = oracle.logits(to_f64(h), to_f64(W), 1.0)
+    cont = np.argmax(z[P - 1:P + C - 1], axis=1)          # the target of row P-1+i is cont[i]
+    b = synth.Batch(rng.integers(0, V, size=P).astype(np.int32), np.array([0, P], np.int32),
+                    cont.astype(np.int32), np.array([0, C], np.int32), V)
+    logp, dh, _ = _full_check(b, h, W, grad_dtype=torch.float32)
+    o = oracle_pack(b)
+    rdh, _ = oracle.token_loss_bwd(to_f64(h), to_f64(W), o["targets"], o["rows"])
+    conf = [t for t in o["rows"] if -0.3 < logp[t] < -1e-2]
+    assert len(conf) >= 30
+    for t in conf:
+        assert rel_frob(dh[t], rdh[t]) <= 2e-2, t
+
+
+@pytest.mark.slow
+def test_medium_vocab_sampled():
+    """~8k masked rows, d = 4096, V = 32003: logp everywhere, dH on sampled
+    rows and dW on sampled vocabulary rows."""
+    rng = np.random.default_rng(31)
+    b = synth.batch_from_lengths(rng, [1000, 777, 2048], [3000, 2500, 2700], 32003)
+    h = synth.rms_hidden_bf16(rng, (b.T, 4096))
+    W = synth.normal_bf16(rng, (32003, 4096), 0.02)
+    logp, _, loss, dh, dw = _gpu(b, h, W, reduction="mean")
+    o = oracle_pack(b)
+    rows = sample_rows(o["rows"], 24, seed=3)
+    rl, _, _ = oracle.token_logprob(to_f32(h), to_f32(W), o["targets"], rows)
+    assert_close_logp(logp[rows], rl[rows])
+    ref = oracle.token_loss_bwd_rows(to_f32(h), to_f32(W), o["targets"], rows, reduction="mean",
+                                     n_mask=o["n_rows"])
+    assert rel_frob(dh[rows], ref) <= 1e-2
+    vocab = np.unique(np.concatenate([[int(o["targets"][o["rows"][0]]), 0, 32002],
+                                      np.random.default_rng(4).integers(0, 32003, size=13)]))
+    refw = oracle.token_loss_bwd_vocab(to_f32(h), to_f32(W), o["targets"], o["rows"], vocab,
+                                       reduction="mean")
+    assert rel_frob(dw[vocab], refw) <= 1e-2
+    assert np.isclose(loss, -logp[o["rows"]].astype(np.float64).mean(), rtol=1e-5)
+
+
+@pytest.mark.slow
+def test_fwdbwd_workload_sampled():
+    """8 x 4096 tokens, d = 4096, V = 151936 (the timed step's configuration)."""
+    b = synth.make_batch("fwdbwd")
+    h = synth.make_hidden("fwdbwd", b.T)
+    W = synth.make_weight("fwdbwd")
+    logp, _, loss, dh, dw = _gpu(b, h, W)
+    o = oracle_pack(b)
+    rows = sample_rows(o["rows"], 24, seed=1)
+    rl, _, _ = oracle.token_logprob(to_f32(h), to_f32(W), o["targets"], rows)
+    assert_close_logp(logp[rows], rl[rows])
+    ref = oracle.token_loss_bwd_rows(to_f32(h), to_f32(W), o["targets"], rows)
+    assert rel_frob(dh[rows], ref) <= 1e-2
+    off = np.setdiff1d(np.arange(b.T), o["rows"])
+    assert not dh[off].any()
+    # sum over the vocabulary of dW is sum_r G[r, :] . hc[r] with sum_v G[r, v] = 0
+    assert np.abs(dw.astype(np.float64).sum(axis=0)).max() <= 2e-2 * np.abs(dw).sum(axis=0).max()
+    assert np.isclose(loss, -logp[o["rows"]].astype(np.float64).sum(), rtol=1e-5)
