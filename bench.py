@@ -1,15 +1,18 @@
 """Throughput of the OLIVE per-token training path on GB300.
 
 One step = the whole hot path over one packed batch: splice/pack of the
-spliced sequences (student prefix || teacher continuation), the LM-head
-forward with online log-sum-exp and the masked continuation loss of Eq.
-(osd-ce), and its backward (d hidden, d W in bf16).  Workload: 8 sequences of
+spliced sequences (student prefix || teacher continuation), then one
+olive_token_loss_fwd_bwd call: the LM-head forward with online log-sum-exp
+and the masked continuation loss of Eq. (osd-ce) (log-probs, lse, loss) and
+its backward (d hidden, d W in bf16), each logit tile computed once.  Workload: 8 sequences of
 4096 tokens, cut ~ U[256, 3840), d = 4096, V = 151936, bf16, synthetic seeded
 data (the "fwdbwd" workload of paper_2609_36246_gb300.synth).
 
 Metric: masked continuation tokens per second, i.e. N_mask * steps / time,
 and the fraction of bf16 dense tensor peak of the counted work
-6 * N_mask * d * V FLOPs per step (logit recomputation is not counted).
+6 * N_mask * d * V FLOPs per step (forward product, dH and dW products).
+The two-call path (olive_token_logprob_fwd + olive_token_loss_bwd, which
+recomputes the logits) is timed beside it for comparison.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -181,8 +184,8 @@ def run_ours(args, world, rank, local):
     hidden = hid_h.to(dev)
     W = W_cpu.to(dev)
     st = B.new_status(dev)
-    ws_f = B.workspace(B.olive_workspace_size("logprob_fwd", T, d, V), dev)
-    ws_b = B.workspace(B.olive_workspace_size("loss_bwd", T, d, V, grad_dtype=torch.bfloat16), dev)
+    ws_fb = B.workspace(B.olive_workspace_size("loss_fwd_bwd", T, d, V, grad_dtype=torch.bfloat16),
+                        dev)
     logp = torch.empty(T, dtype=torch.float32, device=dev)
     lse = torch.empty_like(logp)
     loss = torch.empty(1, dtype=torch.float32, device=dev)
@@ -192,26 +195,23 @@ def run_ours(args, world, rank, local):
     loss_h = torch.empty(1, dtype=torch.float32).pin_memory()
     stream = torch.cuda.current_stream()
 
-    ev = {k: [] for k in ("splice", "fwd", "bwd")}
+    ev = {k: [] for k in ("splice", "fwd_bwd")}
 
     def step(timed: bool, host_io: bool = False):
         if host_io:
             for dst, src in ((pre, pre_h), (poff, poff_h), (con, con_h), (coff, coff_h), (hidden, hid_h)):
                 dst.copy_(src, non_blocking=True)
-        e = [torch.cuda.Event(enable_timing=True) for _ in range(4)] if timed else None
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(3)] if timed else None
         if e: e[0].record(stream)
         pk = B.olive_splice_pack(pre, poff, con, coff, V, T, dev_status=st)
         if e: e[1].record(stream)
-        B.olive_token_logprob_fwd(hidden, W, pk["targets"], pk["rows"], pk["n_rows"], 1.0, "sum",
-                                  ws=ws_f, dev_status=st, out=(logp, lse, loss))
-        if e: e[2].record(stream)
-        B.olive_token_loss_bwd(hidden, W, pk["targets"], pk["rows"], pk["n_rows"], lse, gl, 1.0, "sum",
-                               torch.bfloat16, ws=ws_b, dev_status=st, out=(dh, dw))
+        B.olive_token_loss_fwd_bwd(hidden, W, pk["targets"], pk["rows"], pk["n_rows"], gl, 1.0,
+                                   "sum", torch.bfloat16, ws=ws_fb, dev_status=st,
+                                   out=(logp, lse, loss, dh, dw))
         if e:
-            e[3].record(stream)
+            e[2].record(stream)
             ev["splice"].append((e[0], e[1]))
-            ev["fwd"].append((e[1], e[2]))
-            ev["bwd"].append((e[2], e[3]))
+            ev["fwd_bwd"].append((e[1], e[2]))
         if host_io:
             loss_h.copy_(loss, non_blocking=True)
 
@@ -257,24 +257,31 @@ def run_ours(args, world, rank, local):
     assert math.isfinite(float(loss_h.item()))
 
     avg = lambda k: statistics.mean(a.elapsed_time(b2) for a, b2 in ev[k])
-    fwd_ms, bwd_ms, spl_ms = avg("fwd"), avg("bwd"), avg("splice")
+    fb_ms, spl_ms = avg("fwd_bwd"), avg("splice")
     burst, sustained, src = load_peaks()
     counted = 6.0 * N_mask * d * V
     step_tflops = counted / (ms_per_step / 1e3) / 1e12
-    # dominant kernel: the fused backward (one launch per olive_token_loss_bwd
-    # call, bracketed together with its row gather); algorithmic work per
-    # launch = dH + dW = 4 N_mask d V (the logit recomputation is not counted)
-    bwd_flops = 4.0 * N_mask * d * V
-    ach_bwd = bwd_flops / (bwd_ms / 1e3) / 1e12
-    fwd_flops = 2.0 * N_mask * d * V
-    ach_fwd = fwd_flops / (fwd_ms / 1e3) / 1e12
+    # dominant kernel: bwd_fused_kernel, launched twice per call (forward
+    # tiles, then dH/dW tiles); its algorithmic work per call is the forward
+    # product plus dH and dW, 6 N_mask d V, and the call is bracketed by
+    # events on its stream (so the row gather, the convert pass and the loss
+    # reduction count against it)
+    slabs = -(-((T + 127) // 128 * 128) // B.slab_rows_for(T, V))
+    fb_flops = counted
+    ach_fb = fb_flops / (fb_ms / 1e3) / 1e12
     rev = kernel_rev()
     traffic = profile_traffic("bwd_fused_kernel", rev)
-    launches = 2 + 4 + 2  # splice (scan, fill), forward (gather, GEMM, finalize, loss), backward (gather, fused)
+    # splice (scan, fill) + gather + per slab (forward tiles, convert, dH/dW tiles) + loss reduce
+    launches = 2 + 1 + 3 * slabs + 1
+
+    two_call = None
+    if not args.no_extra:
+        two_call = measure_two_call(dev, hidden, W, pk_fn=lambda: B.olive_splice_pack(
+            pre, poff, con, coff, V, T, dev_status=st), T=T, d=d, V=V, n=N_mask, burst=burst)
 
     extra = {}
     if not args.no_extra:
-        del ws_f, ws_b, dh, dw
+        del ws_fb, dh, dw
         torch.cuda.empty_cache()
         extra["kl_divergence"] = measure_kl(dev, burst)
         torch.cuda.empty_cache()
@@ -300,17 +307,16 @@ def run_ours(args, world, rank, local):
         "pct_bf16_peak": 100.0 * step_tflops / burst,
         "pct_bf16_peak_sustained": 100.0 * step_tflops / sustained,
         "counted_tflops_per_s": step_tflops,
-        "phases_ms": {"splice_pack": spl_ms, "logprob_fwd": fwd_ms, "loss_bwd": bwd_ms},
-        "roofline": {"kernel": "bwd_fused_kernel (recompute + G, dH, dW tiles)", "bound": "tensor",
-                     "achieved": ach_bwd, "peak": sustained, "unit": "TFLOP/s",
-                     "frac": ach_bwd / sustained, "traffic": traffic,
+        "phases_ms": {"splice_pack": spl_ms, "loss_fwd_bwd": fb_ms},
+        "roofline": {"kernel": "bwd_fused_kernel (forward tiles + dH/dW tiles, 2 launches per call)",
+                     "bound": "tensor", "achieved": ach_fb, "peak": sustained, "unit": "TFLOP/s",
+                     "frac": ach_fb / sustained, "traffic": traffic,
                      "peak_source": f"{src} bf16_tflops_sustained",
-                     "flops_per_launch": bwd_flops, "kernel_rev": rev,
-                     "note": "algorithmic FLOPs exclude the logit recomputation (1/3 of executed)"},
-        "roofline_fwd": {"kernel": "gemm_persistent<FwdKern> (LM-head forward + online LSE)",
-                         "bound": "tensor", "achieved": ach_fwd, "peak": sustained,
-                         "unit": "TFLOP/s", "frac": ach_fwd / sustained,
-                         "traffic": profile_traffic("FwdKern", rev), "flops_per_launch": fwd_flops},
+                     "flops_per_call": fb_flops, "kernel_rev": rev,
+                     "note": "per olive_token_loss_fwd_bwd call (its two bwd_fused_kernel launches, "
+                             "timed with the gather, convert and loss kernels around them); "
+                             "traffic is DRAM bytes of both launches"},
+        "two_call_path": two_call,
         "e2e": e2e,
         "gpu_launches": launches * args.steps,
         "clocks": clk.summary(),
@@ -383,6 +389,35 @@ def measure_kl(dev, burst: float, steps: int = 3):
             "pct_bf16_peak": 100.0 * flops / (ms / 1e3) / 1e12 / burst, "steps": steps}
 
 
+def measure_two_call(dev, hidden, W, pk_fn, T, d, V, n, burst, steps: int = 3):
+    """The same step through olive_token_logprob_fwd + olive_token_loss_bwd
+    (the backward recomputes every logit tile), for comparison."""
+    from paper_2609_36246_gb300 import binding as B
+    ws_f = B.workspace(B.olive_workspace_size("logprob_fwd", T, d, V), dev)
+    ws_b = B.workspace(B.olive_workspace_size("loss_bwd", T, d, V), dev)
+    st = B.new_status(dev)
+    gl = torch.ones(1, dtype=torch.float32, device=dev)
+    out_f = (torch.empty(T, device=dev), torch.empty(T, device=dev), torch.empty(1, device=dev))
+    out_b = (torch.empty(T, d, dtype=torch.bfloat16, device=dev),
+             torch.empty(V, d, dtype=torch.bfloat16, device=dev))
+
+    def step():
+        pk = pk_fn()
+        _, lse, _ = B.olive_token_logprob_fwd(hidden, W, pk["targets"], pk["rows"], pk["n_rows"],
+                                              ws=ws_f, dev_status=st, out=out_f)
+        B.olive_token_loss_bwd(hidden, W, pk["targets"], pk["rows"], pk["n_rows"], lse, gl,
+                               ws=ws_b, dev_status=st, out=out_b)
+
+    ms = time_calls(step, steps, 1)
+    if int(st.item()) != 0:
+        raise RuntimeError(f"two-call status {B.status_bits(st)}")
+    del ws_f, ws_b, out_b
+    torch.cuda.empty_cache()
+    return {"workload": "same batch, forward + recomputing backward (two calls)",
+            "value": n / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
+            "pct_bf16_peak": 100.0 * 6.0 * n * d * V / (ms / 1e3) / 1e12 / burst, "steps": steps}
+
+
 def measure_topk_kl(dev, burst: float, steps: int = 3):
     """OPD with the top-16 KL: student and teacher entropy/top-16 sweeps, the
     top-16 compare (overlap, truncated KL, teacher log-probs at the student's
@@ -452,8 +487,9 @@ def measure_scoring(dev, burst: float, steps: int = 5):
 
 
 def measure_varlen(dev, burst: float, steps: int = 2):
-    """splice/pack + forward + backward on the variable-length batch
-    (64 sequences, lengths U[1024,16384], ~557k packed tokens)."""
+    """splice/pack + olive_token_loss_fwd_bwd on the variable-length batch
+    (64 sequences, lengths U[1024,16384], ~557k packed tokens; the masked
+    rows span many G slabs)."""
     from paper_2609_36246_gb300 import binding as B
     from paper_2609_36246_gb300 import synth
     b = synth.make_batch("varlen")
@@ -461,20 +497,17 @@ def measure_varlen(dev, burst: float, steps: int = 2):
     h, W = gpu_inputs(23, T, d, V, dev)
     i32 = lambda a: torch.from_numpy(np.ascontiguousarray(a, dtype=np.int32)).to(dev)
     pre, poff, con, coff = i32(b.prefix_ids), i32(b.prefix_off), i32(b.cont_ids), i32(b.cont_off)
-    ws_f = B.workspace(B.olive_workspace_size("logprob_fwd", T, d, V), dev)
-    ws_b = B.workspace(B.olive_workspace_size("loss_bwd", T, d, V), dev)
+    ws = B.workspace(B.olive_workspace_size("loss_fwd_bwd", T, d, V), dev)
     st = B.new_status(dev)
     gl = torch.ones(1, dtype=torch.float32, device=dev)
-    out_f = (torch.empty(T, device=dev), torch.empty(T, device=dev), torch.empty(1, device=dev))
-    out_b = (torch.empty(T, d, dtype=torch.bfloat16, device=dev),
-             torch.empty(V, d, dtype=torch.bfloat16, device=dev))
+    out = (torch.empty(T, device=dev), torch.empty(T, device=dev), torch.empty(1, device=dev),
+           torch.empty(T, d, dtype=torch.bfloat16, device=dev),
+           torch.empty(V, d, dtype=torch.bfloat16, device=dev))
 
     def step():
         pk = B.olive_splice_pack(pre, poff, con, coff, V, T, dev_status=st)
-        _, lse, _ = B.olive_token_logprob_fwd(h, W, pk["targets"], pk["rows"], pk["n_rows"], 1.0,
-                                              "mean", ws=ws_f, dev_status=st, out=out_f)
-        B.olive_token_loss_bwd(h, W, pk["targets"], pk["rows"], pk["n_rows"], lse, gl, 1.0, "mean",
-                               torch.bfloat16, ws=ws_b, dev_status=st, out=out_b)
+        B.olive_token_loss_fwd_bwd(h, W, pk["targets"], pk["rows"], pk["n_rows"], gl, 1.0, "mean",
+                                   torch.bfloat16, ws=ws, dev_status=st, out=out)
 
     ms = time_calls(step, steps, 1)
     if int(st.item()) != 0:
