@@ -37,6 +37,12 @@ bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t
 // Rows of the G slab used by the backward passes for vocabulary size V.
 int64_t slab_rows(int64_t Tpad, int64_t V);
 inline int64_t vpad(int64_t V) { return align_up(static_cast<size_t>(V), 8); }
+// Slab rows of the forward-KL gradient, whose fp32 slab holds pairs: half of
+// tc in whole 128-row tiles, at least one tile.
+inline int64_t kl_pair_rows(int64_t tc) {
+  const int64_t h = tc / 2 / kRowAlign * kRowAlign;
+  return h > kRowAlign ? h : kRowAlign;
+}
 
 // ---- workspace carving (sizes in bytes; every region 256-byte aligned) ----
 struct FwdWs {
@@ -88,10 +94,11 @@ FbWs carve_fb(void* ws, int64_t T, int64_t d, int64_t V, int grad_dtype);
 struct KlWs {
   void* hcs;      // bf16 [Tpad, d_s]
   void* hct;      // bf16 [Tpad, d_t]
-  float* part;    // [5, kSvMax, Tpad]
-  float* stats;   // [3, Tpad]: lse_s, lse_t, kl per compacted row
-  void* g;        // bf16 [Tc, Vpad] (gradient only)
-  uint32_t* counters;  // tile-scheduler counters (gradient only)
+  float* part;    // [5, kSvMax, Tpad] (value only)
+  float* stats;   // [3, Tpad]: lse_s, lse_t, kl per compacted row (value only)
+  void* g;        // bf16 [Tc, Vpad]: e_s, then G (gradient only)
+  float* s2;      // fp32 [Tc, Vpad]: second slab (gradient only)
+  float* part5;   // [5, Tc, ceil(V/256)] per-tile partials (gradient only)
   int64_t tc;
 };
 size_t kl_ws_bytes(int64_t T, int64_t ds, int64_t dt, int64_t V, int grad);
@@ -191,13 +198,13 @@ olive_status launch_divergence(const Ctx& c, const void* h_s, const void* W_s, i
 // Words of tile-scheduler counters the fused backward needs.
 size_t bwd_counter_words(int64_t Tpad, int64_t tc);
 
-// Divergence backward (fused kernel): d_h_s from the compacted student and
-// teacher rows, the per-row statistics of the forward and a G buffer of tc rows.
-olive_status launch_kl_bwd(const Ctx& c, const void* hcs, const void* hct, const void* W_s,
-                           int32_t d_s, const void* W_t, int32_t d_t, const int32_t* rows,
-                           const int32_t* n_rows, int32_t T, int32_t V, float inv_tau, int reverse,
-                           const float* grad_kl, const float* stats, int32_t ld_stats, void* g,
-                           int64_t tc, uint32_t* counters, void* d_h_s, int grad_dtype,
-                           int32_t* dev_status);
+// Divergence forward + d_h_s in one pass over the logits (fused kernel,
+// per slab: KLZ tiles, conv_kl_kernel, DH tiles); writes kl[t] too.
+olive_status launch_kl_fwd_bwd(const Ctx& c, const void* hcs, const void* hct, const void* W_s,
+                               int32_t d_s, const void* W_t, int32_t d_t, const int32_t* rows,
+                               const int32_t* n_rows, int32_t T, int32_t V, float inv_tau,
+                               int reverse, const float* grad_kl, float* kl, void* g, float* s2,
+                               float* part5, int64_t tc, void* d_h_s, int grad_dtype,
+                               int32_t* dev_status);
 
 }  // namespace olive

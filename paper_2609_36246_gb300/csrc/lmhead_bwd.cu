@@ -8,7 +8,8 @@
 //   dW = G^T . hc     (M = V,    N = d, K = rows)
 // Divergence (OPD's per-token KL, Section 1): G = g_t inv_tau p_s
 // (log p_s - log p_t - KL_t) (reverse) or g_t inv_tau (p_s - p_t) (forward),
-// and dH_s = G . W_s.
+// and dH_s = G . W_s; it always runs in the single-pass form below (KLZ
+// tiles, conv_kl_kernel, DH tiles).
 // Top-K truncated reverse KL (OPD's top-16 approximation as read here, the
 // student's top-K set S held fixed): with l = log p_s, q = log p_t at the ids
 // of S, P_S = sum_S p_s and KL_K the forward value,
@@ -24,8 +25,7 @@
 // workspace.  The masked rows are split into equal slabs of <= tc_max rows;
 // per slab the work is a list of tiles of three kinds, all 128 x 256 fp32
 // accumulators in TMEM:
-//   GRAD    z = hc . W^T (K = d; KL: two products, student and teacher, into
-//           the two 256-column halves of TMEM) -> G tile (bf16) in the slab
+//   GRAD    z = hc . W^T (K = d) -> G tile (bf16) in the slab
 //   DH      G . W  (A = G K-major, B = W MN-major, K = V) -> d_hidden rows
 //   DW      G^T . hc (A = G MN-major, B = hc MN-major, K = slab rows) -> dW
 //           (CE only; stored directly in the output dtype when there is one
@@ -49,7 +49,15 @@
 // term, and turns the slab into G in place (G = g inv_tau (e 2^(m_tile -
 // lse2) - [v == y]), the target entry from the exact fp32 z_y); a second
 // launch runs the DH and DW tiles of the slab.  The launches are stream
-// ordered, so these phases need no tile counters.
+// ordered, so these phases need no tile counters.  The divergence gradient
+// uses the same phases with KLZ tiles (two products per tile, student and
+// teacher, in the two 256-column halves of one TMEM accumulator) and five
+// per-tile partials, from which conv_kl_kernel forms KL and G.  Reverse KL:
+// e_s = 2^(x_s - m_s) in bf16 in the G slab and x_s - x_t in an fp32 slab
+// (G is proportional to p_s, so a bf16 p_s only adds G's own rounding).
+// Forward KL: G = p_s - p_t cancels where the models agree, so both local
+// logits x_s - m_s and x_t - m_t stay fp32 (pairs, in half as many slab rows
+// so the workspace is the same).
 #include <cmath>
 
 #include "gemm_core.cuh"
@@ -63,7 +71,7 @@ constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kBN = 256;
 constexpr int kStages = 4;
 
-enum Kind : int { K_NONE = -1, K_GRAD = 0, K_KLGRAD = 1, K_DH = 2, K_DW = 3, K_ZSAVE = 4 };
+enum Kind : int { K_NONE = -1, K_GRAD = 0, K_KLZ = 1, K_DH = 2, K_DW = 3, K_ZSAVE = 4 };
 // phases: one launch of every tile kind with dependency waits, or one slab's
 // forward (ZSAVE) tiles, or one slab's DH and DW tiles
 enum Phase : int { PH_ALL = 0, PH_Z = 1, PH_DHDW = 2 };
@@ -84,7 +92,6 @@ struct BwdParams {
   const int32_t* targets;    // CE
   const float* lse;          // CE, indexed by packed row
   const float* grad_loss;    // CE, device scalar
-  const float* grad_kl;      // KL, [T]
   const float* sp_coef;      // top-K KL, [T]: softmax coefficient per row
   const float* sp_val;       // top-K KL, [T, sp_k]: full G values at the ids of S
   const int32_t* sp_ids;     // top-K KL, [T, sp_k]: the ids of S
@@ -93,8 +100,9 @@ struct BwdParams {
   float* part_zm;            // PH_Z: [tc, vt] tile max (base 2) per slab row
   float* part_zs;            // PH_Z: [tc, vt] tile sum of 2^(x - max)
   float* zy_s;               // PH_Z: [tc] target logit (natural units)
-  const float* stats;        // KL, [3][ld_stats]: lse_s, lse_t, kl per compacted row
-  int32_t ld_stats;
+  float* s2;                 // KLZ: fp32 slab, [tc, ldg] (reverse) or [tc / 2, 2 ldg] (forward)
+  float* part5;              // KLZ: [5][tc][vt] m_s, s_s, m_t, s_t, A per (row, tile)
+  int64_t plane5;            // tc * vt
   int32_t kl;                // 0: cross-entropy, 1: divergence
   int32_t reverse;           // KL direction
   int32_t T, d, d2, V, reduction, out_dtype, group_rows;
@@ -187,7 +195,7 @@ __device__ Unit decode(const BwdParams& p, const Plan& pl, int u) {
     if (u < ug) {
       const Raster r{mt, pl.vt, p.group_rows};
       r.tile(u, x.i, x.j);
-      x.kind = p.phase == PH_Z ? K_ZSAVE : (p.kl ? K_KLGRAD : K_GRAD);
+      x.kind = p.phase == PH_Z ? (p.kl ? K_KLZ : K_ZSAVE) : K_GRAD;
       return x;
     }
     u -= ug;
@@ -218,7 +226,7 @@ __device__ __forceinline__ void unit_ksteps(const BwdParams& p, const Unit& x, i
   switch (x.kind) {
     case K_GRAD:
     case K_ZSAVE: nk = (p.d + kBK - 1) / kBK; break;
-    case K_KLGRAD:
+    case K_KLZ:
       nk = (p.d + kBK - 1) / kBK;
       nk2 = (p.d2 + kBK - 1) / kBK;
       break;
@@ -318,24 +326,21 @@ __device__ void epi_grad(const BwdParams& p, const Plan& pl, const Unit& x, int 
   }
 }
 
-__device__ void epi_klgrad(const BwdParams& p, const Unit& x, int row, uint32_t taddr) {
+// divergence forward tile: student (columns [0, 256)) and teacher (columns
+// [256, 512)) logits of one 128 x 256 tile; per row the tile maxima m_s, m_t,
+// sums s_s, s_t of 2^(x - m), A = sum e_p (x_p - x_q) in the primary
+// distribution's scale (p = student for the reverse KL, teacher for the
+// forward KL), e_s in bf16 into the G slab and the fp32 second slab
+__device__ void epi_klz(const BwdParams& p, const Plan& pl, const Unit& x, int row,
+                        uint32_t taddr) {
   const int r_local = x.i * kBM + row;
-  const int r = x.row0 + r_local;
   bool valid = r_local < x.in_s;
-  float ls2 = 0.f, lt2 = 0.f, kl = 0.f, coef = 0.f;
   if (valid) {
-    const int t = p.rows[r];
-    if (t >= 0 && t < p.T) {
-      ls2 = p.stats[0 * static_cast<size_t>(p.ld_stats) + r] * kLog2e;
-      lt2 = p.stats[1 * static_cast<size_t>(p.ld_stats) + r] * kLog2e;
-      kl = p.stats[2 * static_cast<size_t>(p.ld_stats) + r];
-      coef = p.grad_kl[t] * p.inv_tau;
-    } else {
-      valid = false;
-    }
+    const int t = p.rows[x.row0 + r_local];
+    valid = t >= 0 && t < p.T;
   }
-  __nv_bfloat16* grow = p.g + static_cast<size_t>(r_local) * p.ldg;
   const int n0 = x.j * kBN;
+  float ms = -INFINITY, mt = -INFINITY;
 #pragma unroll 1
   for (int c = 0; c < kBN; c += 32) {
     const int col0 = n0 + c;
@@ -344,16 +349,73 @@ __device__ void epi_klgrad(const BwdParams& p, const Unit& x, int row, uint32_t 
     tmem_ld_32x32b_x32(taddr + c, a);
     tmem_ld_32x32b_x32(taddr + kBN + c, b);
     tmem_ld_wait();
-    float g[32];
+    const int nv = p.V - col0;
 #pragma unroll
     for (int k = 0; k < 32; ++k) {
-      const float ys = __uint_as_float(a[k]) * p.scale2 - ls2;  // log2 p_s
-      const float yt = __uint_as_float(b[k]) * p.scale2 - lt2;  // log2 p_t
-      const float ps = fast_exp2(ys);
-      const float v = p.reverse ? ps * ((ys - yt) * kLn2 - kl) : ps - fast_exp2(yt);
-      g[k] = valid ? coef * v : 0.f;
+      if (k < nv) {
+        ms = fmaxf(ms, __uint_as_float(a[k]) * p.scale2);
+        mt = fmaxf(mt, __uint_as_float(b[k]) * p.scale2);
+      }
     }
-    store_row32(grow, col0, OLIVE_DTYPE_BF16, p.V - col0, g);
+  }
+  __nv_bfloat16* grow = p.g + static_cast<size_t>(r_local) * p.ldg;
+  float* srow = p.s2 + static_cast<size_t>(r_local) * p.ldg * (p.reverse ? 1 : 2);
+  float ss = 0.f, st = 0.f, A = 0.f;
+#pragma unroll 1
+  for (int c = 0; c < kBN; c += 32) {
+    const int col0 = n0 + c;
+    if (col0 >= p.V) break;
+    uint32_t a[32], b[32];
+    tmem_ld_32x32b_x32(taddr + c, a);
+    tmem_ld_32x32b_x32(taddr + kBN + c, b);
+    tmem_ld_wait();
+    const int nv = p.V - col0;
+    float e[32];
+#pragma unroll
+    for (int k = 0; k < 32; ++k) {
+      const bool ok = valid && k < nv;
+      const float xs = __uint_as_float(a[k]) * p.scale2;
+      const float xt = __uint_as_float(b[k]) * p.scale2;
+      const float es = ok ? fast_exp2(xs - ms) : 0.f;
+      const float et = ok ? fast_exp2(xt - mt) : 0.f;
+      ss += es;
+      st += et;
+      A += p.reverse ? es * (xs - xt) : et * (xt - xs);
+      e[k] = es;
+    }
+    if (p.reverse) {
+      store_row32(grow, col0, OLIVE_DTYPE_BF16, nv, e);
+#pragma unroll
+      for (int k = 0; k < 32; ++k) {
+        const bool ok = valid && k < nv;
+        e[k] = ok ? (__uint_as_float(a[k]) - __uint_as_float(b[k])) * p.scale2 : 0.f;
+      }
+      store_row32(srow, col0, OLIVE_DTYPE_F32, nv, e);
+    } else {
+      // (x_s - m_s, x_t - m_t) pairs, 16 columns per 32-value store
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        float f[32];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+          const int kk = 16 * h + k;
+          const bool ok = valid && kk < nv;
+          f[2 * k] = ok ? __uint_as_float(a[kk]) * p.scale2 - ms : 0.f;
+          f[2 * k + 1] = ok ? __uint_as_float(b[kk]) * p.scale2 - mt : 0.f;
+        }
+        const int nvh = nv - 16 * h;
+        if (nvh > 0) store_row32(srow, 2 * static_cast<size_t>(col0 + 16 * h), OLIVE_DTYPE_F32,
+                                 2 * (nvh < 16 ? nvh : 16), f);
+      }
+    }
+  }
+  if (valid) {
+    const size_t o = static_cast<size_t>(r_local) * pl.vt + x.j;
+    p.part5[o] = ms;
+    p.part5[p.plane5 + o] = ss;
+    p.part5[2 * p.plane5 + o] = mt;
+    p.part5[3 * p.plane5 + o] = st;
+    p.part5[4 * p.plane5 + o] = A;
   }
 }
 
@@ -568,7 +630,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool dep = true;
         if (p.phase != PH_ALL) {
           // phases are separate launches in stream order: nothing to wait for
-        } else if ((x.kind == K_GRAD || x.kind == K_KLGRAD) && x.s > 0) {
+        } else if (x.kind == K_GRAD && x.s > 0) {
           const int pin = slab_in(pl, x.s - 1);
           const int pmt = (pin + 127) / 128;
           dep = wait_counter(ctr_dhdw(p, x.s - 1),
@@ -594,7 +656,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               tma_load_2d(sA, &maps.m[0], fb, k * kBK, x.row0 + x.i * kBM);
               tma_load_2d(sB, &maps.m[1], fb, k * kBK, x.j * kBN);
               break;
-            case K_KLGRAD: {
+            case K_KLZ: {
               const bool second = k >= nk;
               const int kk = (second ? k - nk : k) * kBK;
               tma_load_2d(sA, &maps.m[second ? 4 : 0], fb, kk, x.row0 + x.i * kBM);
@@ -636,7 +698,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t idesc;
         bool a_mn = false, b_mn = false;
         switch (x.kind) {
-          case K_KLGRAD: idesc = idesc_bf16(kBM, kBN, false, false); break;
+          case K_KLZ: idesc = idesc_bf16(kBM, kBN, false, false); break;
           case K_DH: idesc = idesc_bf16(kBM, kBN, false, true); b_mn = true; break;
           case K_DW: idesc = idesc_bf16(kBM, kBN, true, true); a_mn = b_mn = true; break;
           default: idesc = idesc_bf16(kBM, kBN, false, false); break;
@@ -696,7 +758,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       switch (x.kind) {
         case K_GRAD: epi_grad(p, pl, x, row, taddr); break;
-        case K_KLGRAD: epi_klgrad(p, x, row, taddr); break;
+        case K_KLZ: epi_klz(p, pl, x, row, taddr); break;
         case K_ZSAVE: epi_zsave(p, pl, x, row, taddr); break;
         case K_DH: epi_dh(p, x, row, taddr); break;
         case K_DW: epi_dw(p, pl, x, row, taddr, nk); break;
@@ -710,7 +772,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       __threadfence();
       named_bar_sync(1, kEpiThreads);
       if (row == 0 && p.phase == PH_ALL) {
-        if (x.kind == K_GRAD || x.kind == K_KLGRAD) {
+        if (x.kind == K_GRAD) {
           red_release_add(ctr_row(p, x.s, x.i), 1u);
           red_release_add(ctr_grad(p, x.s), 1u);
         } else {
@@ -819,6 +881,148 @@ __global__ void __launch_bounds__(256)
           h2[e] = __floats2bfloat162_rn(a, b);
         }
         grow[idx] = v[q];
+      }
+    }
+  }
+}
+
+// (max, sum, A) triples: A is scaled like the sum
+__device__ __forceinline__ void lse_merge3(float& m, float& s, float& a, float m2, float s2,
+                                           float a2) {
+  if (m2 == -INFINITY) return;
+  if (m == -INFINITY) {
+    m = m2;
+    s = s2;
+    a = a2;
+    return;
+  }
+  const float mn = fmaxf(m, m2);
+  const float f1 = fast_exp2(m - mn), f2 = fast_exp2(m2 - mn);
+  s = s * f1 + s2 * f2;
+  a = a * f1 + a2 * f2;
+  m = mn;
+}
+
+// One warp per masked row of the slab: merges the KLZ partials into lse_s,
+// lse_t and KL = ln2 A / s_p - lse_p + lse_q (p the primary distribution),
+// writes kl[t], then writes the row of G into the G slab:
+//   reverse: G = coef p_s (ln2 (x_s - x_t) - (lse_s - lse_t) - KL), with
+//            p_s = e_s 2^(m_s - lse2_s) from the slab's own e_s
+//   forward: G = coef (p_s - p_t), both from the fp32 (x - m) pairs
+// with coef = grad_kl[t] inv_tau.
+__global__ void __launch_bounds__(256)
+    conv_kl_kernel(const int32_t* __restrict__ n_rows, const int32_t* __restrict__ rows, int T,
+                   int V, int tc, int slab, int vt, int64_t ldg, float inv_tau, int reverse,
+                   const float* __restrict__ grad_kl, const float* __restrict__ part5,
+                   int64_t plane5, const float* __restrict__ s2, __nv_bfloat16* g,
+                   float* __restrict__ kl) {
+  const int n = read_n_rows(n_rows, T, nullptr);
+  const SlabPlan sp(n, tc);
+  if (slab >= sp.n_slabs) return;
+  const int in_s = sp.rows_in(n, slab);
+  const int row0 = slab * sp.rps;
+  const int lane = threadIdx.x & 31;
+  const int warps = (gridDim.x * blockDim.x) >> 5;
+  const int nvec = (V + 7) / 8;
+  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < in_s; r += warps) {
+    const int t = rows[row0 + r];
+    if (t < 0 || t >= T) continue;  // reported by the gather; the G row is zero
+    const float* pms = part5 + static_cast<size_t>(r) * vt;
+    const float* pss = pms + plane5;
+    const float* pmt = pms + 2 * plane5;
+    const float* pst = pms + 3 * plane5;
+    const float* pa = pms + 4 * plane5;
+    float mp = -INFINITY, sp_ = 0.f, A = 0.f, mq = -INFINITY, sq = 0.f;
+    for (int j = lane; j < vt; j += 32) {
+      if (reverse) {
+        lse_merge3(mp, sp_, A, pms[j], pss[j], pa[j]);
+        lse_merge(mq, sq, pmt[j], pst[j]);
+      } else {
+        lse_merge3(mp, sp_, A, pmt[j], pst[j], pa[j]);
+        lse_merge(mq, sq, pms[j], pss[j]);
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, mp, o);
+      const float s2v = __shfl_xor_sync(0xffffffffu, sp_, o);
+      const float a2 = __shfl_xor_sync(0xffffffffu, A, o);
+      lse_merge3(mp, sp_, A, m2, s2v, a2);
+      const float mq2 = __shfl_xor_sync(0xffffffffu, mq, o);
+      const float sq2 = __shfl_xor_sync(0xffffffffu, sq, o);
+      lse_merge(mq, sq, mq2, sq2);
+    }
+    const float lse2_p = mp + log2f(sp_);
+    const float lse2_q = mq + log2f(sq);
+    const float k = kLn2 * (A / sp_) - (lse2_p - lse2_q) * kLn2;
+    const float lse2_s = reverse ? lse2_p : lse2_q;
+    const float lse2_t = reverse ? lse2_q : lse2_p;
+    if (lane == 0) kl[t] = k;
+    const float coef = grad_kl[t] * inv_tau;
+    const float c0 = (lse2_s - lse2_t) * kLn2 + k;
+    uint4* grow = reinterpret_cast<uint4*>(g + static_cast<size_t>(r) * ldg);
+    if (reverse) {
+      const float4* srow = reinterpret_cast<const float4*>(s2 + static_cast<size_t>(r) * ldg);
+#pragma unroll 1
+      for (int base = 0; base < nvec; base += 64) {
+        uint4 v[2];
+        float4 dl[2][2];
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+          const int idx = base + 32 * q + lane;
+          if (idx < nvec) {
+            v[q] = grow[idx];
+            dl[q][0] = srow[2 * idx];
+            dl[q][1] = srow[2 * idx + 1];
+          }
+        }
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+          const int idx = base + 32 * q + lane;
+          if (idx >= nvec) continue;
+          const float scs = coef * fast_exp2(pms[(base >> 5) + q] - lse2_s);
+          const float dd[8] = {dl[q][0].x, dl[q][0].y, dl[q][0].z, dl[q][0].w,
+                               dl[q][1].x, dl[q][1].y, dl[q][1].z, dl[q][1].w};
+          __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&v[q]);
+          const int col = idx * 8;
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float2 u = __bfloat1622float2(h2[e]);
+            float a = scs * u.x * (kLn2 * dd[2 * e] - c0);
+            float b = scs * u.y * (kLn2 * dd[2 * e + 1] - c0);
+            if (col + 2 * e >= V) a = 0.f;
+            if (col + 2 * e + 1 >= V) b = 0.f;
+            h2[e] = __floats2bfloat162_rn(a, b);
+          }
+          grow[idx] = v[q];
+        }
+      }
+    } else {
+      const float4* srow = reinterpret_cast<const float4*>(s2 + static_cast<size_t>(r) * 2 * ldg);
+#pragma unroll 1
+      for (int base = 0; base < nvec; base += 32) {
+        const int idx = base + lane;
+        if (idx >= nvec) continue;
+        float4 pr[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) pr[q] = srow[4 * idx + q];
+        const int j = base >> 5;
+        const float os = pms[j] - lse2_s;
+        const float ot = pmt[j] - lse2_t;
+        const float xy[16] = {pr[0].x, pr[0].y, pr[0].z, pr[0].w, pr[1].x, pr[1].y, pr[1].z, pr[1].w,
+                              pr[2].x, pr[2].y, pr[2].z, pr[2].w, pr[3].x, pr[3].y, pr[3].z, pr[3].w};
+        uint4 out;
+        __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&out);
+        const int col = idx * 8;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          float a = coef * (fast_exp2(xy[4 * e] + os) - fast_exp2(xy[4 * e + 1] + ot));
+          float b = coef * (fast_exp2(xy[4 * e + 2] + os) - fast_exp2(xy[4 * e + 3] + ot));
+          if (col + 2 * e >= V) a = 0.f;
+          if (col + 2 * e + 1 >= V) b = 0.f;
+          h2[e] = __floats2bfloat162_rn(a, b);
+        }
+        grow[idx] = out;
       }
     }
   }
@@ -992,16 +1196,15 @@ olive_status launch_loss_fwd_bwd(const Ctx& c, const void* hidden, const void* W
   return launch_loss_reduce(c, n_rows, T, w.nll, reduction, loss);
 }
 
-olive_status launch_kl_bwd(const Ctx& c, const void* hcs, const void* hct, const void* W_s,
-                           int32_t d_s, const void* W_t, int32_t d_t, const int32_t* rows,
-                           const int32_t* n_rows, int32_t T, int32_t V, float inv_tau, int reverse,
-                           const float* grad_kl, const float* stats, int32_t ld_stats, void* g,
-                           int64_t tc, uint32_t* counters, void* d_h_s, int grad_dtype,
-                           int32_t* dev_status) {
+olive_status launch_kl_fwd_bwd(const Ctx& c, const void* hcs, const void* hct, const void* W_s,
+                               int32_t d_s, const void* W_t, int32_t d_t, const int32_t* rows,
+                               const int32_t* n_rows, int32_t T, int32_t V, float inv_tau,
+                               int reverse, const float* grad_kl, float* kl, void* g, float* s2,
+                               float* part5, int64_t tc, void* d_h_s, int grad_dtype,
+                               int32_t* dev_status) {
   const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
   const int64_t ldg = vpad(V);
-  const size_t nctr = bwd_counter_words(Tpad, tc);
-  if (cudaMemsetAsync(counters, 0, 4 * nctr, c.stream) != cudaSuccess) return OLIVE_ERR_CUDA;
+  const int vt = static_cast<int>(ceil_div(V, kBN));
   BwdMaps maps;
   if (!encode_bf16_2d(&maps.m[0], hcs, d_s, Tpad, 2ull * d_s, 64, 128) ||
       !encode_bf16_2d(&maps.m[1], W_s, d_s, V, 2ull * d_s, 64, 256) ||
@@ -1011,22 +1214,39 @@ olive_status launch_kl_bwd(const Ctx& c, const void* hcs, const void* hct, const
       !encode_bf16_2d(&maps.m[5], W_t, d_t, V, 2ull * d_t, 64, 256))
     return OLIVE_ERR_CUDA;
   BwdParams p = base_params(c, rows, n_rows, T, V, inv_tau, dev_status);
-  p.grad_kl = grad_kl;
-  p.stats = stats;
-  p.ld_stats = ld_stats;
   p.kl = 1;
   p.reverse = reverse;
   p.d = d_s;
   p.d2 = d_t;
   p.out_dtype = grad_dtype;
+  // the forward direction's fp32 pairs take twice the bytes per row: half the rows per slab
+  if (!reverse) tc = kl_pair_rows(tc);
   p.tc_max = static_cast<int32_t>(tc);
-  p.max_slabs = static_cast<int32_t>(ceil_div(Tpad, tc) + 1);
+  const int64_t max_slabs = ceil_div(Tpad, tc);
+  p.max_slabs = static_cast<int32_t>(max_slabs + 1);
   p.max_rt = static_cast<int32_t>(tc / kRowAlign);
   p.ldg = ldg;
   p.g = static_cast<__nv_bfloat16*>(g);
   p.dh_out = d_h_s;
-  p.counters = counters;
-  return launch_bwd_fused(c, maps, p);
+  p.s2 = s2;
+  p.part5 = part5;
+  p.plane5 = tc * vt;
+  int conv_blocks = static_cast<int>(ceil_div(tc, 8));
+  if (conv_blocks > c.num_sms * 16) conv_blocks = c.num_sms * 16;
+  olive_status st;
+  for (int s = 0; s < max_slabs; ++s) {
+    p.slab = s;
+    p.phase = PH_Z;
+    if ((st = launch_bwd_fused(c, maps, p)) != OLIVE_OK) return st;
+    conv_kl_kernel<<<conv_blocks, 256, 0, c.stream>>>(n_rows, rows, T, V, static_cast<int>(tc), s,
+                                                      vt, ldg, inv_tau, reverse, grad_kl, part5,
+                                                      p.plane5, s2,
+                                                      static_cast<__nv_bfloat16*>(g), kl);
+    if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;
+    p.phase = PH_DHDW;
+    if ((st = launch_bwd_fused(c, maps, p)) != OLIVE_OK) return st;
+  }
+  return OLIVE_OK;
 }
 
 }  // namespace olive

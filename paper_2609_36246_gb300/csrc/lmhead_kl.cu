@@ -14,11 +14,11 @@
 // so that KL = ln2 * A / s_p - lse_p + lse_q.  Per-segment partials are
 // merged by the finalize kernel.
 //
-// Gradient: the logits are recomputed per tile and turned into
+// With a gradient request the value and
 //   reverse: G = g_t inv_tau p_s (log p_s - log p_t - KL_t)
-//   forward: G = g_t inv_tau (p_s - p_t)
-// stored as a bf16 slab, then d_h_s = G . W_s; both run in the fused backward
-// kernel of lmhead_bwd.cu.
+//   forward: G = g_t inv_tau (p_s - p_t),   d_h_s = G . W_s
+// come from one pass over the logits in the fused kernel of lmhead_bwd.cu
+// (the forward tiles keep what G needs in the slab; nothing is recomputed).
 #include <cmath>
 
 #include "gemm_core.cuh"
@@ -212,6 +212,16 @@ olive_status launch_divergence(const Ctx& c, const void* h_s, const void* W_s, i
   if ((st = launch_gather_rows(c, h_t, rows, n_rows, T, d_t, w.hct, dev_status)) != OLIVE_OK) return st;
   if (cudaMemsetAsync(kl, 0, sizeof(float) * T, c.stream) != cudaSuccess) return OLIVE_ERR_CUDA;
 
+  if (grad) {
+    // value and gradient in one pass over the logits
+    const size_t elt = grad_dtype == OLIVE_DTYPE_BF16 ? 2 : 4;
+    if (cudaMemsetAsync(d_h_s, 0, elt * T * static_cast<size_t>(d_s), c.stream) != cudaSuccess)
+      return OLIVE_ERR_CUDA;
+    return launch_kl_fwd_bwd(c, w.hcs, w.hct, W_s, d_s, W_t, d_t, rows, n_rows, T, V, inv_tau,
+                             reverse, grad_kl, kl, w.g, w.s2, w.part5, w.tc, d_h_s, grad_dtype,
+                             dev_status);
+  }
+
   CUtensorMap mHs, mWs, mHt, mWt;
   if (!encode_bf16_2d(&mHs, w.hcs, d_s, Tpad, 2ull * d_s, 64, 128)) return OLIVE_ERR_CUDA;
   if (!encode_bf16_2d(&mWs, W_s, d_s, V, 2ull * d_s, 64, KlFwdKern::kBN)) return OLIVE_ERR_CUDA;
@@ -238,13 +248,7 @@ olive_status launch_divergence(const Ctx& c, const void* h_s, const void* W_s, i
   kl_finalize_kernel<<<c.num_sms * 4, 256, 0, c.stream>>>(n_rows, rows, T, vt, c.num_sms, p.ld,
                                                            reverse, w.part, kl, w.stats, dev_status);
   if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;
-  if (!grad) return OLIVE_OK;
-
-  const size_t elt = grad_dtype == OLIVE_DTYPE_BF16 ? 2 : 4;
-  if (cudaMemsetAsync(d_h_s, 0, elt * T * static_cast<size_t>(d_s), c.stream) != cudaSuccess)
-    return OLIVE_ERR_CUDA;
-  return launch_kl_bwd(c, w.hcs, w.hct, W_s, d_s, W_t, d_t, rows, n_rows, T, V, inv_tau, reverse,
-                       grad_kl, w.stats, p.ld, w.g, w.tc, w.counters, d_h_s, grad_dtype, dev_status);
+  return OLIVE_OK;
 }
 
 }  // namespace olive

@@ -3,6 +3,7 @@
 // tensor-map encoder.  All compute is in the kernels of the other files.
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <cstdlib>
 #include <mutex>
 
@@ -209,10 +210,18 @@ static KlWs carve_kl_impl(void* ws, int64_t T, int64_t ds, int64_t dt, int64_t V
   w.tc = slab_rows(Tpad, V);
   w.hcs = c.take(2ull * Tpad * ds);
   w.hct = c.take(2ull * Tpad * dt);
-  w.part = static_cast<float*>(c.take(4ull * 5 * kSvMax * Tpad));
-  w.stats = static_cast<float*>(c.take(4ull * 3 * Tpad));
-  w.g = grad ? c.take(2ull * w.tc * vpad(V)) : nullptr;
-  w.counters = grad ? static_cast<uint32_t*>(c.take(4ull * bwd_counter_words(Tpad, w.tc))) : nullptr;
+  w.part = w.stats = w.s2 = w.part5 = nullptr;
+  w.g = nullptr;
+  if (grad) {
+    w.g = c.take(2ull * w.tc * vpad(V));
+    // reverse: [tc, Vpad] floats; forward: [kl_pair_rows(tc), 2 Vpad] floats
+    const int64_t rows2 = std::max<int64_t>(w.tc, 2 * kl_pair_rows(w.tc));
+    w.s2 = static_cast<float*>(c.take(4ull * rows2 * vpad(V)));
+    w.part5 = static_cast<float*>(c.take(4ull * 5 * w.tc * ceil_div(V, 256)));
+  } else {
+    w.part = static_cast<float*>(c.take(4ull * 5 * kSvMax * Tpad));
+    w.stats = static_cast<float*>(c.take(4ull * 3 * Tpad));
+  }
   if (total) *total = c.off;
   return w;
 }

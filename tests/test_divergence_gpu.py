@@ -85,3 +85,84 @@ def test_kl_workload_sampled_rows():
     assert_close_logp(kl[pick], rkl[pick], "kl")
     assert rel_frob(dhs[pick], rdhs[pick]) <= 1e-2
     assert np.all(kl >= -1e-3)
+
+
+@pytest.mark.parametrize("direction", ["reverse", "forward"])
+def test_several_slabs(direction, monkeypatch):
+    """A lowered slab cap cuts ~1.3k rows into six slabs of the single-pass
+    value + gradient."""
+    monkeypatch.setenv("OLIVE_SLAB_ROWS", "256")
+    hs, Ws, ht, Wt, rows, gk = _case(8, 2000, 64, 96, 1500)
+    assert len(rows) > 5 * 256
+    kl, dhs = _gpu(hs, Ws, ht, Wt, rows, gk, direction, grad_dtype=torch.bfloat16)
+    rkl, rdhs = oracle.token_divergence(to_f64(hs), to_f64(Ws), to_f64(ht), to_f64(Wt), rows,
+                                        1.0, direction, grad_kl=gk.astype(np.float64))
+    assert_close_logp(kl, rkl, "kl")
+    assert_close_grad(dhs, rdhs, "dH_s")
+
+
+def test_value_with_and_without_gradient_agree():
+    """The value-only sweep and the single-pass value + gradient compute KL
+    from the same logits with different tilings of the partials."""
+    hs, Ws, ht, Wt, rows, gk = _case(9, 400, 128, 64, 3001)
+    for direction in ("reverse", "forward"):
+        k1, _ = _gpu(hs, Ws, ht, Wt, rows, None, direction)
+        k2, _ = _gpu(hs, Ws, ht, Wt, rows, gk, direction)
+        assert np.abs(k1 - k2).max() <= 1e-4
+
+
+def test_teacher_shifted_by_a_constant_per_row():
+    """z_t = z_s + c_t with |c_t| up to 24 (an extra hidden unit on a column of
+    ones): the distributions are equal, so KL and its gradient vanish; the
+    log-ratio kept between the passes must not lose them to the shift."""
+    rng = np.random.default_rng(11)
+    T, d, V = 300, 64, 2000
+    hs = synth.normal_bf16(rng, (T, d), 1.0)
+    Ws = synth.normal_bf16(rng, (V, d), 0.3)
+    c = torch.from_numpy(rng.uniform(-24, 24, size=(T, 8)).astype(np.float32)).to(torch.bfloat16)
+    c[:, 1:] = 0
+    ht = torch.cat([hs, c], 1)
+    Wt = torch.cat([Ws, torch.zeros(V, 8, dtype=torch.bfloat16)], 1)
+    Wt[:, d] = 1.0
+    rows = np.arange(T, dtype=np.int32)
+    gk = np.ones(T, dtype=np.float32)
+    for direction in ("reverse", "forward"):
+        kl, dhs = _gpu(hs, Ws, ht, Wt, rows, gk, direction)
+        assert np.abs(kl).max() <= 2e-5, direction
+        assert np.abs(dhs).max() <= 1e-5, direction
+
+
+@pytest.mark.parametrize("direction", ["reverse", "forward"])
+def test_single_row_tile(direction):
+    """T <= 128: one slab of one row tile (the forward direction's pair slab
+    is then larger than half of it)."""
+    hs, Ws, ht, Wt, rows, gk = _case(12, 100, 64, 64, 777)
+    kl, dhs = _gpu(hs, Ws, ht, Wt, rows, gk, direction)
+    rkl, rdhs = oracle.token_divergence(to_f64(hs), to_f64(Ws), to_f64(ht), to_f64(Wt), rows,
+                                        1.0, direction, grad_kl=gk.astype(np.float64))
+    assert_close_logp(kl, rkl, "kl")
+    assert_close_grad(dhs, rdhs, "dH_s")
+
+
+def test_forward_kl_with_a_collapsed_student():
+    """The student puts a logit 100 above the rest on one token (an extra
+    hidden unit), so inside that token's 256-column tile its other
+    probabilities are below 2^-126 of the tile maximum, while the teacher
+    spreads its mass.  Forward-KL gradients there are -p_t, which a p_s kept
+    relative to the tile maximum in 8 exponent bits would lose."""
+    rng = np.random.default_rng(13)
+    T, d, V = 200, 64, 1000
+    h = synth.normal_bf16(rng, (T, d), 1.0)
+    W = synth.normal_bf16(rng, (V, d), 0.3)
+    one = torch.zeros(T, 8, dtype=torch.bfloat16)
+    one[:, 0] = 1.0
+    hs = torch.cat([h, one], 1)
+    Ws = torch.cat([W, torch.zeros(V, 8, dtype=torch.bfloat16)], 1)
+    Ws[300, d] = 100.0
+    rows = np.arange(T, dtype=np.int32)
+    gk = np.ones(T, dtype=np.float32)
+    kl, dhs = _gpu(hs, Ws, h, W, rows, gk, "forward")
+    rkl, rdhs = oracle.token_divergence(to_f64(hs), to_f64(Ws), to_f64(h), to_f64(W), rows, 1.0,
+                                        "forward", grad_kl=gk.astype(np.float64))
+    assert_close_logp(kl, rkl, "kl")
+    assert_close_grad(dhs, rdhs, "dH_s")
