@@ -258,6 +258,8 @@ def run_ours(args, world, rank, local):
 
     avg = lambda k: statistics.mean(a.elapsed_time(b2) for a, b2 in ev[k])
     fb_ms, spl_ms = avg("fwd_bwd"), avg("splice")
+    med_step = statistics.median(a.elapsed_time(b2) for a, b2 in ev["splice"]) + \
+        statistics.median(a.elapsed_time(b2) for a, b2 in ev["fwd_bwd"])
     burst, sustained, src = load_peaks()
     counted = 6.0 * N_mask * d * V
     step_tflops = counted / (ms_per_step / 1e3) / 1e12
@@ -287,6 +289,8 @@ def run_ours(args, world, rank, local):
         torch.cuda.empty_cache()
         extra["topk_kl"] = measure_topk_kl(dev, burst)
         torch.cuda.empty_cache()
+        extra["opd_stats"] = measure_opd_stats(dev, burst)
+        torch.cuda.empty_cache()
         extra["scoring_fwd"], extra["topk_entropy"] = measure_scoring(dev, burst)
         torch.cuda.empty_cache()
         extra["varlen"] = measure_varlen(dev, burst)
@@ -307,6 +311,10 @@ def run_ours(args, world, rank, local):
         "pct_bf16_peak": 100.0 * step_tflops / burst,
         "pct_bf16_peak_sustained": 100.0 * step_tflops / sustained,
         "counted_tflops_per_s": step_tflops,
+        "ms_per_step_median": med_step,
+        "dense_equivalent_tflops_per_s": 6.0 * T * d * V / (ms_per_step / 1e3) / 1e12,
+        "dense_equivalent_note": "6 T d V over the packed T (unmasked rows included); not the "
+                                 "headline, which counts the N_mask scored rows only",
         "phases_ms": {"splice_pack": spl_ms, "loss_fwd_bwd": fb_ms},
         "roofline": {"kernel": "bwd_fused_kernel (forward tiles + dH/dW tiles, 2 launches per call)",
                      "bound": "tensor", "achieved": ach_fb, "peak": sustained, "unit": "TFLOP/s",
@@ -418,11 +426,38 @@ def measure_two_call(dev, hidden, W, pk_fn, T, d, V, n, burst, steps: int = 3):
             "pct_bf16_peak": 100.0 * 6.0 * n * d * V / (ms / 1e3) / 1e12 / burst, "steps": steps}
 
 
+def measure_opd_stats(dev, burst: float, steps: int = 3):
+    """OPD's per-token stats in one sweep with both heads: full KL, both lse,
+    student entropy and top-16, teacher log-probs at those ids, top-16
+    overlap and top-16 KL (16384 rows, student d = 4096, teacher d = 5120,
+    V = 151936)."""
+    from paper_2609_36246_gb300 import binding as B
+    N, ds, dt, V = 16384, 4096, 5120, 151936
+    hs, Ws = gpu_inputs(21, N, ds, V, dev)
+    ht, Wt = gpu_inputs(22, N, dt, V, dev)
+    rows = torch.arange(N, dtype=torch.int32, device=dev)
+    n = torch.tensor([N], dtype=torch.int32, device=dev)
+    ws = B.workspace(B.olive_workspace_size("opd_stats", N, ds, V, d_t=dt), dev)
+    st = B.new_status(dev)
+    ms = time_calls(lambda: B.olive_opd_token_stats(hs, Ws, ht, Wt, rows, n, 16, ws=ws,
+                                                    dev_status=st), steps, 1)
+    if int(st.item()) != 0:
+        raise RuntimeError(f"opd stats status {B.status_bits(st)}")
+    flops = 2.0 * N * V * (ds + dt)
+    return {"workload": "OPD per-token stats (KL, lse, entropy, top-16, overlap, top-16 KL) in one "
+                        "sweep: 16384 rows, d_s=4096, d_t=5120, V=151936",
+            "value": N / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
+            "pct_bf16_peak": 100.0 * flops / (ms / 1e3) / 1e12 / burst, "steps": steps}
+
+
 def measure_topk_kl(dev, burst: float, steps: int = 3):
-    """OPD with the top-16 KL: student and teacher entropy/top-16 sweeps, the
-    top-16 compare (overlap, truncated KL, teacher log-probs at the student's
-    ids) and the gradient w.r.t. h_s and W_s (16384 rows, student d = 4096,
-    teacher d = 5120, V = 151936)."""
+    """OPD with the top-16 KL as a training step: student and teacher
+    entropy/top-16 sweeps, the top-16 compare (overlap, truncated KL, teacher
+    log-probs at the student's ids) and the gradient w.r.t. h_s and W_s
+    (16384 rows, student d = 4096, teacher d = 5120, V = 151936).  The two
+    single-head sweeps are used rather than olive_opd_token_stats: without
+    the full KL they are the faster route (their epilogues overlap the next
+    tile's MMAs)."""
     from paper_2609_36246_gb300 import binding as B
     N, ds, dt, V, K = 16384, 4096, 5120, 151936, 16
     hs, Ws = gpu_inputs(21, N, ds, V, dev)
@@ -561,7 +596,7 @@ def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=20)
-    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-rows", type=int, default=32)
     ap.add_argument("--no-cpu-baseline", action="store_true")

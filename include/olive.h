@@ -25,6 +25,8 @@
  *   olive_token_topk_fwd     per-token entropy and top-K log-probs
  *   olive_topk_compare       student/teacher top-K overlap and top-K KL
  *   olive_topk_kl_bwd        gradient of the top-K KL
+ *   olive_opd_token_stats    OPD's per-token KL, entropy, top-K lists, overlap
+ *                            and top-K KL from one sweep with both heads
  *   olive_token_logprob_fwd_noalloc  the forward without a workspace
  *
  * Conventions shared by every call
@@ -85,7 +87,7 @@ enum { OLIVE_KL_REVERSE = 0, OLIVE_KL_FORWARD = 1 };
 enum { OLIVE_DTYPE_BF16 = 0, OLIVE_DTYPE_F32 = 1 };
 enum { OLIVE_OP_LOGPROB_FWD = 0, OLIVE_OP_LOSS_BWD = 1, OLIVE_OP_DIVERGENCE = 2,
        OLIVE_OP_TOPK_FWD = 3, OLIVE_OP_SPLICE_MASKED = 4, OLIVE_OP_TOPK_KL_BWD = 5,
-       OLIVE_OP_LOSS_FWD_BWD = 6 };
+       OLIVE_OP_LOSS_FWD_BWD = 6, OLIVE_OP_OPD_STATS = 7 };
 
 /* ABI version of the loaded library (OLIVE_ABI_VERSION). */
 OLIVE_API int olive_abi_version(void);
@@ -99,6 +101,7 @@ OLIVE_API const char* olive_status_string(olive_status s);
  *   op  OLIVE_OP_DIVERGENCE: d = student width d_s, d_t = teacher width.
  *   op  OLIVE_OP_TOPK_FWD: d = hidden width, d_t ignored.
  *   op  OLIVE_OP_SPLICE_MASKED: T = T_cap; d, d_t, V ignored.
+ *   op  OLIVE_OP_OPD_STATS: d = student width d_s, d_t = teacher width.
  *   op  OLIVE_OP_TOPK_KL_BWD, OLIVE_OP_LOSS_FWD_BWD: d = (student) hidden
  *       width, grad_dtype as for OLIVE_OP_LOSS_BWD, d_t ignored.
  *   `grad` (bwd / divergence): non-zero when gradients are requested
@@ -242,6 +245,38 @@ OLIVE_API olive_status olive_topk_compare(const void* h_t, const void* W_t, int3
                                           int32_t* dev_status, void* stream);
 
 /*
+ * olive_opd_token_stats -- everything OPD reads per token from one sweep over
+ * the vocabulary with the student (h_s [T, d_s], W_s [V, d_s]) and teacher
+ * (h_t [T, d_t], W_t [V, d_t]) heads, bf16 (Section 1, the per-token KL;
+ * Appendix A, Table opd-config, top-16 log-probs; Section 4.1, the top-K
+ * overlap ratio).  On every masked row t (z = inv_tau h W^T for each head):
+ *   kl[t]               full-vocabulary KL, direction as in
+ *                       olive_token_divergence
+ *   s_lse[t], t_lse[t]  log sum_v exp(z_v) of each head
+ *   s_entropy[t]        -sum_v p_s log p_s
+ *   s_topk_logp[t, j], s_topk_ids[t, j]
+ *                       the student's K most probable tokens (as
+ *                       olive_token_topk_fwd: equal logits, smaller id first)
+ *   t_logp_s[t, j]      log p_t at s_topk_ids[t, j]
+ *   overlap[t], kl_topk[t]
+ *                       as olive_topk_compare (kl_topk: the reverse KL
+ *                       truncated to the student's K tokens)
+ * Every output pointer may be NULL (not written) but not all of them; fp32
+ * [T] or [T, K], ids int32 [T, K]; 0 (ids -1) on rows not in `rows`.
+ * 1 <= K <= 16.  The outputs feed olive_topk_kl_bwd directly.  workspace:
+ * olive_workspace_size(OLIVE_OP_OPD_STATS, T, d_s, d_t, V, 0, 0) bytes.
+ */
+OLIVE_API olive_status olive_opd_token_stats(const void* h_s, const void* W_s, int32_t d_s,
+                                             const void* h_t, const void* W_t, int32_t d_t,
+                                             const int32_t* rows, const int32_t* n_rows,
+                                             int32_t T, int32_t V, float inv_tau, int direction,
+                                             int32_t K, float* kl, float* s_lse, float* t_lse,
+                                             float* s_entropy, float* s_topk_logp,
+                                             int32_t* s_topk_ids, float* t_logp_s,
+                                             float* overlap, float* kl_topk, void* workspace,
+                                             size_t ws_bytes, int32_t* dev_status, void* stream);
+
+/*
  * olive_topk_kl_bwd -- gradient of sum_t g_t kl_topk[t] (the truncated
  * reverse KL of olive_topk_compare) with respect to the student's hidden rows
  * and LM head, the student's top-K set S_t held fixed (it is selected, not
@@ -252,7 +287,8 @@ OLIVE_API olive_status olive_topk_compare(const void* h_t, const void* W_t, int3
  *   d_W_s[u] = sum_t G[t, u] h_s[t]
  * Inputs: h_s [T, d], W_s [V, d] bf16; s_lse fp32 [T], s_ids int32 [T, K],
  * s_logp fp32 [T, K] from olive_token_topk_fwd on the student; t_logp_s
- * fp32 [T, K] and kl_topk fp32 [T] from olive_topk_compare; grad_kl fp32 [T]
+ * fp32 [T, K] and kl_topk fp32 [T] from olive_topk_compare (or all five from
+ * olive_opd_token_stats); grad_kl fp32 [T]
  * the weights g_t.  d_h_s [T, d] and d_W_s [V, d] of grad_dtype as in
  * olive_token_loss_bwd.  The softmax term is recomputed tile by tile as in
  * that backward; the K entries of S_t per row are written over it.  1 <= K

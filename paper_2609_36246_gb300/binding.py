@@ -28,7 +28,7 @@ REDUCE = {"sum": 0, "mean": 1}
 DIRECTION = {"reverse": 0, "forward": 1}
 DTYPE = {torch.bfloat16: 0, torch.float32: 1}
 OP = {"logprob_fwd": 0, "loss_bwd": 1, "divergence": 2, "topk_fwd": 3, "splice_masked": 4,
-      "topk_kl_bwd": 5, "loss_fwd_bwd": 6}
+      "topk_kl_bwd": 5, "loss_fwd_bwd": 6, "opd_stats": 7}
 
 
 class OliveError(RuntimeError):
@@ -76,6 +76,9 @@ def lib() -> ctypes.CDLL:
     L.olive_topk_compare.restype = ctypes.c_int
     L.olive_topk_compare.argtypes = [_P, _P, _I, _P, _P, _I, _I, _F, _I, _P, _P, _P, _P, _P, _P, _P,
                                      _P, _P]
+    L.olive_opd_token_stats.restype = ctypes.c_int
+    L.olive_opd_token_stats.argtypes = [_P, _P, _I, _P, _P, _I, _P, _P, _I, _I, _F, ctypes.c_int, _I,
+                                        _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _S, _P, _P]
     L.olive_token_loss_fwd_bwd.restype = ctypes.c_int
     L.olive_token_loss_fwd_bwd.argtypes = [_P, _P, _P, _P, _P, _I, _I, _I, _F, ctypes.c_int, _P, _P,
                                            _P, _P, _P, _P, ctypes.c_int, _P, _S, _P, _P]
@@ -299,6 +302,44 @@ def olive_topk_compare(h_t, W_t, rows, n_rows, s_ids, s_logp, t_ids, t_lse, inv_
                                   _ptr(t_lse), _ptr(ov), _ptr(kl), _ptr(tlp), _ptr(ds), _stream())
     _check(st, "olive_topk_compare")
     return (ov, kl, tlp) if want_t_logp else (ov, kl)
+
+
+OPD_STATS_KEYS = ("kl", "s_lse", "t_lse", "s_entropy", "s_topk_logp", "s_topk_ids", "t_logp_s",
+                  "overlap", "kl_topk")
+
+
+def olive_opd_token_stats(h_s, W_s, h_t, W_t, rows, n_rows, K: int = 16, inv_tau: float = 1.0,
+                          direction: str = "reverse", want=OPD_STATS_KEYS, ws=None,
+                          dev_status=None) -> dict:
+    """OPD's per-token KL, lse of both heads, student entropy and top-K lists,
+    teacher log-probs at the student's top-K ids, top-K overlap and top-K KL
+    from one sweep.  Returns a dict with the requested keys of OPD_STATS_KEYS."""
+    for t, n in ((h_s, "h_s"), (W_s, "W_s"), (h_t, "h_t"), (W_t, "W_t")):
+        _need(t, torch.bfloat16, n)
+    _need(rows, torch.int32, "rows")
+    _need(n_rows, torch.int32, "n_rows")
+    T, d_s = h_s.shape
+    d_t = h_t.shape[1]
+    V = W_s.shape[0]
+    if W_t.shape[0] != V or h_t.shape[0] != T:
+        raise ValueError("student and teacher shapes disagree")
+    dev = h_s.device
+    shapes = {"s_topk_logp": (T, K), "s_topk_ids": (T, K), "t_logp_s": (T, K)}
+    out = {}
+    for k in OPD_STATS_KEYS:
+        if k in want:
+            dt = torch.int32 if k == "s_topk_ids" else torch.float32
+            out[k] = torch.empty(shapes.get(k, (T,)), dtype=dt, device=dev)
+    if ws is None:
+        ws = workspace(olive_workspace_size("opd_stats", T, d_s, V, d_t=d_t), dev)
+    ds = dev_status if dev_status is not None else new_status(dev)
+    st = lib().olive_opd_token_stats(_ptr(h_s), _ptr(W_s), d_s, _ptr(h_t), _ptr(W_t), d_t,
+                                     _ptr(rows), _ptr(n_rows), T, V, float(inv_tau),
+                                     DIRECTION[direction], int(K),
+                                     *[_ptr(out.get(k)) for k in OPD_STATS_KEYS],
+                                     _ptr(ws), ws.numel(), _ptr(ds), _stream())
+    _check(st, "olive_opd_token_stats")
+    return out
 
 
 def olive_topk_kl_bwd(h_s, W_s, rows, n_rows, s_lse, s_ids, s_logp, t_logp_s, kl_topk, grad_kl,

@@ -77,6 +77,20 @@ size_t bwd_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype);
 BwdWs carve_bwd(void* ws, int64_t T, int64_t d, int64_t V, int grad_dtype);
 size_t topk_kl_bwd_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype);
 
+// OPD per-token stats sweep (dual product with two top lists)
+struct OpdWs {
+  void* hcs;         // bf16 [Tpad, d_s]
+  void* hct;         // bf16 [Tpad, d_t]
+  float* part;       // [6, kSvMax, Tpad]
+  float* part_sv;    // [kSvMax, Tpad, 16]
+  int32_t* part_si;  // [kSvMax, Tpad, 16]
+  float* part_sx;    // [kSvMax, Tpad, 16]
+  float* part_tv;    // [kSvMax, Tpad, 16]
+  int32_t* part_ti;  // [kSvMax, Tpad, 16]
+};
+size_t opd_ws_bytes(int64_t T, int64_t ds, int64_t dt);
+OpdWs carve_opd(void* ws, int64_t T, int64_t ds, int64_t dt);
+
 // fused forward + backward: the backward's regions plus the ZSAVE partials
 struct FbWs {
   void* hc;        // bf16 [Tpad, d]
@@ -172,6 +186,14 @@ struct SparseGrad {
 // Cross-entropy backward (sg == nullptr: targets, grad_loss, reduction used)
 // or, with sg, the top-K KL backward (targets, grad_loss unused; lse is the
 // student's).
+olive_status launch_opd_stats(const Ctx& c, const void* h_s, const void* W_s, int32_t d_s,
+                              const void* h_t, const void* W_t, int32_t d_t, const int32_t* rows,
+                              const int32_t* n_rows, int32_t T, int32_t V, float inv_tau,
+                              int direction, int32_t K, float* kl, float* s_lse, float* t_lse,
+                              float* s_entropy, float* s_topk_logp, int32_t* s_topk_ids,
+                              float* t_logp_s, float* overlap, float* kl_topk, void* ws,
+                              int32_t* dev_status);
+
 olive_status launch_loss_bwd(const Ctx& c, const void* hidden, const void* W,
                              const int32_t* targets, const int32_t* rows, const int32_t* n_rows,
                              int32_t T, int32_t d, int32_t V, float inv_tau, int reduction,

@@ -22,29 +22,13 @@
 
 #include "gemm_core.cuh"
 #include "sched.cuh"
+#include "topk.cuh"
 
 namespace olive {
 namespace {
 
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
-constexpr int kTopMax = 16;  // top-K list length kept per row (K <= 16)
-
-// Inserts (cv, ci) into a list sorted by value descending, then id ascending;
-// the last entry falls off.
-__device__ __forceinline__ void topk_insert(float (&tv)[kTopMax], int (&ti)[kTopMax], float cv,
-                                            int ci) {
-#pragma unroll
-  for (int j = 0; j < kTopMax; ++j) {
-    const bool before = cv > tv[j] || (cv == tv[j] && ci < ti[j]);
-    const float v = tv[j];
-    const int i = ti[j];
-    tv[j] = before ? cv : v;
-    ti[j] = before ? ci : i;
-    cv = before ? v : cv;
-    ci = before ? i : ci;
-  }
-}
 
 template <bool kStats>
 struct FwdKernT {

@@ -170,6 +170,31 @@ BwdWs carve_bwd(void* ws, int64_t T, int64_t d, int64_t V, int grad_dtype) {
   return carve_bwd_impl(ws, T, d, V, grad_dtype, nullptr);
 }
 
+static OpdWs carve_opd_impl(void* ws, int64_t T, int64_t ds, int64_t dt, size_t* total) {
+  const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
+  const size_t lst = 4ull * 16 * kSvMax * Tpad;
+  Carver c{static_cast<char*>(ws)};
+  OpdWs w;
+  w.hcs = c.take(2ull * Tpad * ds);
+  w.hct = c.take(2ull * Tpad * dt);
+  w.part = static_cast<float*>(c.take(4ull * 6 * kSvMax * Tpad));
+  w.part_sv = static_cast<float*>(c.take(lst));
+  w.part_si = static_cast<int32_t*>(c.take(lst));
+  w.part_sx = static_cast<float*>(c.take(lst));
+  w.part_tv = static_cast<float*>(c.take(lst));
+  w.part_ti = static_cast<int32_t*>(c.take(lst));
+  if (total) *total = c.off;
+  return w;
+}
+size_t opd_ws_bytes(int64_t T, int64_t ds, int64_t dt) {
+  size_t n = 0;
+  carve_opd_impl(nullptr, T, ds, dt, &n);
+  return n;
+}
+OpdWs carve_opd(void* ws, int64_t T, int64_t ds, int64_t dt) {
+  return carve_opd_impl(ws, T, ds, dt, nullptr);
+}
+
 static FbWs carve_fb_impl(void* ws, int64_t T, int64_t d, int64_t V, int grad_dtype,
                           size_t* total) {
   const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
@@ -289,6 +314,9 @@ size_t olive_workspace_size(int op, int32_t T, int32_t d, int32_t d_t, int32_t V
     case OLIVE_OP_LOSS_FWD_BWD:
       if (grad_dtype != OLIVE_DTYPE_BF16 && grad_dtype != OLIVE_DTYPE_F32) return 0;
       return fb_ws_bytes(T, d, V, grad_dtype);
+    case OLIVE_OP_OPD_STATS:
+      if (!width_ok(d_t)) return 0;
+      return opd_ws_bytes(T, d, d_t);
     case OLIVE_OP_TOPK_KL_BWD:
       if (grad_dtype != OLIVE_DTYPE_BF16 && grad_dtype != OLIVE_DTYPE_F32) return 0;
       return topk_kl_bwd_ws_bytes(T, d, V, grad_dtype);
@@ -470,6 +498,36 @@ olive_status olive_token_loss_fwd_bwd(const void* hidden, const void* W, const i
   return launch_loss_fwd_bwd(c, hidden, W, targets, rows, n_rows, T, d, V, inv_tau, reduction,
                              grad_loss, logp, lse, loss, d_hidden, d_W, grad_dtype, workspace,
                              dev_status);
+}
+
+olive_status olive_opd_token_stats(const void* h_s, const void* W_s, int32_t d_s, const void* h_t,
+                                   const void* W_t, int32_t d_t, const int32_t* rows,
+                                   const int32_t* n_rows, int32_t T, int32_t V, float inv_tau,
+                                   int direction, int32_t K, float* kl, float* s_lse, float* t_lse,
+                                   float* s_entropy, float* s_topk_logp, int32_t* s_topk_ids,
+                                   float* t_logp_s, float* overlap, float* kl_topk,
+                                   void* workspace, size_t ws_bytes, int32_t* dev_status,
+                                   void* stream) {
+  if (!h_s || !W_s || !h_t || !W_t || !rows || !n_rows || !dev_status) return OLIVE_ERR_INVALID_ARG;
+  if (!kl && !s_lse && !t_lse && !s_entropy && !s_topk_logp && !s_topk_ids && !t_logp_s &&
+      !overlap && !kl_topk)
+    return OLIVE_ERR_INVALID_ARG;
+  if (direction != OLIVE_KL_REVERSE && direction != OLIVE_KL_FORWARD) return OLIVE_ERR_INVALID_ARG;
+  if (T < 1 || V < 1 || d_s < 1 || d_t < 1 || d_s > kMaxDim || d_t > kMaxDim || K < 1 || K > 16 ||
+      K > V)
+    return OLIVE_ERR_SHAPE;
+  if (!(inv_tau > 0.f) || !std::isfinite(inv_tau)) return OLIVE_ERR_INVALID_ARG;
+  if (d_s % 8 != 0 || d_t % 8 != 0 || !aligned16(h_s) || !aligned16(W_s) || !aligned16(h_t) ||
+      !aligned16(W_t))
+    return OLIVE_ERR_ALIGNMENT;
+  olive_status st = check_ws(workspace, ws_bytes, opd_ws_bytes(T, d_s, d_t));
+  if (st != OLIVE_OK) return st;
+  Ctx c;
+  st = make_ctx(stream, &c);
+  if (st != OLIVE_OK) return st;
+  return launch_opd_stats(c, h_s, W_s, d_s, h_t, W_t, d_t, rows, n_rows, T, V, inv_tau, direction,
+                          K, kl, s_lse, t_lse, s_entropy, s_topk_logp, s_topk_ids, t_logp_s,
+                          overlap, kl_topk, workspace, dev_status);
 }
 
 olive_status olive_token_divergence(const void* h_s, const void* W_s, int32_t d_s, const void* h_t,

@@ -170,6 +170,27 @@ def test_new_entry_points_validation(L):
         "logprob_fwd", 4096, 4096, 151936)
 
 
+def test_opd_stats_validation(L):
+    keep, p = _fake()
+    P = ctypes.c_void_p
+    ws = B.olive_workspace_size("opd_stats", 64, 64, 100, d_t=96)
+    assert ws > 0 and B.olive_workspace_size("opd_stats", 64, 64, 100, d_t=90) == 0
+
+    def call(outs=None, **kw):
+        a = dict(K=16, dirn=0, dt=96, ws_bytes=ws)
+        a.update(kw)
+        o = outs if outs is not None else [P(p)] * 9
+        return L.olive_opd_token_stats(P(p), P(p), 64, P(p), P(p), a["dt"], P(p), P(p), 64, 100, 1.0,
+                                       a["dirn"], a["K"], *o, P(p), a["ws_bytes"], P(p), None)
+    assert call(outs=[None] * 9) == 1
+    assert call(dirn=2) == 1
+    assert call(K=0) == 2 and call(K=17) == 2
+    assert call(dt=90) == 3
+    assert call(ws_bytes=ws - 1) == 9
+    if not torch.cuda.is_available():
+        assert call(outs=[None] * 8 + [P(p)]) in (7, 8)
+
+
 def test_fwd_bwd_validation(L):
     keep, p = _fake()
     P = ctypes.c_void_p

@@ -57,14 +57,18 @@ def test_random_shapes(S, V, d, kw):
     _full_check(b, h, W, **kw)
 
 
-def test_two_slabs():
-    # more than 16384 masked rows: G goes through two slabs, dW accumulates
+@pytest.mark.parametrize("slab_rows,grad_dtype", [(4096, torch.float32), (1024, torch.bfloat16)])
+def test_several_slabs(slab_rows, grad_dtype, monkeypatch):
+    """17000 masked rows with the slab cap lowered: G goes through several
+    slabs, which wait on each other inside the one launch, and dW accumulates
+    (fp32 accumulator for a bf16 output)."""
+    monkeypatch.setenv("OLIVE_SLAB_ROWS", str(slab_rows))
     rng = np.random.default_rng(21)
     b = synth.batch_from_lengths(rng, [1] * 10, [1700] * 10, 600)
     h = synth.normal_bf16(rng, (b.T, 64), 1.0)
     W = synth.normal_bf16(rng, (600, 64), 0.1)
-    assert b.n_mask > 16384
-    _full_check(b, h, W, grad_dtype=torch.float32)
+    assert b.n_mask > 4 * slab_rows
+    _full_check(b, h, W, grad_dtype=grad_dtype)
 
 
 def test_empty_mask_gives_zero_grads():
