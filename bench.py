@@ -554,14 +554,25 @@ def measure_varlen(dev, burst: float, steps: int = 2):
             "steps": steps}
 
 
-def kernel_rev() -> str:
-    """Content hash of the CUDA sources (ties a stored ncu traffic figure to them)."""
+def kernel_rev(source: str = "lmhead_bwd.cu") -> str:
+    """Content hash of one kernel's translation unit and the headers it
+    includes (followed transitively), which ties a stored ncu traffic figure
+    to the code that produced it."""
     import hashlib
+    import re as _re
+    csrc = os.path.join(ROOT, "paper_2609_36246_gb300", "csrc")
+    seen, todo = [], [os.path.join(csrc, source)]
+    while todo:
+        path = todo.pop(0)
+        if path in seen or not os.path.exists(path):
+            continue
+        seen.append(path)
+        with open(path) as f:
+            for inc in _re.findall(r'#include "([^"]+)"', f.read()):
+                todo.append(os.path.normpath(os.path.join(os.path.dirname(path), inc)))
     hsh = hashlib.sha256()
-    import glob
-    for p in sorted(glob.glob(os.path.join(ROOT, "paper_2609_36246_gb300", "csrc", "*.cu*"))) + \
-            sorted(glob.glob(os.path.join(ROOT, "paper_2609_36246_gb300", "csrc", "*.h"))):
-        with open(p, "rb") as f:
+    for path in sorted(seen):
+        with open(path, "rb") as f:
             hsh.update(f.read())
     return hsh.hexdigest()[:16]
 
