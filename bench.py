@@ -298,7 +298,7 @@ def run_ours(args, world, rank, local):
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
-        rate, secs, nr = oracle_sample_rate(b, h_cpu, W_cpu, args.cpu_rows)
+        rate, secs, nr = oracle_sample_rate(b, h_cpu, W_cpu, args.cpu_rows or 96)
         cpu = {"value": rate, "unit": "tokens/s", "cores": host_cores(), "kind": "oracle",
                "sample": f"{nr} masked rows of the same batch: fp64 logits, log-probs, dH and dW "
                          f"contributions ({secs:.1f} s)"}
@@ -586,7 +586,7 @@ def run_reference(args, world, rank):
     for _ in range(args.warmup):
         pass  # the oracle has no warm state; warm-up steps would only repeat the sample
     for i in range(args.steps):
-        rate, secs, nr = oracle_sample_rate(b, h, W, args.cpu_rows, seed=i)
+        rate, secs, nr = oracle_sample_rate(b, h, W, args.cpu_rows or 24, seed=i)
         times.append(secs)
         rows += nr
     value = rows / sum(times)
@@ -596,7 +596,7 @@ def run_reference(args, world, rank):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": dict(CONFIG, parallelism="host cores"),
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": host_cores(), "kind": "oracle",
-                         "sample": f"{args.cpu_rows} masked rows per step of the same batch "
+                         "sample": f"{args.cpu_rows or 24} masked rows per step of the same batch "
                                    "(fp64 forward, dH, dW contributions)"},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -609,7 +609,9 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--cpu-rows", type=int, default=32)
+    ap.add_argument("--cpu-rows", type=int, default=None,
+                    help="masked rows in the oracle sample (default: 96 for the cpu_baseline "
+                         "leg, about 10 s; 24 per step for --impl reference)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extra", action="store_true",
                     help="skip the divergence and variable-length measurements")
