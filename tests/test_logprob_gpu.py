@@ -141,3 +141,68 @@ def test_scoring_workload_sampled_rows():
     assert abs(loss + all_lp.sum()) <= 1e-4 * abs(loss)
     sigma2 = 0.02 ** 2 * 2048
     assert abs(all_lp.mean() - (-math.log(151936) - sigma2 / 2)) < 0.05
+
+
+def _integer_case(seed, S=6, V=3001, d=64):
+    """bf16 inputs that are small integers (h in {-2..2}, W in {-1, 0, 1},
+    mostly 0), so every logit is an integer of magnitude <= 2 d that fp32 and
+    fp64 both hold exactly: only the exp / log / accumulation error is left."""
+    rng = np.random.default_rng(seed)
+    b = synth.batch_from_lengths(rng, rng.integers(1, 40, size=S), rng.integers(0, 120, size=S), V)
+    h = torch.from_numpy(rng.integers(-2, 3, size=(b.T, d)).astype(np.float32)).to(torch.bfloat16)
+    Wf = rng.integers(-1, 2, size=(V, d)).astype(np.float32)
+    Wf *= rng.random(size=(V, d)) < 0.05
+    W = torch.from_numpy(Wf).to(torch.bfloat16)
+    return b, h, W
+
+
+@pytest.mark.parametrize("seed", [0, 1])
+def test_exact_integer_logits(seed):
+    """With exact logits the GPU's log-probs carry only fp32 exp/log and
+    accumulation error: 1e-5 + 1e-6 |logp|, 200x tighter than the general
+    bound, for the forward and the single-pass forward + backward."""
+    b, h, W = _integer_case(seed)
+    z = to_f64(h) @ to_f64(W).T
+    assert np.array_equal(z, np.round(z)) and np.abs(z).max() < 2 ** 24
+    _, logp, lse, _ = _run(b, h, W)
+    o = oracle_pack(b)
+    rl, rs, _ = oracle.token_logprob(to_f64(h), to_f64(W), o["targets"], o["rows"])
+    r = o["rows"]
+    assert np.abs(logp[r] - rl[r]).max() <= 1e-5 + 1e-6 * np.abs(rl[r]).max()
+    assert np.abs(lse[r] - rs[r]).max() <= 1e-5 + 1e-6 * np.abs(rs[r]).max()
+    g = gpu_pack(b)
+    gl = torch.ones(1, dtype=torch.float32, device="cuda")
+    logp2, lse2, _, _, _ = B.olive_token_loss_fwd_bwd(h.cuda(), W.cuda(), g["targets"], g["rows"],
+                                                      g["n_rows"], gl, dev_status=g["dev_status"])
+    torch.cuda.synchronize()
+    assert B.status_bits(g["dev_status"]) == []
+    assert np.abs(logp2.cpu().numpy()[r] - rl[r]).max() <= 1e-5 + 1e-6 * np.abs(rl[r]).max()
+
+
+def test_constant_column_shift_invariance():
+    """A hidden unit fixed at 1 with W[:, j] = c adds c to every logit of the
+    row: log-probs and the gradient with respect to the other units do not
+    change (the softmax is shift invariant); lse moves by exactly c."""
+    rng = np.random.default_rng(8)
+    b = synth.batch_from_lengths(rng, rng.integers(1, 40, size=5), rng.integers(1, 150, size=5), 2000)
+    h = synth.normal_bf16(rng, (b.T, 64), 1.0)
+    h[:, 63] = 1.0
+    W = synth.normal_bf16(rng, (2000, 64), 0.3)
+    g = gpu_pack(b)
+    gl = torch.ones(1, dtype=torch.float32, device="cuda")
+    res = []
+    for c in (0.0, 24.0):
+        Wc = W.clone()
+        Wc[:, 63] = c
+        out = B.olive_token_loss_fwd_bwd(h.cuda(), Wc.cuda(), g["targets"], g["rows"], g["n_rows"],
+                                         gl, grad_dtype=torch.float32, dev_status=g["dev_status"])
+        res.append([t.cpu().numpy() for t in out])
+    torch.cuda.synchronize()
+    assert B.status_bits(g["dev_status"]) == []
+    o = oracle_pack(b)
+    r = o["rows"]
+    (l0, s0, _, dh0, dw0), (l1, s1, _, dh1, dw1) = res
+    assert np.abs(l1[r] - l0[r]).max() <= 2e-5 * (1 + np.abs(l0[r]).max())
+    assert np.abs((s1[r] - s0[r]) - 24.0).max() <= 1e-4
+    assert np.linalg.norm(dh1[:, :63] - dh0[:, :63]) <= 2e-2 * np.linalg.norm(dh0[:, :63])
+    assert np.linalg.norm(dw1[:, :63] - dw0[:, :63]) <= 2e-2 * np.linalg.norm(dw0[:, :63])
