@@ -263,7 +263,7 @@ def run_ours(args, world, rank, local):
     burst, sustained, src = load_peaks()
     counted = 6.0 * N_mask * d * V
     step_tflops = counted / (ms_per_step / 1e3) / 1e12
-    # dominant kernel: bwd_fused_kernel, launched twice per call (forward
+    # dominant kernel: lmhead_fused_kernel, launched twice per call (forward
     # tiles, then dH/dW tiles); its algorithmic work per call is the forward
     # product plus dH and dW, 6 N_mask d V, and the call is bracketed by
     # events on its stream (so the row gather, the convert pass and the loss
@@ -272,7 +272,7 @@ def run_ours(args, world, rank, local):
     fb_flops = counted
     ach_fb = fb_flops / (fb_ms / 1e3) / 1e12
     rev = kernel_rev()
-    traffic = profile_traffic("bwd_fused_kernel", rev)
+    traffic = profile_traffic("lmhead_fused_kernel", rev)
     # splice (scan, fill) + gather + per slab (forward tiles, convert, dH/dW tiles) + loss reduce
     launches = 2 + 1 + 3 * slabs + 1
 
@@ -316,12 +316,12 @@ def run_ours(args, world, rank, local):
         "dense_equivalent_note": "6 T d V over the packed T (unmasked rows included); not the "
                                  "headline, which counts the N_mask scored rows only",
         "phases_ms": {"splice_pack": spl_ms, "loss_fwd_bwd": fb_ms},
-        "roofline": {"kernel": "bwd_fused_kernel (forward tiles + dH/dW tiles, 2 launches per call)",
+        "roofline": {"kernel": "lmhead_fused_kernel (forward tiles + dH/dW tiles, 2 launches per call)",
                      "bound": "tensor", "achieved": ach_fb, "peak": sustained, "unit": "TFLOP/s",
                      "frac": ach_fb / sustained, "traffic": traffic,
                      "peak_source": f"{src} bf16_tflops_sustained",
                      "flops_per_call": fb_flops, "kernel_rev": rev,
-                     "note": "per olive_token_loss_fwd_bwd call (its two bwd_fused_kernel launches, "
+                     "note": "per olive_token_loss_fwd_bwd call (its two lmhead_fused_kernel launches, "
                              "timed with the gather, convert and loss kernels around them); "
                              "traffic is DRAM bytes of both launches"},
         "two_call_path": two_call,
@@ -554,7 +554,7 @@ def measure_varlen(dev, burst: float, steps: int = 2):
             "steps": steps}
 
 
-def kernel_rev(source: str = "lmhead_bwd.cu") -> str:
+def kernel_rev(source: str = "lmhead_fused.cu") -> str:
     """Content hash of one kernel's translation unit and the headers it
     includes (followed transitively), which ties a stored ncu traffic figure
     to the code that produced it."""

@@ -2,6 +2,7 @@
 // libolive.so.  Not part of the public ABI (include/olive.h is).
 #pragma once
 
+#include <atomic>
 #include <cstddef>
 #include <cstdint>
 #include <cuda.h>
@@ -28,6 +29,13 @@ struct Ctx {
 
 // Fills ctx for the current device; checks compute capability 10.3.
 olive_status make_ctx(void* stream, Ctx* ctx);
+
+// Raises a kernel's dynamic shared-memory limit to `smem` once per device
+// and process (`done` is the call site's per-device flag array of
+// kMaxDevices entries), so later calls issue no attribute call and can be
+// captured into a CUDA graph.  Returns false if the attribute call fails.
+constexpr int kMaxDevices = 64;
+bool set_smem_once(const void* func, int smem, int device, std::atomic<int>* done);
 
 // Encodes a 2-D bf16 tensor map (row-major [outer, inner], row pitch in
 // bytes) with 128-byte swizzle and the given box.  Returns false on failure.
@@ -109,7 +117,6 @@ struct KlWs {
   void* hcs;      // bf16 [Tpad, d_s]
   void* hct;      // bf16 [Tpad, d_t]
   float* part;    // [5, kSvMax, Tpad] (value only)
-  float* stats;   // [3, Tpad]: lse_s, lse_t, kl per compacted row (value only)
   void* g;        // bf16 [Tc, Vpad]: e_s, then G (gradient only)
   float* s2;      // fp32 [Tc, Vpad]: second slab (gradient only)
   float* part5;   // [5, Tc, ceil(V/256)] per-tile partials (gradient only)

@@ -1,5 +1,6 @@
-// lmhead_bwd.cu -- backward passes of the LM-head losses in one persistent,
-// cooperatively launched kernel with a dynamic tile scheduler.
+// lmhead_fused.cu -- the LM-head losses' backward passes, and their single-pass
+// forward + backward forms, in one persistent tcgen05 kernel
+// (lmhead_fused_kernel) with a static tile schedule.
 //
 // Cross-entropy (Eq. (osd-ce), Section 3.1; the sampled sequences are fixed,
 // so only hidden and W get gradients).  With p = softmax(z) from the
@@ -80,11 +81,11 @@ enum Phase : int { PH_ALL = 0, PH_Z = 1, PH_DHDW = 2 };
 //          3 W MN-major 64x64, 4 G MN-major 64x64, 5 hc MN-major 64x64
 // KL maps: 0 hs K-major 64x128, 1 W_s K-major 64x256, 2 G K-major 64x128,
 //          3 W_s MN-major 64x64, 4 ht K-major 64x128, 5 W_t K-major 64x256
-struct BwdMaps {
+struct FusedMaps {
   CUtensorMap m[6];
 };
 
-struct BwdParams {
+struct FusedParams {
   int32_t* dev_status;
   uint64_t wait_limit_ns;
   const int32_t* n_rows;
@@ -126,15 +127,15 @@ struct Unit {
   int kind, s, i, j, in_s, row0, mt;
 };
 
-__device__ __forceinline__ uint32_t* ctr_grad(const BwdParams& p, int s) { return p.counters + s; }
-__device__ __forceinline__ uint32_t* ctr_dhdw(const BwdParams& p, int s) {
+__device__ __forceinline__ uint32_t* ctr_grad(const FusedParams& p, int s) { return p.counters + s; }
+__device__ __forceinline__ uint32_t* ctr_dhdw(const FusedParams& p, int s) {
   return p.counters + p.max_slabs + s;
 }
-__device__ __forceinline__ uint32_t* ctr_row(const BwdParams& p, int s, int i) {
+__device__ __forceinline__ uint32_t* ctr_row(const FusedParams& p, int s, int i) {
   return p.counters + 2 * p.max_slabs + static_cast<size_t>(s) * p.max_rt + i;
 }
 
-__device__ Plan make_plan(const BwdParams& p) {
+__device__ Plan make_plan(const FusedParams& p) {
   Plan pl;
   pl.n = read_n_rows(p.n_rows, p.T, p.dev_status);
   const SlabPlan sp(pl.n, p.tc_max);
@@ -160,17 +161,17 @@ __device__ __forceinline__ int slab_in(const Plan& pl, int s) {
 }
 __device__ __forceinline__ int units_grad(const Plan& pl, int mt) { return mt * pl.vt; }
 __device__ __forceinline__ int units_dh(const Plan& pl, int mt) { return mt * pl.ntd; }
-__device__ __forceinline__ int units_dw(const BwdParams& p, const Plan& pl, int s, int in_s) {
+__device__ __forceinline__ int units_dw(const FusedParams& p, const Plan& pl, int s, int in_s) {
   return (!p.kl && (s == 0 || in_s > 0)) ? pl.mtv * pl.ntd : 0;
 }
 
 // slabs a launch covers
-__device__ __forceinline__ int slab_lo(const BwdParams& p) { return p.phase == PH_ALL ? 0 : p.slab; }
-__device__ __forceinline__ int slab_hi(const BwdParams& p, const Plan& pl) {
+__device__ __forceinline__ int slab_lo(const FusedParams& p) { return p.phase == PH_ALL ? 0 : p.slab; }
+__device__ __forceinline__ int slab_hi(const FusedParams& p, const Plan& pl) {
   return p.phase == PH_ALL ? pl.n_slabs : (p.slab < pl.n_slabs ? p.slab + 1 : 0);
 }
 
-__device__ int total_units(const BwdParams& p, const Plan& pl) {
+__device__ int total_units(const FusedParams& p, const Plan& pl) {
   int t = 0;
   for (int s = slab_lo(p); s < slab_hi(p, pl); ++s) {
     const int in_s = slab_in(pl, s);
@@ -181,7 +182,7 @@ __device__ int total_units(const BwdParams& p, const Plan& pl) {
   return t;
 }
 
-__device__ Unit decode(const BwdParams& p, const Plan& pl, int u) {
+__device__ Unit decode(const FusedParams& p, const Plan& pl, int u) {
   Unit x;
   x.kind = K_NONE;
   for (int s = slab_lo(p); s < slab_hi(p, pl); ++s) {
@@ -221,7 +222,7 @@ __device__ Unit decode(const BwdParams& p, const Plan& pl, int u) {
 }
 
 // K steps of each product of a unit
-__device__ __forceinline__ void unit_ksteps(const BwdParams& p, const Unit& x, int& nk, int& nk2) {
+__device__ __forceinline__ void unit_ksteps(const FusedParams& p, const Unit& x, int& nk, int& nk2) {
   nk2 = 0;
   switch (x.kind) {
     case K_GRAD:
@@ -280,7 +281,7 @@ __device__ __forceinline__ void store_row32(void* base, size_t off, int dtype, i
 }
 
 // ------------------------------------------------------------- epilogues ---
-__device__ void epi_grad(const BwdParams& p, const Plan& pl, const Unit& x, int row, uint32_t taddr) {
+__device__ void epi_grad(const FusedParams& p, const Plan& pl, const Unit& x, int row, uint32_t taddr) {
   const int r_local = x.i * kBM + row;
   const int r = x.row0 + r_local;
   bool valid = r_local < x.in_s;
@@ -331,7 +332,7 @@ __device__ void epi_grad(const BwdParams& p, const Plan& pl, const Unit& x, int 
 // sums s_s, s_t of 2^(x - m), A = sum e_p (x_p - x_q) in the primary
 // distribution's scale (p = student for the reverse KL, teacher for the
 // forward KL), e_s in bf16 into the G slab and the fp32 second slab
-__device__ void epi_klz(const BwdParams& p, const Plan& pl, const Unit& x, int row,
+__device__ void epi_klz(const FusedParams& p, const Plan& pl, const Unit& x, int row,
                         uint32_t taddr) {
   const int r_local = x.i * kBM + row;
   bool valid = r_local < x.in_s;
@@ -422,7 +423,7 @@ __device__ void epi_klz(const BwdParams& p, const Plan& pl, const Unit& x, int r
 // forward tile of the fused forward + backward: per row the tile's max and
 // sum of 2^(x - max) in base-2 units, e = 2^(x - max) stored in bf16 at the
 // row's G slab columns (zeros on padding rows), and the exact target logit
-__device__ void epi_zsave(const BwdParams& p, const Plan& pl, const Unit& x, int row,
+__device__ void epi_zsave(const FusedParams& p, const Plan& pl, const Unit& x, int row,
                           uint32_t taddr) {
   const int r_local = x.i * kBM + row;
   bool valid = r_local < x.in_s;
@@ -476,7 +477,7 @@ __device__ void epi_zsave(const BwdParams& p, const Plan& pl, const Unit& x, int
   }
 }
 
-__device__ void epi_dh(const BwdParams& p, const Unit& x, int row, uint32_t taddr) {
+__device__ void epi_dh(const FusedParams& p, const Unit& x, int row, uint32_t taddr) {
   const int r_local = x.i * kBM + row;
   int t = -1;
   if (r_local < x.in_s) {
@@ -499,7 +500,7 @@ __device__ void epi_dh(const BwdParams& p, const Unit& x, int row, uint32_t tadd
   }
 }
 
-__device__ void epi_dw(const BwdParams& p, const Plan& pl, const Unit& x, int row, uint32_t taddr,
+__device__ void epi_dw(const FusedParams& p, const Plan& pl, const Unit& x, int row, uint32_t taddr,
                        int nk) {
   const int v = x.i * kBM + row;
   const bool first = x.s == 0;
@@ -547,7 +548,7 @@ __device__ void epi_dw(const BwdParams& p, const Plan& pl, const Unit& x, int ro
 }
 
 // ---------------------------------------------------------------- kernel ---
-struct BwdLayout {
+struct FusedLayout {
   static constexpr int A_BYTES = kBM * kBK * 2;      // 16 KB
   static constexpr int B_BYTES = kBN * kBK * 2;      // 32 KB
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
@@ -561,8 +562,8 @@ struct BwdLayout {
 };
 
 __global__ void __launch_bounds__(kThreads, 1)
-    bwd_fused_kernel(const __grid_constant__ BwdMaps maps, const BwdParams p) {
-  using L = BwdLayout;
+    lmhead_fused_kernel(const __grid_constant__ FusedMaps maps, const FusedParams p) {
+  using L = FusedLayout;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -1028,36 +1029,45 @@ __global__ void __launch_bounds__(256)
   }
 }
 
-olive_status launch_bwd_fused(const Ctx& c, const BwdMaps& maps, const BwdParams& p) {
-  const int smem = BwdLayout::SMEM_BYTES;
-  if (cudaFuncSetAttribute(bwd_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
-      cudaSuccess)
+olive_status launch_lmhead_fused(const Ctx& c, const FusedMaps& maps, const FusedParams& p) {
+  const int smem = FusedLayout::SMEM_BYTES;
+  static std::atomic<int> done[kMaxDevices];
+  if (!set_smem_once(reinterpret_cast<const void*>(lmhead_fused_kernel), smem, c.device, done))
     return OLIVE_ERR_CUDA;
-  int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, bwd_fused_kernel, kThreads, smem) !=
-          cudaSuccess ||
-      per_sm < 1)
-    return OLIVE_ERR_CUDA;
+  // one CTA per SM must fit (the cooperative launch relies on it); checked
+  // once per device
+  static std::atomic<int> fits[kMaxDevices];
+  const bool cached = c.device >= 0 && c.device < kMaxDevices;
+  if (!cached || fits[c.device].load(std::memory_order_acquire) == 0) {
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, lmhead_fused_kernel, kThreads,
+                                                      smem) != cudaSuccess ||
+        per_sm < 1)
+      return OLIVE_ERR_CUDA;
+    if (cached) fits[c.device].store(1, std::memory_order_release);
+  }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(c.num_sms);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = c.stream;
+  // the one-launch form waits across CTAs, so every CTA must be resident: a
+  // cooperative launch; the phase launches have no cross-CTA waits
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeCooperative;
   attr[0].val.cooperative = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  if (cudaLaunchKernelEx(&cfg, bwd_fused_kernel, maps, p) != cudaSuccess) {
+  cfg.numAttrs = p.phase == PH_ALL ? 1 : 0;
+  if (cudaLaunchKernelEx(&cfg, lmhead_fused_kernel, maps, p) != cudaSuccess) {
     cudaGetLastError();
     return OLIVE_ERR_CUDA;
   }
   return OLIVE_OK;
 }
 
-BwdParams base_params(const Ctx& c, const int32_t* rows, const int32_t* n_rows, int32_t T,
+FusedParams base_params(const Ctx& c, const int32_t* rows, const int32_t* n_rows, int32_t T,
                       int32_t V, float inv_tau, int32_t* dev_status) {
-  BwdParams p = {};
+  FusedParams p = {};
   p.dev_status = dev_status;
   p.wait_limit_ns = c.wait_limit_ns;
   p.n_rows = n_rows;
@@ -1096,7 +1106,7 @@ olive_status launch_loss_bwd(const Ctx& c, const void* hidden, const void* W,
   const size_t nctr = bwd_counter_words(Tpad, w.tc);
   if (cudaMemsetAsync(w.counters, 0, 4 * nctr, c.stream) != cudaSuccess) return OLIVE_ERR_CUDA;
 
-  BwdMaps maps;
+  FusedMaps maps;
   if (!encode_bf16_2d(&maps.m[0], w.hc, d, Tpad, 2ull * d, 64, 128) ||
       !encode_bf16_2d(&maps.m[1], W, d, V, 2ull * d, 64, 256) ||
       !encode_bf16_2d(&maps.m[2], w.g, V, w.tc, 2ull * ldg, 64, 128) ||
@@ -1105,7 +1115,7 @@ olive_status launch_loss_bwd(const Ctx& c, const void* hidden, const void* W,
       !encode_bf16_2d(&maps.m[5], w.hc, d, Tpad, 2ull * d, 64, 64))
     return OLIVE_ERR_CUDA;
 
-  BwdParams p = base_params(c, rows, n_rows, T, V, inv_tau, dev_status);
+  FusedParams p = base_params(c, rows, n_rows, T, V, inv_tau, dev_status);
   p.targets = targets;
   p.lse = lse;
   p.grad_loss = grad_loss;
@@ -1129,7 +1139,7 @@ olive_status launch_loss_bwd(const Ctx& c, const void* hidden, const void* W,
   p.dw_out = d_W;
   p.dw_acc = grad_dtype == OLIVE_DTYPE_F32 ? static_cast<float*>(d_W) : w.dw_acc;
   p.counters = w.counters;
-  return launch_bwd_fused(c, maps, p);
+  return launch_lmhead_fused(c, maps, p);
 }
 
 olive_status launch_loss_fwd_bwd(const Ctx& c, const void* hidden, const void* W,
@@ -1151,7 +1161,7 @@ olive_status launch_loss_fwd_bwd(const Ctx& c, const void* hidden, const void* W
       cudaMemsetAsync(lse, 0, sizeof(float) * T, c.stream) != cudaSuccess)
     return OLIVE_ERR_CUDA;
 
-  BwdMaps maps;
+  FusedMaps maps;
   if (!encode_bf16_2d(&maps.m[0], w.hc, d, Tpad, 2ull * d, 64, 128) ||
       !encode_bf16_2d(&maps.m[1], W, d, V, 2ull * d, 64, 256) ||
       !encode_bf16_2d(&maps.m[2], w.g, V, w.tc, 2ull * ldg, 64, 128) ||
@@ -1160,7 +1170,7 @@ olive_status launch_loss_fwd_bwd(const Ctx& c, const void* hidden, const void* W
       !encode_bf16_2d(&maps.m[5], w.hc, d, Tpad, 2ull * d, 64, 64))
     return OLIVE_ERR_CUDA;
 
-  BwdParams p = base_params(c, rows, n_rows, T, V, inv_tau, dev_status);
+  FusedParams p = base_params(c, rows, n_rows, T, V, inv_tau, dev_status);
   p.targets = targets;
   p.kl = 0;
   p.d = d;
@@ -1184,14 +1194,14 @@ olive_status launch_loss_fwd_bwd(const Ctx& c, const void* hidden, const void* W
   for (int s = 0; s < max_slabs; ++s) {
     p.slab = s;
     p.phase = PH_Z;
-    if ((st = launch_bwd_fused(c, maps, p)) != OLIVE_OK) return st;
+    if ((st = launch_lmhead_fused(c, maps, p)) != OLIVE_OK) return st;
     conv_kernel<<<conv_blocks, 256, 0, c.stream>>>(
         n_rows, rows, targets, T, V, static_cast<int>(w.tc), s, vt, ldg, inv_tau, reduction,
         grad_loss, w.part_zm, w.part_zs, w.zy, static_cast<__nv_bfloat16*>(w.g), logp, lse, w.nll,
         dev_status);
     if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;
     p.phase = PH_DHDW;
-    if ((st = launch_bwd_fused(c, maps, p)) != OLIVE_OK) return st;
+    if ((st = launch_lmhead_fused(c, maps, p)) != OLIVE_OK) return st;
   }
   return launch_loss_reduce(c, n_rows, T, w.nll, reduction, loss);
 }
@@ -1205,7 +1215,7 @@ olive_status launch_kl_fwd_bwd(const Ctx& c, const void* hcs, const void* hct, c
   const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
   const int64_t ldg = vpad(V);
   const int vt = static_cast<int>(ceil_div(V, kBN));
-  BwdMaps maps;
+  FusedMaps maps;
   if (!encode_bf16_2d(&maps.m[0], hcs, d_s, Tpad, 2ull * d_s, 64, 128) ||
       !encode_bf16_2d(&maps.m[1], W_s, d_s, V, 2ull * d_s, 64, 256) ||
       !encode_bf16_2d(&maps.m[2], g, V, tc, 2ull * ldg, 64, 128) ||
@@ -1213,7 +1223,7 @@ olive_status launch_kl_fwd_bwd(const Ctx& c, const void* hcs, const void* hct, c
       !encode_bf16_2d(&maps.m[4], hct, d_t, Tpad, 2ull * d_t, 64, 128) ||
       !encode_bf16_2d(&maps.m[5], W_t, d_t, V, 2ull * d_t, 64, 256))
     return OLIVE_ERR_CUDA;
-  BwdParams p = base_params(c, rows, n_rows, T, V, inv_tau, dev_status);
+  FusedParams p = base_params(c, rows, n_rows, T, V, inv_tau, dev_status);
   p.kl = 1;
   p.reverse = reverse;
   p.d = d_s;
@@ -1237,14 +1247,14 @@ olive_status launch_kl_fwd_bwd(const Ctx& c, const void* hcs, const void* hct, c
   for (int s = 0; s < max_slabs; ++s) {
     p.slab = s;
     p.phase = PH_Z;
-    if ((st = launch_bwd_fused(c, maps, p)) != OLIVE_OK) return st;
+    if ((st = launch_lmhead_fused(c, maps, p)) != OLIVE_OK) return st;
     conv_kl_kernel<<<conv_blocks, 256, 0, c.stream>>>(n_rows, rows, T, V, static_cast<int>(tc), s,
                                                       vt, ldg, inv_tau, reverse, grad_kl, part5,
                                                       p.plane5, s2,
                                                       static_cast<__nv_bfloat16*>(g), kl);
     if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;
     p.phase = PH_DHDW;
-    if ((st = launch_bwd_fused(c, maps, p)) != OLIVE_OK) return st;
+    if ((st = launch_lmhead_fused(c, maps, p)) != OLIVE_OK) return st;
   }
   return OLIVE_OK;
 }

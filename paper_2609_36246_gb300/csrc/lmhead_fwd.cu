@@ -377,8 +377,8 @@ template <class K>
 olive_status launch_fwd_core(const Ctx& c, const CUtensorMap& a, const CUtensorMap& b,
                              const typename K::Params& p) {
   const int smem = core_smem_bytes<K>();
-  if (cudaFuncSetAttribute(gemm_persistent<K>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
-      cudaSuccess)
+  static std::atomic<int> done[kMaxDevices];
+  if (!set_smem_once(reinterpret_cast<const void*>(gemm_persistent<K>), smem, c.device, done))
     return OLIVE_ERR_CUDA;
   gemm_persistent<K><<<c.num_sms, kThreads, smem, c.stream>>>(a, b, a, b, p);
   return cudaGetLastError() == cudaSuccess ? OLIVE_OK : OLIVE_ERR_CUDA;

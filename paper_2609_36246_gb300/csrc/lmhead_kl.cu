@@ -17,7 +17,7 @@
 // With a gradient request the value and
 //   reverse: G = g_t inv_tau p_s (log p_s - log p_t - KL_t)
 //   forward: G = g_t inv_tau (p_s - p_t),   d_h_s = G . W_s
-// come from one pass over the logits in the fused kernel of lmhead_bwd.cu
+// come from one pass over the logits in the fused kernel of lmhead_fused.cu
 // (the forward tiles keep what G needs in the slab; nothing is recomputed).
 #include <cmath>
 
@@ -151,9 +151,8 @@ struct KlFwdKern {
 };
 
 __global__ void kl_finalize_kernel(const int32_t* __restrict__ n_rows, const int32_t* __restrict__ rows,
-                                   int T, int vt, int ctas, int ld, int reverse,
-                                   const float* __restrict__ part, float* __restrict__ kl,
-                                   float* __restrict__ stats, int32_t* dev_status) {
+                                   int T, int vt, int ctas, int ld,
+                                   const float* __restrict__ part, float* __restrict__ kl) {
   __shared__ int sh_sv;
   const int n = read_n_rows(n_rows, T, nullptr);
   if (threadIdx.x == 0) sh_sv = choose_split(n, vt, ctas).sv;
@@ -177,9 +176,6 @@ __global__ void kl_finalize_kernel(const int32_t* __restrict__ n_rows, const int
     const float lse_p = (Mp + log2f(Sp)) * kLn2;
     const float lse_q = (Mq + log2f(Sq)) * kLn2;
     const float k = kLn2 * (A / Sp) - lse_p + lse_q;
-    stats[0 * static_cast<size_t>(ld) + r] = reverse ? lse_p : lse_q;  // lse_s
-    stats[1 * static_cast<size_t>(ld) + r] = reverse ? lse_q : lse_p;  // lse_t
-    stats[2 * static_cast<size_t>(ld) + r] = k;
     const int t = rows[r];
     if (t >= 0 && t < T) kl[t] = k;
   }
@@ -189,8 +185,8 @@ template <class K>
 olive_status launch_dual(const Ctx& c, const CUtensorMap& a, const CUtensorMap& b,
                          const CUtensorMap& a2, const CUtensorMap& b2, const typename K::Params& p) {
   const int smem = core_smem_bytes<K>();
-  if (cudaFuncSetAttribute(gemm_persistent<K>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
-      cudaSuccess)
+  static std::atomic<int> done[kMaxDevices];
+  if (!set_smem_once(reinterpret_cast<const void*>(gemm_persistent<K>), smem, c.device, done))
     return OLIVE_ERR_CUDA;
   gemm_persistent<K><<<c.num_sms, kThreads, smem, c.stream>>>(a, b, a2, b2, p);
   return cudaGetLastError() == cudaSuccess ? OLIVE_OK : OLIVE_ERR_CUDA;
@@ -246,7 +242,7 @@ olive_status launch_divergence(const Ctx& c, const void* h_s, const void* W_s, i
 
   const int vt = (V + KlFwdKern::kBN - 1) / KlFwdKern::kBN;
   kl_finalize_kernel<<<c.num_sms * 4, 256, 0, c.stream>>>(n_rows, rows, T, vt, c.num_sms, p.ld,
-                                                           reverse, w.part, kl, w.stats, dev_status);
+                                                           w.part, kl);
   if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;
   return OLIVE_OK;
 }

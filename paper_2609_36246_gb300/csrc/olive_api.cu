@@ -65,6 +65,15 @@ olive_status make_ctx(void* stream, Ctx* ctx) {
   return OLIVE_OK;
 }
 
+bool set_smem_once(const void* func, int smem, int device, std::atomic<int>* done) {
+  const bool cached = device >= 0 && device < kMaxDevices;
+  if (cached && done[device].load(std::memory_order_acquire) == smem) return true;
+  if (cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
+    return false;
+  if (cached) done[device].store(smem, std::memory_order_release);
+  return true;
+}
+
 bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
                     uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
   auto fn = encode_fn();
@@ -235,7 +244,7 @@ static KlWs carve_kl_impl(void* ws, int64_t T, int64_t ds, int64_t dt, int64_t V
   w.tc = slab_rows(Tpad, V);
   w.hcs = c.take(2ull * Tpad * ds);
   w.hct = c.take(2ull * Tpad * dt);
-  w.part = w.stats = w.s2 = w.part5 = nullptr;
+  w.part = w.s2 = w.part5 = nullptr;
   w.g = nullptr;
   if (grad) {
     w.g = c.take(2ull * w.tc * vpad(V));
@@ -245,7 +254,6 @@ static KlWs carve_kl_impl(void* ws, int64_t T, int64_t ds, int64_t dt, int64_t V
     w.part5 = static_cast<float*>(c.take(4ull * 5 * w.tc * ceil_div(V, 256)));
   } else {
     w.part = static_cast<float*>(c.take(4ull * 5 * kSvMax * Tpad));
-    w.stats = static_cast<float*>(c.take(4ull * 3 * Tpad));
   }
   if (total) *total = c.off;
   return w;

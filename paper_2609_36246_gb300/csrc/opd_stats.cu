@@ -357,8 +357,8 @@ olive_status launch_opd_stats(const Ctx& c, const void* h_s, const void* W_s, in
   p.part_tv = w.part_tv;
   p.part_ti = w.part_ti;
   const int smem = core_smem_bytes<OpdKern>();
-  if (cudaFuncSetAttribute(gemm_persistent<OpdKern>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           smem) != cudaSuccess)
+  static std::atomic<int> done[kMaxDevices];
+  if (!set_smem_once(reinterpret_cast<const void*>(gemm_persistent<OpdKern>), smem, c.device, done))
     return OLIVE_ERR_CUDA;
   gemm_persistent<OpdKern><<<c.num_sms, kThreads, smem, c.stream>>>(mHs, mWs, mHt, mWt, p);
   if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;

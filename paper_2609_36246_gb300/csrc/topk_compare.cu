@@ -14,7 +14,7 @@
 // 16-byte loads split across lanes and a shuffle reduction.
 //
 // topk_kl_prep turns those lists into the sparse part of the top-K KL
-// gradient (see lmhead_bwd.cu): per masked row, with g = grad_kl[t] inv_tau,
+// gradient (see lmhead_fused.cu): per masked row, with g = grad_kl[t] inv_tau,
 // P_S = sum_j exp(l_j) and A = kl_topk[t] + P_S,
 //   coef[t]   = -g A                       (multiplies p_s(u) for every u)
 //   val[t, j] = g exp(l_j) (l_j - q_j + 1 - A)   (G at the j-th id of S)

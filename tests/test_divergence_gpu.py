@@ -166,3 +166,23 @@ def test_forward_kl_with_a_collapsed_student():
                                         "forward", grad_kl=gk.astype(np.float64))
     assert_close_logp(kl, rkl, "kl")
     assert_close_grad(dhs, rdhs, "dH_s")
+
+
+@pytest.mark.slow
+def test_kl_medium_sampled_rows():
+    """4096 rows, d_s = 1024, d_t = 1536, V = 65536 (W_s and W_t together
+    larger than L2; ~2 GB on the device): KL and d/dh_s on sampled rows."""
+    rng = np.random.default_rng(41)
+    T, ds, dt, V = 4096, 1024, 1536, 65536
+    hs = synth.rms_hidden_bf16(rng, (T, ds))
+    Ws = synth.normal_bf16(rng, (V, ds), 0.02)
+    ht = synth.rms_hidden_bf16(rng, (T, dt))
+    Wt = synth.normal_bf16(rng, (V, dt), 0.02)
+    rows = np.arange(T, dtype=np.int32)
+    gk = rng.uniform(0.5, 1.5, size=T).astype(np.float32)
+    kl, dhs = _gpu(hs, Ws, ht, Wt, rows, gk, "reverse", grad_dtype=torch.bfloat16)
+    pick = sample_rows(rows, 16, seed=4)
+    rkl, rdhs = oracle.token_divergence(to_f32(hs), to_f32(Ws), to_f32(ht), to_f32(Wt), pick,
+                                        grad_kl=gk.astype(np.float64))
+    assert_close_logp(kl[pick], rkl[pick], "kl")
+    assert rel_frob(dhs[pick], rdhs[pick]) <= 1e-2
