@@ -119,3 +119,19 @@ def test_kl_workload_sampled():
                                       with_dW=False)
     for t in pick:
         assert_close_grad(dh[t], rdh[t], f"dH_s[{t}]")
+
+
+def test_several_slabs(monkeypatch):
+    """The slab cap lowered to 128 rows: the sparse correction and dW's fp32
+    accumulation run across slabs of the one-launch backward."""
+    monkeypatch.setenv("OLIVE_SLAB_ROWS", "128")
+    rng = np.random.default_rng(61)
+    T, ds, dt, V, K = 700, 64, 96, 1500, 8
+    hs, Ws, ht, Wt = _models(rng, T, ds, dt, V)
+    rows = _decided_rows(hs, Ws, ht, Wt, np.arange(T), K, 1.0)
+    assert len(rows) > 4 * 128
+    g = rng.uniform(0.5, 2.0, size=T)
+    dh, dw, _, _, _ = _gpu(hs, Ws, ht, Wt, rows, K, g, grad_dtype=torch.bfloat16)
+    rdh, rdw = oracle.token_topk_kl_bwd(to_f64(hs), to_f64(Ws), to_f64(ht), to_f64(Wt), rows, K, grad=g)
+    assert_close_grad(dh[rows], rdh[rows], "dH_s")
+    assert_close_grad(dw, rdw, "dW_s")

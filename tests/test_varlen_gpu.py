@@ -3,7 +3,8 @@ cut at U[10%,90%] of each length (~557k packed tokens, ~278k masked rows),
 d = 4096, V = 151936: splice/pack -> forward -> backward on the GPU, with the
 bf16 inputs drawn by synth; checked against the oracle on sampled rows and by
 properties that hold at any size.  The masked rows span many G slabs, so dW
-goes through the fp32 accumulator."""
+goes through the fp32 accumulator.  The single-pass call
+(olive_token_loss_fwd_bwd) runs on the same batch and must agree."""
 
 import math
 
@@ -61,3 +62,14 @@ def test_varlen_end_to_end():
     off[o["rows"]] = False
     off_idx = torch.from_numpy(np.nonzero(off)[0][::97]).cuda()
     assert not dh[off_idx].any().item()
+    # the single-pass call (15 slabs of 18304 rows here) against the two calls above
+    logp2, lse2, loss2, dh2, dw2 = B.olive_token_loss_fwd_bwd(h.cuda(), Wc, g["targets"], g["rows"],
+                                                              g["n_rows"], gl, reduction="mean",
+                                                              dev_status=st)
+    torch.cuda.synchronize()
+    assert B.status_bits(st) == []
+    assert np.abs(logp2.cpu().numpy()[o["rows"]] - logp[o["rows"]]).max() <= 2e-4
+    assert abs(float(loss2.item()) - float(loss.item())) <= 1e-5 * abs(float(loss.item()))
+    assert rel_frob(dh2[sub].float().cpu().numpy(), ref) <= 1e-2
+    assert (dh2.float() - dh.float()).norm().item() <= 5e-3 * dh.float().norm().item()
+    assert (dw2.float() - dw.float()).norm().item() <= 5e-3 * dw.float().norm().item()
