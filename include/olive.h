@@ -351,6 +351,17 @@ OLIVE_API olive_status olive_token_loss_fwd_bwd(const void* hidden, const void* 
                                                 int32_t* dev_status, void* stream);
 
 /*
+ * olive_scale -- y[i] = x[i] * (*scale) for i < n, x and y of `dtype`
+ * (OLIVE_DTYPE_BF16: fp32 product, round to nearest even; OLIVE_DTYPE_F32),
+ * x == y allowed, both 16-byte aligned; scale fp32 [1] on the device.  The
+ * paper has no counterpart: this lets a caller that learns the loss gradient
+ * g only after olive_token_loss_fwd_bwd (an autograd backward) run that call
+ * with *grad_loss = 1 and scale d_hidden and d_W by g afterwards.
+ */
+OLIVE_API olive_status olive_scale(const void* x, void* y, size_t n, int dtype,
+                                   const float* scale, void* stream);
+
+/*
  * olive_token_divergence -- OPD's per-token divergence between the student
  * pi_theta and the teacher pi_T over the full vocabulary (Section 1; the
  * paper's top-16 approximation is not used): on masked row t,

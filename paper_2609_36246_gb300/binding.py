@@ -76,6 +76,8 @@ def lib() -> ctypes.CDLL:
     L.olive_topk_compare.restype = ctypes.c_int
     L.olive_topk_compare.argtypes = [_P, _P, _I, _P, _P, _I, _I, _F, _I, _P, _P, _P, _P, _P, _P, _P,
                                      _P, _P]
+    L.olive_scale.restype = ctypes.c_int
+    L.olive_scale.argtypes = [_P, _P, _S, ctypes.c_int, _P, _P]
     L.olive_opd_token_stats.restype = ctypes.c_int
     L.olive_opd_token_stats.argtypes = [_P, _P, _I, _P, _P, _I, _P, _P, _I, _I, _F, ctypes.c_int, _I,
                                         _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _S, _P, _P]
@@ -486,24 +488,57 @@ def olive_token_logprob_fwd_noalloc(hidden, W, targets, rows, n_rows, inv_tau: f
     return logp, lse, loss
 
 
+def olive_scale(x, scale, out=None):
+    """out = x * scale (scale: 1-element fp32 CUDA tensor); bf16 or fp32, in
+    place when out is x."""
+    if x.dtype not in DTYPE:
+        raise TypeError("x must be bf16 or fp32")
+    _need(x, x.dtype, "x")
+    _need(scale, torch.float32, "scale")
+    out = torch.empty_like(x) if out is None else out
+    st = lib().olive_scale(_ptr(x), _ptr(out), x.numel(), DTYPE[x.dtype], _ptr(scale), _stream())
+    _check(st, "olive_scale")
+    return out
+
+
 class FusedLMHeadCE(torch.autograd.Function):
-    """Eq. (osd-ce) loss over the masked rows as an autograd op (bf16 grads)."""
+    """Eq. (osd-ce) loss over the masked rows as an autograd op (gradients in
+    the dtype of hidden).
+
+    With a gradient needed, the forward runs olive_token_loss_fwd_bwd with a
+    unit loss gradient (each logit tile computed once) and the backward scales
+    the stored gradients by the incoming one (olive_scale); otherwise, or with
+    single_pass=False, it runs olive_token_logprob_fwd and the backward
+    recomputes the logits (olive_token_loss_bwd)."""
 
     @staticmethod
-    def forward(ctx, hidden, W, targets, rows, n_rows, inv_tau=1.0, reduction="sum"):
-        logp, lse, loss = olive_token_logprob_fwd(hidden, W, targets, rows, n_rows, inv_tau, reduction)
-        ctx.save_for_backward(hidden, W, targets, rows, n_rows, lse)
+    def forward(ctx, hidden, W, targets, rows, n_rows, inv_tau=1.0, reduction="sum",
+                single_pass=True):
         ctx.inv_tau, ctx.reduction = inv_tau, reduction
+        ctx.single = bool(single_pass and (hidden.requires_grad or W.requires_grad))
+        if ctx.single:
+            one = torch.ones(1, dtype=torch.float32, device=hidden.device)
+            _, _, loss, dh, dw = olive_token_loss_fwd_bwd(hidden, W, targets, rows, n_rows, one,
+                                                          inv_tau, reduction, grad_dtype=hidden.dtype)
+            ctx.save_for_backward(dh, dw)
+        else:
+            _, lse, loss = olive_token_logprob_fwd(hidden, W, targets, rows, n_rows, inv_tau,
+                                                   reduction)
+            ctx.save_for_backward(hidden, W, targets, rows, n_rows, lse)
         return loss[0]
 
     @staticmethod
     def backward(ctx, g):
-        hidden, W, targets, rows, n_rows, lse = ctx.saved_tensors
         gl = g.reshape(1).to(torch.float32).contiguous()
+        if ctx.single:
+            dh1, dw1 = ctx.saved_tensors
+            return (olive_scale(dh1, gl), olive_scale(dw1, gl), None, None, None, None, None, None)
+        hidden, W, targets, rows, n_rows, lse = ctx.saved_tensors
         dh, dw = olive_token_loss_bwd(hidden, W, targets, rows, n_rows, lse, gl, ctx.inv_tau,
                                       ctx.reduction, grad_dtype=hidden.dtype)
-        return dh, dw, None, None, None, None, None
+        return dh, dw, None, None, None, None, None, None
 
 
-def fused_lmhead_ce(hidden, W, targets, rows, n_rows, inv_tau=1.0, reduction="sum"):
-    return FusedLMHeadCE.apply(hidden, W, targets, rows, n_rows, inv_tau, reduction)
+def fused_lmhead_ce(hidden, W, targets, rows, n_rows, inv_tau=1.0, reduction="sum",
+                    single_pass=True):
+    return FusedLMHeadCE.apply(hidden, W, targets, rows, n_rows, inv_tau, reduction, single_pass)

@@ -155,6 +155,10 @@ olive_status launch_logprob_fwd(const Ctx& c, const void* hidden, const void* W,
                                 float* logp, float* lse, float* loss, void* ws,
                                 int32_t* dev_status);
 
+// y = x * (*scale) on n bf16 or fp32 elements (x == y allowed).
+olive_status launch_scale(const Ctx& c, const void* x, void* y, size_t n, int dtype,
+                          const float* scale);
+
 // One block sums the per-row loss terms nll[0, n) in a fixed order (fp64).
 olive_status launch_loss_reduce(const Ctx& c, const int32_t* n_rows, int32_t T, const float* nll,
                                 int reduction, float* loss);

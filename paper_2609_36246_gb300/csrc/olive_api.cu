@@ -538,6 +538,18 @@ olive_status olive_opd_token_stats(const void* h_s, const void* W_s, int32_t d_s
                           overlap, kl_topk, workspace, dev_status);
 }
 
+olive_status olive_scale(const void* x, void* y, size_t n, int dtype, const float* scale,
+                         void* stream) {
+  if (!x || !y || !scale) return OLIVE_ERR_INVALID_ARG;
+  if (dtype != OLIVE_DTYPE_BF16 && dtype != OLIVE_DTYPE_F32) return OLIVE_ERR_INVALID_ARG;
+  if (n < 1) return OLIVE_ERR_SHAPE;
+  if (!aligned16(x) || !aligned16(y)) return OLIVE_ERR_ALIGNMENT;
+  Ctx c;
+  olive_status st = make_ctx(stream, &c);
+  if (st != OLIVE_OK) return st;
+  return launch_scale(c, x, y, n, dtype, scale);
+}
+
 olive_status olive_token_divergence(const void* h_s, const void* W_s, int32_t d_s, const void* h_t,
                                     const void* W_t, int32_t d_t, const int32_t* rows,
                                     const int32_t* n_rows, int32_t T, int32_t V, float inv_tau,

@@ -191,6 +191,17 @@ def test_opd_stats_validation(L):
         assert call(outs=[None] * 8 + [P(p)]) in (7, 8)
 
 
+def test_scale_validation(L):
+    keep, p = _fake()
+    P = ctypes.c_void_p
+    assert L.olive_scale(None, P(p), 8, 0, P(p), None) == 1
+    assert L.olive_scale(P(p), P(p), 8, 3, P(p), None) == 1
+    assert L.olive_scale(P(p), P(p), 0, 0, P(p), None) == 2
+    assert L.olive_scale(P(p + 2), P(p), 8, 0, P(p), None) == 3
+    if not torch.cuda.is_available():
+        assert L.olive_scale(P(p), P(p), 8, 1, P(p), None) in (7, 8)
+
+
 def test_fwd_bwd_validation(L):
     keep, p = _fake()
     P = ctypes.c_void_p
