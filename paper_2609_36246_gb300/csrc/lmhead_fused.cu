@@ -21,9 +21,9 @@
 // overwrites the (at most K) entries of S that fall in its tile.  dH and dW
 // are then the cross-entropy tiles unchanged.
 //
-// The logits are recomputed tile by tile and turned into G in the epilogue;
-// G exists only as a bf16 slab of at most tc_max compacted rows in the
-// workspace.  The masked rows are split into equal slabs of <= tc_max rows;
+// One-launch form (olive_token_loss_bwd, olive_topk_kl_bwd): the logits are
+// recomputed tile by tile and turned into G in the epilogue; G exists only as
+// a bf16 slab of at most tc_max compacted rows in the workspace.  The masked rows are split into equal slabs of <= tc_max rows;
 // per slab the work is a list of tiles of three kinds, all 128 x 256 fp32
 // accumulators in TMEM:
 //   GRAD    z = hc . W^T (K = d) -> G tile (bf16) in the slab
