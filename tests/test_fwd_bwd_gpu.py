@@ -176,3 +176,24 @@ def test_fwdbwd_workload_sampled():
     # sum over the vocabulary of dW is sum_r G[r, :] . hc[r] with sum_v G[r, v] = 0
     assert np.abs(dw.astype(np.float64).sum(axis=0)).max() <= 2e-2 * np.abs(dw).sum(axis=0).max()
     assert np.isclose(loss, -logp[o["rows"]].astype(np.float64).sum(), rtol=1e-5)
+
+
+def test_runs_are_bitwise_reproducible():
+    """Every reduction on these paths runs in a fixed order (per-row merges in
+    tile order, the loss in one block, dW per slab): two runs agree bit for
+    bit, for the single-pass call and for the two-call path."""
+    b, h, W = synth.random_case(91, 8, 5000, 192, max_prefix=50, max_cont=400, std_w=0.1)
+    g = gpu_pack(b)
+    hc, Wc = h.cuda(), W.cuda()
+    gl = torch.tensor([0.7], dtype=torch.float32, device="cuda")
+    runs = []
+    for _ in range(2):
+        a = B.olive_token_loss_fwd_bwd(hc, Wc, g["targets"], g["rows"], g["n_rows"], gl, 1.1, "mean")
+        _, lse, loss = B.olive_token_logprob_fwd(hc, Wc, g["targets"], g["rows"], g["n_rows"], 1.1,
+                                                 "mean")
+        dh, dw = B.olive_token_loss_bwd(hc, Wc, g["targets"], g["rows"], g["n_rows"], lse, gl, 1.1,
+                                        "mean")
+        runs.append([t.clone() for t in (*a, lse, loss, dh, dw)])
+    torch.cuda.synchronize()
+    for x, y in zip(*runs):
+        assert torch.equal(x, y)
