@@ -186,3 +186,7 @@ def test_kl_medium_sampled_rows():
                                         grad_kl=gk.astype(np.float64))
     assert_close_logp(kl[pick], rkl[pick], "kl")
     assert rel_frob(dhs[pick], rdhs[pick]) <= 1e-2
+    # the value-only sweep on the same rows
+    kl0, none = _gpu(hs, Ws, ht, Wt, rows, None, "reverse")
+    assert none is None
+    assert np.abs(kl0 - kl).max() <= 1e-4
