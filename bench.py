@@ -240,7 +240,7 @@ def run_ours(args, world, rank, local):
     # computes (two device input sets), as a training loop would overlap them
     barrier(world)
     torch.cuda.synchronize()
-    e_steps = max(1, min(args.steps, 5))
+    e_steps = max(1, min(args.steps, 10))
     host_in = (pre_h, poff_h, con_h, coff_h, hid_h)
     dev_in = [(pre, poff, con, coff, hidden), tuple(torch.empty_like(x) for x in (pre, poff, con, coff, hidden))]
     copy_stream = torch.cuda.Stream()
@@ -254,27 +254,35 @@ def run_ours(args, world, rank, local):
                 dst.copy_(src, non_blocking=True)
         ready[k].record(copy_stream)
 
-    for k in (0, 1):
-        free[k].record(stream)
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    copy_stream.wait_event(e0)
-    copy_in(0)
-    for i in range(e_steps):
-        k = i % 2
-        if i + 1 < e_steps:
-            copy_in(1 - k)
-        stream.wait_event(ready[k])
-        p_, po_, c_, co_, h_ = dev_in[k]
-        pk_e = B.olive_splice_pack(p_, po_, c_, co_, V, T, dev_status=st)
-        B.olive_token_loss_fwd_bwd(h_, W, pk_e["targets"], pk_e["rows"], pk_e["n_rows"], gl, 1.0,
-                                   "sum", torch.bfloat16, ws=ws_fb, dev_status=st,
-                                   out=(logp, lse, loss, dh, dw))
-        free[k].record(stream)
-        loss_h.copy_(loss, non_blocking=True)
-    e1.record(stream)
-    torch.cuda.synchronize()
+    def e2e_steps(n):
+        for k in (0, 1):
+            free[k].record(stream)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        copy_stream.wait_event(e0)
+        copy_in(0)
+        for i in range(n):
+            k = i % 2
+            if i + 1 < n:
+                copy_in(1 - k)
+            stream.wait_event(ready[k])
+            p_, po_, c_, co_, h_ = dev_in[k]
+            pk_e = B.olive_splice_pack(p_, po_, c_, co_, V, T, dev_status=st)
+            B.olive_token_loss_fwd_bwd(h_, W, pk_e["targets"], pk_e["rows"], pk_e["n_rows"], gl,
+                                       1.0, "sum", torch.bfloat16, ws=ws_fb, dev_status=st,
+                                       out=(logp, lse, loss, dh, dw))
+            free[k].record(stream)
+            loss_h.copy_(loss, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0, e1
+
+    # untimed warm-up of this loop (the first use of the copy stream and of the
+    # second input set costs ~14 ms once), then the timed steps
+    e2e_steps(2)
+    barrier(world)
+    e0, e1 = e2e_steps(e_steps)
     e_ms = max_over_ranks(e0.elapsed_time(e1), world)
     h2d = sum(x.numel() * x.element_size() for x in host_in)
     e2e = {"value": N_mask * e_steps * world / (e_ms / 1e3), "unit": "tokens/s",
