@@ -1,7 +1,6 @@
 """fused_lmhead_ce (the Eq. (osd-ce) loss as a torch autograd op over the C
 ABI) and olive_scale, against the oracle."""
 
-import numpy as np
 import pytest
 import torch
 

@@ -2,7 +2,6 @@
 64-wide TMA box), a single-entry vocabulary, a long reduction (d = 8192) and
 a vocabulary of 2^18 + 3 entries (ragged last tile, many segments)."""
 
-import math
 
 import numpy as np
 import pytest

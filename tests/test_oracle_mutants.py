@@ -8,7 +8,6 @@ for the real oracle and at least one must fail for every mutant.  Everything
 runs on the CPU.
 """
 
-import importlib.util
 import json
 import math
 import os

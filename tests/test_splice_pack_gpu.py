@@ -5,7 +5,6 @@ import os
 
 import numpy as np
 import pytest
-import torch
 
 from paper_2609_36246_gb300 import binding as B
 from paper_2609_36246_gb300 import synth
