@@ -1,15 +1,18 @@
 // gemm_core.cuh -- persistent warp-specialised tcgen05 GEMM pipeline shared by
 // the LM-head kernels.
 //
-// One CTA per SM (192 threads):
-//   warps 0-3  epilogue: warp w owns TMEM lanes [32w, 32w+32), i.e. one
-//              accumulator row per thread; a kernel-specific policy turns each
-//              finished 128 x BN fp32 tile into its result.
-//   warp 4     producer: TMA loads of 128 x 64 A and BN x 64 B bf16 tiles
-//              (128-byte swizzle) into a kStages-deep shared-memory ring.
-//   warp 5     MMA issuer: owns the TMEM allocation and issues tcgen05.mma
-//              (M=128, N=BN, K=16) into one of two TMEM accumulators, so the
-//              epilogue of tile n overlaps the MMAs of tile n+1.
+// One CTA per SM, E = Kern::kEpiWarps epilogue warps (4 or 8) + 2:
+//   warps 0..E-1  epilogue: warp w reads TMEM lanes [32 (w % 4), +32), one
+//                 accumulator row per thread; with 8 warps the two warps of a
+//                 lane quadrant split each tile's columns in halves (part
+//                 w / 4), so two threads share a row and the policy merges
+//                 their per-row state at the end of a unit.  A kernel-specific
+//                 policy turns each finished 128 x BN fp32 tile into its result.
+//   warp E        producer: TMA loads of 128 x 64 A and BN x 64 B bf16 tiles
+//                 (128-byte swizzle) into a kStages-deep shared-memory ring.
+//   warp E+1      MMA issuer: owns the TMEM allocation and issues tcgen05.mma
+//                 (M=128, N=BN, K=16) into one of two TMEM accumulators, so
+//                 the epilogue of tile n overlaps the MMAs of tile n+1.
 // A "dual" policy runs two products per tile (e.g. student and teacher
 // logits): K steps [0, nk) use (mapA, mapB) into accumulator columns
 // [0, BN), steps [nk, nk+nk2) use (mapA2, mapB2) into columns [BN, 2 BN).
@@ -19,10 +22,12 @@
 //
 // A Kern policy supplies:
 //   Params (with int32_t* dev_status and uint64_t wait_limit_ns), kBN, kAMn,
-//   kBMn, kDual, kStages, Sched, make_sched(p) (thread 0; may read device
-//   counters such as n_rows), num_units(p,s), unit_len(p,s,u), tile(p,s,u,t),
-//   kEpiSmem (bytes of shared-memory scratch for the epilogue) and Epi with
-//   init(smem), begin(p,s,u,row), tile(p,s,u,t,tc,taddr), end(p,s,u).
+//   kBMn, kDual, kStages, kEpiWarps, Sched, make_sched(p) (thread 0; may read
+//   device counters such as n_rows), num_units(p,s), unit_len(p,s,u),
+//   tile(p,s,u,t), kEpiSmem (bytes of shared-memory scratch for the epilogue)
+//   and Epi with init(smem, part), begin(p,s,u,row), tile(p,s,u,t,tc,taddr),
+//   end(p,s,u).  Every wait of the epilogue ends in one decision of all its
+//   warps, so Epi::end may synchronise them (named barrier 2).
 #pragma once
 
 #include "sm103.cuh"
@@ -46,6 +51,18 @@ constexpr int kProducerWarp = 4;
 constexpr int kMmaWarp = 5;
 constexpr int kStatusTimeoutBit = 1 << 6;  // (1 << OLIVE_ERR_TIMEOUT)
 
+// Thread layout of a policy's CTA.
+template <class Kern>
+struct CoreThreads {
+  static constexpr int kEpiWarps = Kern::kEpiWarps;
+  static_assert(kEpiWarps == 4 || kEpiWarps == 8, "4 or 8 epilogue warps");
+  static constexpr int kEpi = 32 * kEpiWarps;   // epilogue threads
+  static constexpr int kParts = kEpiWarps / 4;  // threads per accumulator row
+  static constexpr int kProducer = kEpiWarps;
+  static constexpr int kMma = kEpiWarps + 1;
+  static constexpr int kAll = 32 * (kEpiWarps + 2);
+};
+
 template <class Kern>
 struct CoreLayout {
   static constexpr int A_BYTES = kBM * kBK * 2;
@@ -67,13 +84,14 @@ struct CoreLayout {
 };
 
 template <class Kern>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(CoreThreads<Kern>::kAll, 1)
     gemm_persistent(const __grid_constant__ CUtensorMap mapA,
                     const __grid_constant__ CUtensorMap mapB,
                     const __grid_constant__ CUtensorMap mapA2,
                     const __grid_constant__ CUtensorMap mapB2,
                     const typename Kern::Params p) {
   using L = CoreLayout<Kern>;
+  using CT = CoreThreads<Kern>;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -102,14 +120,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(tfull_bar(b), 1);
-      mbar_init(tempty_bar(b), kEpiThreads);
+      mbar_init(tempty_bar(b), CT::kEpi);
     }
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
     *sched_smem = Kern::make_sched(p);
     fence_mbar_init();
   }
-  if (warp == kProducerWarp && lane == 0) {
+  if (warp == CT::kProducer && lane == 0) {
     tma_prefetch_desc(&mapA);
     tma_prefetch_desc(&mapB);
     if constexpr (Kern::kDual) {
@@ -117,7 +135,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&mapB2);
     }
   }
-  if (warp == kMmaWarp) {
+  if (warp == CT::kMma) {
     tmem_alloc(smem_u32(tmem_slot), L::TMEM_COLS);
     tmem_relinquish();
   }
@@ -130,7 +148,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const WaitCtl ctl{abort_flag, p.wait_limit_ns};
   const int n_units = Kern::num_units(p, sched);
 
-  if (warp == kProducerWarp) {
+  if (warp == CT::kProducer) {
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
@@ -176,7 +194,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     __syncwarp();
-  } else if (warp == kMmaWarp) {
+  } else if (warp == CT::kMma) {
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16(kBM, Kern::kBN, Kern::kAMn, Kern::kBMn);
       int stage = 0;
@@ -226,21 +244,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncwarp();
   } else {
-    // epilogue warps 0-3: thread = accumulator row = TMEM lane
-    const int row = threadIdx.x;
-    const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
+    // epilogue warps: thread = accumulator row = TMEM lane (quadrant warp % 4)
+    const int quad = warp & 3;
+    const int row = quad * 32 + lane;
+    const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16);
     int buf = 0;
     uint32_t aphase = 0;
     bool ok = true;
     typename Kern::Epi epi;
-    epi.init(misc + L::MISC_BYTES);
+    epi.init(misc + L::MISC_BYTES, warp >> 2);
     for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
       const int nt = Kern::unit_len(p, sched, u);
       epi.begin(p, sched, u, row);
       for (int t = 0; t < nt; ++t) {
         const TileC tc = Kern::tile(p, sched, u, t);
-        // warp-uniform decision: tcgen05.ld below is a warp-collective
-        if (!__all_sync(0xffffffffu, mbar_wait(tfull_bar(buf), aphase, ctl))) { ok = false; break; }
+        // one decision for all epilogue threads: tcgen05.ld below is a warp
+        // collective and Epi::end may synchronise the epilogue warps
+        if (!named_bar_and(1, CT::kEpi, mbar_wait(tfull_bar(buf), aphase, ctl))) { ok = false; break; }
         tc_fence_after();
         epi.tile(p, sched, u, t, tc, lane_addr + static_cast<uint32_t>(buf * L::ACC_COLS));
         tc_fence_before();
@@ -255,7 +275,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   if (threadIdx.x == 0 && *abort_flag) atomicOr(p.dev_status, kStatusTimeoutBit);
-  if (warp == kMmaWarp) {
+  if (warp == CT::kMma) {
     tc_fence_after();
     tmem_dealloc(tmem_base, L::TMEM_COLS);
   }
@@ -264,6 +284,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 template <class Kern>
 inline int core_smem_bytes() {
   return CoreLayout<Kern>::SMEM_BYTES;
+}
+
+template <class Kern>
+inline int core_threads() {
+  return CoreThreads<Kern>::kAll;
 }
 
 }  // namespace olive

@@ -103,8 +103,8 @@ OpdWs carve_opd(void* ws, int64_t T, int64_t ds, int64_t dt);
 struct FbWs {
   void* hc;        // bf16 [Tpad, d]
   void* g;         // bf16 [Tc, Vpad]: e = 2^(x - m_tile), then G
-  float* part_zm;  // [Tc, vt] tile max (base 2)
-  float* part_zs;  // [Tc, vt] tile sums
+  float* part_zm;  // [Tc, ceil(V/128)] half-tile max (base 2)
+  float* part_zs;  // [Tc, ceil(V/128)] half-tile sums
   float* zy;       // [Tc] target logits of the slab
   float* nll;      // [Tpad] per-row loss terms
   float* dw_acc;   // fp32 [V, d] (bf16 output only)
@@ -119,7 +119,7 @@ struct KlWs {
   float* part;    // [5, kSvMax, Tpad] (value only)
   void* g;        // bf16 [Tc, Vpad]: e_s, then G (gradient only)
   float* s2;      // fp32 [Tc, Vpad]: second slab (gradient only)
-  float* part5;   // [5, Tc, ceil(V/256)] per-tile partials (gradient only)
+  float* part5;   // [5, Tc, ceil(V/128)] per-half-tile partials (gradient only)
   int64_t tc;
 };
 size_t kl_ws_bytes(int64_t T, int64_t ds, int64_t dt, int64_t V, int grad);

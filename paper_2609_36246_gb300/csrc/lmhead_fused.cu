@@ -71,6 +71,16 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kBN = 256;
 constexpr int kStages = 4;
+// Eight epilogue warps: the two warps of a TMEM lane quadrant (warp % 4) take
+// the two 128-column halves (part = warp / 4) of every tile, which halves the
+// epilogue of the tile kinds whose accumulator cannot be double-buffered
+// (KLZ).  Warp 8 is the producer, warp 9 the MMA issuer.
+constexpr int kFEpiWarps = 8;
+constexpr int kFEpi = 32 * kFEpiWarps;
+constexpr int kFProducer = kFEpiWarps;
+constexpr int kFMma = kFEpiWarps + 1;
+constexpr int kFThreads = 32 * (kFEpiWarps + 2);
+constexpr int kHalf = kBN / 2;
 
 enum Kind : int { K_NONE = -1, K_GRAD = 0, K_KLZ = 1, K_DH = 2, K_DW = 3, K_ZSAVE = 4 };
 // phases: one launch of every tile kind with dependency waits, or one slab's
@@ -98,12 +108,12 @@ struct FusedParams {
   const int32_t* sp_ids;     // top-K KL, [T, sp_k]: the ids of S
   int32_t sp_k;              // 0: cross-entropy targets; K: top-K KL
   int32_t phase, slab;       // Phase; the slab of PH_Z / PH_DHDW
-  float* part_zm;            // PH_Z: [tc, vt] tile max (base 2) per slab row
-  float* part_zs;            // PH_Z: [tc, vt] tile sum of 2^(x - max)
+  float* part_zm;            // PH_Z: [tc, vh] half-tile max (base 2) per slab row
+  float* part_zs;            // PH_Z: [tc, vh] half-tile sum of 2^(x - max)
   float* zy_s;               // PH_Z: [tc] target logit (natural units)
   float* s2;                 // KLZ: fp32 slab, [tc, ldg] (reverse) or [tc / 2, 2 ldg] (forward)
-  float* part5;              // KLZ: [5][tc][vt] m_s, s_s, m_t, s_t, A per (row, tile)
-  int64_t plane5;            // tc * vt
+  float* part5;              // KLZ: [5][tc][vh] m_s, s_s, m_t, s_t, A per (row, half-tile)
+  int64_t plane5;            // tc * vh
   int32_t kl;                // 0: cross-entropy, 1: divergence
   int32_t reverse;           // KL direction
   int32_t T, d, d2, V, reduction, out_dtype, group_rows;
@@ -119,7 +129,7 @@ struct FusedParams {
 };
 
 struct Plan {
-  int n, n_slabs, rps, vt, ntd, mtv, bn_grad;
+  int n, n_slabs, rps, vt, vh, ntd, mtv, bn_grad;
   float coef;  // CE: g * inv_tau (/ N_mask for the mean)
 };
 
@@ -144,6 +154,7 @@ __device__ Plan make_plan(const FusedParams& p) {
   pl.rps = sp.rps;
   pl.bn_grad = 256;
   pl.vt = (p.V + pl.bn_grad - 1) / pl.bn_grad;
+  pl.vh = (p.V + kHalf - 1) / kHalf;
   pl.ntd = (p.d + kBN - 1) / kBN;
   pl.mtv = (p.V + kBM - 1) / kBM;
   pl.coef = 0.f;
@@ -281,7 +292,8 @@ __device__ __forceinline__ void store_row32(void* base, size_t off, int dtype, i
 }
 
 // ------------------------------------------------------------- epilogues ---
-__device__ void epi_grad(const FusedParams& p, const Plan& pl, const Unit& x, int row, uint32_t taddr) {
+__device__ void epi_grad(const FusedParams& p, const Plan& pl, const Unit& x, int row, int part,
+                         uint32_t taddr) {
   const int r_local = x.i * kBM + row;
   const int r = x.row0 + r_local;
   bool valid = r_local < x.in_s;
@@ -300,7 +312,7 @@ __device__ void epi_grad(const FusedParams& p, const Plan& pl, const Unit& x, in
   __nv_bfloat16* grow = p.g + static_cast<size_t>(r_local) * p.ldg;
   const int n0 = x.j * kBN;
 #pragma unroll 1
-  for (int c = 0; c < kBN; c += 32) {
+  for (int c = part * kHalf; c < (part + 1) * kHalf; c += 32) {
     const int col0 = n0 + c;
     if (col0 >= p.V) break;
     uint32_t a[32];
@@ -315,14 +327,15 @@ __device__ void epi_grad(const FusedParams& p, const Plan& pl, const Unit& x, in
     store_row32(grow, col0, OLIVE_DTYPE_BF16, p.V - col0, g);
   }
   if (p.sp_k > 0 && valid) {
-    // the entries of S in this tile: same thread, same addresses, so these
-    // stores land after the softmax values written above
-    const int n1 = min(n0 + kBN, p.V);
+    // the entries of S in this half tile: same thread, same addresses, so
+    // these stores land after the softmax values written above
+    const int h0 = n0 + part * kHalf;
+    const int h1 = min(h0 + kHalf, p.V);
     const size_t o = static_cast<size_t>(t) * p.sp_k;
 #pragma unroll 1
     for (int k = 0; k < p.sp_k; ++k) {
       const int u = p.sp_ids[o + k];
-      if (u >= n0 && u < n1) grow[u] = __float2bfloat16_rn(p.sp_val[o + k]);
+      if (u >= h0 && u < h1) grow[u] = __float2bfloat16_rn(p.sp_val[o + k]);
     }
   }
 }
@@ -332,7 +345,7 @@ __device__ void epi_grad(const FusedParams& p, const Plan& pl, const Unit& x, in
 // sums s_s, s_t of 2^(x - m), A = sum e_p (x_p - x_q) in the primary
 // distribution's scale (p = student for the reverse KL, teacher for the
 // forward KL), e_s in bf16 into the G slab and the fp32 second slab
-__device__ void epi_klz(const FusedParams& p, const Plan& pl, const Unit& x, int row,
+__device__ void epi_klz(const FusedParams& p, const Plan& pl, const Unit& x, int row, int part,
                         uint32_t taddr) {
   const int r_local = x.i * kBM + row;
   bool valid = r_local < x.in_s;
@@ -343,7 +356,7 @@ __device__ void epi_klz(const FusedParams& p, const Plan& pl, const Unit& x, int
   const int n0 = x.j * kBN;
   float ms = -INFINITY, mt = -INFINITY;
 #pragma unroll 1
-  for (int c = 0; c < kBN; c += 32) {
+  for (int c = part * kHalf; c < (part + 1) * kHalf; c += 32) {
     const int col0 = n0 + c;
     if (col0 >= p.V) break;
     uint32_t a[32], b[32];
@@ -363,7 +376,7 @@ __device__ void epi_klz(const FusedParams& p, const Plan& pl, const Unit& x, int
   float* srow = p.s2 + static_cast<size_t>(r_local) * p.ldg * (p.reverse ? 1 : 2);
   float ss = 0.f, st = 0.f, A = 0.f;
 #pragma unroll 1
-  for (int c = 0; c < kBN; c += 32) {
+  for (int c = part * kHalf; c < (part + 1) * kHalf; c += 32) {
     const int col0 = n0 + c;
     if (col0 >= p.V) break;
     uint32_t a[32], b[32];
@@ -410,8 +423,8 @@ __device__ void epi_klz(const FusedParams& p, const Plan& pl, const Unit& x, int
       }
     }
   }
-  if (valid) {
-    const size_t o = static_cast<size_t>(r_local) * pl.vt + x.j;
+  if (valid && n0 + part * kHalf < p.V) {  // a half past V has no partial slot
+    const size_t o = static_cast<size_t>(r_local) * pl.vh + 2 * x.j + part;
     p.part5[o] = ms;
     p.part5[p.plane5 + o] = ss;
     p.part5[2 * p.plane5 + o] = mt;
@@ -423,7 +436,7 @@ __device__ void epi_klz(const FusedParams& p, const Plan& pl, const Unit& x, int
 // forward tile of the fused forward + backward: per row the tile's max and
 // sum of 2^(x - max) in base-2 units, e = 2^(x - max) stored in bf16 at the
 // row's G slab columns (zeros on padding rows), and the exact target logit
-__device__ void epi_zsave(const FusedParams& p, const Plan& pl, const Unit& x, int row,
+__device__ void epi_zsave(const FusedParams& p, const Plan& pl, const Unit& x, int row, int part,
                           uint32_t taddr) {
   const int r_local = x.i * kBM + row;
   bool valid = r_local < x.in_s;
@@ -436,7 +449,7 @@ __device__ void epi_zsave(const FusedParams& p, const Plan& pl, const Unit& x, i
   const int n0 = x.j * kBN;
   float tm = -INFINITY;
 #pragma unroll 1
-  for (int c = 0; c < kBN; c += 32) {
+  for (int c = part * kHalf; c < (part + 1) * kHalf; c += 32) {
     const int col0 = n0 + c;
     if (col0 >= p.V) break;
     uint32_t a[32];
@@ -455,7 +468,7 @@ __device__ void epi_zsave(const FusedParams& p, const Plan& pl, const Unit& x, i
   __nv_bfloat16* grow = p.g + static_cast<size_t>(r_local) * p.ldg;
   float ts = 0.f;
 #pragma unroll 1
-  for (int c = 0; c < kBN; c += 32) {
+  for (int c = part * kHalf; c < (part + 1) * kHalf; c += 32) {
     const int col0 = n0 + c;
     if (col0 >= p.V) break;
     uint32_t a[32];
@@ -470,14 +483,14 @@ __device__ void epi_zsave(const FusedParams& p, const Plan& pl, const Unit& x, i
     }
     store_row32(grow, col0, OLIVE_DTYPE_BF16, nv, e);
   }
-  if (valid) {
-    const size_t o = static_cast<size_t>(r_local) * pl.vt + x.j;
+  if (valid && n0 + part * kHalf < p.V) {  // a half past V has no partial slot
+    const size_t o = static_cast<size_t>(r_local) * pl.vh + 2 * x.j + part;
     p.part_zm[o] = tm;
     p.part_zs[o] = ts;
   }
 }
 
-__device__ void epi_dh(const FusedParams& p, const Unit& x, int row, uint32_t taddr) {
+__device__ void epi_dh(const FusedParams& p, const Unit& x, int row, int part, uint32_t taddr) {
   const int r_local = x.i * kBM + row;
   int t = -1;
   if (r_local < x.in_s) {
@@ -486,7 +499,7 @@ __device__ void epi_dh(const FusedParams& p, const Unit& x, int row, uint32_t ta
   }
   const int n0 = x.j * kBN;
 #pragma unroll 1
-  for (int c = 0; c < kBN; c += 32) {
+  for (int c = part * kHalf; c < (part + 1) * kHalf; c += 32) {
     const int col0 = n0 + c;
     if (col0 >= p.d) break;
     uint32_t a[32];
@@ -500,14 +513,14 @@ __device__ void epi_dh(const FusedParams& p, const Unit& x, int row, uint32_t ta
   }
 }
 
-__device__ void epi_dw(const FusedParams& p, const Plan& pl, const Unit& x, int row, uint32_t taddr,
-                       int nk) {
+__device__ void epi_dw(const FusedParams& p, const Plan& pl, const Unit& x, int row, int part,
+                       uint32_t taddr, int nk) {
   const int v = x.i * kBM + row;
   const bool first = x.s == 0;
   const bool last = x.s == pl.n_slabs - 1;
   const int n0 = x.j * kBN;
 #pragma unroll 1
-  for (int c = 0; c < kBN; c += 32) {
+  for (int c = part * kHalf; c < (part + 1) * kHalf; c += 32) {
     const int col0 = n0 + c;
     if (col0 >= p.d) break;
     float g[32];
@@ -561,7 +574,7 @@ struct FusedLayout {
   static constexpr uint32_t TMEM_COLS = 512;
 };
 
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kFThreads, 1)
     lmhead_fused_kernel(const __grid_constant__ FusedMaps maps, const FusedParams p) {
   using L = FusedLayout;
   extern __shared__ uint8_t smem_raw[];
@@ -591,18 +604,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(tfull_bar(b), 1);
-      mbar_init(tempty_bar(b), kEpiThreads);
+      mbar_init(tempty_bar(b), kFEpi);
     }
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
     *plan_smem = make_plan(p);
     fence_mbar_init();
   }
-  if (warp == kProducerWarp && lane == 0) {
+  if (warp == kFProducer && lane == 0) {
 #pragma unroll
     for (int m = 0; m < 6; ++m) tma_prefetch_desc(&maps.m[m]);
   }
-  if (warp == kMmaWarp) {
+  if (warp == kFMma) {
     tmem_alloc(smem_u32(tmem_slot), L::TMEM_COLS);
     tmem_relinquish();
   }
@@ -620,7 +633,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int total = total_units(p, pl);
 
-  if (warp == kProducerWarp) {
+  if (warp == kFProducer) {
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
@@ -687,7 +700,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     __syncwarp();
-  } else if (warp == kMmaWarp) {
+  } else if (warp == kFMma) {
     if (lane == 0) {
       int stage = 0, buf = 0;
       uint32_t phase = 0, aphase = 0;
@@ -738,8 +751,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncwarp();
   } else {
-    const int row = threadIdx.x;
-    const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
+    const int quad = warp & 3;
+    const int part = warp >> 2;
+    const int row = quad * 32 + lane;
+    const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16);
     int buf = 0;
     uint32_t aphase = 0;
     // every wait below ends in one group decision (bar.red.and), so the 128
@@ -748,21 +763,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       const Unit x = decode(p, pl, u);
       int nk, nk2;
       unit_ksteps(p, x, nk, nk2);
-      if (!named_bar_and(1, kEpiThreads, mbar_wait(tfull_bar(buf), aphase, ctl))) break;
+      if (!named_bar_and(1, kFEpi, mbar_wait(tfull_bar(buf), aphase, ctl))) break;
       tc_fence_after();
       __syncwarp();
       const uint32_t taddr = lane_addr + static_cast<uint32_t>(buf * kBN);
       if (x.kind == K_DW && x.s > 0 && p.phase == PH_ALL) {
         // the fp32 partial of the previous slab must be visible before it is read
-        const bool seen = row == 0 ? wait_counter(ctr_grad(p, x.s), units_grad(pl, x.mt), ctl) : true;
-        if (!named_bar_and(1, kEpiThreads, seen)) break;
+        const bool seen =
+            threadIdx.x == 0 ? wait_counter(ctr_grad(p, x.s), units_grad(pl, x.mt), ctl) : true;
+        if (!named_bar_and(1, kFEpi, seen)) break;
       }
       switch (x.kind) {
-        case K_GRAD: epi_grad(p, pl, x, row, taddr); break;
-        case K_KLZ: epi_klz(p, pl, x, row, taddr); break;
-        case K_ZSAVE: epi_zsave(p, pl, x, row, taddr); break;
-        case K_DH: epi_dh(p, x, row, taddr); break;
-        case K_DW: epi_dw(p, pl, x, row, taddr, nk); break;
+        case K_GRAD: epi_grad(p, pl, x, row, part, taddr); break;
+        case K_KLZ: epi_klz(p, pl, x, row, part, taddr); break;
+        case K_ZSAVE: epi_zsave(p, pl, x, row, part, taddr); break;
+        case K_DH: epi_dh(p, x, row, part, taddr); break;
+        case K_DW: epi_dw(p, pl, x, row, part, taddr, nk); break;
         default: break;
       }
       tc_fence_before();
@@ -771,8 +787,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       // publish: every epilogue thread's stores, then one release increment
       fence_proxy_async_global();
       __threadfence();
-      named_bar_sync(1, kEpiThreads);
-      if (row == 0 && p.phase == PH_ALL) {
+      named_bar_sync(1, kFEpi);
+      if (threadIdx.x == 0 && p.phase == PH_ALL) {
         if (x.kind == K_GRAD) {
           red_release_add(ctr_row(p, x.s, x.i), 1u);
           red_release_add(ctr_grad(p, x.s), 1u);
@@ -786,7 +802,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   if (threadIdx.x == 0 && *abort_flag) atomicOr(p.dev_status, kStatusTimeoutBit);
-  if (warp == kMmaWarp) {
+  if (warp == kFMma) {
     tc_fence_after();
     tmem_dealloc(tmem_base, L::TMEM_COLS);
   }
@@ -812,7 +828,7 @@ __device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2
 // max is one broadcast load).  The target entry uses the exact z_y.
 __global__ void __launch_bounds__(256)
     conv_kernel(const int32_t* __restrict__ n_rows, const int32_t* __restrict__ rows,
-                const int32_t* __restrict__ targets, int T, int V, int tc, int slab, int vt,
+                const int32_t* __restrict__ targets, int T, int V, int tc, int slab, int vh,
                 int64_t ldg, float inv_tau, int reduction, const float* __restrict__ grad_loss,
                 const float* __restrict__ part_zm, const float* __restrict__ part_zs,
                 const float* __restrict__ zy_s, __nv_bfloat16* g, float* __restrict__ logp,
@@ -835,10 +851,10 @@ __global__ void __launch_bounds__(256)
       continue;
     }
     const int y = targets[t];
-    const float* zm = part_zm + static_cast<size_t>(r) * vt;
-    const float* zs = part_zs + static_cast<size_t>(r) * vt;
+    const float* zm = part_zm + static_cast<size_t>(r) * vh;
+    const float* zs = part_zs + static_cast<size_t>(r) * vh;
     float m = -INFINITY, sum = 0.f;
-    for (int j = lane; j < vt; j += 32) lse_merge(m, sum, zm[j], zs[j]);
+    for (int j = lane; j < vh; j += 32) lse_merge(m, sum, zm[j], zs[j]);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
@@ -869,7 +885,7 @@ __global__ void __launch_bounds__(256)
       for (int q = 0; q < 4; ++q) {
         const int idx = base + 32 * q + lane;
         if (idx >= nvec) continue;
-        const float sc = coef * fast_exp2(zm[(base >> 5) + q] - lse2);
+        const float sc = coef * fast_exp2(zm[idx >> 4] - lse2);  // 16 vectors per half tile
         __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&v[q]);
         const int col = idx * 8;
 #pragma unroll
@@ -913,7 +929,7 @@ __device__ __forceinline__ void lse_merge3(float& m, float& s, float& a, float m
 // with coef = grad_kl[t] inv_tau.
 __global__ void __launch_bounds__(256)
     conv_kl_kernel(const int32_t* __restrict__ n_rows, const int32_t* __restrict__ rows, int T,
-                   int V, int tc, int slab, int vt, int64_t ldg, float inv_tau, int reverse,
+                   int V, int tc, int slab, int vh, int64_t ldg, float inv_tau, int reverse,
                    const float* __restrict__ grad_kl, const float* __restrict__ part5,
                    int64_t plane5, const float* __restrict__ s2, __nv_bfloat16* g,
                    float* __restrict__ kl) {
@@ -928,13 +944,13 @@ __global__ void __launch_bounds__(256)
   for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < in_s; r += warps) {
     const int t = rows[row0 + r];
     if (t < 0 || t >= T) continue;  // reported by the gather; the G row is zero
-    const float* pms = part5 + static_cast<size_t>(r) * vt;
+    const float* pms = part5 + static_cast<size_t>(r) * vh;
     const float* pss = pms + plane5;
     const float* pmt = pms + 2 * plane5;
     const float* pst = pms + 3 * plane5;
     const float* pa = pms + 4 * plane5;
     float mp = -INFINITY, sp_ = 0.f, A = 0.f, mq = -INFINITY, sq = 0.f;
-    for (int j = lane; j < vt; j += 32) {
+    for (int j = lane; j < vh; j += 32) {
       if (reverse) {
         lse_merge3(mp, sp_, A, pms[j], pss[j], pa[j]);
         lse_merge(mq, sq, pmt[j], pst[j]);
@@ -981,7 +997,7 @@ __global__ void __launch_bounds__(256)
         for (int q = 0; q < 2; ++q) {
           const int idx = base + 32 * q + lane;
           if (idx >= nvec) continue;
-          const float scs = coef * fast_exp2(pms[(base >> 5) + q] - lse2_s);
+          const float scs = coef * fast_exp2(pms[idx >> 4] - lse2_s);  // 16 vectors per half tile
           const float dd[8] = {dl[q][0].x, dl[q][0].y, dl[q][0].z, dl[q][0].w,
                                dl[q][1].x, dl[q][1].y, dl[q][1].z, dl[q][1].w};
           __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&v[q]);
@@ -1007,7 +1023,7 @@ __global__ void __launch_bounds__(256)
         float4 pr[4];
 #pragma unroll
         for (int q = 0; q < 4; ++q) pr[q] = srow[4 * idx + q];
-        const int j = base >> 5;
+        const int j = idx >> 4;  // 16 vectors per half tile
         const float os = pms[j] - lse2_s;
         const float ot = pmt[j] - lse2_t;
         const float xy[16] = {pr[0].x, pr[0].y, pr[0].z, pr[0].w, pr[1].x, pr[1].y, pr[1].z, pr[1].w,
@@ -1040,7 +1056,7 @@ olive_status launch_lmhead_fused(const Ctx& c, const FusedMaps& maps, const Fuse
   const bool cached = c.device >= 0 && c.device < kMaxDevices;
   if (!cached || fits[c.device].load(std::memory_order_acquire) == 0) {
     int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, lmhead_fused_kernel, kThreads,
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, lmhead_fused_kernel, kFThreads,
                                                       smem) != cudaSuccess ||
         per_sm < 1)
       return OLIVE_ERR_CUDA;
@@ -1048,7 +1064,7 @@ olive_status launch_lmhead_fused(const Ctx& c, const FusedMaps& maps, const Fuse
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(c.num_sms);
-  cfg.blockDim = dim3(kThreads);
+  cfg.blockDim = dim3(kFThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = c.stream;
   // the one-launch form waits across CTAs, so every CTA must be resident: a
@@ -1152,7 +1168,7 @@ olive_status launch_loss_fwd_bwd(const Ctx& c, const void* hidden, const void* W
   const FbWs w = carve_fb(ws, T, d, V, grad_dtype);
   const int64_t ldg = vpad(V);
   const size_t elt = grad_dtype == OLIVE_DTYPE_BF16 ? 2 : 4;
-  const int vt = static_cast<int>(ceil_div(V, kBN));
+  const int vh = static_cast<int>(ceil_div(V, kHalf));
 
   olive_status st = launch_gather_rows(c, hidden, rows, n_rows, T, d, w.hc, dev_status);
   if (st != OLIVE_OK) return st;
@@ -1196,7 +1212,7 @@ olive_status launch_loss_fwd_bwd(const Ctx& c, const void* hidden, const void* W
     p.phase = PH_Z;
     if ((st = launch_lmhead_fused(c, maps, p)) != OLIVE_OK) return st;
     conv_kernel<<<conv_blocks, 256, 0, c.stream>>>(
-        n_rows, rows, targets, T, V, static_cast<int>(w.tc), s, vt, ldg, inv_tau, reduction,
+        n_rows, rows, targets, T, V, static_cast<int>(w.tc), s, vh, ldg, inv_tau, reduction,
         grad_loss, w.part_zm, w.part_zs, w.zy, static_cast<__nv_bfloat16*>(w.g), logp, lse, w.nll,
         dev_status);
     if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;
@@ -1214,7 +1230,7 @@ olive_status launch_kl_fwd_bwd(const Ctx& c, const void* hcs, const void* hct, c
                                int32_t* dev_status) {
   const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
   const int64_t ldg = vpad(V);
-  const int vt = static_cast<int>(ceil_div(V, kBN));
+  const int vh = static_cast<int>(ceil_div(V, kHalf));
   FusedMaps maps;
   if (!encode_bf16_2d(&maps.m[0], hcs, d_s, Tpad, 2ull * d_s, 64, 128) ||
       !encode_bf16_2d(&maps.m[1], W_s, d_s, V, 2ull * d_s, 64, 256) ||
@@ -1240,7 +1256,7 @@ olive_status launch_kl_fwd_bwd(const Ctx& c, const void* hcs, const void* hct, c
   p.dh_out = d_h_s;
   p.s2 = s2;
   p.part5 = part5;
-  p.plane5 = tc * vt;
+  p.plane5 = tc * vh;
   int conv_blocks = static_cast<int>(ceil_div(tc, 8));
   if (conv_blocks > c.num_sms * 16) conv_blocks = c.num_sms * 16;
   olive_status st;
@@ -1249,7 +1265,7 @@ olive_status launch_kl_fwd_bwd(const Ctx& c, const void* hcs, const void* hct, c
     p.phase = PH_Z;
     if ((st = launch_lmhead_fused(c, maps, p)) != OLIVE_OK) return st;
     conv_kl_kernel<<<conv_blocks, 256, 0, c.stream>>>(n_rows, rows, T, V, static_cast<int>(tc), s,
-                                                      vt, ldg, inv_tau, reverse, grad_kl, part5,
+                                                      vh, ldg, inv_tau, reverse, grad_kl, part5,
                                                       p.plane5, s2,
                                                       static_cast<__nv_bfloat16*>(g), kl);
     if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;

@@ -38,6 +38,7 @@ struct FwdKernT {
   static constexpr bool kDual = false;
   static constexpr int kStages = 4;
   static constexpr int kAccBufs = 2;
+  static constexpr int kEpiWarps = 4;
   // stats: per-thread candidate buffer of 32 (value, id) pairs, slot-major
   static constexpr int kEpiSmem = kStats ? 32 * kEpiThreads * 8 : 0;
 
@@ -101,7 +102,7 @@ struct FwdKernT {
     int ti[kStats ? kTopMax : 1];
     float2* buf;  // stats: this thread's candidate slots, stride kEpiThreads
 
-    __device__ void init(uint8_t* smem) {
+    __device__ void init(uint8_t* smem, int) {
       buf = reinterpret_cast<float2*>(smem) + threadIdx.x;
     }
 
@@ -380,7 +381,7 @@ olive_status launch_fwd_core(const Ctx& c, const CUtensorMap& a, const CUtensorM
   static std::atomic<int> done[kMaxDevices];
   if (!set_smem_once(reinterpret_cast<const void*>(gemm_persistent<K>), smem, c.device, done))
     return OLIVE_ERR_CUDA;
-  gemm_persistent<K><<<c.num_sms, kThreads, smem, c.stream>>>(a, b, a, b, p);
+  gemm_persistent<K><<<c.num_sms, core_threads<K>(), smem, c.stream>>>(a, b, a, b, p);
   return cudaGetLastError() == cudaSuccess ? OLIVE_OK : OLIVE_ERR_CUDA;
 }
 

@@ -32,8 +32,11 @@ constexpr float kLn2 = 0.6931471805599453f;
 
 // 128 x 256 tiles per product (student and teacher), both products in one
 // 512-column TMEM accumulator pair: a tile moves the same bytes per FLOP as
-// the cross-entropy forward; the epilogue (a few microseconds against ~45 of
-// MMAs per tile at d_s + d_t = 9216) is not overlapped.
+// the cross-entropy forward, but the epilogue cannot overlap the next tile's
+// MMAs.  Eight epilogue warps shorten it: the two warps of a TMEM lane
+// quadrant take the two 128-column halves of every tile, and at the end of a
+// unit the second half's (m_p, s_p, A, m_q, s_q) is merged into the first's
+// through shared memory.
 struct KlFwdKern {
   static constexpr int kBN = 256;
   static constexpr bool kAMn = false;
@@ -41,7 +44,9 @@ struct KlFwdKern {
   static constexpr bool kDual = true;
   static constexpr int kStages = 4;
   static constexpr int kAccBufs = 1;
-  static constexpr int kEpiSmem = 0;
+  static constexpr int kEpiWarps = 8;
+  static constexpr int kEpiT = 32 * kEpiWarps;
+  static constexpr int kEpiSmem = 5 * 128 * 4;  // the merge area
 
   struct Params {
     int32_t* dev_status;
@@ -83,9 +88,13 @@ struct KlFwdKern {
     return c;
   }
   struct Epi {
-    int r, sg;
+    int r, sg, part;
     float mp, sp, mq, sq, A;
-    __device__ void init(uint8_t*) {}
+    float* merge;  // [5][128]
+    __device__ void init(uint8_t* smem, int prt) {
+      merge = reinterpret_cast<float*>(smem);
+      part = prt;
+    }
     __device__ void begin(const Params& p, const Sched& s, int u, int row) {
       int i;
       unit_pos(p, s, u, i, sg);
@@ -127,7 +136,7 @@ struct KlFwdKern {
     }
     __device__ void tile(const Params& p, const Sched&, int, int, const TileC& tc, uint32_t taddr) {
 #pragma unroll 1
-      for (int c = 0; c < kBN; c += 32) {
+      for (int c = part * (kBN / 2); c < (part + 1) * (kBN / 2); c += 32) {
         const int col0 = tc.n0 + c;
         if (col0 >= p.V) break;
         uint32_t a[32], b[32];
@@ -137,7 +146,38 @@ struct KlFwdKern {
         chunk(p, a, b, col0);
       }
     }
+    // (m, s, a) + (m2, s2, a2) in base 2; an empty side (m = -inf) adds nothing
+    static __device__ __forceinline__ void merge3(float& m, float& s, float& a, float m2, float s2,
+                                                  float a2) {
+      if (m2 == -INFINITY) return;
+      if (m == -INFINITY) {
+        m = m2;
+        s = s2;
+        a = a2;
+        return;
+      }
+      const float mn = fmaxf(m, m2);
+      const float f1 = fast_exp2(m - mn), f2 = fast_exp2(m2 - mn);
+      s = s * f1 + s2 * f2;
+      a = a * f1 + a2 * f2;
+      m = mn;
+    }
     __device__ void end(const Params& p, const Sched& s, int) {
+      // the row's two halves meet here; every epilogue thread takes both barriers
+      const int row = threadIdx.x & 127;
+      named_bar_sync(2, kEpiT);
+      if (part == 1) {
+        merge[0 * 128 + row] = mp;
+        merge[1 * 128 + row] = sp;
+        merge[2 * 128 + row] = A;
+        merge[3 * 128 + row] = mq;
+        merge[4 * 128 + row] = sq;
+      }
+      named_bar_sync(2, kEpiT);
+      if (part == 1) return;
+      merge3(mp, sp, A, merge[0 * 128 + row], merge[1 * 128 + row], merge[2 * 128 + row]);
+      float unused = 0.f;
+      merge3(mq, sq, unused, merge[3 * 128 + row], merge[4 * 128 + row], 0.f);
       if (r >= s.sp.n) return;
       const size_t plane = static_cast<size_t>(kSvMax) * p.ld;
       const size_t o = static_cast<size_t>(sg) * p.ld + r;
@@ -188,7 +228,7 @@ olive_status launch_dual(const Ctx& c, const CUtensorMap& a, const CUtensorMap& 
   static std::atomic<int> done[kMaxDevices];
   if (!set_smem_once(reinterpret_cast<const void*>(gemm_persistent<K>), smem, c.device, done))
     return OLIVE_ERR_CUDA;
-  gemm_persistent<K><<<c.num_sms, kThreads, smem, c.stream>>>(a, b, a2, b2, p);
+  gemm_persistent<K><<<c.num_sms, core_threads<K>(), smem, c.stream>>>(a, b, a2, b2, p);
   return cudaGetLastError() == cudaSuccess ? OLIVE_OK : OLIVE_ERR_CUDA;
 }
 

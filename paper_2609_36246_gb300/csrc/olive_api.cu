@@ -207,14 +207,14 @@ OpdWs carve_opd(void* ws, int64_t T, int64_t ds, int64_t dt) {
 static FbWs carve_fb_impl(void* ws, int64_t T, int64_t d, int64_t V, int grad_dtype,
                           size_t* total) {
   const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
-  const int64_t vt = ceil_div(V, 256);
+  const int64_t vh = ceil_div(V, 128);  // partials per 128-column half tile
   Carver c{static_cast<char*>(ws)};
   FbWs w;
   w.tc = slab_rows(Tpad, V);
   w.hc = c.take(2ull * Tpad * d);
   w.g = c.take(2ull * w.tc * vpad(V));
-  w.part_zm = static_cast<float*>(c.take(4ull * w.tc * vt));
-  w.part_zs = static_cast<float*>(c.take(4ull * w.tc * vt));
+  w.part_zm = static_cast<float*>(c.take(4ull * w.tc * vh));
+  w.part_zs = static_cast<float*>(c.take(4ull * w.tc * vh));
   w.zy = static_cast<float*>(c.take(4ull * w.tc));
   w.nll = static_cast<float*>(c.take(4ull * Tpad));
   w.dw_acc = grad_dtype == OLIVE_DTYPE_BF16 ? static_cast<float*>(c.take(4ull * V * d)) : nullptr;
@@ -251,7 +251,7 @@ static KlWs carve_kl_impl(void* ws, int64_t T, int64_t ds, int64_t dt, int64_t V
     // reverse: [tc, Vpad] floats; forward: [kl_pair_rows(tc), 2 Vpad] floats
     const int64_t rows2 = std::max<int64_t>(w.tc, 2 * kl_pair_rows(w.tc));
     w.s2 = static_cast<float*>(c.take(4ull * rows2 * vpad(V)));
-    w.part5 = static_cast<float*>(c.take(4ull * 5 * w.tc * ceil_div(V, 256)));
+    w.part5 = static_cast<float*>(c.take(4ull * 5 * w.tc * ceil_div(V, 128)));
   } else {
     w.part = static_cast<float*>(c.take(4ull * 5 * kSvMax * Tpad));
   }

@@ -57,6 +57,7 @@ struct OpdKern {
   static constexpr bool kDual = true;
   static constexpr int kStages = 4;
   static constexpr int kAccBufs = 1;
+  static constexpr int kEpiWarps = 4;
   static constexpr int kEpiSmem = 0;
 
   struct Params {
@@ -110,7 +111,7 @@ struct OpdKern {
     float sv[kTopMax], sx[kTopMax], tv[kTopMax];
     int si[kTopMax], ti[kTopMax];
 
-    __device__ void init(uint8_t*) {}
+    __device__ void init(uint8_t*, int) {}
     __device__ void begin(const Params& p, const Sched& s, int u, int row) {
       int i;
       unit_pos(p, s, u, i, sg);
@@ -360,7 +361,7 @@ olive_status launch_opd_stats(const Ctx& c, const void* h_s, const void* W_s, in
   static std::atomic<int> done[kMaxDevices];
   if (!set_smem_once(reinterpret_cast<const void*>(gemm_persistent<OpdKern>), smem, c.device, done))
     return OLIVE_ERR_CUDA;
-  gemm_persistent<OpdKern><<<c.num_sms, kThreads, smem, c.stream>>>(mHs, mWs, mHt, mWt, p);
+  gemm_persistent<OpdKern><<<c.num_sms, core_threads<OpdKern>(), smem, c.stream>>>(mHs, mWs, mHt, mWt, p);
   if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;
 
   const int vt = (V + OpdKern::kBN - 1) / OpdKern::kBN;
