@@ -25,6 +25,8 @@
  *   olive_token_topk_fwd     per-token entropy and top-K log-probs
  *   olive_topk_compare       student/teacher top-K overlap and top-K KL
  *   olive_topk_kl_bwd        gradient of the top-K KL
+ *   olive_topk_kl_fwd_bwd    the student's top-K lists, the top-K KL and its
+ *                            gradient from one sweep of the student's logits
  *   olive_opd_token_stats    OPD's per-token KL, entropy, top-K lists, overlap
  *                            and top-K KL from one sweep with both heads
  *   olive_token_logprob_fwd_noalloc  the forward without a workspace
@@ -87,7 +89,7 @@ enum { OLIVE_KL_REVERSE = 0, OLIVE_KL_FORWARD = 1 };
 enum { OLIVE_DTYPE_BF16 = 0, OLIVE_DTYPE_F32 = 1 };
 enum { OLIVE_OP_LOGPROB_FWD = 0, OLIVE_OP_LOSS_BWD = 1, OLIVE_OP_DIVERGENCE = 2,
        OLIVE_OP_TOPK_FWD = 3, OLIVE_OP_SPLICE_MASKED = 4, OLIVE_OP_TOPK_KL_BWD = 5,
-       OLIVE_OP_LOSS_FWD_BWD = 6, OLIVE_OP_OPD_STATS = 7 };
+       OLIVE_OP_LOSS_FWD_BWD = 6, OLIVE_OP_OPD_STATS = 7, OLIVE_OP_TOPK_KL_FWD_BWD = 8 };
 
 /* ABI version of the loaded library (OLIVE_ABI_VERSION). */
 OLIVE_API int olive_abi_version(void);
@@ -102,8 +104,9 @@ OLIVE_API const char* olive_status_string(olive_status s);
  *   op  OLIVE_OP_TOPK_FWD: d = hidden width, d_t ignored.
  *   op  OLIVE_OP_SPLICE_MASKED: T = T_cap; d, d_t, V ignored.
  *   op  OLIVE_OP_OPD_STATS: d = student width d_s, d_t = teacher width.
- *   op  OLIVE_OP_TOPK_KL_BWD, OLIVE_OP_LOSS_FWD_BWD: d = (student) hidden
- *       width, grad_dtype as for OLIVE_OP_LOSS_BWD, d_t ignored.
+ *   op  OLIVE_OP_TOPK_KL_BWD, OLIVE_OP_LOSS_FWD_BWD,
+ *       OLIVE_OP_TOPK_KL_FWD_BWD: d = (student) hidden width, grad_dtype as
+ *       for OLIVE_OP_LOSS_BWD, d_t ignored.
  *   `grad` (bwd / divergence): non-zero when gradients are requested
  *   (OLIVE_OP_LOSS_BWD always computes them); `grad_dtype` is the dtype of
  *   d_W for OLIVE_OP_LOSS_BWD (bf16 output needs an fp32 accumulator).
@@ -349,6 +352,42 @@ OLIVE_API olive_status olive_token_loss_fwd_bwd(const void* hidden, const void* 
                                                 float* loss, void* d_hidden, void* d_W,
                                                 int grad_dtype, void* workspace, size_t ws_bytes,
                                                 int32_t* dev_status, void* stream);
+
+/*
+ * olive_topk_kl_fwd_bwd -- olive_token_topk_fwd on the student,
+ * olive_topk_compare and olive_topk_kl_bwd of one OPD training step in a
+ * single call, for callers that know the weights g_t = grad_kl[t] before the
+ * forward runs and have the teacher's lse (and top-K ids) from
+ * olive_token_topk_fwd on the teacher.  Each student logit tile is computed
+ * once: the forward product stores e = exp(z - tile max) in bf16 in the G
+ * slab of the workspace; per masked row the C = min(K + 8, 24) largest
+ * entries of e (read only in the 128-column blocks whose maximum can hold
+ * one) are the candidates whose logits are recomputed exactly (fp32 dot
+ * products), S_t is the K largest of those, and the teacher's log-probs at
+ * S_t come from h_t . W_t[v] - t_lse[t]; a bandwidth-bound pass writes G
+ * (the formula of olive_topk_kl_bwd) and the dH and dW products follow.
+ * Inputs: h_s [T, d_s], W_s [V, d_s], h_t [T, d_t], W_t [V, d_t] bf16 (d_s,
+ * d_t multiples of 8); t_lse fp32 [T]; t_ids int32 [T, K] (nullable: no
+ * overlap); grad_kl fp32 [T].  Outputs: s_lse fp32 [T]; s_ids int32 [T, K] and
+ * s_logp fp32 [T, K] (S_t by decreasing log-prob, ties by id); t_logp_s fp32
+ * [T, K]; kl_topk fp32 [T]; overlap fp32 [T] (written when t_ids is given;
+ * may be NULL otherwise); d_h_s [T, d_s] and d_W_s [V, d_s] of grad_dtype.
+ * Rows not in `rows` get 0 (ids -1).  S_t differs from the exact top-K only
+ * where C - K or more logits lie within bf16 resolution (~2^-8 relative of
+ * exp) below the K-th largest.  1 <= K <= min(16, V).  workspace:
+ * olive_workspace_size(OLIVE_OP_TOPK_KL_FWD_BWD, T, d_s, 0, V, 1, grad_dtype)
+ * bytes.
+ */
+OLIVE_API olive_status olive_topk_kl_fwd_bwd(const void* h_s, const void* W_s, int32_t d_s,
+                                             const void* h_t, const void* W_t, int32_t d_t,
+                                             const int32_t* rows, const int32_t* n_rows,
+                                             int32_t T, int32_t V, float inv_tau, int32_t K,
+                                             const float* t_lse, const int32_t* t_ids,
+                                             const float* grad_kl, float* s_lse, int32_t* s_ids,
+                                             float* s_logp, float* t_logp_s, float* kl_topk,
+                                             float* overlap, void* d_h_s, void* d_W_s,
+                                             int grad_dtype, void* workspace, size_t ws_bytes,
+                                             int32_t* dev_status, void* stream);
 
 /*
  * olive_scale -- y[i] = x[i] * (*scale) for i < n, x and y of `dtype`

@@ -28,7 +28,7 @@ REDUCE = {"sum": 0, "mean": 1}
 DIRECTION = {"reverse": 0, "forward": 1}
 DTYPE = {torch.bfloat16: 0, torch.float32: 1}
 OP = {"logprob_fwd": 0, "loss_bwd": 1, "divergence": 2, "topk_fwd": 3, "splice_masked": 4,
-      "topk_kl_bwd": 5, "loss_fwd_bwd": 6, "opd_stats": 7}
+      "topk_kl_bwd": 5, "loss_fwd_bwd": 6, "opd_stats": 7, "topk_kl_fwd_bwd": 8}
 
 
 class OliveError(RuntimeError):
@@ -84,6 +84,10 @@ def lib() -> ctypes.CDLL:
     L.olive_token_loss_fwd_bwd.restype = ctypes.c_int
     L.olive_token_loss_fwd_bwd.argtypes = [_P, _P, _P, _P, _P, _I, _I, _I, _F, ctypes.c_int, _P, _P,
                                            _P, _P, _P, _P, ctypes.c_int, _P, _S, _P, _P]
+    L.olive_topk_kl_fwd_bwd.restype = ctypes.c_int
+    L.olive_topk_kl_fwd_bwd.argtypes = [_P, _P, _I, _P, _P, _I, _P, _P, _I, _I, _F, _I, _P, _P, _P,
+                                        _P, _P, _P, _P, _P, _P, _P, _P, ctypes.c_int, _P, _S, _P,
+                                        _P]
     L.olive_topk_kl_bwd.restype = ctypes.c_int
     L.olive_topk_kl_bwd.argtypes = [_P, _P, _P, _P, _I, _I, _I, _F, _I, _P, _P, _P, _P, _P, _P, _P,
                                     _P, ctypes.c_int, _P, _S, _P, _P]
@@ -372,6 +376,48 @@ def olive_topk_kl_bwd(h_s, W_s, rows, n_rows, s_lse, s_ids, s_logp, t_logp_s, kl
                                  DTYPE[grad_dtype], _ptr(ws), ws.numel(), _ptr(ds), _stream())
     _check(st, "olive_topk_kl_bwd")
     return dh, dw
+
+
+def olive_topk_kl_fwd_bwd(h_s, W_s, h_t, W_t, rows, n_rows, K, t_lse, grad_kl, t_ids=None,
+                          inv_tau: float = 1.0, grad_dtype=torch.bfloat16, ws=None,
+                          dev_status=None, out=None):
+    """The student's top-K lists, the top-K KL against the teacher and its
+    gradient in one sweep of the student's logits.  t_lse (and t_ids, for the
+    overlap) come from olive_token_topk_fwd on the teacher.  Returns a dict
+    with s_lse, s_ids, s_logp, t_logp_s, kl_topk, overlap (None without
+    t_ids), d_h_s and d_W_s."""
+    _need(h_s, torch.bfloat16, "h_s")
+    _need(W_s, torch.bfloat16, "W_s")
+    _need(h_t, torch.bfloat16, "h_t")
+    _need(W_t, torch.bfloat16, "W_t")
+    _need(t_lse, torch.float32, "t_lse")
+    _need(grad_kl, torch.float32, "grad_kl")
+    if t_ids is not None:
+        _need(t_ids, torch.int32, "t_ids")
+    T, ds = h_s.shape
+    V = W_s.shape[0]
+    dt = h_t.shape[1]
+    dev = h_s.device
+    if out is None:
+        f = lambda *shape: torch.empty(*shape, dtype=torch.float32, device=dev)
+        out = dict(s_lse=f(T), s_ids=torch.empty(T, K, dtype=torch.int32, device=dev),
+                   s_logp=f(T, K), t_logp_s=f(T, K), kl_topk=f(T),
+                   overlap=f(T) if t_ids is not None else None,
+                   d_h_s=torch.empty(T, ds, dtype=grad_dtype, device=dev),
+                   d_W_s=torch.empty(V, ds, dtype=grad_dtype, device=dev))
+    if ws is None:
+        ws = workspace(olive_workspace_size("topk_kl_fwd_bwd", T, ds, V, grad_dtype=grad_dtype), dev)
+    st_buf = dev_status if dev_status is not None else new_status(dev)
+    o = out
+    st = lib().olive_topk_kl_fwd_bwd(
+        _ptr(h_s), _ptr(W_s), ds, _ptr(h_t), _ptr(W_t), dt, _ptr(rows), _ptr(n_rows), T, V,
+        float(inv_tau), K, _ptr(t_lse), _ptr(t_ids) if t_ids is not None else None, _ptr(grad_kl),
+        _ptr(o["s_lse"]), _ptr(o["s_ids"]), _ptr(o["s_logp"]), _ptr(o["t_logp_s"]),
+        _ptr(o["kl_topk"]), _ptr(o["overlap"]) if o["overlap"] is not None else None,
+        _ptr(o["d_h_s"]), _ptr(o["d_W_s"]), DTYPE[grad_dtype], _ptr(ws), ws.numel(),
+        _ptr(st_buf), _stream())
+    _check(st, "olive_topk_kl_fwd_bwd")
+    return out
 
 
 def olive_token_loss_bwd(hidden, W, targets, rows, n_rows, lse, grad_loss, inv_tau: float = 1.0,

@@ -231,6 +231,19 @@ olive_status launch_divergence(const Ctx& c, const void* h_s, const void* W_s, i
 // Words of tile-scheduler counters the fused backward needs.
 size_t bwd_counter_words(int64_t Tpad, int64_t tc);
 
+// Top-K KL forward and backward over one sweep of the student's logits
+// (lmhead_fused.cu): workspace = the fused forward + backward regions, then
+// coef [T] and val [T, 16].
+size_t topk_kl_fb_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype);
+olive_status launch_topk_kl_fwd_bwd(const Ctx& c, const void* h_s, const void* W_s, int32_t d_s,
+                                    const void* h_t, const void* W_t, int32_t d_t,
+                                    const int32_t* rows, const int32_t* n_rows, int32_t T,
+                                    int32_t V, float inv_tau, int32_t K, const float* t_lse,
+                                    const int32_t* t_ids, const float* grad_kl, float* s_lse,
+                                    int32_t* s_ids, float* s_logp, float* t_logp_s,
+                                    float* kl_topk, float* overlap, void* d_h_s, void* d_W_s,
+                                    int grad_dtype, void* ws, int32_t* dev_status);
+
 // Divergence forward + d_h_s in one pass over the logits (fused kernel,
 // per slab: KLZ tiles, conv_kl_kernel, DH tiles); writes kl[t] too.
 olive_status launch_kl_fwd_bwd(const Ctx& c, const void* hcs, const void* hct, const void* W_s,

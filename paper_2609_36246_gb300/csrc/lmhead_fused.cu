@@ -59,6 +59,7 @@
 // Forward KL: G = p_s - p_t cancels where the models agree, so both local
 // logits x_s - m_s and x_t - m_t stay fp32 (pairs, in half as many slab rows
 // so the workspace is the same).
+#include <climits>
 #include <cmath>
 
 #include "gemm_core.cuh"
@@ -443,7 +444,7 @@ __device__ void epi_zsave(const FusedParams& p, const Plan& pl, const Unit& x, i
   int y = -1;
   if (valid) {
     const int t = p.rows[x.row0 + r_local];
-    if (t >= 0 && t < p.T) y = p.targets[t];
+    if (t >= 0 && t < p.T) y = p.targets ? p.targets[t] : -1;  // no targets: top-K KL
     else valid = false;
   }
   const int n0 = x.j * kBN;
@@ -1045,6 +1046,364 @@ __global__ void __launch_bounds__(256)
   }
 }
 
+// ------------------------------------------------ top-K KL in one pass ---
+// The student's forward tiles (no targets) leave e = 2^(x - m_half) in bf16
+// in the G slab and the half-tile (max, sum) partials.  Per masked row,
+// topk_kl_rows_kernel then
+//   1. merges the partials into lse_s and takes tau, the C-th largest
+//      half-tile maximum (C = min(K + 8, 24)): C distinct logits reach tau,
+//      so the row's C largest logits all lie in half tiles whose maximum is
+//      at least tau, and only those (about C of ~V/128) are read,
+//   2. takes from them the C largest approximate logits x ~ log2(e) + m_half
+//      (bf16 e resolves x to a few thousandths),
+//   3. recomputes those candidates' logits exactly (fp32 dot products
+//      h_s . W_s[u]) and keeps the K largest: the student's top-K set S,
+//      exact wherever fewer than C - K logits lie within bf16 resolution
+//      below the K-th largest,
+//   4. takes the teacher's log-probs at S (dot products h_t . W_t[u] minus
+//      the teacher's lse) and forms the truncated KL, the overlap with the
+//      teacher's top-K ids and the gradient terms of the top-K KL: with
+//      g = grad_kl inv_tau, P_S = sum_S p_s and A = KL_K + P_S,
+//      G[u] = -g A p_s(u) for every u, plus g p_s(u) (l_u - q_u + 1) on S.
+// topk_kl_conv_kernel then writes G over the slab.
+
+constexpr int kTkCand = 24;  // most candidates taken to the exact recomputation (K <= 16)
+
+__device__ __forceinline__ float dot8(uint4 x, uint4 y, float s) {
+  const __nv_bfloat162* px = reinterpret_cast<const __nv_bfloat162*>(&x);
+  const __nv_bfloat162* py = reinterpret_cast<const __nv_bfloat162*>(&y);
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const float2 u = __bfloat1622float2(px[q]);
+    const float2 v = __bfloat1622float2(py[q]);
+    s = fmaf(u.x, v.x, s);
+    s = fmaf(u.y, v.y, s);
+  }
+  return s;
+}
+
+// h . w over d8 16-byte groups, split across the warp; four groups per lane
+// in flight
+__device__ __forceinline__ float dot_row_bf16(const uint4* __restrict__ h,
+                                              const uint4* __restrict__ w, int d8, int lane) {
+  float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+  int c = lane;
+  for (; c + 96 < d8; c += 128) {
+    const uint4 w0 = __ldg(w + c), w1 = __ldg(w + c + 32), w2 = __ldg(w + c + 64),
+                w3 = __ldg(w + c + 96);
+    const uint4 h0 = __ldg(h + c), h1 = __ldg(h + c + 32), h2 = __ldg(h + c + 64),
+                h3 = __ldg(h + c + 96);
+    s0 = dot8(h0, w0, s0);
+    s1 = dot8(h1, w1, s1);
+    s2 = dot8(h2, w2, s2);
+    s3 = dot8(h3, w3, s3);
+  }
+  for (; c < d8; c += 32) s0 = dot8(__ldg(h + c), __ldg(w + c), s0);
+  float s = (s0 + s1) + (s2 + s3);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  return s;
+}
+
+// Inserts (v, id) into a lane-local list of N entries sorted by (value
+// descending, id ascending).
+template <int N>
+__device__ __forceinline__ void lane_list_insert(float (&lv)[N], int (&li)[N], float v, int id) {
+#pragma unroll
+  for (int j = 0; j < N; ++j) {
+    const bool before = v > lv[j] || (v == lv[j] && id < li[j]);
+    const float tv = lv[j];
+    const int ti = li[j];
+    lv[j] = before ? v : tv;
+    li[j] = before ? id : ti;
+    v = before ? tv : v;
+    id = before ? ti : id;
+  }
+}
+
+// Pops the warp's best head of the lanes' sorted lists (value descending,
+// id ascending); the lane that held it advances.  Returns the id (INT_MAX
+// once every list is exhausted) and the value in *v.
+template <int N>
+__device__ __forceinline__ int warp_pop(const float (&lv)[N], const int (&li)[N], int& head,
+                                        float* v) {
+  float bv = -INFINITY;
+  int bi = INT_MAX;
+#pragma unroll
+  for (int j = 0; j < N; ++j)
+    if (j == head) {
+      bv = lv[j];
+      bi = li[j];
+    }
+  float wv = bv;
+  int wi = bi;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ov = __shfl_xor_sync(0xffffffffu, wv, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, wi, o);
+    if (ov > wv || (ov == wv && oi < wi)) {
+      wv = ov;
+      wi = oi;
+    }
+  }
+  if (wi != INT_MAX && wi == bi) ++head;  // ids are unique across lanes
+  *v = wv;
+  return wi;
+}
+
+struct TopkKlRows {
+  const int32_t* n_rows;
+  const int32_t* rows;
+  int T, V, tc, slab, vh, K;
+  int64_t ldg;
+  float inv_tau;
+  const float* part_zm;
+  const float* part_zs;
+  const __nv_bfloat16* g;  // e of the slab
+  const uint4* h_s;
+  const uint4* W_s;
+  int ds8;
+  const uint4* h_t;
+  const uint4* W_t;
+  int dt8;
+  const float* t_lse;
+  const int32_t* t_ids;  // nullable: no overlap
+  const float* grad_kl;
+  float* s_lse;
+  int32_t* s_ids;
+  float* s_logp;
+  float* t_logp_s;
+  float* kl_topk;
+  float* overlap;  // nullable
+  float* coef;
+  float* val;
+};
+
+__global__ void __launch_bounds__(256) topk_kl_rows_kernel(const TopkKlRows a) {
+  const int n = read_n_rows(a.n_rows, a.T, nullptr);
+  const SlabPlan sp(n, a.tc);
+  if (a.slab >= sp.n_slabs) return;
+  const int in_s = sp.rows_in(n, a.slab);
+  const int row0 = a.slab * sp.rps;
+  const int lane = threadIdx.x & 31;
+  const int warps = (gridDim.x * blockDim.x) >> 5;
+  const int K = a.K;
+  const int C = min(K + 8, kTkCand);
+  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < in_s; r += warps) {
+    const int t = a.rows[row0 + r];
+    if (t < 0 || t >= a.T) continue;  // reported by the gather
+    const float* zm = a.part_zm + static_cast<size_t>(r) * a.vh;
+    const float* zs = a.part_zs + static_cast<size_t>(r) * a.vh;
+    // 1. lse_s, and tau = the C-th largest half-tile maximum: C distinct
+    //    logits reach it, so every logit of the row's top C is >= tau and
+    //    lies in a half tile whose maximum is >= tau
+    float m = -INFINITY, sum = 0.f;
+    float tv[kTkCand];
+    int ti[kTkCand];
+#pragma unroll
+    for (int j = 0; j < kTkCand; ++j) {
+      tv[j] = -INFINITY;
+      ti[j] = INT_MAX;
+    }
+    for (int j = lane; j < a.vh; j += 32) {
+      const float mj = zm[j];
+      lse_merge(m, sum, mj, zs[j]);
+      if (mj > tv[kTkCand - 1]) lane_list_insert(tv, ti, mj, j);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+      const float s2 = __shfl_xor_sync(0xffffffffu, sum, o);
+      lse_merge(m, sum, m2, s2);
+    }
+    const float lse_s = (m + log2f(sum)) * kLn2;
+    float tau = -INFINITY;
+    {
+      int head = 0;
+      for (int k = 0; k < C; ++k) warp_pop(tv, ti, head, &tau);
+    }
+    // 2. candidates from the half tiles whose maximum reaches tau: each lane
+    //    takes 4 columns of a tile and keeps its 16 best approximate logits
+    //    x = log2(e) + m_half (bf16 e: x to within a few thousandths)
+    float lv[16];
+    int li[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      lv[j] = -INFINITY;
+      li[j] = INT_MAX;
+    }
+    const __nv_bfloat16* grow = a.g + static_cast<size_t>(r) * a.ldg;
+    for (int base = 0; base < a.vh; base += 32) {
+      const int j = base + lane;
+      unsigned b = __ballot_sync(0xffffffffu, j < a.vh && zm[j] >= tau);
+      while (b) {
+        int js[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          js[q] = b ? base + __ffs(b) - 1 : -1;
+          b &= b ? b - 1 : 0u;
+        }
+        uint2 v[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          // rows are only vpad(V) wide: columns from V on are not read
+          const int c = js[q] * kHalf + 4 * lane;
+          v[q] = js[q] >= 0 && c < a.V ? *reinterpret_cast<const uint2*>(grow + c)
+                                       : make_uint2(0u, 0u);
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          if (js[q] < 0) continue;
+          const float mh = zm[js[q]];
+          const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&v[q]);
+          const int c0 = js[q] * kHalf + 4 * lane;
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const float2 u = __bfloat1622float2(h2[e]);
+            const float x0 = log2f(u.x) + mh, x1 = log2f(u.y) + mh;
+            if (c0 + 2 * e < a.V && x0 >= tau) lane_list_insert(lv, li, x0, c0 + 2 * e);
+            if (c0 + 2 * e + 1 < a.V && x1 >= tau) lane_list_insert(lv, li, x1, c0 + 2 * e + 1);
+          }
+        }
+      }
+    }
+    // the warp's C best: lane k keeps the k-th candidate
+    int cid = -1;
+    {
+      int head = 0;
+      float dummy;
+      for (int k = 0; k < C; ++k) {
+        const int w = warp_pop(lv, li, head, &dummy);
+        if (lane == k) cid = w == INT_MAX ? -1 : w;
+      }
+    }
+    // 3. exact logits of the candidates, then the K largest by rank
+    const uint4* hs = a.h_s + static_cast<size_t>(t) * a.ds8;
+    float l = -INFINITY;
+    for (int k = 0; k < C; ++k) {
+      const int u = __shfl_sync(0xffffffffu, cid, k);
+      if (u < 0) break;  // the list ends (fewer columns than candidates)
+      const float x = dot_row_bf16(hs, a.W_s + static_cast<size_t>(u) * a.ds8, a.ds8, lane);
+      if (lane == k) l = x * a.inv_tau - lse_s;
+    }
+    int rank = 0;
+    for (int k = 0; k < C; ++k) {
+      const float lk = __shfl_sync(0xffffffffu, l, k);
+      const int ik = __shfl_sync(0xffffffffu, cid, k);
+      if (ik >= 0 && (lk > l || (lk == l && ik < cid))) ++rank;
+    }
+    const bool mine = cid >= 0 && rank < K;
+    // 4. lane j < K takes the j-th member of S, then the teacher's log-prob there
+    int sid = -1;
+    float slp = 0.f;
+    for (int j = 0; j < K; ++j) {
+      const unsigned b = __ballot_sync(0xffffffffu, mine && rank == j);
+      const int src = b ? __ffs(b) - 1 : 0;
+      const int u = __shfl_sync(0xffffffffu, cid, src);
+      const float lu = __shfl_sync(0xffffffffu, l, src);
+      if (lane == j && b) {
+        sid = u;
+        slp = lu;
+      }
+    }
+    const uint4* ht = a.h_t + static_cast<size_t>(t) * a.dt8;
+    const float lse_t = a.t_lse[t];
+    float q = 0.f;
+    for (int j = 0; j < K; ++j) {
+      const int u = __shfl_sync(0xffffffffu, sid, j);
+      if (u < 0) continue;
+      const float x = dot_row_bf16(ht, a.W_t + static_cast<size_t>(u) * a.dt8, a.dt8, lane);
+      if (lane == j) q = x * a.inv_tau - lse_t;
+    }
+    const bool in_k = lane < K && sid >= 0;
+    const float p = in_k ? expf(slp) : 0.f;
+    float kl = in_k ? p * (slp - q) : 0.f, P = p;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      kl += __shfl_xor_sync(0xffffffffu, kl, o);
+      P += __shfl_xor_sync(0xffffffffu, P, o);
+    }
+    const float gk = a.grad_kl[t] * a.inv_tau;
+    const float A = kl + P;
+    const size_t o = static_cast<size_t>(t) * K + lane;
+    if (lane < K) {
+      a.s_ids[o] = sid;
+      a.s_logp[o] = in_k ? slp : -INFINITY;
+      a.t_logp_s[o] = in_k ? q : -INFINITY;
+      a.val[o] = in_k ? gk * p * (slp - q + 1.f - A) : 0.f;
+    }
+    if (a.overlap) {
+      const int tid = lane < K ? a.t_ids[static_cast<size_t>(t) * K + lane] : -2;
+      bool found = false;
+      for (int k = 0; k < K; ++k) found |= __shfl_sync(0xffffffffu, tid, k) == sid;
+      const int common = __popc(__ballot_sync(0xffffffffu, in_k && found));
+      if (lane == 0) a.overlap[t] = static_cast<float>(common) / static_cast<float>(K);
+    }
+    if (lane == 0) {
+      a.s_lse[t] = lse_s;
+      a.kl_topk[t] = kl;
+      a.coef[t] = -gk * A;
+    }
+  }
+}
+
+// One warp per masked row of the slab: G = coef[t] e 2^(m_half - lse2_s) for
+// every column (zero past V), then the K full values at the ids of S.
+__global__ void __launch_bounds__(256)
+    topk_kl_conv_kernel(const int32_t* __restrict__ n_rows, const int32_t* __restrict__ rows, int T,
+                        int V, int tc, int slab, int vh, int64_t ldg, int K,
+                        const float* __restrict__ part_zm, const float* __restrict__ s_lse,
+                        const float* __restrict__ coef, const float* __restrict__ val,
+                        const int32_t* __restrict__ ids, __nv_bfloat16* g) {
+  const int n = read_n_rows(n_rows, T, nullptr);
+  const SlabPlan sp(n, tc);
+  if (slab >= sp.n_slabs) return;
+  const int in_s = sp.rows_in(n, slab);
+  const int row0 = slab * sp.rps;
+  const int lane = threadIdx.x & 31;
+  const int warps = (gridDim.x * blockDim.x) >> 5;
+  const int nvec = (V + 7) / 8;
+  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < in_s; r += warps) {
+    const int t = rows[row0 + r];
+    if (t < 0 || t >= T) continue;  // the G row stays zero
+    const float* zm = part_zm + static_cast<size_t>(r) * vh;
+    const float lse2 = s_lse[t] * kLog2e;
+    const float cf = coef[t];
+    uint4* grow = reinterpret_cast<uint4*>(g + static_cast<size_t>(r) * ldg);
+#pragma unroll 1
+    for (int base = 0; base < nvec; base += 128) {
+      uint4 v[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int idx = base + 32 * q + lane;
+        if (idx < nvec) v[q] = grow[idx];
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int idx = base + 32 * q + lane;
+        if (idx >= nvec) continue;
+        const float sc = cf * fast_exp2(zm[idx >> 4] - lse2);
+        __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&v[q]);
+        const int col = idx * 8;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 u = __bfloat1622float2(h2[e]);
+          const float a = col + 2 * e < V ? u.x * sc : 0.f;
+          const float b = col + 2 * e + 1 < V ? u.y * sc : 0.f;
+          h2[e] = __floats2bfloat162_rn(a, b);
+        }
+        grow[idx] = v[q];
+      }
+    }
+    __syncwarp();  // the row's dense values are written before the K overrides
+    if (lane < K) {
+      const size_t o = static_cast<size_t>(t) * K + lane;
+      const int u = ids[o];
+      if (u >= 0 && u < V) g[static_cast<size_t>(r) * ldg + u] = __float2bfloat16_rn(val[o]);
+    }
+  }
+}
+
 olive_status launch_lmhead_fused(const Ctx& c, const FusedMaps& maps, const FusedParams& p) {
   const int smem = FusedLayout::SMEM_BYTES;
   static std::atomic<int> done[kMaxDevices];
@@ -1268,6 +1627,112 @@ olive_status launch_kl_fwd_bwd(const Ctx& c, const void* hcs, const void* hct, c
                                                       vh, ldg, inv_tau, reverse, grad_kl, part5,
                                                       p.plane5, s2,
                                                       static_cast<__nv_bfloat16*>(g), kl);
+    if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;
+    p.phase = PH_DHDW;
+    if ((st = launch_lmhead_fused(c, maps, p)) != OLIVE_OK) return st;
+  }
+  return OLIVE_OK;
+}
+
+olive_status launch_topk_kl_fwd_bwd(const Ctx& c, const void* h_s, const void* W_s, int32_t d_s,
+                                    const void* h_t, const void* W_t, int32_t d_t,
+                                    const int32_t* rows, const int32_t* n_rows, int32_t T,
+                                    int32_t V, float inv_tau, int32_t K, const float* t_lse,
+                                    const int32_t* t_ids, const float* grad_kl, float* s_lse,
+                                    int32_t* s_ids, float* s_logp, float* t_logp_s,
+                                    float* kl_topk, float* overlap, void* d_h_s, void* d_W_s,
+                                    int grad_dtype, void* ws, int32_t* dev_status) {
+  const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
+  const FbWs w = carve_fb(ws, T, d_s, V, grad_dtype);
+  char* sparse = static_cast<char*>(ws) + fb_ws_bytes(T, d_s, V, grad_dtype);
+  float* coef = reinterpret_cast<float*>(sparse);
+  float* val = reinterpret_cast<float*>(sparse + align_up(4ull * T, kWsAlign));
+  const int64_t ldg = vpad(V);
+  const size_t elt = grad_dtype == OLIVE_DTYPE_BF16 ? 2 : 4;
+  const int vh = static_cast<int>(ceil_div(V, kHalf));
+  const size_t tk = static_cast<size_t>(T) * K;
+
+  olive_status st = launch_gather_rows(c, h_s, rows, n_rows, T, d_s, w.hc, dev_status);
+  if (st != OLIVE_OK) return st;
+  if (cudaMemsetAsync(d_h_s, 0, elt * T * static_cast<size_t>(d_s), c.stream) != cudaSuccess ||
+      cudaMemsetAsync(s_lse, 0, sizeof(float) * T, c.stream) != cudaSuccess ||
+      cudaMemsetAsync(kl_topk, 0, sizeof(float) * T, c.stream) != cudaSuccess ||
+      (overlap && cudaMemsetAsync(overlap, 0, sizeof(float) * T, c.stream) != cudaSuccess) ||
+      cudaMemsetAsync(s_logp, 0, sizeof(float) * tk, c.stream) != cudaSuccess ||
+      cudaMemsetAsync(t_logp_s, 0, sizeof(float) * tk, c.stream) != cudaSuccess ||
+      cudaMemsetAsync(s_ids, 0xff, sizeof(int32_t) * tk, c.stream) != cudaSuccess)
+    return OLIVE_ERR_CUDA;
+
+  FusedMaps maps;
+  if (!encode_bf16_2d(&maps.m[0], w.hc, d_s, Tpad, 2ull * d_s, 64, 128) ||
+      !encode_bf16_2d(&maps.m[1], W_s, d_s, V, 2ull * d_s, 64, 256) ||
+      !encode_bf16_2d(&maps.m[2], w.g, V, w.tc, 2ull * ldg, 64, 128) ||
+      !encode_bf16_2d(&maps.m[3], W_s, d_s, V, 2ull * d_s, 64, 64) ||
+      !encode_bf16_2d(&maps.m[4], w.g, V, w.tc, 2ull * ldg, 64, 64) ||
+      !encode_bf16_2d(&maps.m[5], w.hc, d_s, Tpad, 2ull * d_s, 64, 64))
+    return OLIVE_ERR_CUDA;
+
+  FusedParams p = base_params(c, rows, n_rows, T, V, inv_tau, dev_status);
+  p.targets = nullptr;  // the forward tiles keep e and the partials only
+  p.kl = 0;
+  p.d = d_s;
+  p.reduction = OLIVE_REDUCE_SUM;
+  p.out_dtype = grad_dtype;
+  p.tc_max = static_cast<int32_t>(w.tc);
+  const int64_t max_slabs = ceil_div(Tpad, w.tc);
+  p.max_slabs = static_cast<int32_t>(max_slabs + 1);
+  p.max_rt = static_cast<int32_t>(w.tc / kRowAlign);
+  p.ldg = ldg;
+  p.g = static_cast<__nv_bfloat16*>(w.g);
+  p.dh_out = d_h_s;
+  p.dw_out = d_W_s;
+  p.dw_acc = grad_dtype == OLIVE_DTYPE_F32 ? static_cast<float*>(d_W_s) : w.dw_acc;
+  p.part_zm = w.part_zm;
+  p.part_zs = w.part_zs;
+  p.zy_s = w.zy;
+
+  TopkKlRows ra = {};
+  ra.n_rows = n_rows;
+  ra.rows = rows;
+  ra.T = T;
+  ra.V = V;
+  ra.tc = static_cast<int>(w.tc);
+  ra.vh = vh;
+  ra.K = K;
+  ra.ldg = ldg;
+  ra.inv_tau = inv_tau;
+  ra.part_zm = w.part_zm;
+  ra.part_zs = w.part_zs;
+  ra.g = static_cast<const __nv_bfloat16*>(w.g);
+  ra.h_s = static_cast<const uint4*>(h_s);
+  ra.W_s = static_cast<const uint4*>(W_s);
+  ra.ds8 = d_s / 8;
+  ra.h_t = static_cast<const uint4*>(h_t);
+  ra.W_t = static_cast<const uint4*>(W_t);
+  ra.dt8 = d_t / 8;
+  ra.t_lse = t_lse;
+  ra.t_ids = t_ids;
+  ra.grad_kl = grad_kl;
+  ra.s_lse = s_lse;
+  ra.s_ids = s_ids;
+  ra.s_logp = s_logp;
+  ra.t_logp_s = t_logp_s;
+  ra.kl_topk = kl_topk;
+  ra.overlap = t_ids ? overlap : nullptr;
+  ra.coef = coef;
+  ra.val = val;
+
+  int conv_blocks = static_cast<int>(ceil_div(w.tc, 8));
+  if (conv_blocks > c.num_sms * 16) conv_blocks = c.num_sms * 16;
+  for (int s = 0; s < max_slabs; ++s) {
+    p.slab = s;
+    p.phase = PH_Z;
+    if ((st = launch_lmhead_fused(c, maps, p)) != OLIVE_OK) return st;
+    ra.slab = s;
+    topk_kl_rows_kernel<<<conv_blocks, 256, 0, c.stream>>>(ra);
+    topk_kl_conv_kernel<<<conv_blocks, 256, 0, c.stream>>>(
+        n_rows, rows, T, V, static_cast<int>(w.tc), s, vh, ldg, K, w.part_zm, s_lse, coef, val,
+        s_ids, static_cast<__nv_bfloat16*>(w.g));
     if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;
     p.phase = PH_DHDW;
     if ((st = launch_lmhead_fused(c, maps, p)) != OLIVE_OK) return st;

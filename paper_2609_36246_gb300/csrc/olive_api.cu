@@ -236,6 +236,12 @@ size_t topk_kl_bwd_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype) {
          align_up(4ull * 16 * T, kWsAlign);
 }
 
+// the fused forward + backward's regions, then coef [T] and val [T, 16]
+size_t topk_kl_fb_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype) {
+  return fb_ws_bytes(T, d, V, grad_dtype) + align_up(4ull * T, kWsAlign) +
+         align_up(4ull * 16 * T, kWsAlign);
+}
+
 static KlWs carve_kl_impl(void* ws, int64_t T, int64_t ds, int64_t dt, int64_t V, int grad,
                           size_t* total) {
   const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
@@ -328,6 +334,9 @@ size_t olive_workspace_size(int op, int32_t T, int32_t d, int32_t d_t, int32_t V
     case OLIVE_OP_TOPK_KL_BWD:
       if (grad_dtype != OLIVE_DTYPE_BF16 && grad_dtype != OLIVE_DTYPE_F32) return 0;
       return topk_kl_bwd_ws_bytes(T, d, V, grad_dtype);
+    case OLIVE_OP_TOPK_KL_FWD_BWD:
+      if (grad_dtype != OLIVE_DTYPE_BF16 && grad_dtype != OLIVE_DTYPE_F32) return 0;
+      return topk_kl_fb_ws_bytes(T, d, V, grad_dtype);
     default: return 0;
   }
 }
@@ -457,6 +466,36 @@ olive_status olive_topk_kl_bwd(const void* h_s, const void* W_s, const int32_t* 
   const SparseGrad sg{coef, val, s_ids, K};
   return launch_loss_bwd(c, h_s, W_s, nullptr, rows, n_rows, T, d, V, inv_tau, OLIVE_REDUCE_SUM,
                          s_lse, nullptr, d_h_s, d_W_s, grad_dtype, workspace, dev_status, &sg);
+}
+
+olive_status olive_topk_kl_fwd_bwd(const void* h_s, const void* W_s, int32_t d_s, const void* h_t,
+                                   const void* W_t, int32_t d_t, const int32_t* rows,
+                                   const int32_t* n_rows, int32_t T, int32_t V, float inv_tau,
+                                   int32_t K, const float* t_lse, const int32_t* t_ids,
+                                   const float* grad_kl, float* s_lse, int32_t* s_ids,
+                                   float* s_logp, float* t_logp_s, float* kl_topk, float* overlap,
+                                   void* d_h_s, void* d_W_s, int grad_dtype, void* workspace,
+                                   size_t ws_bytes, int32_t* dev_status, void* stream) {
+  if (!h_s || !W_s || !h_t || !W_t || !rows || !n_rows || !t_lse || !grad_kl || !s_lse ||
+      !s_ids || !s_logp || !t_logp_s || !kl_topk || (t_ids && !overlap) || !d_h_s || !d_W_s ||
+      !dev_status)
+    return OLIVE_ERR_INVALID_ARG;
+  if (grad_dtype != OLIVE_DTYPE_BF16 && grad_dtype != OLIVE_DTYPE_F32) return OLIVE_ERR_INVALID_ARG;
+  if (T < 1 || V < 1 || d_s < 1 || d_s > kMaxDim || d_t < 1 || d_t > kMaxDim || K < 1 ||
+      K > 16 || K > V)
+    return OLIVE_ERR_SHAPE;
+  if (!(inv_tau > 0.f) || !std::isfinite(inv_tau)) return OLIVE_ERR_INVALID_ARG;
+  if (d_s % 8 != 0 || d_t % 8 != 0 || !aligned16(h_s) || !aligned16(W_s) || !aligned16(h_t) ||
+      !aligned16(W_t) || !aligned16(d_h_s) || !aligned16(d_W_s))
+    return OLIVE_ERR_ALIGNMENT;
+  olive_status st = check_ws(workspace, ws_bytes, topk_kl_fb_ws_bytes(T, d_s, V, grad_dtype));
+  if (st != OLIVE_OK) return st;
+  Ctx c;
+  st = make_ctx(stream, &c);
+  if (st != OLIVE_OK) return st;
+  return launch_topk_kl_fwd_bwd(c, h_s, W_s, d_s, h_t, W_t, d_t, rows, n_rows, T, V, inv_tau, K,
+                                t_lse, t_ids, grad_kl, s_lse, s_ids, s_logp, t_logp_s, kl_topk,
+                                overlap, d_h_s, d_W_s, grad_dtype, workspace, dev_status);
 }
 
 olive_status olive_token_loss_bwd(const void* hidden, const void* W, const int32_t* targets,

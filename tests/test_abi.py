@@ -191,6 +191,31 @@ def test_opd_stats_validation(L):
         assert call(outs=[None] * 8 + [P(p)]) in (7, 8)
 
 
+def test_topk_kl_fwd_bwd_validation(L):
+    keep, p = _fake()
+    P = ctypes.c_void_p
+    ws = B.olive_workspace_size("topk_kl_fwd_bwd", 64, 64, 100, grad_dtype=torch.bfloat16)
+    assert ws >= B.olive_workspace_size("loss_fwd_bwd", 64, 64, 100, grad_dtype=torch.bfloat16)
+    assert L.olive_workspace_size(8, 64, 64, 0, 100, 1, 2) == 0  # no fp16 gradients
+
+    def call(**kw):
+        a = dict(ds=64, dt=96, K=8, tids=P(p), ov=P(p), dt_=0, dh=P(p), ws_bytes=ws, tlse=P(p))
+        a.update(kw)
+        return L.olive_topk_kl_fwd_bwd(P(p), P(p), a["ds"], P(p), P(p), a["dt"], P(p), P(p), 64,
+                                       100, 1.0, a["K"], a["tlse"], a["tids"], P(p), P(p), P(p),
+                                       P(p), P(p), P(p), a["ov"], a["dh"], P(p), a["dt_"], P(p),
+                                       a["ws_bytes"], P(p), None)
+    assert call(tlse=None) == 1
+    assert call(ov=None) == 1          # teacher ids without an overlap output
+    assert call(dt_=2) == 1
+    assert call(K=0) == 2 and call(K=17) == 2 and call(K=16, dt=64) != 2
+    assert call(ds=60) == 3 and call(dt=90) == 3 and call(dh=P(p + 4)) == 3
+    assert call(ws_bytes=ws - 1) == 9
+    if not torch.cuda.is_available():
+        assert call() in (7, 8)
+        assert call(tids=None, ov=None) in (7, 8)
+
+
 def test_scale_validation(L):
     keep, p = _fake()
     P = ctypes.c_void_p
