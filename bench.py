@@ -299,18 +299,19 @@ def run_ours(args, world, rank, local):
     burst, sustained, src = load_peaks()
     counted = 6.0 * N_mask * d * V
     step_tflops = counted / (ms_per_step / 1e3) / 1e12
-    # dominant kernel: lmhead_fused_kernel, launched twice per call (forward
-    # tiles, then dH/dW tiles); its algorithmic work per call is the forward
-    # product plus dH and dW, 6 N_mask d V, and the call is bracketed by
-    # events on its stream (so the row gather, the convert pass and the loss
-    # reduction count against it)
+    # dominant kernel: lmhead_fused_kernel, launched three times per slab
+    # (the reference tiles, the forward tiles, the dH/dW tiles); its
+    # algorithmic work per call is the forward product plus dH and dW,
+    # 6 N_mask d V, and the call is bracketed by events on its stream (so the
+    # row gather, the per-row fix-up and the loss reduction count against it)
     slabs = -(-((T + 127) // 128 * 128) // B.slab_rows_for(T, V))
     fb_flops = counted
     ach_fb = fb_flops / (fb_ms / 1e3) / 1e12
     rev = kernel_rev()
     traffic = profile_traffic("lmhead_fused_kernel", rev)
-    # splice (scan, fill) + gather + per slab (forward tiles, convert, dH/dW tiles) + loss reduce
-    launches = 2 + 1 + 3 * slabs + 1
+    # splice (scan, fill) + gather + per slab (reference tiles, forward tiles, fix-up,
+    # dH/dW tiles) + loss reduce
+    launches = 2 + 1 + 4 * slabs + 1
 
     two_call = None
     if not args.no_extra:
@@ -352,14 +353,15 @@ def run_ours(args, world, rank, local):
         "dense_equivalent_note": "6 T d V over the packed T (unmasked rows included); not the "
                                  "headline, which counts the N_mask scored rows only",
         "phases_ms": {"splice_pack": spl_ms, "loss_fwd_bwd": fb_ms},
-        "roofline": {"kernel": "lmhead_fused_kernel (forward tiles + dH/dW tiles, 2 launches per call)",
+        "roofline": {"kernel": "lmhead_fused_kernel (reference, forward and dH/dW tiles, 3 launches "
+                               "per slab)",
                      "bound": "tensor", "achieved": ach_fb, "peak": sustained, "unit": "TFLOP/s",
                      "frac": ach_fb / sustained, "traffic": traffic,
                      "peak_source": f"{src} bf16_tflops_sustained",
                      "flops_per_call": fb_flops, "kernel_rev": rev,
-                     "note": "per olive_token_loss_fwd_bwd call (its two lmhead_fused_kernel launches, "
-                             "timed with the gather, convert and loss kernels around them); "
-                             "traffic is DRAM bytes of both launches"},
+                     "note": "per olive_token_loss_fwd_bwd call (its lmhead_fused_kernel launches, "
+                             "timed with the gather, fix-up and loss kernels around them); "
+                             "traffic is DRAM bytes of those launches"},
         "two_call_path": two_call,
         "e2e": e2e,
         "gpu_launches": launches * args.steps,

@@ -108,6 +108,9 @@ struct FbWs {
   float* zy;       // [Tc] target logits of the slab
   float* nll;      // [Tpad] per-row loss terms
   float* dw_acc;   // fp32 [V, d] (bf16 output only)
+  float* zref;     // [Tc, 2] reference maxima of the slab rows (base 2)
+  float* lam;      // [Tc] dH row scale of the slab rows
+  void* hs;        // bf16 [Tpad, d]: hc rows scaled by their lam (dW operand)
   int64_t tc;
 };
 size_t fb_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype);

@@ -44,13 +44,20 @@
 // resident.
 //
 // Forward + backward in one call (olive_token_loss_fwd_bwd) avoids the logit
-// recomputation: per slab, a launch of ZSAVE tiles (the forward product) stores
-// e = 2^(x - m_tile) in bf16 in the G slab with the tile's (max, sum) per row;
-// conv_kernel merges the partials into lse, writes logp and the row's loss
-// term, and turns the slab into G in place (G = g inv_tau (e 2^(m_tile -
-// lse2) - [v == y]), the target entry from the exact fp32 z_y); a second
-// launch runs the DH and DW tiles of the slab.  The launches are stream
-// ordered, so these phases need no tile counters.  The divergence gradient
+// recomputation: per slab, a launch of ZREF tiles (the first vocabulary tile of
+// every row tile) takes each row's reference R = its maximum there; a launch
+// of ZSAVE tiles (the forward product) stores e' = 2^(x - R) in bf16 in the G
+// slab with each half tile's (R, sum of 2^(x - R)) per row.  Since
+// G = g inv_tau (p - [v == y]) = lam e' off the target with one scale per row,
+// lam = g inv_tau 2^(R - lse2), the slab is not rewritten: ref_fix_kernel
+// merges the partials into lse, writes logp and the row's loss term, puts
+// G_y / lam at the target (from the exact fp32 z_y), and stores lam and the
+// rows hs = lam hc; the DH and DW launch then computes dH = lam (e' . W) (the
+// scale in the DH epilogue) and dW = e'^T . hs.  A half tile whose maximum
+// exceeds R by more than kRefMax keeps its own maximum as reference, and its
+// row is rewritten in full relative to lse2 by ref_fix_kernel (lam = g
+// inv_tau).  The launches are stream ordered, so these phases need no tile
+// counters.  The divergence gradient
 // uses the same phases with KLZ tiles (two products per tile, student and
 // teacher, in the two 256-column halves of one TMEM accumulator) and five
 // per-tile partials, from which conv_kl_kernel forms KL and G.  Reverse KL:
@@ -83,10 +90,16 @@ constexpr int kFMma = kFEpiWarps + 1;
 constexpr int kFThreads = 32 * (kFEpiWarps + 2);
 constexpr int kHalf = kBN / 2;
 
-enum Kind : int { K_NONE = -1, K_GRAD = 0, K_KLZ = 1, K_DH = 2, K_DW = 3, K_ZSAVE = 4 };
+enum Kind : int { K_NONE = -1, K_GRAD = 0, K_KLZ = 1, K_DH = 2, K_DW = 3, K_ZSAVE = 4, K_ZREF = 5 };
 // phases: one launch of every tile kind with dependency waits, or one slab's
-// forward (ZSAVE) tiles, or one slab's DH and DW tiles
-enum Phase : int { PH_ALL = 0, PH_Z = 1, PH_DHDW = 2 };
+// forward (ZSAVE) tiles, or one slab's DH and DW tiles, or the first vocabulary
+// tile of every row tile of one slab (the rows' reference maxima)
+enum Phase : int { PH_ALL = 0, PH_Z = 1, PH_DHDW = 2, PH_R = 3 };
+
+// A half tile whose maximum exceeds the row's reference by more than this
+// (base 2) keeps its own maximum as reference: 2^(x - ref) stays below 2^100,
+// so sums of e . W over the vocabulary stay finite in fp32.
+constexpr float kRefMax = 100.f;
 
 // CE maps: 0 hc K-major 64x128, 1 W K-major 64x256, 2 G K-major 64x128,
 //          3 W MN-major 64x64, 4 G MN-major 64x64, 5 hc MN-major 64x64
@@ -112,6 +125,10 @@ struct FusedParams {
   float* part_zm;            // PH_Z: [tc, vh] half-tile max (base 2) per slab row
   float* part_zs;            // PH_Z: [tc, vh] half-tile sum of 2^(x - max)
   float* zy_s;               // PH_Z: [tc] target logit (natural units)
+  float* zref;               // CE single pass: [tc, 2] per slab row, the maxima (base 2) of the
+                             // two halves of its first vocabulary tile (PH_R); null: ZSAVE
+                             // tiles store e relative to each half tile's own maximum
+  const float* lam;          // CE single pass: [tc] dH row scale (null: none)
   float* s2;                 // KLZ: fp32 slab, [tc, ldg] (reverse) or [tc / 2, 2 ldg] (forward)
   float* part5;              // KLZ: [5][tc][vh] m_s, s_s, m_t, s_t, A per (row, half-tile)
   int64_t plane5;            // tc * vh
@@ -188,6 +205,10 @@ __device__ int total_units(const FusedParams& p, const Plan& pl) {
   for (int s = slab_lo(p); s < slab_hi(p, pl); ++s) {
     const int in_s = slab_in(pl, s);
     const int mt = (in_s + 127) / 128;
+    if (p.phase == PH_R) {
+      t += mt;
+      continue;
+    }
     if (p.phase != PH_DHDW) t += units_grad(pl, mt);
     if (p.phase != PH_Z) t += units_dh(pl, mt) + units_dw(p, pl, s, in_s);
   }
@@ -204,6 +225,16 @@ __device__ Unit decode(const FusedParams& p, const Plan& pl, int u) {
     x.in_s = in_s;
     x.row0 = s * pl.rps;
     x.mt = mt;
+    if (p.phase == PH_R) {
+      if (u < mt) {
+        x.i = u;
+        x.j = 0;
+        x.kind = K_ZREF;
+        return x;
+      }
+      u -= mt;
+      continue;
+    }
     const int ug = p.phase == PH_DHDW ? 0 : units_grad(pl, mt);
     if (u < ug) {
       const Raster r{mt, pl.vt, p.group_rows};
@@ -238,7 +269,8 @@ __device__ __forceinline__ void unit_ksteps(const FusedParams& p, const Unit& x,
   nk2 = 0;
   switch (x.kind) {
     case K_GRAD:
-    case K_ZSAVE: nk = (p.d + kBK - 1) / kBK; break;
+    case K_ZSAVE:
+    case K_ZREF: nk = (p.d + kBK - 1) / kBK; break;
     case K_KLZ:
       nk = (p.d + kBK - 1) / kBK;
       nk2 = (p.d2 + kBK - 1) / kBK;
@@ -442,10 +474,12 @@ __device__ void epi_zsave(const FusedParams& p, const Plan& pl, const Unit& x, i
   const int r_local = x.i * kBM + row;
   bool valid = r_local < x.in_s;
   int y = -1;
+  float R = 0.f;
   if (valid) {
     const int t = p.rows[x.row0 + r_local];
     if (t >= 0 && t < p.T) y = p.targets ? p.targets[t] : -1;  // no targets: top-K KL
     else valid = false;
+    if (p.zref) R = fmaxf(p.zref[2 * r_local], p.zref[2 * r_local + 1]);
   }
   const int n0 = x.j * kBN;
   float tm = -INFINITY;
@@ -466,6 +500,10 @@ __device__ void epi_zsave(const FusedParams& p, const Plan& pl, const Unit& x, i
         if (col0 + k == y) p.zy_s[r_local] = __uint_as_float(a[k]) * p.inv_tau;
     }
   }
+  // the reference of the stored e and of the partial sum: the row's reference
+  // maximum when one is given and tm does not exceed it by more than kRefMax,
+  // else the half tile's own maximum
+  const float ref = (p.zref && !(tm - R > kRefMax)) ? R : tm;
   __nv_bfloat16* grow = p.g + static_cast<size_t>(r_local) * p.ldg;
   float ts = 0.f;
 #pragma unroll 1
@@ -479,16 +517,36 @@ __device__ void epi_zsave(const FusedParams& p, const Plan& pl, const Unit& x, i
     float e[32];
 #pragma unroll
     for (int k = 0; k < 32; ++k) {
-      e[k] = (valid && k < nv) ? fast_exp2(__uint_as_float(a[k]) * p.scale2 - tm) : 0.f;
+      e[k] = (valid && k < nv) ? fast_exp2(__uint_as_float(a[k]) * p.scale2 - ref) : 0.f;
       ts += e[k];
     }
     store_row32(grow, col0, OLIVE_DTYPE_BF16, nv, e);
   }
   if (valid && n0 + part * kHalf < p.V) {  // a half past V has no partial slot
     const size_t o = static_cast<size_t>(r_local) * pl.vh + 2 * x.j + part;
-    p.part_zm[o] = tm;
+    p.part_zm[o] = ref;
     p.part_zs[o] = ts;
   }
+}
+
+// reference tile (the first vocabulary tile of a row tile): each row's
+// maximum over its half, base 2, for the ZSAVE tiles that follow
+__device__ void epi_zref(const FusedParams& p, const Unit& x, int row, int part, uint32_t taddr) {
+  const int r_local = x.i * kBM + row;
+  const bool valid = r_local < x.in_s;
+  float tm = -INFINITY;
+#pragma unroll 1
+  for (int c = part * kHalf; c < (part + 1) * kHalf; c += 32) {
+    if (c >= p.V) break;
+    uint32_t a[32];
+    tmem_ld_32x32b_x32(taddr + c, a);
+    tmem_ld_wait();
+    const int nv = p.V - c;
+#pragma unroll
+    for (int k = 0; k < 32; ++k)
+      if (k < nv) tm = fmaxf(tm, __uint_as_float(a[k]) * p.scale2);
+  }
+  if (valid) p.zref[2 * r_local + part] = tm;
 }
 
 __device__ void epi_dh(const FusedParams& p, const Unit& x, int row, int part, uint32_t taddr) {
@@ -507,9 +565,10 @@ __device__ void epi_dh(const FusedParams& p, const Unit& x, int row, int part, u
     tmem_ld_32x32b_x32(taddr + c, a);
     tmem_ld_wait();
     if (t < 0) continue;
+    const float sc = p.lam ? p.lam[r_local] : 1.f;
     float g[32];
 #pragma unroll
-    for (int k = 0; k < 32; ++k) g[k] = __uint_as_float(a[k]);
+    for (int k = 0; k < 32; ++k) g[k] = __uint_as_float(a[k]) * sc;
     store_row32(p.dh_out, static_cast<size_t>(t) * p.d + col0, p.out_dtype, p.d - col0, g);
   }
 }
@@ -668,6 +727,7 @@ __global__ void __launch_bounds__(kFThreads, 1)
           switch (x.kind) {
             case K_GRAD:
             case K_ZSAVE:
+            case K_ZREF:
               tma_load_2d(sA, &maps.m[0], fb, k * kBK, x.row0 + x.i * kBM);
               tma_load_2d(sB, &maps.m[1], fb, k * kBK, x.j * kBN);
               break;
@@ -778,6 +838,7 @@ __global__ void __launch_bounds__(kFThreads, 1)
         case K_GRAD: epi_grad(p, pl, x, row, part, taddr); break;
         case K_KLZ: epi_klz(p, pl, x, row, part, taddr); break;
         case K_ZSAVE: epi_zsave(p, pl, x, row, part, taddr); break;
+        case K_ZREF: epi_zref(p, x, row, part, taddr); break;
         case K_DH: epi_dh(p, x, row, part, taddr); break;
         case K_DW: epi_dw(p, pl, x, row, part, taddr, nk); break;
         default: break;
@@ -822,22 +883,30 @@ __device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2
   m = mn;
 }
 
-// One warp per masked row of the slab: merges the ZSAVE partials into lse,
-// writes logp, lse and the row's loss term, then rewrites the row's slab
-// entries e = 2^(x - m_tile) as G = coef (e 2^(m_tile - lse2) - [v == y]) in
-// place (32 lanes x 8 columns cover one 256-wide tile per step, so the tile
-// max is one broadcast load).  The target entry uses the exact z_y.
+// One warp per row tile row of the slab, after ZSAVE tiles with a row
+// reference R (base 2): the row's stored e' = 2^(x - R) give
+// G = lam e' with lam = coef 2^(R - lse2), so instead of rewriting the row
+// this merges the partials into lse, writes logp, lse and the loss term, puts
+// G_y / lam = expm1(logp) 2^(lse2 - R) at the target (G_y from the exact z_y),
+// stores lam for the dH tiles and writes hs = lam hc, the dW product's scaled
+// rows.  A row where some half tile kept its own maximum as reference (it
+// exceeded R by more than kRefMax) is rewritten in full relative to lse2
+// (e'' = p, lam = coef).  Rows past the slab's masked rows get lam = 0 and
+// hs = 0 up to the row tile's end.
 __global__ void __launch_bounds__(256)
-    conv_kernel(const int32_t* __restrict__ n_rows, const int32_t* __restrict__ rows,
-                const int32_t* __restrict__ targets, int T, int V, int tc, int slab, int vh,
-                int64_t ldg, float inv_tau, int reduction, const float* __restrict__ grad_loss,
-                const float* __restrict__ part_zm, const float* __restrict__ part_zs,
-                const float* __restrict__ zy_s, __nv_bfloat16* g, float* __restrict__ logp,
-                float* __restrict__ lse, float* __restrict__ nll, int32_t* dev_status) {
+    ref_fix_kernel(const int32_t* __restrict__ n_rows, const int32_t* __restrict__ rows,
+                   const int32_t* __restrict__ targets, int T, int V, int tc, int slab, int vh,
+                   int64_t ldg, float inv_tau, int reduction, const float* __restrict__ grad_loss,
+                   const float* __restrict__ part_zm, const float* __restrict__ part_zs,
+                   const float* __restrict__ zy_s, const float* __restrict__ zref,
+                   const uint4* __restrict__ hc, int d8, __nv_bfloat16* g, float* __restrict__ lam,
+                   uint4* __restrict__ hs, float* __restrict__ logp, float* __restrict__ lse,
+                   float* __restrict__ nll, int32_t* dev_status) {
   const int n = read_n_rows(n_rows, T, nullptr);
   const SlabPlan sp(n, tc);
   if (slab >= sp.n_slabs) return;
   const int in_s = sp.rows_in(n, slab);
+  const int row_end = min((in_s + kBM - 1) / kBM * kBM, tc);
   const int row0 = slab * sp.rps;
   float gs = *grad_loss;
   if (reduction == OLIVE_REDUCE_MEAN && n > 0) gs = gs / static_cast<float>(n);
@@ -845,23 +914,35 @@ __global__ void __launch_bounds__(256)
   const int lane = threadIdx.x & 31;
   const int warps = (gridDim.x * blockDim.x) >> 5;
   const int nvec = (V + 7) / 8;
-  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < in_s; r += warps) {
-    const int t = rows[row0 + r];
+  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < row_end; r += warps) {
+    const int t = r < in_s ? rows[row0 + r] : -1;
+    uint4* hrow = hs + static_cast<size_t>(row0 + r) * d8;
     if (t < 0 || t >= T) {
-      if (lane == 0) nll[row0 + r] = 0.f;  // reported by the gather; the G row is zero
+      // reported by the gather (masked rows); the G row is zero
+      if (lane == 0) {
+        lam[r] = 0.f;
+        if (r < in_s) nll[row0 + r] = 0.f;
+      }
+      for (int c = lane; c < d8; c += 32) hrow[c] = make_uint4(0u, 0u, 0u, 0u);
       continue;
     }
     const int y = targets[t];
+    const float R = fmaxf(zref[2 * r], zref[2 * r + 1]);
     const float* zm = part_zm + static_cast<size_t>(r) * vh;
     const float* zs = part_zs + static_cast<size_t>(r) * vh;
     float m = -INFINITY, sum = 0.f;
-    for (int j = lane; j < vh; j += 32) lse_merge(m, sum, zm[j], zs[j]);
+    bool own = false;  // some half tile kept its own maximum
+    for (int j = lane; j < vh; j += 32) {
+      own |= zm[j] != R;
+      lse_merge(m, sum, zm[j], zs[j]);
+    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
       const float s2 = __shfl_xor_sync(0xffffffffu, sum, o);
       lse_merge(m, sum, m2, s2);
     }
+    own = __any_sync(0xffffffffu, own);
     const float lse2 = m + log2f(sum);
     const float l = lse2 * kLn2;
     const bool ybad = y < 0 || y >= V;
@@ -872,34 +953,38 @@ __global__ void __launch_bounds__(256)
       nll[row0 + r] = -lp;
       if (ybad) atomicOr(dev_status, 1 << OLIVE_ERR_TOKEN_RANGE);
     }
-    const float gy = coef * expm1f(lp);
-    uint4* grow = reinterpret_cast<uint4*>(g + static_cast<size_t>(r) * ldg);
-#pragma unroll 1
-    for (int base = 0; base < nvec; base += 128) {
-      uint4 v[4];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int idx = base + 32 * q + lane;
-        if (idx < nvec) v[q] = grow[idx];
-      }
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int idx = base + 32 * q + lane;
-        if (idx >= nvec) continue;
-        const float sc = coef * fast_exp2(zm[idx >> 4] - lse2);  // 16 vectors per half tile
-        __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&v[q]);
-        const int col = idx * 8;
+    const float lm = own ? coef : coef * fast_exp2(R - lse2);
+    if (own) {
+      // G / coef = e 2^(ref - lse2) = p, in place
+      uint4* grow = reinterpret_cast<uint4*>(g + static_cast<size_t>(r) * ldg);
+      for (int idx = lane; idx < nvec; idx += 32) {
+        uint4 v = grow[idx];
+        const float sc = fast_exp2(zm[idx >> 4] - lse2);  // 16 vectors per half tile
+        __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&v);
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           const float2 u = __bfloat1622float2(h2[e]);
-          float a = col + 2 * e < V ? u.x * sc : 0.f;
-          float b = col + 2 * e + 1 < V ? u.y * sc : 0.f;
-          if (col + 2 * e == y) a = gy;
-          if (col + 2 * e + 1 == y) b = gy;
-          h2[e] = __floats2bfloat162_rn(a, b);
+          const int c = idx * 8 + 2 * e;
+          h2[e] = __floats2bfloat162_rn(c < V ? u.x * sc : 0.f, c + 1 < V ? u.y * sc : 0.f);
         }
-        grow[idx] = v[q];
+        grow[idx] = v;
       }
+      __syncwarp();  // the dense rewrite precedes the target entry
+    }
+    if (lane == 0 && !ybad)
+      g[static_cast<size_t>(r) * ldg + y] =
+          __float2bfloat16_rn(own ? expm1f(lp) : expm1f(lp) * fast_exp2(lse2 - R));
+    if (lane == 0) lam[r] = lm;
+    const uint4* hin = hc + static_cast<size_t>(row0 + r) * d8;
+    for (int c = lane; c < d8; c += 32) {
+      uint4 v = hin[c];
+      __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&v);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float2 u = __bfloat1622float2(h2[e]);
+        h2[e] = __floats2bfloat162_rn(u.x * lm, u.y * lm);
+      }
+      hrow[c] = v;
     }
   }
 }
@@ -1542,7 +1627,7 @@ olive_status launch_loss_fwd_bwd(const Ctx& c, const void* hidden, const void* W
       !encode_bf16_2d(&maps.m[2], w.g, V, w.tc, 2ull * ldg, 64, 128) ||
       !encode_bf16_2d(&maps.m[3], W, d, V, 2ull * d, 64, 64) ||
       !encode_bf16_2d(&maps.m[4], w.g, V, w.tc, 2ull * ldg, 64, 64) ||
-      !encode_bf16_2d(&maps.m[5], w.hc, d, Tpad, 2ull * d, 64, 64))
+      !encode_bf16_2d(&maps.m[5], w.hs, d, Tpad, 2ull * d, 64, 64))
     return OLIVE_ERR_CUDA;
 
   FusedParams p = base_params(c, rows, n_rows, T, V, inv_tau, dev_status);
@@ -1563,16 +1648,21 @@ olive_status launch_loss_fwd_bwd(const Ctx& c, const void* hidden, const void* W
   p.part_zm = w.part_zm;
   p.part_zs = w.part_zs;
   p.zy_s = w.zy;
+  p.zref = w.zref;
+  p.lam = w.lam;
 
   int conv_blocks = static_cast<int>(ceil_div(w.tc, 8));
   if (conv_blocks > c.num_sms * 16) conv_blocks = c.num_sms * 16;
   for (int s = 0; s < max_slabs; ++s) {
     p.slab = s;
+    p.phase = PH_R;
+    if ((st = launch_lmhead_fused(c, maps, p)) != OLIVE_OK) return st;
     p.phase = PH_Z;
     if ((st = launch_lmhead_fused(c, maps, p)) != OLIVE_OK) return st;
-    conv_kernel<<<conv_blocks, 256, 0, c.stream>>>(
+    ref_fix_kernel<<<conv_blocks, 256, 0, c.stream>>>(
         n_rows, rows, targets, T, V, static_cast<int>(w.tc), s, vh, ldg, inv_tau, reduction,
-        grad_loss, w.part_zm, w.part_zs, w.zy, static_cast<__nv_bfloat16*>(w.g), logp, lse, w.nll,
+        grad_loss, w.part_zm, w.part_zs, w.zy, w.zref, static_cast<const uint4*>(w.hc), d / 8,
+        static_cast<__nv_bfloat16*>(w.g), w.lam, static_cast<uint4*>(w.hs), logp, lse, w.nll,
         dev_status);
     if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;
     p.phase = PH_DHDW;

@@ -218,6 +218,9 @@ static FbWs carve_fb_impl(void* ws, int64_t T, int64_t d, int64_t V, int grad_dt
   w.zy = static_cast<float*>(c.take(4ull * w.tc));
   w.nll = static_cast<float*>(c.take(4ull * Tpad));
   w.dw_acc = grad_dtype == OLIVE_DTYPE_BF16 ? static_cast<float*>(c.take(4ull * V * d)) : nullptr;
+  w.zref = static_cast<float*>(c.take(8ull * w.tc));
+  w.lam = static_cast<float*>(c.take(4ull * w.tc));
+  w.hs = c.take(2ull * Tpad * d);
   if (total) *total = c.off;
   return w;
 }

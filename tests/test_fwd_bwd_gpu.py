@@ -111,6 +111,29 @@ def test_empty_mask():
     assert loss == 0.0 and not logp.any() and not dh.any() and not dw.any()
 
 
+@pytest.mark.parametrize("spike", [0.2, 0.5])
+def test_rows_far_above_their_first_tile(spike):
+    """Each row's stored e' = 2^(x - R) is relative to the maximum R over the
+    row's first 256 vocabulary entries.  Here one id far down the vocabulary
+    (1000) has a logit 31-39 nats (spike 0.2: e' up to ~2^57, the scaled form)
+    or 78-101 nats (spike 0.5: more than 2^100 above R, so its half tile keeps
+    its own maximum and the row is rewritten relative to lse) above the first
+    tile on half of the rows; the other rows stay unremarkable."""
+    rng = np.random.default_rng(int(spike * 10))
+    S, V, d = 6, 3000, 64
+    b = synth.batch_from_lengths(rng, [20] * S, [60] * S, V)
+    h = synth.normal_bf16(rng, (b.T, d), 1.0).float()
+    h[::2] += 3.0                                   # sum over d ~ 192 on even rows
+    h = h.to(torch.bfloat16)
+    W = synth.normal_bf16(rng, (V, d), 0.05).float()
+    W[1000] = spike
+    W = W.to(torch.bfloat16)
+    z = oracle.logits(to_f64(h), to_f64(W), 1.0)
+    gap = (z.max(axis=1) - z[:, :256].max(axis=1))[::2]
+    assert gap.min() > (25 if spike < 0.3 else 75)
+    _full_check(b, h, W, grad_dtype=torch.float32)
+
+
 def test_confident_rows_keep_their_accuracy():
     """Targets equal to a dominant logit (p_y close to 1): G_y = g (p_y - 1) is
     small and formed from the fp32 target logit (a bf16-rounded p_y would be
