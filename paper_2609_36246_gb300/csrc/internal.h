@@ -236,7 +236,7 @@ size_t bwd_counter_words(int64_t Tpad, int64_t tc);
 
 // Top-K KL forward and backward over one sweep of the student's logits
 // (lmhead_fused.cu): workspace = the fused forward + backward regions, then
-// coef [T] and val [T, 16].
+// the slab rows' true half-tile maxima [tc, ceil(V/128)].
 size_t topk_kl_fb_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype);
 olive_status launch_topk_kl_fwd_bwd(const Ctx& c, const void* h_s, const void* W_s, int32_t d_s,
                                     const void* h_t, const void* W_t, int32_t d_t,

@@ -97,9 +97,14 @@ enum Kind : int { K_NONE = -1, K_GRAD = 0, K_KLZ = 1, K_DH = 2, K_DW = 3, K_ZSAV
 enum Phase : int { PH_ALL = 0, PH_Z = 1, PH_DHDW = 2, PH_R = 3 };
 
 // A half tile whose maximum exceeds the row's reference by more than this
-// (base 2) keeps its own maximum as reference: 2^(x - ref) stays below 2^100,
-// so sums of e . W over the vocabulary stay finite in fp32.
-constexpr float kRefMax = 100.f;
+// (base 2) keeps its own maximum as reference: e' = 2^(x - ref) stays below
+// 2^64 and the row scale 2^(R - lse2) above 2^-82 (V < 2^18), so neither the
+// bf16 operands nor the fp32 sums leave their normal range.
+constexpr float kRefMax = 64.f;
+// Such a half tile's reference when its small entries are still wanted (the
+// top-K candidates): 110 below its maximum, so e' spans 2^-133 .. 2^110 and
+// its sum stays below 2^117.
+constexpr float kOwnShift = 110.f;
 
 // CE maps: 0 hc K-major 64x128, 1 W K-major 64x256, 2 G K-major 64x128,
 //          3 W MN-major 64x64, 4 G MN-major 64x64, 5 hc MN-major 64x64
@@ -129,6 +134,8 @@ struct FusedParams {
                              // two halves of its first vocabulary tile (PH_R); null: ZSAVE
                              // tiles store e relative to each half tile's own maximum
   const float* lam;          // CE single pass: [tc] dH row scale (null: none)
+  float* part_tm;            // PH_Z: [tc, vh] true half-tile maximum (base 2), when kept
+  int32_t dw_coef;           // 1: DW tiles scale by g inv_tau (/ N_mask), the CE single pass
   float* s2;                 // KLZ: fp32 slab, [tc, ldg] (reverse) or [tc / 2, 2 ldg] (forward)
   float* part5;              // KLZ: [5][tc][vh] m_s, s_s, m_t, s_t, A per (row, half-tile)
   int64_t plane5;            // tc * vh
@@ -176,7 +183,7 @@ __device__ Plan make_plan(const FusedParams& p) {
   pl.ntd = (p.d + kBN - 1) / kBN;
   pl.mtv = (p.V + kBM - 1) / kBM;
   pl.coef = 0.f;
-  if (!p.kl && p.sp_k == 0 && p.phase == PH_ALL) {
+  if (!p.kl && p.sp_k == 0 && (p.phase == PH_ALL || p.dw_coef) && p.grad_loss) {
     float g = *p.grad_loss;
     if (p.reduction == OLIVE_REDUCE_MEAN && pl.n > 0) g = g / static_cast<float>(pl.n);
     pl.coef = g * p.inv_tau;
@@ -502,8 +509,10 @@ __device__ void epi_zsave(const FusedParams& p, const Plan& pl, const Unit& x, i
   }
   // the reference of the stored e and of the partial sum: the row's reference
   // maximum when one is given and tm does not exceed it by more than kRefMax,
-  // else the half tile's own maximum
-  const float ref = (p.zref && !(tm - R > kRefMax)) ? R : tm;
+  // else the half tile's own maximum (kOwnShift below it when the true maxima
+  // are kept for a top-K selection)
+  float ref = tm;
+  if (p.zref) ref = !(tm - R > kRefMax) ? R : (p.part_tm ? tm - kOwnShift : tm);
   __nv_bfloat16* grow = p.g + static_cast<size_t>(r_local) * p.ldg;
   float ts = 0.f;
 #pragma unroll 1
@@ -526,6 +535,7 @@ __device__ void epi_zsave(const FusedParams& p, const Plan& pl, const Unit& x, i
     const size_t o = static_cast<size_t>(r_local) * pl.vh + 2 * x.j + part;
     p.part_zm[o] = ref;
     p.part_zs[o] = ts;
+    if (p.part_tm) p.part_tm[o] = tm;
   }
 }
 
@@ -579,6 +589,7 @@ __device__ void epi_dw(const FusedParams& p, const Plan& pl, const Unit& x, int 
   const bool first = x.s == 0;
   const bool last = x.s == pl.n_slabs - 1;
   const int n0 = x.j * kBN;
+  const float sc = p.dw_coef ? pl.coef : 1.f;
 #pragma unroll 1
   for (int c = part * kHalf; c < (part + 1) * kHalf; c += 32) {
     const int col0 = n0 + c;
@@ -589,7 +600,7 @@ __device__ void epi_dw(const FusedParams& p, const Plan& pl, const Unit& x, int 
       tmem_ld_32x32b_x32(taddr + c, a);
       tmem_ld_wait();
 #pragma unroll
-      for (int k = 0; k < 32; ++k) g[k] = __uint_as_float(a[k]);
+      for (int k = 0; k < 32; ++k) g[k] = __uint_as_float(a[k]) * sc;
     } else {
 #pragma unroll
       for (int k = 0; k < 32; ++k) g[k] = 0.f;
@@ -884,15 +895,16 @@ __device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2
 }
 
 // One warp per row tile row of the slab, after ZSAVE tiles with a row
-// reference R (base 2): the row's stored e' = 2^(x - R) give
-// G = lam e' with lam = coef 2^(R - lse2), so instead of rewriting the row
-// this merges the partials into lse, writes logp, lse and the loss term, puts
-// G_y / lam = expm1(logp) 2^(lse2 - R) at the target (G_y from the exact z_y),
-// stores lam for the dH tiles and writes hs = lam hc, the dW product's scaled
-// rows.  A row where some half tile kept its own maximum as reference (it
+// reference R (base 2): the row's stored e' = 2^(x - R) give G = coef s e'
+// off the target, with coef = g inv_tau (/ N_mask) and s = 2^(R - lse2) per
+// row, so instead of rewriting the row this merges the partials into lse,
+// writes logp, lse and the loss term, puts G_y / (coef s) = expm1(logp) / s at
+// the target (G_y from the exact z_y), stores lam = coef s for the dH tiles
+// and writes hs = s hc, the dW product's scaled rows (the DW tiles apply
+// coef).  A row where some half tile kept its own maximum as reference (it
 // exceeded R by more than kRefMax) is rewritten in full relative to lse2
-// (e'' = p, lam = coef).  Rows past the slab's masked rows get lam = 0 and
-// hs = 0 up to the row tile's end.
+// (e'' = p, s = 1).  Rows past the slab's masked rows get lam = 0 and hs = 0
+// up to the row tile's end.
 __global__ void __launch_bounds__(256)
     ref_fix_kernel(const int32_t* __restrict__ n_rows, const int32_t* __restrict__ rows,
                    const int32_t* __restrict__ targets, int T, int V, int tc, int slab, int vh,
@@ -953,7 +965,7 @@ __global__ void __launch_bounds__(256)
       nll[row0 + r] = -lp;
       if (ybad) atomicOr(dev_status, 1 << OLIVE_ERR_TOKEN_RANGE);
     }
-    const float lm = own ? coef : coef * fast_exp2(R - lse2);
+    const float sr = own ? 1.f : fast_exp2(R - lse2);
     if (own) {
       // G / coef = e 2^(ref - lse2) = p, in place
       uint4* grow = reinterpret_cast<uint4*>(g + static_cast<size_t>(r) * ldg);
@@ -974,7 +986,7 @@ __global__ void __launch_bounds__(256)
     if (lane == 0 && !ybad)
       g[static_cast<size_t>(r) * ldg + y] =
           __float2bfloat16_rn(own ? expm1f(lp) : expm1f(lp) * fast_exp2(lse2 - R));
-    if (lane == 0) lam[r] = lm;
+    if (lane == 0) lam[r] = coef * sr;
     const uint4* hin = hc + static_cast<size_t>(row0 + r) * d8;
     for (int c = lane; c < d8; c += 32) {
       uint4 v = hin[c];
@@ -982,7 +994,7 @@ __global__ void __launch_bounds__(256)
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const float2 u = __bfloat1622float2(h2[e]);
-        h2[e] = __floats2bfloat162_rn(u.x * lm, u.y * lm);
+        h2[e] = __floats2bfloat162_rn(u.x * sr, u.y * sr);
       }
       hrow[c] = v;
     }
@@ -1132,15 +1144,16 @@ __global__ void __launch_bounds__(256)
 }
 
 // ------------------------------------------------ top-K KL in one pass ---
-// The student's forward tiles (no targets) leave e = 2^(x - m_half) in bf16
-// in the G slab and the half-tile (max, sum) partials.  Per masked row,
-// topk_kl_rows_kernel then
+// The student's forward tiles (no targets) leave e' = 2^(x - ref) in bf16 in
+// the G slab (ref = the row's reference R, or the half tile's own maximum
+// where that exceeds R by more than kRefMax), each half tile's (ref, sum) and
+// its true maximum m_half.  Per masked row, topk_kl_rows_kernel then
 //   1. merges the partials into lse_s and takes tau, the C-th largest
 //      half-tile maximum (C = min(K + 8, 24)): C distinct logits reach tau,
 //      so the row's C largest logits all lie in half tiles whose maximum is
 //      at least tau, and only those (about C of ~V/128) are read,
-//   2. takes from them the C largest approximate logits x ~ log2(e) + m_half
-//      (bf16 e resolves x to a few thousandths),
+//   2. takes from them the C largest approximate logits x ~ log2(e') + ref
+//      (bf16 e' resolves x to a few thousandths),
 //   3. recomputes those candidates' logits exactly (fp32 dot products
 //      h_s . W_s[u]) and keeps the K largest: the student's top-K set S,
 //      exact wherever fewer than C - K logits lie within bf16 resolution
@@ -1149,8 +1162,12 @@ __global__ void __launch_bounds__(256)
 //      the teacher's lse) and forms the truncated KL, the overlap with the
 //      teacher's top-K ids and the gradient terms of the top-K KL: with
 //      g = grad_kl inv_tau, P_S = sum_S p_s and A = KL_K + P_S,
-//      G[u] = -g A p_s(u) for every u, plus g p_s(u) (l_u - q_u + 1) on S.
-// topk_kl_conv_kernel then writes G over the slab.
+//      G[u] = -g A p_s(u) for every u, plus g p_s(u) (l_u - q_u + 1) on S,
+//   5. writes G without rewriting the row: off S, G = lam e' with
+//      lam = -g A 2^(R - lse2), so only the K entries of S are stored (as
+//      G / lam), lam goes to the dH tiles and hs = lam h_s to the dW tiles.
+//      Where lam is out of range (|lam| < 2^-96, |A| < 2^-20) or a half tile
+//      kept its own maximum, the row is rewritten as G itself (lam = 1).
 
 constexpr int kTkCand = 24;  // most candidates taken to the exact recomputation (K <= 16)
 
@@ -1242,9 +1259,13 @@ struct TopkKlRows {
   int T, V, tc, slab, vh, K;
   int64_t ldg;
   float inv_tau;
-  const float* part_zm;
-  const float* part_zs;
-  const __nv_bfloat16* g;  // e of the slab
+  const float* part_zm;  // [tc, vh] reference of each half tile's e'
+  const float* part_zs;  // [tc, vh] sum of 2^(x - ref)
+  const float* part_tm;  // [tc, vh] true half-tile maximum
+  const float* zref;     // [tc, 2] the row's reference halves
+  __nv_bfloat16* g;      // e' of the slab, then G / lam
+  float* lam;            // [tc] dH row scale
+  uint4* hs;             // [Tpad, ds8] lam h_s rows (dW operand)
   const uint4* h_s;
   const uint4* W_s;
   int ds8;
@@ -1260,8 +1281,6 @@ struct TopkKlRows {
   float* t_logp_s;
   float* kl_topk;
   float* overlap;  // nullable
-  float* coef;
-  float* val;
 };
 
 __global__ void __launch_bounds__(256) topk_kl_rows_kernel(const TopkKlRows a) {
@@ -1269,20 +1288,31 @@ __global__ void __launch_bounds__(256) topk_kl_rows_kernel(const TopkKlRows a) {
   const SlabPlan sp(n, a.tc);
   if (a.slab >= sp.n_slabs) return;
   const int in_s = sp.rows_in(n, a.slab);
+  const int row_end = min((in_s + kBM - 1) / kBM * kBM, a.tc);
   const int row0 = a.slab * sp.rps;
   const int lane = threadIdx.x & 31;
   const int warps = (gridDim.x * blockDim.x) >> 5;
   const int K = a.K;
   const int C = min(K + 8, kTkCand);
-  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < in_s; r += warps) {
-    const int t = a.rows[row0 + r];
-    if (t < 0 || t >= a.T) continue;  // reported by the gather
+  const int nvec = (a.V + 7) / 8;
+  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < row_end; r += warps) {
+    const int t = r < in_s ? a.rows[row0 + r] : -1;
+    uint4* hrow = a.hs + static_cast<size_t>(row0 + r) * a.ds8;
+    if (t < 0 || t >= a.T) {
+      // reported by the gather (masked rows); the G row is zero
+      if (lane == 0) a.lam[r] = 0.f;
+      for (int c = lane; c < a.ds8; c += 32) hrow[c] = make_uint4(0u, 0u, 0u, 0u);
+      continue;
+    }
     const float* zm = a.part_zm + static_cast<size_t>(r) * a.vh;
     const float* zs = a.part_zs + static_cast<size_t>(r) * a.vh;
+    const float* tmx = a.part_tm + static_cast<size_t>(r) * a.vh;
+    const float R = fmaxf(a.zref[2 * r], a.zref[2 * r + 1]);
     // 1. lse_s, and tau = the C-th largest half-tile maximum: C distinct
     //    logits reach it, so every logit of the row's top C is >= tau and
     //    lies in a half tile whose maximum is >= tau
     float m = -INFINITY, sum = 0.f;
+    bool own = false;  // some half tile kept its own maximum as reference
     float tv[kTkCand];
     int ti[kTkCand];
 #pragma unroll
@@ -1291,8 +1321,9 @@ __global__ void __launch_bounds__(256) topk_kl_rows_kernel(const TopkKlRows a) {
       ti[j] = INT_MAX;
     }
     for (int j = lane; j < a.vh; j += 32) {
-      const float mj = zm[j];
-      lse_merge(m, sum, mj, zs[j]);
+      const float mj = tmx[j];
+      own |= mj - R > kRefMax;  // the forward tiles' own test
+      lse_merge(m, sum, zm[j], zs[j]);
       if (mj > tv[kTkCand - 1]) lane_list_insert(tv, ti, mj, j);
     }
 #pragma unroll
@@ -1301,7 +1332,9 @@ __global__ void __launch_bounds__(256) topk_kl_rows_kernel(const TopkKlRows a) {
       const float s2 = __shfl_xor_sync(0xffffffffu, sum, o);
       lse_merge(m, sum, m2, s2);
     }
-    const float lse_s = (m + log2f(sum)) * kLn2;
+    own = __any_sync(0xffffffffu, own);
+    const float lse2 = m + log2f(sum);
+    const float lse_s = lse2 * kLn2;
     float tau = -INFINITY;
     {
       int head = 0;
@@ -1309,7 +1342,7 @@ __global__ void __launch_bounds__(256) topk_kl_rows_kernel(const TopkKlRows a) {
     }
     // 2. candidates from the half tiles whose maximum reaches tau: each lane
     //    takes 4 columns of a tile and keeps its 16 best approximate logits
-    //    x = log2(e) + m_half (bf16 e: x to within a few thousandths)
+    //    x = log2(e') + ref (bf16 e': x to within a few thousandths)
     float lv[16];
     int li[16];
 #pragma unroll
@@ -1317,10 +1350,10 @@ __global__ void __launch_bounds__(256) topk_kl_rows_kernel(const TopkKlRows a) {
       lv[j] = -INFINITY;
       li[j] = INT_MAX;
     }
-    const __nv_bfloat16* grow = a.g + static_cast<size_t>(r) * a.ldg;
+    __nv_bfloat16* grow = a.g + static_cast<size_t>(r) * a.ldg;
     for (int base = 0; base < a.vh; base += 32) {
       const int j = base + lane;
-      unsigned b = __ballot_sync(0xffffffffu, j < a.vh && zm[j] >= tau);
+      unsigned b = __ballot_sync(0xffffffffu, j < a.vh && tmx[j] >= tau);
       while (b) {
         int js[4];
 #pragma unroll
@@ -1363,12 +1396,12 @@ __global__ void __launch_bounds__(256) topk_kl_rows_kernel(const TopkKlRows a) {
       }
     }
     // 3. exact logits of the candidates, then the K largest by rank
-    const uint4* hs = a.h_s + static_cast<size_t>(t) * a.ds8;
+    const uint4* hs_in = a.h_s + static_cast<size_t>(t) * a.ds8;
     float l = -INFINITY;
     for (int k = 0; k < C; ++k) {
       const int u = __shfl_sync(0xffffffffu, cid, k);
       if (u < 0) break;  // the list ends (fewer columns than candidates)
-      const float x = dot_row_bf16(hs, a.W_s + static_cast<size_t>(u) * a.ds8, a.ds8, lane);
+      const float x = dot_row_bf16(hs_in, a.W_s + static_cast<size_t>(u) * a.ds8, a.ds8, lane);
       if (lane == k) l = x * a.inv_tau - lse_s;
     }
     int rank = 0;
@@ -1410,12 +1443,12 @@ __global__ void __launch_bounds__(256) topk_kl_rows_kernel(const TopkKlRows a) {
     }
     const float gk = a.grad_kl[t] * a.inv_tau;
     const float A = kl + P;
+    const float val = in_k ? gk * p * (slp - q + 1.f - A) : 0.f;  // G at the lane's id of S
     const size_t o = static_cast<size_t>(t) * K + lane;
     if (lane < K) {
       a.s_ids[o] = sid;
       a.s_logp[o] = in_k ? slp : -INFINITY;
       a.t_logp_s[o] = in_k ? q : -INFINITY;
-      a.val[o] = in_k ? gk * p * (slp - q + 1.f - A) : 0.f;
     }
     if (a.overlap) {
       const int tid = lane < K ? a.t_ids[static_cast<size_t>(t) * K + lane] : -2;
@@ -1427,64 +1460,42 @@ __global__ void __launch_bounds__(256) topk_kl_rows_kernel(const TopkKlRows a) {
     if (lane == 0) {
       a.s_lse[t] = lse_s;
       a.kl_topk[t] = kl;
-      a.coef[t] = -gk * A;
     }
-  }
-}
-
-// One warp per masked row of the slab: G = coef[t] e 2^(m_half - lse2_s) for
-// every column (zero past V), then the K full values at the ids of S.
-__global__ void __launch_bounds__(256)
-    topk_kl_conv_kernel(const int32_t* __restrict__ n_rows, const int32_t* __restrict__ rows, int T,
-                        int V, int tc, int slab, int vh, int64_t ldg, int K,
-                        const float* __restrict__ part_zm, const float* __restrict__ s_lse,
-                        const float* __restrict__ coef, const float* __restrict__ val,
-                        const int32_t* __restrict__ ids, __nv_bfloat16* g) {
-  const int n = read_n_rows(n_rows, T, nullptr);
-  const SlabPlan sp(n, tc);
-  if (slab >= sp.n_slabs) return;
-  const int in_s = sp.rows_in(n, slab);
-  const int row0 = slab * sp.rps;
-  const int lane = threadIdx.x & 31;
-  const int warps = (gridDim.x * blockDim.x) >> 5;
-  const int nvec = (V + 7) / 8;
-  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < in_s; r += warps) {
-    const int t = rows[row0 + r];
-    if (t < 0 || t >= T) continue;  // the G row stays zero
-    const float* zm = part_zm + static_cast<size_t>(r) * vh;
-    const float lse2 = s_lse[t] * kLog2e;
-    const float cf = coef[t];
-    uint4* grow = reinterpret_cast<uint4*>(g + static_cast<size_t>(r) * ldg);
-#pragma unroll 1
-    for (int base = 0; base < nvec; base += 128) {
-      uint4 v[4];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int idx = base + 32 * q + lane;
-        if (idx < nvec) v[q] = grow[idx];
-      }
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int idx = base + 32 * q + lane;
-        if (idx >= nvec) continue;
-        const float sc = cf * fast_exp2(zm[idx >> 4] - lse2);
-        __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&v[q]);
-        const int col = idx * 8;
+    // 5. G: the scaled form, or the row rewritten as G itself
+    const float cf = -gk * A;
+    float lm = own ? 0.f : cf * fast_exp2(R - lse2);
+    const bool rewrite =
+        own || !(fabsf(lm) >= 0x1p-96f) || !(fabsf(lm) < 0x1p96f) || !(fabsf(A) >= 0x1p-20f);
+    if (rewrite) {
+      lm = 1.f;
+      uint4* g4 = reinterpret_cast<uint4*>(grow);
+      for (int idx = lane; idx < nvec; idx += 32) {
+        uint4 v = g4[idx];
+        const float sc = fast_exp2(zm[idx >> 4] - lse2);  // 16 vectors per half tile
+        __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&v);
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           const float2 u = __bfloat1622float2(h2[e]);
-          const float a = col + 2 * e < V ? u.x * sc : 0.f;
-          const float b = col + 2 * e + 1 < V ? u.y * sc : 0.f;
-          h2[e] = __floats2bfloat162_rn(a, b);
+          const int c = idx * 8 + 2 * e;
+          // p = e' 2^(ref - lse2) first, then the row coefficient
+          h2[e] = __floats2bfloat162_rn(c < a.V ? (u.x * sc) * cf : 0.f,
+                                        c + 1 < a.V ? (u.y * sc) * cf : 0.f);
         }
-        grow[idx] = v[q];
+        g4[idx] = v;
       }
     }
-    __syncwarp();  // the row's dense values are written before the K overrides
-    if (lane < K) {
-      const size_t o = static_cast<size_t>(t) * K + lane;
-      const int u = ids[o];
-      if (u >= 0 && u < V) g[static_cast<size_t>(r) * ldg + u] = __float2bfloat16_rn(val[o]);
+    __syncwarp();  // the candidate reads and any dense rewrite precede the K entries
+    if (in_k) grow[sid] = __float2bfloat16_rn(val / lm);
+    if (lane == 0) a.lam[r] = lm;
+    for (int c = lane; c < a.ds8; c += 32) {
+      uint4 v = hs_in[c];
+      __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&v);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float2 u = __bfloat1622float2(h2[e]);
+        h2[e] = __floats2bfloat162_rn(u.x * lm, u.y * lm);
+      }
+      hrow[c] = v;
     }
   }
 }
@@ -1648,8 +1659,10 @@ olive_status launch_loss_fwd_bwd(const Ctx& c, const void* hidden, const void* W
   p.part_zm = w.part_zm;
   p.part_zs = w.part_zs;
   p.zy_s = w.zy;
+  p.grad_loss = grad_loss;  // the DW tiles' coefficient
   p.zref = w.zref;
   p.lam = w.lam;
+  p.dw_coef = 1;
 
   int conv_blocks = static_cast<int>(ceil_div(w.tc, 8));
   if (conv_blocks > c.num_sms * 16) conv_blocks = c.num_sms * 16;
@@ -1734,9 +1747,8 @@ olive_status launch_topk_kl_fwd_bwd(const Ctx& c, const void* h_s, const void* W
                                     int grad_dtype, void* ws, int32_t* dev_status) {
   const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
   const FbWs w = carve_fb(ws, T, d_s, V, grad_dtype);
-  char* sparse = static_cast<char*>(ws) + fb_ws_bytes(T, d_s, V, grad_dtype);
-  float* coef = reinterpret_cast<float*>(sparse);
-  float* val = reinterpret_cast<float*>(sparse + align_up(4ull * T, kWsAlign));
+  float* part_tm =
+      reinterpret_cast<float*>(static_cast<char*>(ws) + fb_ws_bytes(T, d_s, V, grad_dtype));
   const int64_t ldg = vpad(V);
   const size_t elt = grad_dtype == OLIVE_DTYPE_BF16 ? 2 : 4;
   const int vh = static_cast<int>(ceil_div(V, kHalf));
@@ -1759,7 +1771,7 @@ olive_status launch_topk_kl_fwd_bwd(const Ctx& c, const void* h_s, const void* W
       !encode_bf16_2d(&maps.m[2], w.g, V, w.tc, 2ull * ldg, 64, 128) ||
       !encode_bf16_2d(&maps.m[3], W_s, d_s, V, 2ull * d_s, 64, 64) ||
       !encode_bf16_2d(&maps.m[4], w.g, V, w.tc, 2ull * ldg, 64, 64) ||
-      !encode_bf16_2d(&maps.m[5], w.hc, d_s, Tpad, 2ull * d_s, 64, 64))
+      !encode_bf16_2d(&maps.m[5], w.hs, d_s, Tpad, 2ull * d_s, 64, 64))
     return OLIVE_ERR_CUDA;
 
   FusedParams p = base_params(c, rows, n_rows, T, V, inv_tau, dev_status);
@@ -1780,6 +1792,9 @@ olive_status launch_topk_kl_fwd_bwd(const Ctx& c, const void* h_s, const void* W
   p.part_zm = w.part_zm;
   p.part_zs = w.part_zs;
   p.zy_s = w.zy;
+  p.zref = w.zref;
+  p.lam = w.lam;
+  p.part_tm = part_tm;
 
   TopkKlRows ra = {};
   ra.n_rows = n_rows;
@@ -1793,7 +1808,11 @@ olive_status launch_topk_kl_fwd_bwd(const Ctx& c, const void* h_s, const void* W
   ra.inv_tau = inv_tau;
   ra.part_zm = w.part_zm;
   ra.part_zs = w.part_zs;
-  ra.g = static_cast<const __nv_bfloat16*>(w.g);
+  ra.part_tm = part_tm;
+  ra.zref = w.zref;
+  ra.g = static_cast<__nv_bfloat16*>(w.g);
+  ra.lam = w.lam;
+  ra.hs = static_cast<uint4*>(w.hs);
   ra.h_s = static_cast<const uint4*>(h_s);
   ra.W_s = static_cast<const uint4*>(W_s);
   ra.ds8 = d_s / 8;
@@ -1809,20 +1828,17 @@ olive_status launch_topk_kl_fwd_bwd(const Ctx& c, const void* h_s, const void* W
   ra.t_logp_s = t_logp_s;
   ra.kl_topk = kl_topk;
   ra.overlap = t_ids ? overlap : nullptr;
-  ra.coef = coef;
-  ra.val = val;
 
   int conv_blocks = static_cast<int>(ceil_div(w.tc, 8));
   if (conv_blocks > c.num_sms * 16) conv_blocks = c.num_sms * 16;
   for (int s = 0; s < max_slabs; ++s) {
     p.slab = s;
+    p.phase = PH_R;
+    if ((st = launch_lmhead_fused(c, maps, p)) != OLIVE_OK) return st;
     p.phase = PH_Z;
     if ((st = launch_lmhead_fused(c, maps, p)) != OLIVE_OK) return st;
     ra.slab = s;
     topk_kl_rows_kernel<<<conv_blocks, 256, 0, c.stream>>>(ra);
-    topk_kl_conv_kernel<<<conv_blocks, 256, 0, c.stream>>>(
-        n_rows, rows, T, V, static_cast<int>(w.tc), s, vh, ldg, K, w.part_zm, s_lse, coef, val,
-        s_ids, static_cast<__nv_bfloat16*>(w.g));
     if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;
     p.phase = PH_DHDW;
     if ((st = launch_lmhead_fused(c, maps, p)) != OLIVE_OK) return st;

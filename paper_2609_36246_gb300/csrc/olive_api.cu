@@ -239,10 +239,12 @@ size_t topk_kl_bwd_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype) {
          align_up(4ull * 16 * T, kWsAlign);
 }
 
-// the fused forward + backward's regions, then coef [T] and val [T, 16]
+// the fused forward + backward's regions, then the true half-tile maxima
+// [tc, ceil(V/128)] of the slab rows
 size_t topk_kl_fb_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype) {
-  return fb_ws_bytes(T, d, V, grad_dtype) + align_up(4ull * T, kWsAlign) +
-         align_up(4ull * 16 * T, kWsAlign);
+  const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
+  return fb_ws_bytes(T, d, V, grad_dtype) +
+         align_up(4ull * slab_rows(Tpad, V) * ceil_div(V, 128), kWsAlign);
 }
 
 static KlWs carve_kl_impl(void* ws, int64_t T, int64_t ds, int64_t dt, int64_t V, int grad,

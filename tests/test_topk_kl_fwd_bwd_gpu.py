@@ -196,6 +196,47 @@ def test_several_slabs(monkeypatch):
     _full_check(hs, Ws, ht, Wt, rows, K, g, 1.0, grad_dtype=torch.bfloat16)
 
 
+@pytest.mark.parametrize("spike", [0.2, 0.5])
+def test_rows_far_above_their_first_tile(spike):
+    """One student id far down the vocabulary (1000) sits 31-39 nats (spike
+    0.2: the scaled form, e' up to ~2^57) or 78-101 nats (spike 0.5: beyond
+    the reference window, the row is rewritten as G) above the row's first
+    256 logits on half of the rows."""
+    rng = np.random.default_rng(int(spike * 10) + 40)
+    T, d, V, K = 160, 64, 3000, 8
+    hs = synth.normal_bf16(rng, (T, d), 1.0).float()
+    hs[::2] += 3.0
+    hs = hs.to(torch.bfloat16)
+    Ws = synth.normal_bf16(rng, (V, d), 0.05).float()
+    Ws[1000] = spike
+    Ws = Ws.to(torch.bfloat16)
+    ht = synth.normal_bf16(rng, (T, d), 1.0)
+    Wt = synth.normal_bf16(rng, (V, d), 0.3)
+    z = oracle.logits(to_f64(hs), to_f64(Ws), 1.0)
+    gap = (z.max(axis=1) - z[:, :256].max(axis=1))[::2]
+    assert gap.min() > (25 if spike < 0.3 else 75)
+    rows = _decided_rows(hs, Ws, ht, Wt, np.arange(T), K, 1.0)
+    g = rng.uniform(0.5, 2.0, size=T)
+    _full_check(hs, Ws, ht, Wt, rows, K, g, 1.0)
+
+
+def test_tiny_weights_take_the_rewritten_form():
+    """Rows with g_t = 1e-30 put the row scale below 2^-96, so their G is
+    written out in full; each such row still matches on its own."""
+    rng = np.random.default_rng(77)
+    T, ds, dt, V, K = 120, 64, 96, 2000, 16
+    hs, Ws, ht, Wt = _models(rng, T, ds, dt, V)
+    rows = _decided_rows(hs, Ws, ht, Wt, np.arange(T), K, 1.0)
+    g = np.where(np.arange(T) % 3 == 0, 1e-30, rng.uniform(0.5, 2.0, size=T))
+    o = _full_check(hs, Ws, ht, Wt, rows, K, g, 1.0)
+    rdh, _ = oracle.token_topk_kl_bwd(to_f64(hs), to_f64(Ws), to_f64(ht), to_f64(Wt), rows, K, grad=g,
+                                      with_dW=False)
+    tiny = [t for t in rows if t % 3 == 0][:8]
+    assert len(tiny) >= 4
+    for t in tiny:
+        assert rel_frob(o["d_h_s"][t], rdh[t]) <= 2e-2, t
+
+
 def test_empty_mask():
     rng = np.random.default_rng(3)
     hs, Ws, ht, Wt = _models(rng, 40, 64, 64, 300)
