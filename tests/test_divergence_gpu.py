@@ -7,7 +7,8 @@ import torch
 import oracle
 from paper_2609_36246_gb300 import binding as B
 from paper_2609_36246_gb300 import synth
-from tests.parity import assert_close_grad, assert_close_logp, rel_frob, sample_rows, to_f32, to_f64
+from tests.parity import (FULL_SIZE_ROWS, assert_close_grad, assert_close_logp, rel_frob, sample_rows,
+                          to_f32, to_f64)
 
 pytestmark = pytest.mark.gpu
 
@@ -71,7 +72,8 @@ def test_no_gradient_requested_bf16():
 
 @pytest.mark.slow
 def test_kl_workload_sampled_rows():
-    """16384 rows, d_s = 4096, d_t = 5120, V = 151936: sampled oracle rows."""
+    """16384 rows, d_s = 4096, d_t = 5120, V = 151936: KL and dH_s on 2048
+    sampled rows."""
     T = 16384
     hs = synth.make_hidden("kl", T)
     Ws = synth.make_weight("kl")
@@ -79,7 +81,7 @@ def test_kl_workload_sampled_rows():
     rows = np.arange(T, dtype=np.int32)
     gk = np.ones(T, dtype=np.float32)
     kl, dhs = _gpu(hs, Ws, ht, Wt, rows, gk, "reverse", grad_dtype=torch.bfloat16)
-    pick = sample_rows(rows, 16, seed=2)
+    pick = sample_rows(rows, FULL_SIZE_ROWS, seed=2)
     rkl, rdhs = oracle.token_divergence(to_f32(hs), to_f32(Ws), to_f32(ht), to_f32(Wt), pick,
                                         grad_kl=np.ones(T))
     assert_close_logp(kl[pick], rkl[pick], "kl")

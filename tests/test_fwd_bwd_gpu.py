@@ -9,8 +9,8 @@ import torch
 import oracle
 from paper_2609_36246_gb300 import binding as B
 from paper_2609_36246_gb300 import synth
-from tests.parity import (assert_close_grad, assert_close_logp, assert_close_loss, gpu_pack,
-                          oracle_pack, rel_frob, sample_rows, to_f32, to_f64)
+from tests.parity import (FULL_SIZE_ROWS, assert_close_grad, assert_close_logp, assert_close_loss,
+                          gpu_pack, oracle_pack, rel_frob, sample_rows, to_f32, to_f64)
 
 pytestmark = pytest.mark.gpu
 
@@ -183,16 +183,20 @@ def test_medium_vocab_sampled():
 
 @pytest.mark.slow
 def test_fwdbwd_workload_sampled():
-    """8 x 4096 tokens, d = 4096, V = 151936 (the timed step's configuration)."""
+    """8 x 4096 tokens, d = 4096, V = 151936 (the timed step's configuration):
+    log-probs, lse and dH on 2048 sampled masked rows, dW through the
+    vocabulary-sum property, dH = 0 off the mask, loss = -sum logp."""
     b = synth.make_batch("fwdbwd")
     h = synth.make_hidden("fwdbwd", b.T)
     W = synth.make_weight("fwdbwd")
-    logp, _, loss, dh, dw = _gpu(b, h, W)
+    logp, lse, loss, dh, dw = _gpu(b, h, W)
     o = oracle_pack(b)
-    rows = sample_rows(o["rows"], 24, seed=1)
-    rl, _, _ = oracle.token_logprob(to_f32(h), to_f32(W), o["targets"], rows)
+    rows = sample_rows(o["rows"], FULL_SIZE_ROWS, seed=1)
+    hf, Wf = to_f32(h), to_f32(W)
+    rl, rlse, _ = oracle.token_logprob(hf, Wf, o["targets"], rows)
     assert_close_logp(logp[rows], rl[rows])
-    ref = oracle.token_loss_bwd_rows(to_f32(h), to_f32(W), o["targets"], rows)
+    assert_close_logp(lse[rows], rlse[rows], "lse")
+    ref = oracle.token_loss_bwd_rows(hf, Wf, o["targets"], rows)
     assert rel_frob(dh[rows], ref) <= 1e-2
     off = np.setdiff1d(np.arange(b.T), o["rows"])
     assert not dh[off].any()
