@@ -86,6 +86,6 @@ def test_kl_workload_sampled():
     ht, Wt = synth.make_teacher("kl", T)
     rows = np.arange(T)
     ov, kl = _gpu(hs, Ws, ht, Wt, rows, 16)
-    pick = sample_rows(rows, 12, seed=8)
+    pick = sample_rows(rows, 256, seed=8)
     ref = oracle.token_topk_compare(to_f32(hs), to_f32(Ws), to_f32(ht), to_f32(Wt), pick, 16)
     _check(ov, kl, ref, pick, min_decided=0.5)

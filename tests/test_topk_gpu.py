@@ -103,7 +103,7 @@ def test_scoring_workload_sampled_rows():
     W = synth.make_weight("scoring")
     o = oracle.splice_pack(b.prefix_ids, b.prefix_off, b.cont_ids, b.cont_off, b.V)
     gpu = _gpu(h, W, o["rows"], 16)
-    pick = sample_rows(o["rows"], 16, seed=6)
+    pick = sample_rows(o["rows"], 512, seed=6)
     lp, lse = oracle.log_softmax_rows(oracle.logits(to_f32(h[torch.from_numpy(pick)]).astype(np.float64), to_f32(W), 1.0))
     H = -(np.exp(lp) * lp).sum(axis=1)
     _check_rows(pick, 16, gpu, lse, H, lp)
