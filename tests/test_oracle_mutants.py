@@ -49,6 +49,17 @@ MUTANTS = {
     "kl_grad_forward_sign": ("                dz = ps - pt", "                dz = pt - ps"),
     "topk_grad_drops_mass_term": ("            G[k] = -ps[k] * (kl + P_S)", "            G[k] = -ps[k] * kl"),
     "topk_grad_drops_plus_one": ("(lps[k, S] - lpt[k, S] + 1.0)", "(lps[k, S] - lpt[k, S])"),
+    "entropy_wrong_sign": ("H[rr] = -(np.exp(lp) * lp).sum(axis=1)", "H[rr] = (np.exp(lp) * lp).sum(axis=1)"),
+    "topk_ties_by_descending_id": ("order = np.lexsort((ids, -lp[k]))[:K]",
+                                   "order = np.lexsort((-ids, -lp[k]))[:K]"),
+    "topk_takes_smallest": ("order = np.lexsort((ids, -lp[k]))[:K]", "order = np.lexsort((ids, lp[k]))[:K]"),
+    "overlap_over_union": ("overlap[r] = len(set(S.tolist()) & set(Tk.tolist())) / K",
+                           "overlap[r] = len(set(S.tolist()) & set(Tk.tolist())) / "
+                           "len(set(S.tolist()) | set(Tk.tolist()))"),
+    "topk_kl_renormalised": ("kl[r] = float((np.exp(lps[k, S]) * (lps[k, S] - lpt[k, S])).sum())",
+                             "ls_ = lps[k, S] - np.logaddexp.reduce(lps[k, S]); "
+                             "lt_ = lpt[k, S] - np.logaddexp.reduce(lpt[k, S]); "
+                             "kl[r] = float((np.exp(ls_) * (ls_ - lt_)).sum())"),
 }
 
 
@@ -161,8 +172,29 @@ def pin_topk_kl_grad(O):
                 and np.allclose(dW, Ws_t.grad.numpy(), atol=1e-12))
 
 
+def pin_topk_closed_forms(O):
+    """Uniform logits (entropy ln V, ties by ascending id) and a three-token row whose
+    top-K overlap, truncated KL, top-K log-probs and entropy are worked out by hand."""
+    V = 50
+    h = np.random.default_rng(5).standard_normal((2, 3))
+    _, H, tv, ti = O.token_topk(h, np.zeros((V, 3)), [0, 1], 4)
+    ok = np.allclose(H, math.log(V), atol=1e-12) and np.array_equal(ti, np.tile(np.arange(4), (2, 1)))
+    ok &= np.allclose(tv, -math.log(V), atol=1e-12)
+    hs = np.ones((1, 1))
+    Ws, Wt = np.array([[2.0], [1.0], [0.0]]), np.array([[0.0], [1.0], [2.0]])
+    Z = math.e ** 2 + math.e + 1
+    p0, p2 = math.e ** 2 / Z, 1 / Z
+    for K, (ov_ref, kl_ref) in {1: (0.0, 2 * p0), 2: (0.5, 2 * p0), 3: (1.0, 2 * p0 - 2 * p2)}.items():
+        ov, kl, _, _ = O.token_topk_compare(hs, Ws, hs, Wt, [0], K)
+        ok &= ov[0] == ov_ref and abs(kl[0] - kl_ref) < 1e-12
+    _, H3, tv3, ti3 = O.token_topk(hs, Ws, [0], 2)
+    ok &= ti3[0].tolist() == [0, 1] and abs(tv3[0, 0] - (2 - math.log(Z))) < 1e-12
+    ok &= abs(H3[0] - (math.log(Z) - (2 * math.e ** 2 + math.e) / Z)) < 1e-12
+    return bool(ok)
+
+
 PINS = [pin_golden_splice, pin_turns_golden, pin_uniform, pin_scipy, pin_torch_ce_and_autograd, pin_kl,
-        pin_topk_kl_grad]
+        pin_topk_kl_grad, pin_topk_closed_forms]
 
 
 def test_real_oracle_passes_every_pin():

@@ -412,6 +412,31 @@ def test_topk_compare_pins():
         assert gs[r] > 0 and gt[r] > 0
 
 
+def test_topk_compare_three_token_closed_form():
+    """V = 3, student logits (2, 1, 0), teacher logits (0, 1, 2): both rows have the same
+    log-sum-exp Z = ln(e^2 + e + 1), so log p_s(v) - log p_t(v) = z_s(v) - z_t(v) = (2, 0, -2).
+    K = 1: S = {0}, teacher top-1 = {2}: overlap 0, KL_1 = 2 p_s(0).
+    K = 2: S = {0, 1}, teacher {2, 1}: overlap 1/2, KL_2 = 2 p_s(0) + 0 p_s(1) = KL_1.
+    K = 3: overlap 1, KL_3 = 2 p_s(0) - 2 p_s(2), the full reverse KL.
+    Without renormalisation over S the truncated terms keep the full-vocabulary p_s."""
+    hs, ht = np.ones((1, 1)), np.ones((1, 1))
+    Ws = np.array([[2.0], [1.0], [0.0]])
+    Wt = np.array([[0.0], [1.0], [2.0]])
+    Z = math.e ** 2 + math.e + 1
+    p0, p2 = math.e ** 2 / Z, 1 / Z
+    expect = {1: (0.0, 2 * p0), 2: (0.5, 2 * p0), 3: (1.0, 2 * p0 - 2 * p2)}
+    for K, (ov_ref, kl_ref) in expect.items():
+        ov, kl, _, _ = oracle.token_topk_compare(hs, Ws, ht, Wt, [0], K)
+        assert ov[0] == ov_ref
+        assert kl[0] == pytest.approx(kl_ref, rel=1e-13)
+    # the top-K lists themselves: descending log-probs with their ids
+    _, H, tv, ti = oracle.token_topk(hs, Ws, [0], 2)
+    assert ti[0].tolist() == [0, 1]
+    assert tv[0] == pytest.approx([2 - math.log(Z), 1 - math.log(Z)], rel=1e-13)
+    # entropy: ln Z - sum_v p_v z_v
+    assert H[0] == pytest.approx(math.log(Z) - (2 * math.e ** 2 + math.e) / Z, rel=1e-13)
+
+
 def test_topk_kl_bwd_matches_autograd_with_fixed_set():
     rng = np.random.default_rng(19)
     T, ds, dt, V, K = 5, 7, 9, 40, 6
