@@ -62,6 +62,29 @@ def test_random_turn_flags(seed, S, maxlen):
     _compare(b, flags, T_cap=b.T + 100)
 
 
+def _turn_runs(n, seed, action_len=200, obs_len=60):
+    """Alternating runs over the continuation ids: teacher actions (flag 1) and
+    observations (flag 0), each run's length geometric with the given mean."""
+    rng = np.random.default_rng(seed)
+    flags = np.empty(n, np.uint8)
+    i, on = 0, True
+    while i < n:
+        L = int(rng.geometric(1.0 / (action_len if on else obs_len)))
+        flags[i:i + L] = 1 if on else 0
+        i += L
+        on = not on
+    return flags
+
+
+def test_varlen_batch_with_turn_runs():
+    """The largest packing input (64 sequences, 528k packed tokens) with teacher actions
+    and observations alternating along every continuation: bit-exact against the oracle."""
+    b = synth.make_batch("varlen")
+    flags = _turn_runs(len(b.cont_ids), 310)
+    g, o = _compare(b, flags)
+    assert 0 < o["n_rows"] < b.n_mask
+
+
 def test_all_ones_matches_plain_and_all_zero_is_empty():
     rng = np.random.default_rng(9)
     b = synth.batch_from_lengths(rng, rng.integers(1, 500, size=9), rng.integers(0, 900, size=9), 800)
