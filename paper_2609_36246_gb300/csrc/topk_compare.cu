@@ -74,8 +74,19 @@ __global__ void topk_compare_kernel(const uint4* __restrict__ h_t, const uint4* 
         continue;
       }
       const uint4* wrow = W_t + static_cast<size_t>(v) * d8;
-      float part = 0.f;
-      for (int c = lane; c < d8; c += 32) part += dot_bf16x8(__ldg(hrow + c), __ldg(wrow + c));
+      // four 16-byte groups per lane in flight
+      float p0 = 0.f, p1 = 0.f, p2 = 0.f, p3 = 0.f;
+      int c = lane;
+      for (; c + 96 < d8; c += 128) {
+        const uint4 w0 = __ldg(wrow + c), w1 = __ldg(wrow + c + 32), w2 = __ldg(wrow + c + 64),
+                    w3 = __ldg(wrow + c + 96);
+        p0 += dot_bf16x8(__ldg(hrow + c), w0);
+        p1 += dot_bf16x8(__ldg(hrow + c + 32), w1);
+        p2 += dot_bf16x8(__ldg(hrow + c + 64), w2);
+        p3 += dot_bf16x8(__ldg(hrow + c + 96), w3);
+      }
+      for (; c < d8; c += 32) p0 += dot_bf16x8(__ldg(hrow + c), __ldg(wrow + c));
+      float part = (p0 + p1) + (p2 + p3);
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
       const float lpt = part * inv_tau - lse_t;
