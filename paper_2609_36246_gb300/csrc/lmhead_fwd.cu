@@ -184,8 +184,8 @@ struct FwdKernT {
           const float2 e = buf[q * kEpiThreads];
           const float cv = e.x;
           const int ci = __float_as_int(e.y);
-          if (cv > tv[kTopMax - 1] || (cv == tv[kTopMax - 1] && ci < ti[kTopMax - 1]))
-            topk_insert(tv, ti, cv, ci);
+          // a unit visits its ids in ascending order: values alone order the list
+          if (cv > tv[kTopMax - 1]) topk_insert_asc(tv, ti, cv, ci);
         }
       } else {
 #pragma unroll

@@ -159,27 +159,29 @@ struct OpdKern {
       A = A * (p.reverse ? rs : rt) + e_a;
       ms = msn;
       mt = mtn;
+      // a unit visits its ids in ascending order, so a new id is larger than
+      // every listed one: values alone decide the candidates and their places
       uint32_t cand_s = 0u, cand_t = 0u;
+      const float last_s = sv[kTopMax - 1], last_t = tv[kTopMax - 1];
 #pragma unroll
       for (int k = 0; k < 32; ++k) {
         const bool ok = k < nvalid;
-        if (ok && topk_beats_last(sv, si, __uint_as_float(a[k]), col0 + k)) cand_s |= 1u << k;
-        if (ok && topk_beats_last(tv, ti, __uint_as_float(b[k]), col0 + k)) cand_t |= 1u << k;
+        if (ok && __uint_as_float(a[k]) > last_s) cand_s |= 1u << k;
+        if (ok && __uint_as_float(b[k]) > last_t) cand_t |= 1u << k;
       }
 #pragma unroll 1
       while (cand_s) {
         const int k = __ffs(cand_s) - 1;
         cand_s &= cand_s - 1u;
         const float v = __uint_as_float(pick32(a, k));
-        if (topk_beats_last(sv, si, v, col0 + k))
-          topk_insert3(sv, si, sx, v, col0 + k, __uint_as_float(pick32(b, k)));
+        if (v > sv[kTopMax - 1]) topk_insert3_asc(sv, si, sx, v, col0 + k, __uint_as_float(pick32(b, k)));
       }
 #pragma unroll 1
       while (cand_t) {
         const int k = __ffs(cand_t) - 1;
         cand_t &= cand_t - 1u;
         const float w = __uint_as_float(pick32(b, k));
-        if (topk_beats_last(tv, ti, w, col0 + k)) topk_insert(tv, ti, w, col0 + k);
+        if (w > tv[kTopMax - 1]) topk_insert_asc(tv, ti, w, col0 + k);
       }
     }
 

@@ -47,4 +47,39 @@ __device__ __forceinline__ void topk_insert3(float (&tv)[kTopMax], int (&ti)[kTo
   }
 }
 
+// The same two insertions for a sweep that visits ids in ascending order
+// within the list's lifetime: the new id is larger than every id already
+// listed, so among equal values it belongs last, and the value alone decides
+// its place (no id comparisons).
+__device__ __forceinline__ void topk_insert_asc(float (&tv)[kTopMax], int (&ti)[kTopMax], float cv,
+                                                int ci) {
+#pragma unroll
+  for (int j = 0; j < kTopMax; ++j) {
+    const bool before = cv > tv[j];
+    const float v = tv[j];
+    const int i = ti[j];
+    tv[j] = before ? cv : v;
+    ti[j] = before ? ci : i;
+    cv = before ? v : cv;
+    ci = before ? i : ci;
+  }
+}
+
+__device__ __forceinline__ void topk_insert3_asc(float (&tv)[kTopMax], int (&ti)[kTopMax],
+                                                 float (&tx)[kTopMax], float cv, int ci, float cx) {
+#pragma unroll
+  for (int j = 0; j < kTopMax; ++j) {
+    const bool before = cv > tv[j];
+    const float v = tv[j];
+    const int i = ti[j];
+    const float x = tx[j];
+    tv[j] = before ? cv : v;
+    ti[j] = before ? ci : i;
+    tx[j] = before ? cx : x;
+    cv = before ? v : cv;
+    ci = before ? i : ci;
+    cx = before ? x : cx;
+  }
+}
+
 }  // namespace olive
