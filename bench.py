@@ -4,15 +4,19 @@ One step = the whole hot path over one packed batch: splice/pack of the
 spliced sequences (student prefix || teacher continuation), then one
 olive_token_loss_fwd_bwd call: the LM-head forward with online log-sum-exp
 and the masked continuation loss of Eq. (osd-ce) (log-probs, lse, loss) and
-its backward (d hidden, d W in bf16), each logit tile computed once.  Workload: 8 sequences of
-4096 tokens, cut ~ U[256, 3840), d = 4096, V = 151936, bf16, synthetic seeded
-data (the "fwdbwd" workload of paper_2609_36246_gb300.synth).
+its backward (d hidden, d W in bf16), the logit gradient formed and consumed
+on chip (no [rows, V] array is stored; the logits are computed twice, once
+per pass).  Workload: 8 sequences of 4096 tokens, cut ~ U[256, 3840),
+d = 4096, V = 151936, bf16, synthetic seeded data (the "fwdbwd" workload of
+paper_2609_36246_gb300.synth).
 
 Metric: masked continuation tokens per second, i.e. N_mask * steps / time,
 and the fraction of bf16 dense tensor peak of the counted work
 6 * N_mask * d * V FLOPs per step (forward product, dH and dW products).
-The two-call path (olive_token_logprob_fwd + olive_token_loss_bwd, which
-recomputes the logits) is timed beside it for comparison.
+Secondary lines on the same batch: the slab form
+(olive_token_loss_fwd_bwd_slab, which keeps e' = exp(z - R) for every masked
+row in HBM and computes each logit once) and the two-call path
+(olive_token_logprob_fwd + olive_token_loss_bwd).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -144,20 +148,28 @@ def make_inputs(rank: int):
 
 # --------------------------------------------------------------------------- oracle legs
 def oracle_sample_rate(b, h, W, n_rows: int, seed: int = 0):
-    """fp64 oracle on a sample of masked rows: forward log-probs, dH of those
-    rows and their dW contribution (the same per-row work as one step).
-    Returns (masked tokens per second, seconds, rows)."""
+    """fp64 oracle on samples of masked rows: forward log-probs, dH of those
+    rows and their dW contribution (the same per-row work as one step).  Each
+    oracle call also pays a fixed cost (W widened to fp64, the [V, d] fp64 dW
+    zeroed and written: seconds at V = 151936, d = 4096), so the rate is
+    differential: the same computation on n and on 3n rows, rate =
+    2n / (t(3n) - t(n)), fixed = t(n) - n / rate.
+    Returns (masked tokens per second, fixed seconds, seconds in all, rows)."""
     import oracle
     o = oracle.splice_pack(b.prefix_ids, b.prefix_off, b.cont_ids, b.cont_off, b.V)
     rng = np.random.default_rng(seed)
-    rows = np.sort(rng.choice(o["rows"], size=min(n_rows, len(o["rows"])), replace=False))
     hf = h.float().numpy()
     Wf = W.float().numpy()
-    t0 = time.perf_counter()
-    oracle.token_logprob(hf, Wf, o["targets"], rows)
-    oracle.token_loss_bwd(hf, Wf, o["targets"], rows)
-    dt = time.perf_counter() - t0
-    return len(rows) / dt, dt, len(rows)
+    times = []
+    for k in (n_rows, 3 * n_rows):
+        rows = np.sort(rng.choice(o["rows"], size=min(k, len(o["rows"])), replace=False))
+        t0 = time.perf_counter()
+        oracle.token_logprob(hf, Wf, o["targets"], rows)
+        oracle.token_loss_bwd(hf, Wf, o["targets"], rows)
+        times.append(time.perf_counter() - t0)
+    rate = 2 * n_rows / max(times[1] - times[0], 1e-9)
+    fixed = max(times[0] - n_rows / rate, 0.0)
+    return rate, fixed, sum(times), 4 * n_rows
 
 
 def host_cores() -> int:
@@ -287,8 +299,11 @@ def run_ours(args, world, rank, local):
     h2d = sum(x.numel() * x.element_size() for x in host_in)
     e2e = {"value": N_mask * e_steps * world / (e_ms / 1e3), "unit": "tokens/s",
            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": 4,
-           "note": "pinned host inputs copied every step on a second stream, overlapped with "
-                   "the previous step's compute (two device input sets); loss read back every step"}
+           "note": "pinned host inputs (ids and hidden rows) copied every step on a second "
+                   "stream, overlapped with the previous step's compute (two device input sets); "
+                   "the loss read back every step; W, d_hidden and d_W stay on the device by "
+                   "design (a training step that feeds an on-device optimizer), so they are "
+                   "neither copied in nor read back"}
     assert math.isfinite(float(loss_h.item()))
     del dev_in
 
@@ -299,22 +314,28 @@ def run_ours(args, world, rank, local):
     burst, sustained, src = load_peaks()
     counted = 6.0 * N_mask * d * V
     step_tflops = counted / (ms_per_step / 1e3) / 1e12
-    # dominant kernel: lmhead_fused_kernel, launched three times per slab
-    # (the reference tiles, the forward tiles, the dH/dW tiles); its
+    # dominant kernel: lmhead_group_kernel, launched four times per call (the
+    # rows' reference maxima, pass A: lse, logp and dH, its redo launch, empty
+    # unless a row's maximum exceeds its reference by 2^64, pass B: dW).  Its
     # algorithmic work per call is the forward product plus dH and dW,
-    # 6 N_mask d V, and the call is bracketed by events on its stream (so the
-    # row gather, the per-row fix-up and the loss reduction count against it)
-    slabs = -(-((T + 127) // 128 * 128) // B.slab_rows_for(T, V))
+    # 6 N_mask d V; it executes 8 N_mask d V (each pass computes the logits).
+    # The call is bracketed by events on its stream, so the row gather, the
+    # memsets and the loss reduction count against it.  The call lasts tens of
+    # milliseconds, so the denominator is the burst peak.
     fb_flops = counted
     ach_fb = fb_flops / (fb_ms / 1e3) / 1e12
-    rev = kernel_rev()
-    traffic = profile_traffic("lmhead_fused_kernel", rev)
-    # splice (scan, fill) + gather + per slab (reference tiles, forward tiles, fix-up,
-    # dH/dW tiles) + loss reduce
-    launches = 2 + 1 + 4 * slabs + 1
+    rev = kernel_rev("lmhead_group.cu")
+    traffic = profile_traffic("lmhead_group_kernel", rev)
+    # algorithmic DRAM bytes of a call: W read, hc read (once per pass), dW and
+    # dH written (bf16)
+    alg_bytes = 2.0 * V * d + 2 * 2.0 * N_mask * d + 2.0 * V * d + 2.0 * N_mask * d
+    # splice (scan, fill) + row gather + 4 lmhead_group_kernel + loss reduce
+    launches = 2 + 1 + 4 + 1
 
-    two_call = None
+    two_call = slab = None
     if not args.no_extra:
+        slab = measure_slab(dev, hidden, W, pk_fn=lambda: B.olive_splice_pack(
+            pre, poff, con, coff, V, T, dev_status=st), T=T, d=d, V=V, n=N_mask, burst=burst)
         two_call = measure_two_call(dev, hidden, W, pk_fn=lambda: B.olive_splice_pack(
             pre, poff, con, coff, V, T, dev_status=st), T=T, d=d, V=V, n=N_mask, burst=burst)
 
@@ -335,10 +356,13 @@ def run_ours(args, world, rank, local):
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
-        rate, secs, nr = oracle_sample_rate(b, h_cpu, W_cpu, args.cpu_rows or 96)
+        nr = args.cpu_rows or 24
+        rate, fixed, secs, _ = oracle_sample_rate(b, h_cpu, W_cpu, nr)
         cpu = {"value": rate, "unit": "tokens/s", "cores": host_cores(), "kind": "oracle",
-               "sample": f"{nr} masked rows of the same batch: fp64 logits, log-probs, dH and dW "
-                         f"contributions ({secs:.1f} s)"}
+               "sample": f"{nr} and {3 * nr} masked rows of the same batch: fp64 logits, "
+                         f"log-probs, dH and dW contributions; per-row rate from the difference "
+                         f"({secs:.1f} s in all)",
+               "fixed_s_per_call": fixed}
 
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
@@ -353,16 +377,21 @@ def run_ours(args, world, rank, local):
         "dense_equivalent_note": "6 T d V over the packed T (unmasked rows included); not the "
                                  "headline, which counts the N_mask scored rows only",
         "phases_ms": {"splice_pack": spl_ms, "loss_fwd_bwd": fb_ms},
-        "roofline": {"kernel": "lmhead_fused_kernel (row-maximum tiles, forward tiles, dH/dW "
-                               "tiles: 3 launches per slab)",
-                     "bound": "tensor", "achieved": ach_fb, "peak": sustained, "unit": "TFLOP/s",
-                     "frac": ach_fb / sustained, "traffic": traffic,
-                     "peak_source": f"{src} bf16_tflops_sustained",
-                     "flops_per_call": fb_flops, "kernel_rev": rev,
-                     "note": "per olive_token_loss_fwd_bwd call (its lmhead_fused_kernel launches, "
-                             "timed with the gather, fix-up and loss kernels around them); "
-                             "traffic is DRAM bytes of those launches"},
+        "roofline": {"kernel": "lmhead_group_kernel (reference maxima, pass A: lse/logp/dH, "
+                               "its redo launch, pass B: dW)",
+                     "bound": "tensor", "achieved": ach_fb, "peak": burst, "unit": "TFLOP/s",
+                     "frac": ach_fb / burst, "traffic": traffic,
+                     "algorithmic_bytes": alg_bytes,
+                     "traffic_over_algorithmic": (traffic / alg_bytes) if traffic else None,
+                     "peak_source": f"{src} bf16_tflops (burst: one call lasts tens of ms)",
+                     "flops_per_call": fb_flops, "executed_flops_per_call": 8.0 * N_mask * d * V,
+                     "executed_frac": 8.0 * N_mask * d * V / (fb_ms / 1e3) / 1e12 / burst,
+                     "kernel_rev": rev,
+                     "note": "per olive_token_loss_fwd_bwd call (its lmhead_group_kernel launches, "
+                             "timed with the gather, memsets and loss reduction around them); "
+                             "traffic is DRAM bytes of those launches from an ncu capture"},
         "two_call_path": two_call,
+        "slab_path": slab,
         "e2e": e2e,
         "gpu_launches": launches * args.steps,
         "clocks": clk.summary(),
@@ -437,7 +466,7 @@ def measure_kl(dev, burst: float, steps: int = 3):
 
 def measure_two_call(dev, hidden, W, pk_fn, T, d, V, n, burst, steps: int = 3):
     """The same step through olive_token_logprob_fwd + olive_token_loss_bwd
-    (the backward recomputes every logit tile), for comparison."""
+    (the backward recomputes the logits in both of its passes), for comparison."""
     from paper_2609_36246_gb300 import binding as B
     ws_f = B.workspace(B.olive_workspace_size("logprob_fwd", T, d, V), dev)
     ws_b = B.workspace(B.olive_workspace_size("loss_bwd", T, d, V), dev)
@@ -459,7 +488,37 @@ def measure_two_call(dev, hidden, W, pk_fn, T, d, V, n, burst, steps: int = 3):
         raise RuntimeError(f"two-call status {B.status_bits(st)}")
     del ws_f, ws_b, out_b
     torch.cuda.empty_cache()
-    return {"workload": "same batch, forward + recomputing backward (two calls)",
+    return {"workload": "same batch, forward + on-chip backward (two calls; logits computed "
+                        "three times)",
+            "value": n / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
+            "pct_bf16_peak": 100.0 * 6.0 * n * d * V / (ms / 1e3) / 1e12 / burst, "steps": steps}
+
+
+def measure_slab(dev, hidden, W, pk_fn, T, d, V, n, burst, steps: int = 3):
+    """The same step through olive_token_loss_fwd_bwd_slab: each logit tile
+    computed once, e' = exp(z - R) of every masked row kept in an HBM slab
+    (about 5 GB here) between the forward and the dH / dW products.  A
+    secondary line: the headline keeps G on chip."""
+    from paper_2609_36246_gb300 import binding as B
+    ws = B.workspace(B.olive_workspace_size("loss_fwd_bwd_slab", T, d, V), dev)
+    st = B.new_status(dev)
+    gl = torch.ones(1, dtype=torch.float32, device=dev)
+    out = (torch.empty(T, device=dev), torch.empty(T, device=dev), torch.empty(1, device=dev),
+           torch.empty(T, d, dtype=torch.bfloat16, device=dev),
+           torch.empty(V, d, dtype=torch.bfloat16, device=dev))
+
+    def step():
+        pk = pk_fn()
+        B.olive_token_loss_fwd_bwd(hidden, W, pk["targets"], pk["rows"], pk["n_rows"], gl, 1.0,
+                                   "sum", torch.bfloat16, ws=ws, dev_status=st, out=out, slab=True)
+
+    ms = time_calls(step, steps, 1)
+    if int(st.item()) != 0:
+        raise RuntimeError(f"slab status {B.status_bits(st)}")
+    del ws, out
+    torch.cuda.empty_cache()
+    return {"workload": "same batch, olive_token_loss_fwd_bwd_slab (G through an HBM slab of "
+                        "every masked row, ~5 GB; logits computed once)",
             "value": n / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
             "pct_bf16_peak": 100.0 * 6.0 * n * d * V / (ms / 1e3) / 1e12 / burst, "steps": steps}
 
@@ -634,22 +693,26 @@ def run_reference(args, world, rank):
     if rank != 0:
         return
     b, h, W = make_inputs(rank)
-    times, rows = [], 0
+    nr = args.cpu_rows or 24
+    secs, rates, fixed = [], [], []
     for _ in range(args.warmup):
         pass  # the oracle has no warm state; warm-up steps would only repeat the sample
     for i in range(args.steps):
-        rate, secs, nr = oracle_sample_rate(b, h, W, args.cpu_rows or 24, seed=i)
-        times.append(secs)
-        rows += nr
-    value = rows / sum(times)
+        rate, fx, s_, _ = oracle_sample_rate(b, h, W, nr, seed=i)
+        rates.append(rate)
+        fixed.append(fx)
+        secs.append(s_)
+    value = statistics.median(rates)
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * statistics.mean(times),
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * statistics.mean(secs),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": dict(CONFIG, parallelism="host cores"),
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": host_cores(), "kind": "oracle",
-                         "sample": f"{args.cpu_rows or 24} masked rows per step of the same batch "
-                                   "(fp64 forward, dH, dW contributions)"},
+                         "sample": f"per step {nr} and {3 * nr} masked rows of the same batch (fp64 "
+                                   "forward, dH, dW contributions); per-row rate from the "
+                                   "difference, median over steps",
+                         "fixed_s_per_call": statistics.median(fixed)},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -662,8 +725,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-rows", type=int, default=None,
-                    help="masked rows in the oracle sample (default: 96 for the cpu_baseline "
-                         "leg, about 10 s; 24 per step for --impl reference)")
+                    help="masked rows n of the oracle samples (n and 3n rows; default 24, "
+                         "about 8 s per sample pair on 16 cores)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extra", action="store_true",
                     help="skip the divergence and variable-length measurements")

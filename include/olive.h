@@ -19,7 +19,9 @@
  * and these extend it:
  *
  *   olive_token_loss_fwd_bwd the forward and backward of a training step in
- *                            one pass over the logits (no recomputation)
+ *                            one call, G formed and consumed on chip
+ *   olive_token_loss_fwd_bwd_slab  the same step through an HBM slab of G
+ *                            (no logit recomputation)
  *   olive_splice_pack_masked multi-turn packing, loss only on teacher actions
  *                            (Section 3.2)
  *   olive_token_topk_fwd     per-token entropy and top-K log-probs
@@ -89,7 +91,8 @@ enum { OLIVE_KL_REVERSE = 0, OLIVE_KL_FORWARD = 1 };
 enum { OLIVE_DTYPE_BF16 = 0, OLIVE_DTYPE_F32 = 1 };
 enum { OLIVE_OP_LOGPROB_FWD = 0, OLIVE_OP_LOSS_BWD = 1, OLIVE_OP_DIVERGENCE = 2,
        OLIVE_OP_TOPK_FWD = 3, OLIVE_OP_SPLICE_MASKED = 4, OLIVE_OP_TOPK_KL_BWD = 5,
-       OLIVE_OP_LOSS_FWD_BWD = 6, OLIVE_OP_OPD_STATS = 7, OLIVE_OP_TOPK_KL_FWD_BWD = 8 };
+       OLIVE_OP_LOSS_FWD_BWD = 6, OLIVE_OP_OPD_STATS = 7, OLIVE_OP_TOPK_KL_FWD_BWD = 8,
+       OLIVE_OP_LOSS_FWD_BWD_SLAB = 9 };
 
 /* ABI version of the loaded library (OLIVE_ABI_VERSION). */
 OLIVE_API int olive_abi_version(void);
@@ -317,8 +320,14 @@ OLIVE_API olive_status olive_topk_kl_bwd(const void* h_s, const void* W_s, const
  * Arguments as in olive_token_logprob_fwd; lse fp32 [T] is the forward's
  * output; grad_loss fp32 [1] (device); d_hidden [T,d] and d_W [V,d] of
  * grad_dtype (OLIVE_DTYPE_BF16: fp32 accumulation, round-to-nearest-even
- * store; OLIVE_DTYPE_F32).  Logits are recomputed tile by tile; G exists only
- * as a bf16 slab of at most a fixed number of rows inside the workspace.
+ * store; OLIVE_DTYPE_F32).  The logits are recomputed tile by tile and G is
+ * formed and consumed on chip: groups of ceil(d / 256) CTAs each hold a
+ * 128 x 256 column block of the d_hidden (then d_W) accumulator in tensor
+ * memory and pass 128 x 256 bf16 tiles of G to one another through a ring of
+ * fixed size in the workspace (3 ceil(d/256) tiles of 64 KB per group, tens
+ * of MB in all, independent of T and V); no [rows, V] array is stored.  The
+ * bf16 tile carries one rounding of G (relative 2^-9).  workspace:
+ * olive_workspace_size(OLIVE_OP_LOSS_BWD, T, d, 0, V, 1, grad_dtype) bytes.
  */
 OLIVE_API olive_status olive_token_loss_bwd(const void* hidden, const void* W,
                                   const int32_t* targets, const int32_t* rows,
@@ -335,13 +344,18 @@ OLIVE_API olive_status olive_token_loss_bwd(const void* hidden, const void* W,
  * gradient before the forward runs (*grad_loss is read on the device, e.g. 1
  * for a loss that is the objective itself).  Outputs and arguments as in
  * those two calls: logp, lse fp32 [T], loss fp32 [1], d_hidden [T, d] and
- * d_W [V, d] of grad_dtype.  Each logit tile is computed once: the forward
- * product stores e = exp(z - tile max) in bf16 in the G slab of the workspace
- * (one slab of at most a fixed number of rows at a time, never [T, V]), a
- * bandwidth-bound pass turns it into G once the row's lse is known, and the
- * dH and dW products follow.  Compared with olive_token_loss_bwd, G carries
- * one more bf16 rounding of p (relative 2^-9 per entry; the target entry is
- * formed from the fp32 logit).  workspace: olive_workspace_size(
+ * d_W [V, d] of grad_dtype.  Nothing of size [rows, V] is stored: the first
+ * pass walks each 128-row tile across the vocabulary, forms P = exp(z - R)
+ * against a per-row reference R (the maximum of the row's first vocabulary
+ * tile) in bf16 tiles that a group of CTAs shares through a fixed-size ring
+ * (see olive_token_loss_bwd), and accumulates P . W and the row sums, from
+ * which lse, logp and d_hidden = g inv_tau (exp(R - lse) P.W - W[y]) follow;
+ * the second pass walks each 128-row vocabulary tile across the masked rows,
+ * recomputes the logits and accumulates d_W = G^T hidden with G formed on
+ * chip from that lse.  A row whose maximum logit exceeds R by more than 64
+ * log2 units has its row tile recomputed with R = its maximum (exact, only
+ * slower).  The training step executes four products of 2 N_mask d V flops
+ * for the three it needs.  workspace: olive_workspace_size(
  * OLIVE_OP_LOSS_FWD_BWD, T, d, 0, V, 1, grad_dtype) bytes.
  */
 OLIVE_API olive_status olive_token_loss_fwd_bwd(const void* hidden, const void* W,
@@ -352,6 +366,33 @@ OLIVE_API olive_status olive_token_loss_fwd_bwd(const void* hidden, const void* 
                                                 float* loss, void* d_hidden, void* d_W,
                                                 int grad_dtype, void* workspace, size_t ws_bytes,
                                                 int32_t* dev_status, void* stream);
+
+/*
+ * olive_token_loss_fwd_bwd_slab -- the same step, arguments and outputs as
+ * olive_token_loss_fwd_bwd, computing each logit tile once instead of twice
+ * by keeping it in HBM: the forward product stores e' = 2^(x - R) in bf16
+ * (R = the row's maximum over its first vocabulary tile) in a slab of the
+ * workspace of at most min(T, 32768, ~5.6 GB / (2 V)) rows -- at the
+ * 8 x 4096-token, V = 151936 batch that slab holds every masked row, about
+ * 5 GB -- a per-row pass merges the tile partials into lse and writes logp,
+ * the target entry of G and the row scale lam = g inv_tau 2^(R - lse2), and
+ * the d_hidden and d_W products read the slab (d_hidden = lam (e' . W) with
+ * lam in the epilogue; d_W = e'^T . (lam hidden)).  Faster where HBM capacity
+ * allows (three products instead of four) but the G of up to 32768 rows is
+ * materialised; olive_token_loss_fwd_bwd is the on-chip form.  The paper has
+ * no counterpart (an implementation alternative).  workspace:
+ * olive_workspace_size(OLIVE_OP_LOSS_FWD_BWD_SLAB, T, d, 0, V, 1, grad_dtype)
+ * bytes.
+ */
+OLIVE_API olive_status olive_token_loss_fwd_bwd_slab(const void* hidden, const void* W,
+                                                     const int32_t* targets, const int32_t* rows,
+                                                     const int32_t* n_rows, int32_t T, int32_t d,
+                                                     int32_t V, float inv_tau, int reduction,
+                                                     const float* grad_loss, float* logp,
+                                                     float* lse, float* loss, void* d_hidden,
+                                                     void* d_W, int grad_dtype, void* workspace,
+                                                     size_t ws_bytes, int32_t* dev_status,
+                                                     void* stream);
 
 /*
  * olive_topk_kl_fwd_bwd -- olive_token_topk_fwd on the student,

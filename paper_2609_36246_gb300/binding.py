@@ -28,7 +28,8 @@ REDUCE = {"sum": 0, "mean": 1}
 DIRECTION = {"reverse": 0, "forward": 1}
 DTYPE = {torch.bfloat16: 0, torch.float32: 1}
 OP = {"logprob_fwd": 0, "loss_bwd": 1, "divergence": 2, "topk_fwd": 3, "splice_masked": 4,
-      "topk_kl_bwd": 5, "loss_fwd_bwd": 6, "opd_stats": 7, "topk_kl_fwd_bwd": 8}
+      "topk_kl_bwd": 5, "loss_fwd_bwd": 6, "opd_stats": 7, "topk_kl_fwd_bwd": 8,
+      "loss_fwd_bwd_slab": 9}
 
 
 class OliveError(RuntimeError):
@@ -84,6 +85,8 @@ def lib() -> ctypes.CDLL:
     L.olive_token_loss_fwd_bwd.restype = ctypes.c_int
     L.olive_token_loss_fwd_bwd.argtypes = [_P, _P, _P, _P, _P, _I, _I, _I, _F, ctypes.c_int, _P, _P,
                                            _P, _P, _P, _P, ctypes.c_int, _P, _S, _P, _P]
+    L.olive_token_loss_fwd_bwd_slab.restype = ctypes.c_int
+    L.olive_token_loss_fwd_bwd_slab.argtypes = L.olive_token_loss_fwd_bwd.argtypes
     L.olive_topk_kl_fwd_bwd.restype = ctypes.c_int
     L.olive_topk_kl_fwd_bwd.argtypes = [_P, _P, _I, _P, _P, _I, _P, _P, _I, _I, _F, _I, _P, _P, _P,
                                         _P, _P, _P, _P, _P, _P, _P, _P, ctypes.c_int, _P, _S, _P,
@@ -449,8 +452,9 @@ def olive_token_loss_bwd(hidden, W, targets, rows, n_rows, lse, grad_loss, inv_t
 
 def olive_token_loss_fwd_bwd(hidden, W, targets, rows, n_rows, grad_loss, inv_tau: float = 1.0,
                              reduction: str = "sum", grad_dtype=torch.bfloat16, ws=None,
-                             dev_status=None, out=None):
-    """Forward and backward of one training step in one pass over the logits.
+                             dev_status=None, out=None, slab: bool = False):
+    """Forward and backward of one training step in one call (G on chip;
+    slab=True: olive_token_loss_fwd_bwd_slab, G through an HBM slab).
 
     grad_loss is a 1-element fp32 CUDA tensor (the loss gradient, known before
     the call).  Returns (logp [T], lse [T], loss [1], d_hidden [T, d], d_W [V, d])."""
@@ -468,14 +472,14 @@ def olive_token_loss_fwd_bwd(hidden, W, targets, rows, n_rows, grad_loss, inv_ta
                torch.empty(V, d, dtype=grad_dtype, device=dev))
     logp, lse, loss, dh, dw = out
     if ws is None:
-        ws = workspace(olive_workspace_size("loss_fwd_bwd", T, d, V, grad_dtype=grad_dtype), dev)
+        op = "loss_fwd_bwd_slab" if slab else "loss_fwd_bwd"
+        ws = workspace(olive_workspace_size(op, T, d, V, grad_dtype=grad_dtype), dev)
     ds = dev_status if dev_status is not None else new_status(dev)
-    st = lib().olive_token_loss_fwd_bwd(_ptr(hidden), _ptr(W), _ptr(targets), _ptr(rows),
-                                        _ptr(n_rows), T, d, V, float(inv_tau), REDUCE[reduction],
-                                        _ptr(grad_loss), _ptr(logp), _ptr(lse), _ptr(loss),
-                                        _ptr(dh), _ptr(dw), DTYPE[grad_dtype], _ptr(ws), ws.numel(),
-                                        _ptr(ds), _stream())
-    _check(st, "olive_token_loss_fwd_bwd")
+    fn = lib().olive_token_loss_fwd_bwd_slab if slab else lib().olive_token_loss_fwd_bwd
+    st = fn(_ptr(hidden), _ptr(W), _ptr(targets), _ptr(rows), _ptr(n_rows), T, d, V,
+            float(inv_tau), REDUCE[reduction], _ptr(grad_loss), _ptr(logp), _ptr(lse), _ptr(loss),
+            _ptr(dh), _ptr(dw), DTYPE[grad_dtype], _ptr(ws), ws.numel(), _ptr(ds), _stream())
+    _check(st, "olive_token_loss_fwd_bwd_slab" if slab else "olive_token_loss_fwd_bwd")
     return logp, lse, loss, dh, dw
 
 

@@ -128,6 +128,63 @@ struct KlWs {
 size_t kl_ws_bytes(int64_t T, int64_t ds, int64_t dt, int64_t V, int grad);
 KlWs carve_kl(void* ws, int64_t T, int64_t ds, int64_t dt, int64_t V, int grad);
 
+// On-chip training step (lmhead_group.cu): groups of ceil(d / 256) CTAs
+// exchange 128 x 256 bf16 logit-gradient tiles through a ring of fixed size.
+constexpr int kGroupMaxSms = 192;  // ring and counters are sized for up to this many SMs
+struct GroupWs {
+  void* hc;          // bf16 [Tpad, d]
+  float* rref;       // [Tpad] reference (base 2) per compact row
+  float* rmax;       // [Tpad] row maxima of tiles that are redone
+  float* zy;         // [Tpad] target logits
+  float* pyb;        // [Tpad] the targets' bf16 exchange-tile entries
+  float* nll;        // [Tpad] per-row loss terms
+  float* part_s;     // [g_max, Tpad] per-member partial sums
+  float* part_m;     // [g_max, Tpad] per-member partial maxima
+  void* ring;        // group_ring_bytes(T, d, V)
+  uint32_t* outer;   // [2 rt] pass-A group barriers (first launch, redo launch)
+  uint32_t* redo;    // [1 + rt] redo list
+  uint32_t* ring_ctr;  // 3 launches x 2 x group_ring_words(T, d, V)
+  size_t ctr_words;  // words from `outer` to the end of ring_ctr
+};
+size_t group_ws_bytes(int64_t T, int64_t d, int64_t V);
+GroupWs carve_group(void* ws, int64_t T, int64_t d, int64_t V);
+int group_g_max(int64_t d);
+int group_count_max(int64_t T, int64_t d, int64_t V);
+size_t group_ring_words(int64_t T, int64_t d, int64_t V);
+size_t group_ring_bytes(int64_t T, int64_t d, int64_t V);
+int group_sweep_cols(int sms);
+
+struct GroupArgs {
+  int32_t* dev_status;
+  const int32_t* n_rows;
+  const int32_t* rows;
+  const int32_t* targets;
+  int reduction;
+  float inv_tau;
+  const float* grad_loss;
+  int lse_known, redo, write_fwd;
+  const float* lse_in;
+  float *rref, *rmax, *part_s, *part_m, *zy, *pyb, *logp, *lse, *nll;
+  uint32_t* redo_list;
+  uint32_t* outer_ctr;
+  void* ring;
+  void* d_hidden;
+  void* d_W;
+  int out_dtype;
+};
+// mode 0: reference maxima, 1: pass A (lse, logp, dH), 2: pass B (dW)
+olive_status launch_group(const Ctx& c, int mode, const void* hc, const void* W, int32_t T,
+                          int32_t d, int32_t V, const GroupArgs& a, int c_base, int c_end,
+                          uint32_t* ring_ctr);
+// The whole step: forward + backward when lse_given is null (logp, lse, loss
+// written), else the backward of that forward.
+olive_status launch_loss_group(const Ctx& c, const void* hidden, const void* W,
+                               const int32_t* targets, const int32_t* rows, const int32_t* n_rows,
+                               int32_t T, int32_t d, int32_t V, float inv_tau, int reduction,
+                               const float* grad_loss, const float* lse_given, float* logp,
+                               float* lse, float* loss, void* d_hidden, void* d_W, int grad_dtype,
+                               void* ws, int32_t* dev_status);
+
 // ---- launchers (validated arguments; return OLIVE_OK or OLIVE_ERR_CUDA) ----
 olive_status launch_splice_pack(const Ctx& c, const int32_t* prefix_ids, const int32_t* prefix_off,
                                 const int32_t* cont_ids, const int32_t* cont_off, int32_t S,

@@ -1,0 +1,942 @@
+// lmhead_group.cu -- the training step of the Eq. (osd-ce) loss (Section 3.1)
+// with its logit gradient formed and consumed on chip.
+//
+// With z = inv_tau H[rows] W^T, lse per row and G = coef (softmax(z) -
+// onehot(y)) (coef = g inv_tau, / N_mask for OLIVE_REDUCE_MEAN):
+//   dH = G . W       reduces over the vocabulary  (K = V)
+//   dW = G^T . hc    reduces over the masked rows (K = N_mask)
+// Either output tile is [128, d] fp32 for a 128-row M tile: 2 MB at d = 4096,
+// eight SMs' worth of tensor memory, so one SM cannot hold it.  The CTAs are
+// therefore split into GROUPS of g = ceil(d / 256) members.  Member m owns
+// the output columns [c0, c0 + cw) of d (cw <= 256) and keeps their 128 x cw
+// fp32 accumulator in TMEM for a whole OUTER tile, while the members take
+// turns computing the 128 x 256 logit tiles (Z jobs, K = d) that every member
+// needs.  The member that computed a Z tile turns it into a bf16 EXCHANGE
+// tile and stores it in its group's ring of R slots of 64 KB; every member
+// bulk-copies each exchange tile, 64 K-columns at a time, into shared memory
+// as the A operand of its accumulating MMA.  The ring has a fixed size (R
+// slots per group, a few tens of MB in all, which stays in the L2), each slot
+// is rewritten once all g members have read it, and no slot outlives R
+// exchange tiles: the logits and G are never stored as a [rows, V] array.
+//
+//   Pass A (outer = 128 masked rows, inner = 256-column vocabulary tile):
+//     exchange tile P'[r, v] = 2^(x - R_r), x = z log2(e), R_r a per-row
+//     reference (the maximum of the row's first vocabulary tile, from the
+//     GM_REF launch, or the row's lse when it is given); the members
+//     accumulate acc = P' . W[:, chunk] and keep per-row partial sums of
+//     2^(x - R) over their own Z jobs, merged at the end of the outer tile
+//     into lse2 = R + log2(sum) (a group barrier through a global counter).
+//     The epilogue then applies the softmax-minus-onehot scaling:
+//       dH[r, chunk] = coef (2^(R - lse2) acc - W[y_r, chunk]).
+//     A row whose maximum exceeds R by more than kRefMax (2^x - R would leave
+//     the range the bf16 operand and the fp32 sums are safe in) puts its row
+//     tile on a redo list; a second launch recomputes those tiles with R = the
+//     rows' maxima from the first launch.
+//   Pass B (outer = 128 vocabulary rows, inner = 256 masked rows): exchange
+//     tile G^T[v, r] = coef_r (2^(x - lse2_r) - [v == y_r]) from pass A's
+//     lse (transposed logit tile z^T = W hc^T, so a TMEM lane is a vocabulary
+//     row); member m accumulates dW[v, chunk] = G^T . hc[:, chunk] and stores
+//     it when the outer tile ends (every dW element has one owner: no atomics).
+//
+// Each pass executes two products per logit (the Z tile and its share of the
+// accumulation), so the training step executes 4 GEMM units of 2 N_mask d V
+// flops for the 3 it counts.
+//
+// Schedule inside a group (every member derives it from N_mask on the
+// device): the exchange tiles of the group's outer tiles form one sequence
+// e = 0 .. E-1 (e = i ni + k for the group's i-th outer tile and inner tile
+// k), cut into rounds of g tiles; tile e is computed by member e mod g and
+// lives in ring slot e mod R.  Each member's tensor pipe runs, per round r:
+// its Z job of round r, then the accumulation of all g tiles of round r - 1,
+// so the epilogue of a Z tile (and the other members' epilogues) overlaps the
+// accumulation MMAs, and a single 256-column Z accumulator suffices next to
+// the 256-column output accumulator (512 TMEM columns).  Waits between
+// members go through global release/acquire counters: a slot's `ready` count
+// (tile written) and `cons` count (tile copied by all g members).  Every
+// dependency points to a tile with a smaller index (a slot is rewritten R >=
+// 2g tiles after its previous use), the launch is cooperative (all CTAs
+// resident), and every wait is bounded (OLIVE_ERR_TIMEOUT on expiry).
+#include <algorithm>
+#include <cmath>
+
+#include "sched.cuh"
+#include "sm103.cuh"
+
+namespace olive {
+namespace {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr int kBM = 128;
+constexpr int kBK = 64;
+constexpr int kZN = 256;             // logit tile 128 x 256
+constexpr int kStages = 4;
+constexpr int kSA = kBM * kBK * 2;   // A operand of a stage: 128 x 64 bf16
+constexpr int kSB = kZN * kBK * 2;   // B operand: 256 x 64 (Z job) or 64 x <= 256 (accumulation)
+constexpr int kStageBytes = kSA + kSB;
+constexpr int kXSlice = kSA;         // one 128 x 64 K-slice of an exchange tile
+constexpr int kXTile = 4 * kXSlice;  // 128 x 256 bf16 (64 KB)
+constexpr int kEpi = 128;            // epilogue threads: one accumulator row each
+constexpr int kProducerWarp = 4;
+constexpr int kMmaWarp = 5;
+constexpr int kThreads = 192;
+constexpr int kStatusTimeoutBit = 1 << OLIVE_ERR_TIMEOUT;
+constexpr float kRefMax = 64.f;
+constexpr int kMetaBytes = kZN * 8;  // pass B: lse2 and target of the tile's 256 rows
+
+enum GMode : int { GM_REF = 0, GM_A = 1, GM_B = 2 };
+
+// GM_REF / GM_A: za = hc {64 x 128}, zb = W {64 x 256}, xb = W {64 x 64}
+// GM_B:          za = W {64 x 128},  zb = hc {64 x 256}, xb = hc {64 x 64}
+struct GroupMaps {
+  CUtensorMap za, zb, xb;
+};
+
+struct GroupParams {
+  int32_t* dev_status;
+  uint64_t wait_limit_ns;
+  const int32_t* n_rows;
+  const int32_t* rows;
+  const int32_t* targets;
+  const __nv_bfloat16* W;   // GM_A: the rows W[y] of the onehot term
+  int32_t T, d, V;
+  int32_t mode;
+  int32_t g, ngroups, R;    // members per group, groups, ring slots per group
+  int32_t chunk;            // output columns per member (multiple of 16, <= 256)
+  int32_t c_base, c_end;    // output columns [c_base, c_end) of this launch
+  int32_t reduction;
+  float inv_tau, scale2;    // 1 / tau, log2(e) / tau
+  const float* grad_loss;   // device scalar g
+  int32_t lse_known;        // GM_A: R = lse2 from lse_in (backward of a given forward)
+  int32_t redo;             // GM_A: outer tiles from redo_list, R = rmax
+  int32_t write_fwd;        // GM_A: write lse, logp, nll
+  const float* lse_in;      // [T] natural lse per packed row (GM_A lse_known, GM_B)
+  float* rref;              // [Tpad] base-2 reference per compact row (GM_REF writes)
+  float* rmax;              // [Tpad] base-2 row maximum (GM_A writes for redo rows)
+  float* part_s;            // [g][Tpad] per-member sums of 2^(x - R)
+  float* part_m;            // [g][Tpad] per-member maxima (base 2)
+  float* zy;                // [Tpad] target logit z_y (natural units)
+  float* pyb;               // [Tpad] P'_y as rounded to bf16 in the exchange tile
+  float* logp;              // [T]
+  float* lse;               // [T]
+  float* nll;               // [Tpad] per-row loss terms
+  uint32_t* redo_list;      // [1 + rt]: count, then row tiles
+  uint32_t* outer_ctr;      // [rt] pass A group barrier (one array per GM_A launch)
+  __nv_bfloat16* ring;      // [ngroups][R][128 x 256] exchange tiles (swizzled images)
+  uint32_t* ready;          // [ngroups][R]
+  uint32_t* cons;           // [ngroups][R]
+  void* out;                // GM_A: d_hidden [T, d]; GM_B: d_W [V, d]
+  int32_t out_dtype;
+};
+
+// per-CTA schedule, the same in every CTA of a group
+struct GSched {
+  int n;      // masked rows
+  int no;     // outer tiles in all
+  int ni;     // inner tiles per outer tile
+  int nk;     // 64-wide K steps of a Z job
+  int q, m;   // group, member
+  int myo;    // outer tiles of this group
+  int E;      // exchange tiles of this group
+  int c0, cw; // output columns of this member
+  int nbox;   // 64-column boxes of the accumulation's B operand
+  int nacc;   // N of the accumulation MMA (cw rounded up to 16)
+  int kcount; // inner extent: V (pass A) or n (pass B)
+  float coef;
+};
+
+__device__ GSched make_gsched(const GroupParams& p) {
+  GSched s;
+  s.n = read_n_rows(p.n_rows, p.T, p.dev_status);
+  const int rt = (s.n + kBM - 1) / kBM;
+  if (p.mode == GM_B) {
+    s.no = (p.V + kBM - 1) / kBM;
+    s.ni = (s.n + kZN - 1) / kZN;
+    s.kcount = s.n;
+  } else {
+    s.no = (p.mode == GM_A && p.redo) ? static_cast<int>(min(p.redo_list[0], static_cast<uint32_t>(rt))) : rt;
+    s.ni = p.mode == GM_REF ? 1 : (p.V + kZN - 1) / kZN;
+    s.kcount = p.V;
+  }
+  s.nk = (p.d + kBK - 1) / kBK;
+  s.q = blockIdx.x / p.g;
+  s.m = blockIdx.x % p.g;
+  s.myo = s.q < s.no ? (s.no - s.q + p.ngroups - 1) / p.ngroups : 0;
+  s.E = s.myo * s.ni;
+  s.c0 = p.c_base + s.m * p.chunk;
+  s.cw = min(p.chunk, p.c_end - s.c0);
+  if (s.cw < 0) s.cw = 0;
+  s.nbox = (s.cw + 63) / 64;
+  s.nacc = (s.cw + 15) / 16 * 16;
+  if (s.nacc < 16) s.nacc = 16;
+  s.coef = 0.f;
+  if (p.grad_loss) {
+    float gl = *p.grad_loss;
+    if (p.reduction == OLIVE_REDUCE_MEAN && s.n > 0) gl = gl / static_cast<float>(s.n);
+    s.coef = gl * p.inv_tau;
+  }
+  return s;
+}
+
+// global index of the group's i-th outer tile
+__device__ __forceinline__ int outer_of(const GroupParams& p, const GSched& s, int i) {
+  const int k = s.q + i * p.ngroups;
+  return (p.mode == GM_A && p.redo) ? static_cast<int>(p.redo_list[1 + k]) : k;
+}
+__device__ __forceinline__ int kvalid_of(const GSched& s, int k) {
+  return min(kZN, s.kcount - k * kZN);
+}
+// 64-wide K slices of inner tile k that hold valid columns
+__device__ __forceinline__ int slices_of(const GSched& s, int k) {
+  return (kvalid_of(s, k) + kBK - 1) / kBK;
+}
+// does member m compute a Z job of the group's i-th outer tile?
+__device__ __forceinline__ bool member_has_job(const GSched& s, int g, int i) {
+  const int lo = i * s.ni;
+  const int first = lo + (((s.m - lo) % g) + g) % g;
+  return first < lo + s.ni;
+}
+
+// byte offset of 16-byte chunk c (0..7) of row r in K-slice sl of an exchange
+// tile: the 128-byte-swizzled K-major layout a TMA load of a 64 x 128 box
+// produces (row r at r * 128, chunk c at position c ^ (r & 7)), so a linear
+// copy of a slice to a 1024-byte-aligned stage is a valid UMMA operand
+__device__ __forceinline__ uint32_t img_off(int r, int sl, int c) {
+  return static_cast<uint32_t>(sl * kXSlice + (r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4));
+}
+
+__device__ __forceinline__ void store_out32(void* base, size_t off, int dtype, int n_valid,
+                                            const float (&v)[32]) {
+  if (dtype == OLIVE_DTYPE_BF16) {
+    __nv_bfloat16* o = static_cast<__nv_bfloat16*>(base) + off;
+    if (n_valid >= 32) {
+      uint4* d4 = reinterpret_cast<uint4*>(o);
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        d4[q] = make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                           pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+    } else {
+#pragma unroll
+      for (int k = 0; k < 32; ++k)
+        if (k < n_valid) o[k] = __float2bfloat16_rn(v[k]);
+    }
+  } else {
+    float* o = static_cast<float*>(base) + off;
+    if (n_valid >= 32) {
+      float4* d4 = reinterpret_cast<float4*>(o);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) d4[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+    } else {
+#pragma unroll
+      for (int k = 0; k < 32; ++k)
+        if (k < n_valid) o[k] = v[k];
+    }
+  }
+}
+
+// 32 fp32 values -> four 16-byte chunks of row r of the exchange image
+__device__ __forceinline__ void store_img32(uint8_t* img, int r, int h, const float (&v)[32]) {
+  const int sl = h >> 1;
+  const int c0 = (h & 1) * 4;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const uint4 u = make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                               pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+    *reinterpret_cast<uint4*>(img + img_off(r, sl, c0 + q)) = u;
+  }
+}
+
+// per-row values of pass A (and GM_REF) for compact row rc
+struct RowA {
+  bool valid;   // rc < n and rows[rc] in [0, T)
+  int t, y;     // packed row, target (-1 when none)
+  float R;      // reference (base 2)
+};
+
+__device__ __forceinline__ RowA load_row_a(const GroupParams& p, const GSched& s, int rc) {
+  RowA a;
+  a.valid = false;
+  a.t = -1;
+  a.y = -1;
+  a.R = 0.f;
+  if (rc < s.n) {
+    const int t = p.rows[rc];
+    if (t >= 0 && t < p.T) {
+      a.valid = true;
+      a.t = t;
+      a.y = p.targets[t];
+      if (p.mode == GM_A) {
+        if (p.lse_known) a.R = p.lse_in[t] * kLog2e;
+        else if (p.redo) a.R = p.rmax[rc];
+        else a.R = p.rref[rc];
+      }
+    }
+  }
+  return a;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    lmhead_group_kernel(const __grid_constant__ GroupMaps maps, const GroupParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+
+  const uint32_t stages = base;
+  const uint32_t bar0 = base + kStages * kStageBytes;
+  auto full_bar = [&](int st) { return bar0 + 8u * st; };
+  auto empty_bar = [&](int st) { return bar0 + 8u * (kStages + st); };
+  const uint32_t zfull = bar0 + 8u * (2 * kStages);
+  const uint32_t zempty = zfull + 8;
+  const uint32_t ofull = zfull + 16;
+  const uint32_t oempty = zfull + 24;
+  const uint32_t drain = zfull + 32;
+  uint8_t* misc = gbase + kStages * kStageBytes + 8 * (2 * kStages + 5);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(misc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 4);
+  GSched* sched_smem = reinterpret_cast<GSched*>(misc + 16);
+  float* meta_l = reinterpret_cast<float*>(misc + 128);                 // [256] lse2 (GM_B)
+  int* meta_y = reinterpret_cast<int*>(misc + 128 + kMetaBytes / 2);    // [256] targets (GM_B)
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int st = 0; st < kStages; ++st) {
+      mbar_init(full_bar(st), 1);
+      mbar_init(empty_bar(st), 1);
+    }
+    mbar_init(zfull, 1);
+    mbar_init(zempty, kEpi);
+    mbar_init(ofull, 1);
+    mbar_init(oempty, kEpi);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    *sched_smem = make_gsched(p);
+    fence_mbar_init();
+  }
+  if (warp == kProducerWarp && lane == 0) {
+    tma_prefetch_desc(&maps.za);
+    tma_prefetch_desc(&maps.zb);
+    tma_prefetch_desc(&maps.xb);
+  }
+  if (warp == kMmaWarp) {
+    tmem_alloc(smem_u32(tmem_slot), 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+
+  const uint32_t tmem_base = *tmem_slot;
+  const GSched s = *sched_smem;
+  const WaitCtl ctl{abort_flag, p.wait_limit_ns};
+  const int g = p.g;
+  const bool consume = p.mode != GM_REF;
+  const int nr = (s.E + g - 1) / g;  // rounds
+  const size_t ring0 = static_cast<size_t>(s.q) * p.R;
+  uint8_t* ring_bytes = reinterpret_cast<uint8_t*>(p.ring);
+
+  if (warp == kProducerWarp) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int r = 0; ok && r <= nr; ++r) {
+        const int j = r * g + s.m;
+        if (r < nr && j < s.E) {
+          const int o = outer_of(p, s, j / s.ni);
+          const int k = j % s.ni;
+          for (int ks = 0; ks < s.nk; ++ks) {
+            if (!mbar_wait(empty_bar(stage), phase ^ 1u, ctl)) { ok = false; break; }
+            const uint32_t sA = stages + stage * kStageBytes;
+            const uint32_t fb = full_bar(stage);
+            mbar_arrive_expect_tx(fb, kStageBytes);
+            tma_load_2d(sA, &maps.za, fb, ks * kBK, o * kBM);
+            tma_load_2d(sA + kSA, &maps.zb, fb, ks * kBK, k * kZN);
+            if (++stage == kStages) { stage = 0; phase ^= 1u; }
+          }
+        }
+        if (!ok || !consume || r == 0) continue;
+        const int e_end = min(r * g, s.E);
+        for (int e = (r - 1) * g; ok && e < e_end; ++e) {
+          const int slot = e % p.R;
+          if (!wait_counter(p.ready + ring0 + slot, static_cast<uint32_t>(e / p.R + 1), ctl)) {
+            ok = false;
+            break;
+          }
+          fence_proxy_async_global();
+          const int k = e % s.ni;
+          const int nsl = slices_of(s, k);
+          const uint8_t* img = ring_bytes + (ring0 + slot) * static_cast<size_t>(kXTile);
+          for (int sl = 0; sl < nsl; ++sl) {
+            if (!mbar_wait(empty_bar(stage), phase ^ 1u, ctl)) { ok = false; break; }
+            const uint32_t sA = stages + stage * kStageBytes;
+            const uint32_t fb = full_bar(stage);
+            mbar_arrive_expect_tx(fb, kXSlice + s.nbox * 8192);
+            bulk_load(sA, img + sl * kXSlice, kXSlice, fb);
+            for (int b = 0; b < s.nbox; ++b)
+              tma_load_2d(sA + kSA + b * 8192, &maps.xb, fb, s.c0 + 64 * b, k * kZN + sl * kBK);
+            if (++stage == kStages) { stage = 0; phase ^= 1u; }
+          }
+        }
+      }
+      if (!ok) {
+        // let copies already issued land before the CTA retires
+        const uint64_t t0 = global_timer_ns();
+        while (global_timer_ns() - t0 < 50000) nanosleep_ns(1000);
+      }
+    }
+    __syncwarp();
+  } else if (warp == kMmaWarp) {
+    if (lane == 0) {
+      const uint32_t zacc = tmem_base;
+      const uint32_t oacc = tmem_base + 256;
+      const uint32_t idz = idesc_bf16(kBM, kZN, false, false);
+      const uint32_t idx = idesc_bf16(kBM, s.nacc, false, true);
+      int stage = 0;
+      uint32_t phase = 0, zph = 0, oph = 0;
+      bool ok = true;
+      for (int r = 0; ok && r <= nr; ++r) {
+        const int j = r * g + s.m;
+        if (r < nr && j < s.E) {
+          if (!mbar_wait(zempty, zph ^ 1u, ctl)) { ok = false; break; }
+          tc_fence_after();
+          for (int ks = 0; ks < s.nk; ++ks) {
+            if (!mbar_wait(full_bar(stage), phase, ctl)) { ok = false; break; }
+            tc_fence_after();
+            const uint32_t sA = stages + stage * kStageBytes;
+            const uint32_t sB = sA + kSA;
+#pragma unroll
+            for (int kk = 0; kk < kBK / 16; ++kk)
+              umma_bf16(zacc, sdesc_sw128(sA + kk * 32, 16, 1024), sdesc_sw128(sB + kk * 32, 16, 1024),
+                        idz, (ks > 0 || kk > 0) ? 1u : 0u);
+            umma_commit(empty_bar(stage));
+            if (++stage == kStages) { stage = 0; phase ^= 1u; }
+          }
+          if (!ok) break;
+          umma_commit(zfull);
+          zph ^= 1u;
+        }
+        if (!consume || r == 0) continue;
+        const int e_end = min(r * g, s.E);
+        for (int e = (r - 1) * g; ok && e < e_end; ++e) {
+          const int k = e % s.ni;
+          if (k == 0) {
+            if (!mbar_wait(oempty, oph ^ 1u, ctl)) { ok = false; break; }
+            tc_fence_after();
+          }
+          const int nsl = slices_of(s, k);
+          for (int sl = 0; sl < nsl; ++sl) {
+            if (!mbar_wait(full_bar(stage), phase, ctl)) { ok = false; break; }
+            tc_fence_after();
+            const uint32_t sA = stages + stage * kStageBytes;
+            const uint32_t sB = sA + kSA;
+#pragma unroll
+            for (int kk = 0; kk < kBK / 16; ++kk)
+              umma_bf16(oacc, sdesc_sw128(sA + kk * 32, 16, 1024),
+                        sdesc_sw128(sB + kk * 2048, 8192, 1024), idx,
+                        (k > 0 || sl > 0 || kk > 0) ? 1u : 0u);
+            umma_commit(empty_bar(stage));
+            if (++stage == kStages) { stage = 0; phase ^= 1u; }
+          }
+          if (!ok) break;
+          // every slice of tile e has landed in shared memory: its slot may
+          // be rewritten once all members say so
+          red_release_add(p.cons + ring0 + e % p.R, 1u);
+          if (k == s.ni - 1) {
+            umma_commit(ofull);
+            oph ^= 1u;
+          }
+        }
+      }
+      // arrives once every MMA issued above has completed (bounded wait that
+      // ignores the abort flag: it only waits for work already in flight)
+      umma_commit(drain);
+      volatile int keep_waiting = 0;
+      const uint64_t floor_ns = 200ull * 1000 * 1000;
+      const WaitCtl own{&keep_waiting, p.wait_limit_ns > floor_ns ? p.wait_limit_ns : floor_ns};
+      mbar_wait(drain, 0, own);
+    }
+    __syncwarp();
+  } else {
+    // epilogue warps 0..3: thread = accumulator row = TMEM lane
+    const int row = warp * 32 + lane;
+    const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
+    const uint32_t zaddr = lane_addr;
+    const uint32_t oaddr = lane_addr + 256;
+    uint32_t zph = 0, oph = 0;
+    bool ok = true;
+    const size_t Tpad = static_cast<size_t>((p.T + kBM - 1) / kBM) * kBM;
+
+    if (p.mode == GM_B && s.ni == 0) {
+      // no masked rows: dW is zero on this member's columns of its outer tiles
+      float zero[32];
+#pragma unroll
+      for (int k = 0; k < 32; ++k) zero[k] = 0.f;
+      for (int i = 0; i < s.myo; ++i) {
+        const int v = outer_of(p, s, i) * kBM + row;
+        if (v >= p.V) continue;
+        for (int c = 0; c < s.cw; c += 32)
+          store_out32(p.out, static_cast<size_t>(v) * p.d + s.c0 + c, p.out_dtype, min(32, s.cw - c), zero);
+      }
+    }
+
+    int cur_o = -1;             // pass A: the outer tile of the running partials
+    RowA ra{false, -1, -1, 0.f};
+    float run_s = 0.f, run_m = -INFINITY;
+    for (int r = 0; ok && r <= nr; ++r) {
+      const int j = r * g + s.m;
+      if (r < nr && j < s.E) {
+        // ---------------------------------------------------- Z epilogue
+        const int i = j / s.ni;
+        const int k = j % s.ni;
+        const int o = outer_of(p, s, i);
+        const int slot = j % p.R;
+        const int kv = kvalid_of(s, k);
+        // 32-column blocks to read: every block of the slices the members
+        // copy, so columns >= kv are written as zeros, never left stale
+        const int hend = 2 * slices_of(s, k);
+        if (consume) {
+          // the slot's previous tile must have been copied by every member
+          const bool free_ok =
+              threadIdx.x == 0
+                  ? wait_counter(p.cons + ring0 + slot, static_cast<uint32_t>(g * (j / p.R)), ctl)
+                  : true;
+          if (!named_bar_and(1, kEpi, free_ok)) { ok = false; break; }
+        }
+        if (p.mode == GM_B) {
+          // lse2 and target of the tile's 256 masked rows (+inf / -1 beyond n)
+          for (int c = threadIdx.x; c < kZN; c += kEpi) {
+            const int rc = k * kZN + c;
+            float l2 = INFINITY;
+            int yy = -1;
+            if (rc < s.n) {
+              const int t = p.rows[rc];
+              if (t >= 0 && t < p.T) {
+                l2 = p.lse_in[t] * kLog2e;
+                yy = p.targets[t];
+              }
+            }
+            meta_l[c] = l2;
+            meta_y[c] = yy;
+          }
+        }
+        if (!named_bar_and(1, kEpi, mbar_wait(zfull, zph, ctl))) { ok = false; break; }
+        zph ^= 1u;
+        tc_fence_after();
+        uint8_t* img = ring_bytes + (ring0 + slot) * static_cast<size_t>(kXTile);
+        if (p.mode == GM_B) {
+          const int v = o * kBM + row;
+#pragma unroll 1
+          for (int h = 0; h < hend; ++h) {
+            uint32_t a[32];
+            tmem_ld_32x32b_x32(zaddr + h * 32, a);
+            tmem_ld_wait();
+            float gv[32];
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+              const int col = h * 32 + c;
+              const float xl = fmaf(__uint_as_float(a[c]), p.scale2, -meta_l[col]);
+              // the target entry p - 1 from expm1, exact where p is near 1
+              const float pm = meta_y[col] == v ? expm1f(xl * kLn2) : fast_exp2(xl);
+              gv[c] = col < kv ? s.coef * pm : 0.f;
+            }
+            store_img32(img, row, h, gv);
+          }
+        } else {
+          if (o != cur_o) {
+            cur_o = o;
+            ra = load_row_a(p, s, o * kBM + row);
+            run_s = 0.f;
+            run_m = -INFINITY;
+          }
+          const int v0 = k * kZN;
+#pragma unroll 1
+          for (int h = 0; h < hend; ++h) {
+            uint32_t a[32];
+            tmem_ld_32x32b_x32(zaddr + h * 32, a);
+            tmem_ld_wait();
+            float pv[32];
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+              const int col = h * 32 + c;
+              const float x = __uint_as_float(a[c]) * p.scale2;
+              const bool in = col < kv;
+              run_m = in ? fmaxf(run_m, x) : run_m;
+              const float e = fast_exp2(x - ra.R);
+              pv[c] = in ? e : 0.f;
+              run_s += pv[c];
+            }
+            const int yo = ra.y - (v0 + h * 32);
+            if (p.mode == GM_A && yo >= 0 && yo < 32) {
+              // the target's exact logit and the bf16 value of P'_y the MMA
+              // sees: the epilogue replaces that term by p_y - 1 from the
+              // logit, so rows with p_y near 1 keep their accuracy
+#pragma unroll
+              for (int c = 0; c < 32; ++c)
+                if (c == yo) {
+                  p.zy[o * kBM + row] = __uint_as_float(a[c]) * p.inv_tau;
+                  p.pyb[o * kBM + row] = __bfloat162float(__float2bfloat16_rn(pv[c]));
+                }
+            }
+            if (p.mode == GM_A) store_img32(img, row, h, pv);
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(zempty);
+        if (p.mode == GM_REF) {
+          if (o * kBM + row < s.n) p.rref[o * kBM + row] = run_m;
+        } else {
+          if (p.mode == GM_A && ra.valid) {
+            p.part_s[static_cast<size_t>(s.m) * Tpad + o * kBM + row] = run_s;
+            p.part_m[static_cast<size_t>(s.m) * Tpad + o * kBM + row] = run_m;
+          }
+          // publish the tile: every thread's stores, then one release
+          fence_proxy_async_global();
+          __threadfence();
+          named_bar_sync(1, kEpi);
+          if (threadIdx.x == 0) red_release_add(p.ready + ring0 + slot, 1u);
+        }
+      }
+      if (!consume || r == 0) continue;
+      // ------------------------------------------- outer tiles completed
+      const int e_end = min(r * g, s.E);
+      for (int e = (r - 1) * g; ok && e < e_end; ++e) {
+        if (e % s.ni != s.ni - 1) continue;
+        const int i = e / s.ni;
+        const int o = outer_of(p, s, i);
+        if (p.mode == GM_B) {
+          if (!named_bar_and(1, kEpi, mbar_wait(ofull, oph, ctl))) { ok = false; break; }
+          oph ^= 1u;
+          tc_fence_after();
+          const int v = o * kBM + row;
+#pragma unroll 1
+          for (int c = 0; c < s.cw; c += 32) {
+            uint32_t a[32];
+            tmem_ld_32x32b_x32(oaddr + c, a);
+            tmem_ld_wait();
+            float ov[32];
+#pragma unroll
+            for (int q = 0; q < 32; ++q) ov[q] = __uint_as_float(a[q]);
+            if (v < p.V)
+              store_out32(p.out, static_cast<size_t>(v) * p.d + s.c0 + c, p.out_dtype,
+                          min(32, s.cw - c), ov);
+          }
+          tc_fence_before();
+          mbar_arrive(oempty);
+          continue;
+        }
+        // pass A: merge the members' partials, then dH
+        const int rc = o * kBM + row;
+        const RowA rw = load_row_a(p, s, rc);
+        // every member's partials (and the target's z_y, P'_y from the
+        // member that met it) are published before any member reads them
+        if (rw.valid && !member_has_job(s, g, i)) {
+          p.part_s[static_cast<size_t>(s.m) * Tpad + rc] = 0.f;
+          p.part_m[static_cast<size_t>(s.m) * Tpad + rc] = -INFINITY;
+        }
+        __threadfence();
+        named_bar_sync(1, kEpi);
+        if (threadIdx.x == 0) red_release_add(p.outer_ctr + o, 1u);
+        const bool seen =
+            threadIdx.x == 0 ? wait_counter(p.outer_ctr + o, static_cast<uint32_t>(g), ctl) : true;
+        if (!named_bar_and(1, kEpi, seen)) { ok = false; break; }
+        if (!named_bar_and(1, kEpi, mbar_wait(ofull, oph, ctl))) { ok = false; break; }
+        oph ^= 1u;
+        tc_fence_after();
+        float lse2 = rw.R, mx = -INFINITY;
+        if (!p.lse_known && rw.valid) {
+          float sum = 0.f;
+          for (int mm = 0; mm < g; ++mm) {
+            sum += __ldcg(p.part_s + static_cast<size_t>(mm) * Tpad + rc);
+            mx = fmaxf(mx, __ldcg(p.part_m + static_cast<size_t>(mm) * Tpad + rc));
+          }
+          lse2 = rw.R + log2f(sum);
+        }
+        // (the redo launch, with R = the rows' maxima, never flags)
+        const bool row_ok = !rw.valid || p.lse_known || p.redo ||
+                            (mx - rw.R <= kRefMax && isfinite(lse2));
+        const bool tile_ok = named_bar_and(1, kEpi, row_ok);
+        if (!tile_ok) {
+          // the reference was too low for some row: the redo launch
+          // recomputes this row tile with R = the rows' maxima
+          if (s.m == 0) {
+            if (rw.valid) p.rmax[rc] = mx;
+            if (threadIdx.x == 0) {
+              const uint32_t at = atomicAdd(p.redo_list, 1u);
+              p.redo_list[1 + at] = static_cast<uint32_t>(o);
+            }
+          }
+        } else {
+          const bool has_y = rw.valid && rw.y >= 0 && rw.y < p.V;
+          if (s.m == 0 && rw.valid) {
+            if (!has_y) atomicOr(p.dev_status, 1 << OLIVE_ERR_TOKEN_RANGE);
+            if (p.write_fwd) {
+              const float l = lse2 * kLn2;
+              const float lp = has_y ? __ldcg(p.zy + rc) - l : NAN;
+              p.lse[rw.t] = l;
+              p.logp[rw.t] = lp;
+              p.nll[rc] = -lp;
+            }
+          }
+          const float scale = fast_exp2(rw.R - lse2);
+          // dH = coef (scale acc - W[y]) with the target's term taken out of
+          // acc (scale P'_y, P'_y as the MMA saw it) and put back as p_y W[y]:
+          // together coef (scale acc + corr W[y]), corr = (p_y - 1) - scale P'_y
+          float corr = 0.f;
+          if (has_y) {
+            const float lnat = p.lse_known ? p.lse_in[rw.t] : lse2 * kLn2;
+            corr = expm1f(__ldcg(p.zy + rc) - lnat) - scale * __ldcg(p.pyb + rc);
+          }
+          const uint4* wy =
+              has_y ? reinterpret_cast<const uint4*>(p.W + static_cast<size_t>(rw.y) * p.d + s.c0) : nullptr;
+#pragma unroll 1
+          for (int c = 0; c < s.cw; c += 32) {
+            uint32_t a[32];
+            tmem_ld_32x32b_x32(oaddr + c, a);
+            tmem_ld_wait();
+            float dv[32];
+            const int nv = min(32, s.cw - c);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              uint4 w4 = make_uint4(0, 0, 0, 0);
+              if (wy && 8 * q < nv) w4 = __ldg(wy + c / 8 + q);
+              const __nv_bfloat162* w2 = reinterpret_cast<const __nv_bfloat162*>(&w4);
+#pragma unroll
+              for (int u = 0; u < 4; ++u) {
+                const float2 wf = __bfloat1622float2(w2[u]);
+                dv[8 * q + 2 * u] = s.coef * fmaf(scale, __uint_as_float(a[8 * q + 2 * u]), corr * wf.x);
+                dv[8 * q + 2 * u + 1] =
+                    s.coef * fmaf(scale, __uint_as_float(a[8 * q + 2 * u + 1]), corr * wf.y);
+              }
+            }
+            if (rw.valid)
+              store_out32(p.out, static_cast<size_t>(rw.t) * p.d + s.c0 + c, p.out_dtype, nv, dv);
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(oempty);
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x == 0 && *abort_flag) atomicOr(p.dev_status, kStatusTimeoutBit);
+  if (warp == kMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, 512);
+  }
+}
+
+constexpr int kGroupSmem = 1024 + kStages * kStageBytes + 8 * (2 * kStages + 5) + 128 + kMetaBytes;
+static_assert(kGroupSmem <= 227 * 1024, "shared memory budget");
+
+int ring_slots_for(int g) { return 3 * g > 4 ? 3 * g : 4; }
+
+// groups of ceil(cols / 256) members, as many as `sms` SMs hold
+struct GroupShape {
+  int g, chunk, ngroups, R;
+};
+
+GroupShape group_shape(int cols, int sms) {
+  GroupShape gs;
+  gs.g = (cols + kZN - 1) / kZN;
+  if (gs.g < 1) gs.g = 1;
+  gs.chunk = ((cols + gs.g - 1) / gs.g + 15) / 16 * 16;
+  gs.ngroups = sms / gs.g;
+  gs.R = ring_slots_for(gs.g);
+  return gs;
+}
+
+}  // namespace
+
+// widest group a launch forms (ring and counters are sized for it)
+int group_g_max(int64_t d) {
+  const int64_t cols = d < static_cast<int64_t>(kGroupMaxSms) * kZN ? d : static_cast<int64_t>(kGroupMaxSms) * kZN;
+  return static_cast<int>((cols + kZN - 1) / kZN);
+}
+
+int ring_slots(int g) { return ring_slots_for(g); }
+
+// groups a launch forms at most: as many as the SMs hold, and no more than
+// the outer tiles of either pass (row tiles of T rows, vocabulary tiles)
+int group_count_max(int64_t T, int64_t d, int64_t V) {
+  const int g = group_g_max(d);
+  const int64_t outer = std::max(ceil_div(T, kBM), ceil_div(V, kBM));
+  return static_cast<int>(std::min<int64_t>(kGroupMaxSms / g, std::max<int64_t>(outer, 1)));
+}
+
+size_t group_ring_words(int64_t T, int64_t d, int64_t V) {
+  return static_cast<size_t>(group_count_max(T, d, V)) * ring_slots_for(group_g_max(d));
+}
+
+size_t group_ring_bytes(int64_t T, int64_t d, int64_t V) { return group_ring_words(T, d, V) * kXTile; }
+
+int group_sweep_cols(int sms) { return (sms < kGroupMaxSms ? sms : kGroupMaxSms) * kZN; }
+
+olive_status launch_group(const Ctx& c, int mode, const void* hc, const void* W, int32_t T,
+                          int32_t d, int32_t V, const GroupArgs& a, int c_base, int c_end,
+                          uint32_t* ring_ctr) {
+  const int sms = c.num_sms < kGroupMaxSms ? c.num_sms : kGroupMaxSms;
+  const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
+  GroupShape gs;
+  if (mode == GM_REF) {
+    gs.g = 1;
+    gs.chunk = kZN;
+    gs.ngroups = sms;
+    gs.R = 1;
+  } else {
+    gs = group_shape(c_end - c_base, sms);
+    gs.ngroups = std::min(gs.ngroups, group_count_max(T, d, V));
+    if (gs.ngroups < 1) return OLIVE_ERR_SHAPE;
+  }
+  GroupMaps maps;
+  const bool rowsA = mode != GM_B;
+  const void* zaBase = rowsA ? hc : W;
+  const void* zbBase = rowsA ? W : hc;
+  const uint64_t zaRows = rowsA ? Tpad : V;
+  const uint64_t zbRows = rowsA ? V : Tpad;
+  if (!encode_bf16_2d(&maps.za, zaBase, d, zaRows, 2ull * d, 64, 128) ||
+      !encode_bf16_2d(&maps.zb, zbBase, d, zbRows, 2ull * d, 64, 256) ||
+      !encode_bf16_2d(&maps.xb, zbBase, d, zbRows, 2ull * d, 64, 64))
+    return OLIVE_ERR_CUDA;
+
+  GroupParams p = {};
+  p.dev_status = a.dev_status;
+  p.wait_limit_ns = c.wait_limit_ns;
+  p.n_rows = a.n_rows;
+  p.rows = a.rows;
+  p.targets = a.targets;
+  p.W = static_cast<const __nv_bfloat16*>(W);
+  p.T = T;
+  p.d = d;
+  p.V = V;
+  p.mode = mode;
+  p.g = gs.g;
+  p.ngroups = gs.ngroups;
+  p.R = gs.R;
+  p.chunk = gs.chunk;
+  p.c_base = c_base;
+  p.c_end = c_end;
+  p.reduction = a.reduction;
+  p.inv_tau = a.inv_tau;
+  p.scale2 = a.inv_tau * kLog2e;
+  p.grad_loss = a.grad_loss;
+  p.lse_known = a.lse_known;
+  p.redo = a.redo;
+  p.write_fwd = a.write_fwd;
+  p.lse_in = a.lse_in;
+  p.rref = a.rref;
+  p.rmax = a.rmax;
+  p.part_s = a.part_s;
+  p.part_m = a.part_m;
+  p.zy = a.zy;
+  p.pyb = a.pyb;
+  p.logp = a.logp;
+  p.lse = a.lse;
+  p.nll = a.nll;
+  p.redo_list = a.redo_list;
+  p.outer_ctr = a.outer_ctr + (mode == GM_A && a.redo ? (T + kBM - 1) / kBM : 0);
+  p.ring = static_cast<__nv_bfloat16*>(a.ring);
+  p.ready = ring_ctr;
+  p.cons = ring_ctr ? ring_ctr + static_cast<size_t>(gs.ngroups) * gs.R : nullptr;
+  p.out = mode == GM_B ? a.d_W : a.d_hidden;
+  p.out_dtype = a.out_dtype;
+
+  static std::atomic<int> done[kMaxDevices];
+  if (!set_smem_once(reinterpret_cast<const void*>(lmhead_group_kernel), kGroupSmem, c.device, done))
+    return OLIVE_ERR_CUDA;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(gs.ngroups * gs.g);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kGroupSmem;
+  cfg.stream = c.stream;
+  // members of a group wait on one another: every CTA must be resident
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = mode == GM_REF ? 0 : 1;
+  if (cudaLaunchKernelEx(&cfg, lmhead_group_kernel, maps, p) != cudaSuccess) {
+    cudaGetLastError();
+    return OLIVE_ERR_CUDA;
+  }
+  return OLIVE_OK;
+}
+
+}  // namespace olive
+
+namespace olive {
+
+olive_status launch_loss_group(const Ctx& c, const void* hidden, const void* W,
+                               const int32_t* targets, const int32_t* rows, const int32_t* n_rows,
+                               int32_t T, int32_t d, int32_t V, float inv_tau, int reduction,
+                               const float* grad_loss, const float* lse_given, float* logp,
+                               float* lse, float* loss, void* d_hidden, void* d_W, int grad_dtype,
+                               void* ws, int32_t* dev_status) {
+  const bool fwd = lse_given == nullptr;
+  const GroupWs w = carve_group(ws, T, d, V);
+  const size_t elt = grad_dtype == OLIVE_DTYPE_BF16 ? 2 : 4;
+  olive_status st = launch_gather_rows(c, hidden, rows, n_rows, T, d, w.hc, dev_status);
+  if (st != OLIVE_OK) return st;
+  if (cudaMemsetAsync(d_hidden, 0, elt * T * static_cast<size_t>(d), c.stream) != cudaSuccess ||
+      cudaMemsetAsync(w.outer, 0, 4 * w.ctr_words, c.stream) != cudaSuccess)
+    return OLIVE_ERR_CUDA;
+  if (fwd && (cudaMemsetAsync(logp, 0, sizeof(float) * T, c.stream) != cudaSuccess ||
+              cudaMemsetAsync(lse, 0, sizeof(float) * T, c.stream) != cudaSuccess))
+    return OLIVE_ERR_CUDA;
+
+  GroupArgs a = {};
+  a.dev_status = dev_status;
+  a.n_rows = n_rows;
+  a.rows = rows;
+  a.targets = targets;
+  a.reduction = reduction;
+  a.inv_tau = inv_tau;
+  a.grad_loss = grad_loss;
+  a.lse_in = fwd ? lse : lse_given;
+  a.rref = w.rref;
+  a.rmax = w.rmax;
+  a.part_s = w.part_s;
+  a.part_m = w.part_m;
+  a.zy = w.zy;
+  a.pyb = w.pyb;
+  a.logp = logp;
+  a.lse = lse;
+  a.nll = w.nll;
+  a.redo_list = w.redo;
+  a.outer_ctr = w.outer;
+  a.ring = w.ring;
+  a.d_hidden = d_hidden;
+  a.d_W = d_W;
+  a.out_dtype = grad_dtype;
+
+  if (fwd && (st = launch_group(c, GM_REF, w.hc, W, T, d, V, a, 0, d, nullptr)) != OLIVE_OK)
+    return st;
+  // one sweep of both passes per range of output columns the SMs can hold
+  // (every d up to 38912 at 152 SMs takes one)
+  const int cols = group_sweep_cols(c.num_sms);
+  const size_t rw = 2 * group_ring_words(T, d, V);
+  for (int cb = 0; cb < d; cb += cols) {
+    const int ce = d - cb < cols ? d : cb + cols;
+    if (cb > 0 && cudaMemsetAsync(w.outer, 0, 4 * w.ctr_words, c.stream) != cudaSuccess)
+      return OLIVE_ERR_CUDA;
+    a.lse_known = (!fwd || cb > 0) ? 1 : 0;
+    a.write_fwd = (fwd && cb == 0) ? 1 : 0;
+    a.redo = 0;
+    if ((st = launch_group(c, GM_A, w.hc, W, T, d, V, a, cb, ce, w.ring_ctr)) != OLIVE_OK) return st;
+    if (fwd && cb == 0) {
+      a.redo = 1;
+      if ((st = launch_group(c, GM_A, w.hc, W, T, d, V, a, cb, ce, w.ring_ctr + rw)) != OLIVE_OK)
+        return st;
+      a.redo = 0;
+    }
+    if ((st = launch_group(c, GM_B, w.hc, W, T, d, V, a, cb, ce, w.ring_ctr + 2 * rw)) != OLIVE_OK)
+      return st;
+  }
+  return fwd ? launch_loss_reduce(c, n_rows, T, w.nll, reduction, loss) : OLIVE_OK;
+}
+
+}  // namespace olive

@@ -247,6 +247,42 @@ size_t topk_kl_fb_ws_bytes(int64_t T, int64_t d, int64_t V, int grad_dtype) {
          align_up(4ull * slab_rows(Tpad, V) * ceil_div(V, 128), kWsAlign);
 }
 
+static GroupWs carve_group_impl(void* ws, int64_t T, int64_t d, int64_t V, size_t* total) {
+  const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
+  const int64_t rt = Tpad / kRowAlign;
+  const int gmax = group_g_max(d);
+  Carver c{static_cast<char*>(ws)};
+  GroupWs w;
+  w.hc = c.take(2ull * Tpad * d);
+  w.rref = static_cast<float*>(c.take(4ull * Tpad));
+  w.rmax = static_cast<float*>(c.take(4ull * Tpad));
+  w.zy = static_cast<float*>(c.take(4ull * Tpad));
+  w.pyb = static_cast<float*>(c.take(4ull * Tpad));
+  w.nll = static_cast<float*>(c.take(4ull * Tpad));
+  w.part_s = static_cast<float*>(c.take(4ull * gmax * Tpad));
+  w.part_m = static_cast<float*>(c.take(4ull * gmax * Tpad));
+  w.ring = c.take(group_ring_bytes(T, d, V));
+  // counters in one region, zeroed by one memset per column sweep: group
+  // barriers [2 rt] (first and redo launch), the redo list [1 + rt], then the
+  // ring counters of the three launches of a sweep
+  const size_t rw = 2 * group_ring_words(T, d, V);
+  w.ctr_words = static_cast<size_t>(3 * rt + 1) + 3 * rw;
+  uint32_t* ctr = static_cast<uint32_t*>(c.take(4ull * w.ctr_words));
+  w.outer = ctr;
+  w.redo = ctr ? ctr + 2 * rt : nullptr;
+  w.ring_ctr = ctr ? ctr + 3 * rt + 1 : nullptr;
+  if (total) *total = c.off;
+  return w;
+}
+size_t group_ws_bytes(int64_t T, int64_t d, int64_t V) {
+  size_t n = 0;
+  carve_group_impl(nullptr, T, d, V, &n);
+  return n;
+}
+GroupWs carve_group(void* ws, int64_t T, int64_t d, int64_t V) {
+  return carve_group_impl(ws, T, d, V, nullptr);
+}
+
 static KlWs carve_kl_impl(void* ws, int64_t T, int64_t ds, int64_t dt, int64_t V, int grad,
                           size_t* total) {
   const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
@@ -325,12 +361,15 @@ size_t olive_workspace_size(int op, int32_t T, int32_t d, int32_t d_t, int32_t V
     case OLIVE_OP_LOGPROB_FWD: return fwd_ws_bytes(T, d);
     case OLIVE_OP_LOSS_BWD:
       if (grad_dtype != OLIVE_DTYPE_BF16 && grad_dtype != OLIVE_DTYPE_F32) return 0;
-      return bwd_ws_bytes(T, d, V, grad_dtype);
+      return group_ws_bytes(T, d, V);
     case OLIVE_OP_DIVERGENCE:
       if (!width_ok(d_t)) return 0;
       return kl_ws_bytes(T, d, d_t, V, grad);
     case OLIVE_OP_TOPK_FWD: return topk_ws_bytes(T, d);
     case OLIVE_OP_LOSS_FWD_BWD:
+      if (grad_dtype != OLIVE_DTYPE_BF16 && grad_dtype != OLIVE_DTYPE_F32) return 0;
+      return group_ws_bytes(T, d, V);
+    case OLIVE_OP_LOSS_FWD_BWD_SLAB:
       if (grad_dtype != OLIVE_DTYPE_BF16 && grad_dtype != OLIVE_DTYPE_F32) return 0;
       return fb_ws_bytes(T, d, V, grad_dtype);
     case OLIVE_OP_OPD_STATS:
@@ -518,13 +557,14 @@ olive_status olive_token_loss_bwd(const void* hidden, const void* W, const int32
   if (!(inv_tau > 0.f) || !std::isfinite(inv_tau)) return OLIVE_ERR_INVALID_ARG;
   if (d % 8 != 0 || !aligned16(hidden) || !aligned16(W) || !aligned16(d_hidden) || !aligned16(d_W))
     return OLIVE_ERR_ALIGNMENT;
-  olive_status st = check_ws(workspace, ws_bytes, bwd_ws_bytes(T, d, V, grad_dtype));
+  olive_status st = check_ws(workspace, ws_bytes, group_ws_bytes(T, d, V));
   if (st != OLIVE_OK) return st;
   Ctx c;
   st = make_ctx(stream, &c);
   if (st != OLIVE_OK) return st;
-  return launch_loss_bwd(c, hidden, W, targets, rows, n_rows, T, d, V, inv_tau, reduction, lse,
-                         grad_loss, d_hidden, d_W, grad_dtype, workspace, dev_status);
+  return launch_loss_group(c, hidden, W, targets, rows, n_rows, T, d, V, inv_tau, reduction,
+                           grad_loss, lse, nullptr, nullptr, nullptr, d_hidden, d_W, grad_dtype,
+                           workspace, dev_status);
 }
 
 olive_status olive_token_loss_fwd_bwd(const void* hidden, const void* W, const int32_t* targets,
@@ -533,6 +573,31 @@ olive_status olive_token_loss_fwd_bwd(const void* hidden, const void* W, const i
                                       const float* grad_loss, float* logp, float* lse, float* loss,
                                       void* d_hidden, void* d_W, int grad_dtype, void* workspace,
                                       size_t ws_bytes, int32_t* dev_status, void* stream) {
+  if (!hidden || !W || !targets || !rows || !n_rows || !grad_loss || !logp || !lse || !loss ||
+      !d_hidden || !d_W || !dev_status)
+    return OLIVE_ERR_INVALID_ARG;
+  if (reduction != OLIVE_REDUCE_SUM && reduction != OLIVE_REDUCE_MEAN) return OLIVE_ERR_INVALID_ARG;
+  if (grad_dtype != OLIVE_DTYPE_BF16 && grad_dtype != OLIVE_DTYPE_F32) return OLIVE_ERR_INVALID_ARG;
+  if (T < 1 || V < 1 || d < 1 || d > kMaxDim) return OLIVE_ERR_SHAPE;
+  if (!(inv_tau > 0.f) || !std::isfinite(inv_tau)) return OLIVE_ERR_INVALID_ARG;
+  if (d % 8 != 0 || !aligned16(hidden) || !aligned16(W) || !aligned16(d_hidden) || !aligned16(d_W))
+    return OLIVE_ERR_ALIGNMENT;
+  olive_status st = check_ws(workspace, ws_bytes, group_ws_bytes(T, d, V));
+  if (st != OLIVE_OK) return st;
+  Ctx c;
+  st = make_ctx(stream, &c);
+  if (st != OLIVE_OK) return st;
+  return launch_loss_group(c, hidden, W, targets, rows, n_rows, T, d, V, inv_tau, reduction,
+                           grad_loss, nullptr, logp, lse, loss, d_hidden, d_W, grad_dtype,
+                           workspace, dev_status);
+}
+
+olive_status olive_token_loss_fwd_bwd_slab(const void* hidden, const void* W, const int32_t* targets,
+                                           const int32_t* rows, const int32_t* n_rows, int32_t T,
+                                           int32_t d, int32_t V, float inv_tau, int reduction,
+                                           const float* grad_loss, float* logp, float* lse, float* loss,
+                                           void* d_hidden, void* d_W, int grad_dtype, void* workspace,
+                                           size_t ws_bytes, int32_t* dev_status, void* stream) {
   if (!hidden || !W || !targets || !rows || !n_rows || !grad_loss || !logp || !lse || !loss ||
       !d_hidden || !d_W || !dev_status)
     return OLIVE_ERR_INVALID_ARG;

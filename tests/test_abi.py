@@ -47,8 +47,15 @@ def test_workspace_sizes(L):
     bwd32 = B.olive_workspace_size("loss_bwd", T, d, V, grad_dtype=torch.float32)
     kl = B.olive_workspace_size("divergence", 16384, 4096, V, d_t=5120, grad=True)
     assert fwd >= 2 * T * d and fwd % 256 == 0
-    # bf16 dW needs the fp32 accumulator on top
-    assert bwd16 - bwd32 >= 4 * V * d
+    # the on-chip backward stores no [rows, V] array and no [V, d]
+    # accumulator: its workspace does not grow with V or the gradient dtype
+    assert bwd16 == bwd32
+    assert bwd16 == B.olive_workspace_size("loss_bwd", T, d, 8192)
+    fb = B.olive_workspace_size("loss_fwd_bwd", T, d, V)
+    assert fb == bwd16 and fb < 2 * T * d + 256 * 2**20
+    # the slab variant holds G for up to 32768 rows (~5.6 GB at this V)
+    slab = B.olive_workspace_size("loss_fwd_bwd_slab", T, d, V)
+    assert slab >= 2 * 18304 * V
     assert kl > B.olive_workspace_size("divergence", 16384, 4096, V, d_t=5120, grad=False)
     # invalid requests give 0
     assert B.olive_workspace_size("logprob_fwd", 0, d, V) == 0
@@ -143,7 +150,7 @@ def test_new_entry_points_validation(L):
     assert st == 2
     # top-K KL backward: missing t_logp_s, bad K, bad dtype, misaligned d_W_s, workspace
     ws = B.olive_workspace_size("topk_kl_bwd", 64, 64, 100, grad_dtype=torch.float32)
-    assert ws > B.olive_workspace_size("loss_bwd", 64, 64, 100, grad_dtype=torch.float32)
+    assert ws > 2 * 64 * 100  # its G slab
 
     def kl_bwd(**kw):
         a = dict(tlp=P(p), K=4, dt=1, dw=P(p), ws_bytes=1 << 20)
@@ -195,7 +202,7 @@ def test_topk_kl_fwd_bwd_validation(L):
     keep, p = _fake()
     P = ctypes.c_void_p
     ws = B.olive_workspace_size("topk_kl_fwd_bwd", 64, 64, 100, grad_dtype=torch.bfloat16)
-    assert ws >= B.olive_workspace_size("loss_fwd_bwd", 64, 64, 100, grad_dtype=torch.bfloat16)
+    assert ws >= B.olive_workspace_size("loss_fwd_bwd_slab", 64, 64, 100, grad_dtype=torch.bfloat16)
     assert L.olive_workspace_size(8, 64, 64, 0, 100, 1, 2) == 0  # no fp16 gradients
 
     def call(**kw):
