@@ -718,6 +718,35 @@ def run_reference(args, world, rank):
     print(json.dumps(line), flush=True)
 
 
+def run_profile_case(args):
+    """A small case for profilers: `--steps` calls of olive_token_loss_fwd_bwd
+    (or the slab form with --slab) on N masked rows (every row masked,
+    RMS-normalised N(0,1) hidden, W ~ N(0, 0.02), d = 4096, V = 151936); no
+    JSON line.  At N = 4096 the device holds ~3 GB."""
+    from paper_2609_36246_gb300 import binding as B
+    from paper_2609_36246_gb300 import build as _build
+    _build.build()
+    dev = torch.device("cuda", torch.cuda.current_device())
+    N, d, V = args.profile_rows, 4096, 151936
+    h, W = gpu_inputs(31, N, d, V, dev)
+    rows = torch.arange(N, dtype=torch.int32, device=dev)
+    n = torch.tensor([N], dtype=torch.int32, device=dev)
+    g = torch.Generator(device=dev).manual_seed(32)
+    targets = torch.randint(0, V, (N,), generator=g, device=dev, dtype=torch.int32)
+    gl = torch.ones(1, dtype=torch.float32, device=dev)
+    op = "loss_fwd_bwd_slab" if args.slab else "loss_fwd_bwd"
+    ws = B.workspace(B.olive_workspace_size(op, N, d, V), dev)
+    st = B.new_status(dev)
+    out = None
+    for _ in range(args.steps):
+        out = B.olive_token_loss_fwd_bwd(h, W, targets, rows, n, gl, ws=ws, dev_status=st, out=out,
+                                         slab=args.slab)
+    torch.cuda.synchronize()
+    if int(st.item()) != 0:
+        raise RuntimeError(f"device status {B.status_bits(st)}")
+    print(f"profile case: {args.steps} calls of {op} on {N} rows, loss {float(out[2].item()):.4f}")
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -730,7 +759,16 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extra", action="store_true",
                     help="skip the divergence and variable-length measurements")
+    ap.add_argument("--profile-rows", type=int, default=0,
+                    help="run only the training-step call on this many masked rows (a small "
+                         "case for ncu) and print no JSON line")
+    ap.add_argument("--slab", action="store_true", help="with --profile-rows: the slab form")
     args = ap.parse_args()
+    if args.profile_rows > 0:
+        if torch.cuda.is_available():
+            torch.cuda.set_device(0)
+        run_profile_case(args)
+        return
     world, rank, local = dist_setup()
     if args.impl == "reference":
         run_reference(args, world, rank)

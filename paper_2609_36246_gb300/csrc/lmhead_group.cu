@@ -79,7 +79,8 @@ constexpr int kXTile = 4 * kXSlice;  // 128 x 256 bf16 (64 KB)
 constexpr int kEpi = 128;            // epilogue threads: one accumulator row each
 constexpr int kProducerWarp = 4;
 constexpr int kMmaWarp = 5;
-constexpr int kThreads = 192;
+constexpr int kSignalWarp = 6;       // posts the members' "tile copied" counts
+constexpr int kThreads = 224;
 constexpr int kStatusTimeoutBit = 1 << OLIVE_ERR_TIMEOUT;
 constexpr float kRefMax = 64.f;
 constexpr int kMetaBytes = kZN * 8;  // pass B: lse2 and target of the tile's 256 rows
@@ -275,6 +276,27 @@ __device__ __forceinline__ RowA load_row_a(const GroupParams& p, const GSched& s
   return a;
 }
 
+// All lanes of a warp: wait until the exchange tiles [e_lo, e_end) of a
+// round are written (ready[e mod R] > e / R), lane i checking tiles i, i+32,
+// ...  Returns the warp's common decision (false: limit ran out or abort).
+__device__ bool wait_round_ready(const uint32_t* ready, int R, int e_lo, int e_end, int lane,
+                                 const WaitCtl& ctl) {
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+    bool mine = true;
+    for (int e = e_lo + lane; e < e_end; e += 32)
+      mine = mine && ld_acquire(ready + e % R) >= static_cast<uint32_t>(e / R + 1);
+    if (__all_sync(0xffffffffu, mine)) return true;
+    bool stop = *ctl.abort != 0;
+    if (!stop && global_timer_ns() - t0 > ctl.limit_ns) {
+      if (lane == 0) *ctl.abort = 1;
+      stop = true;
+    }
+    if (__any_sync(0xffffffffu, stop)) return false;
+    nanosleep_ns(64);
+  }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     lmhead_group_kernel(const __grid_constant__ GroupMaps maps, const GroupParams p) {
   extern __shared__ uint8_t smem_raw[];
@@ -294,6 +316,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* misc = gbase + kStages * kStageBytes + 8 * (2 * kStages + 5);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 4);
+  volatile uint32_t* copied = reinterpret_cast<volatile uint32_t*>(misc + 8);  // tiles copied
   GSched* sched_smem = reinterpret_cast<GSched*>(misc + 16);
   float* meta_l = reinterpret_cast<float*>(misc + 128);                 // [256] lse2 (GM_B)
   int* meta_y = reinterpret_cast<int*>(misc + 128 + kMetaBytes / 2);    // [256] targets (GM_B)
@@ -312,6 +335,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(oempty, kEpi);
     mbar_init(drain, 1);
     *abort_flag = 0;
+    *copied = 0;
     *sched_smem = make_gsched(p);
     fence_mbar_init();
   }
@@ -338,13 +362,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* ring_bytes = reinterpret_cast<uint8_t*>(p.ring);
 
   if (warp == kProducerWarp) {
-    if (lane == 0) {
-      int stage = 0;
-      uint32_t phase = 0;
-      bool ok = true;
-      for (int r = 0; ok && r <= nr; ++r) {
-        const int j = r * g + s.m;
-        if (r < nr && j < s.E) {
+    // lane 0 issues every copy; the whole warp checks the `ready` flags of a
+    // round's g exchange tiles at once (one L2 round trip per round instead
+    // of one blocking acquire per tile, which left the stage ring empty)
+    int stage = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    for (int r = 0; ok && r <= nr; ++r) {
+      const int j = r * g + s.m;
+      if (r < nr && j < s.E) {
+        if (lane == 0) {
           const int o = outer_of(p, s, j / s.ni);
           const int k = j % s.ni;
           for (int ks = 0; ks < s.nk; ++ks) {
@@ -357,15 +384,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (++stage == kStages) { stage = 0; phase ^= 1u; }
           }
         }
-        if (!ok || !consume || r == 0) continue;
-        const int e_end = min(r * g, s.E);
-        for (int e = (r - 1) * g; ok && e < e_end; ++e) {
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+      }
+      if (!ok || !consume || r == 0) continue;
+      const int e_lo = (r - 1) * g;
+      const int e_end = min(r * g, s.E);
+      ok = wait_round_ready(p.ready + ring0, p.R, e_lo, e_end, lane, ctl);
+      if (!ok) break;
+      if (lane == 0) {
+        fence_proxy_async_global();
+        for (int e = e_lo; ok && e < e_end; ++e) {
           const int slot = e % p.R;
-          if (!wait_counter(p.ready + ring0 + slot, static_cast<uint32_t>(e / p.R + 1), ctl)) {
-            ok = false;
-            break;
-          }
-          fence_proxy_async_global();
           const int k = e % s.ni;
           const int nsl = slices_of(s, k);
           const uint8_t* img = ring_bytes + (ring0 + slot) * static_cast<size_t>(kXTile);
@@ -381,10 +410,35 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
-      if (!ok) {
-        // let copies already issued land before the CTA retires
-        const uint64_t t0 = global_timer_ns();
-        while (global_timer_ns() - t0 < 50000) nanosleep_ns(1000);
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+    }
+    if (!ok && lane == 0) {
+      // let copies already issued land before the CTA retires
+      const uint64_t t0 = global_timer_ns();
+      while (global_timer_ns() - t0 < 50000) nanosleep_ns(1000);
+    }
+    __syncwarp();
+  } else if (warp == kSignalWarp) {
+    // for every exchange tile, in order, once the MMA warp has seen all its
+    // slices land: one release increment of the slot's `cons` count
+    if (lane == 0 && consume) {
+      uint32_t sent = 0;
+      const uint32_t total = static_cast<uint32_t>(s.E);
+      const uint64_t t0 = global_timer_ns();
+      uint64_t last = t0;
+      while (sent < total) {
+        const uint32_t c = *copied;
+        if (c > sent) {
+          for (; sent < c; ++sent) red_release_add(p.cons + ring0 + sent % p.R, 1u);
+          last = global_timer_ns();
+          continue;
+        }
+        if (*abort_flag) break;
+        nanosleep_ns(100);
+        if (global_timer_ns() - last > p.wait_limit_ns) {
+          *abort_flag = 1;
+          break;
+        }
       }
     }
     __syncwarp();
@@ -441,9 +495,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (++stage == kStages) { stage = 0; phase ^= 1u; }
           }
           if (!ok) break;
-          // every slice of tile e has landed in shared memory: its slot may
-          // be rewritten once all members say so
-          red_release_add(p.cons + ring0 + e % p.R, 1u);
+          // every slice of tile e has landed in shared memory: the signal
+          // warp tells the group (its slot may be rewritten once all members
+          // have said so)
+          *copied = static_cast<uint32_t>(e + 1);
           if (k == s.ni - 1) {
             umma_commit(ofull);
             oph ^= 1u;
