@@ -143,7 +143,7 @@ struct GroupWs {
   void* ring;        // group_ring_bytes(T, d, V)
   uint32_t* outer;   // [2 rt] pass-A group barriers (first launch, redo launch)
   uint32_t* redo;    // [1 + rt] redo list
-  uint32_t* ring_ctr;  // 3 launches x 2 x group_ring_words(T, d, V)
+  uint32_t* ring_ctr;  // 3 launches x group_ctr_words(T, d, V)
   size_t ctr_words;  // words from `outer` to the end of ring_ctr
 };
 size_t group_ws_bytes(int64_t T, int64_t d, int64_t V);
@@ -152,6 +152,7 @@ int group_g_max(int64_t d);
 int group_count_max(int64_t T, int64_t d, int64_t V);
 size_t group_ring_words(int64_t T, int64_t d, int64_t V);
 size_t group_ring_bytes(int64_t T, int64_t d, int64_t V);
+size_t group_ctr_words(int64_t T, int64_t d, int64_t V);
 int group_sweep_cols(int sms);
 
 struct GroupArgs {

@@ -84,6 +84,14 @@ constexpr int kThreads = 224;
 constexpr int kStatusTimeoutBit = 1 << OLIVE_ERR_TIMEOUT;
 constexpr float kRefMax = 64.f;
 constexpr int kMetaBytes = kZN * 8;  // pass B: lse2 and target of the tile's 256 rows
+// Pacing across groups: every group walks the same sequence of inner tiles
+// (vocabulary tiles of W in pass A, row pairs of hc in pass B), so while the
+// groups stay within kPaceLag rounds of one another one DRAM fetch of a tile
+// serves all of them from the L2; a group that runs ahead waits, at most
+// kPaceLimitNs per round (a hint: giving up only costs bandwidth).
+constexpr int kPaceLag = 1;
+constexpr uint64_t kPaceLimitNs = 2000000;
+constexpr uint32_t kPaceDone = 0x40000000u;
 
 enum GMode : int { GM_REF = 0, GM_A = 1, GM_B = 2 };
 
@@ -126,6 +134,7 @@ struct GroupParams {
   __nv_bfloat16* ring;      // [ngroups][R][128 x 256] exchange tiles (swizzled images)
   uint32_t* ready;          // [ngroups][R]
   uint32_t* cons;           // [ngroups][R]
+  uint32_t* pace;           // [ngroups] rounds each group has begun (a pacing hint)
   void* out;                // GM_A: d_hidden [T, d]; GM_B: d_W [V, d]
   int32_t out_dtype;
 };
@@ -297,6 +306,21 @@ __device__ bool wait_round_ready(const uint32_t* ready, int R, int e_lo, int e_e
   }
 }
 
+// All lanes of a warp: wait (at most kPaceLimitNs) until every group has
+// begun round `need` (pace[q] >= need), lane i checking groups i, i+32, ...
+__device__ void pace_wait(const uint32_t* pace, int ngroups, int need, int lane) {
+  if (need <= 0) return;
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+    bool mine = true;
+    for (int q = lane; q < ngroups; q += 32)
+      mine = mine && *reinterpret_cast<const volatile uint32_t*>(pace + q) >= static_cast<uint32_t>(need);
+    if (__all_sync(0xffffffffu, mine)) return;
+    if (global_timer_ns() - t0 > kPaceLimitNs) return;
+    nanosleep_ns(128);
+  }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     lmhead_group_kernel(const __grid_constant__ GroupMaps maps, const GroupParams p) {
   extern __shared__ uint8_t smem_raw[];
@@ -368,8 +392,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
+    const bool paced = consume && p.ngroups > 1;
     for (int r = 0; ok && r <= nr; ++r) {
       const int j = r * g + s.m;
+      if (paced && r < nr) {
+        pace_wait(p.pace, p.ngroups, r - kPaceLag, lane);
+        if (s.m == 0 && lane == 0)
+          *reinterpret_cast<volatile uint32_t*>(p.pace + s.q) = static_cast<uint32_t>(r + 1);
+      }
       if (r < nr && j < s.E) {
         if (lane == 0) {
           const int o = outer_of(p, s, j / s.ni);
@@ -412,6 +442,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       ok = __shfl_sync(0xffffffffu, ok, 0);
     }
+    if (paced && s.m == 0 && lane == 0) *reinterpret_cast<volatile uint32_t*>(p.pace + s.q) = kPaceDone;
     if (!ok && lane == 0) {
       // let copies already issued land before the CTA retires
       const uint64_t t0 = global_timer_ns();
@@ -829,6 +860,11 @@ size_t group_ring_words(int64_t T, int64_t d, int64_t V) {
 
 size_t group_ring_bytes(int64_t T, int64_t d, int64_t V) { return group_ring_words(T, d, V) * kXTile; }
 
+// counter words of one launch: ready and cons per ring slot, pace per group
+size_t group_ctr_words(int64_t T, int64_t d, int64_t V) {
+  return 2 * group_ring_words(T, d, V) + static_cast<size_t>(group_count_max(T, d, V));
+}
+
 int group_sweep_cols(int sms) { return (sms < kGroupMaxSms ? sms : kGroupMaxSms) * kZN; }
 
 olive_status launch_group(const Ctx& c, int mode, const void* hc, const void* W, int32_t T,
@@ -897,6 +933,7 @@ olive_status launch_group(const Ctx& c, int mode, const void* hc, const void* W,
   p.ring = static_cast<__nv_bfloat16*>(a.ring);
   p.ready = ring_ctr;
   p.cons = ring_ctr ? ring_ctr + static_cast<size_t>(gs.ngroups) * gs.R : nullptr;
+  p.pace = ring_ctr ? ring_ctr + 2 * static_cast<size_t>(gs.ngroups) * gs.R : nullptr;
   p.out = mode == GM_B ? a.d_W : a.d_hidden;
   p.out_dtype = a.out_dtype;
 
@@ -973,7 +1010,7 @@ olive_status launch_loss_group(const Ctx& c, const void* hidden, const void* W,
   // one sweep of both passes per range of output columns the SMs can hold
   // (every d up to 38912 at 152 SMs takes one)
   const int cols = group_sweep_cols(c.num_sms);
-  const size_t rw = 2 * group_ring_words(T, d, V);
+  const size_t rw = group_ctr_words(T, d, V);
   for (int cb = 0; cb < d; cb += cols) {
     const int ce = d - cb < cols ? d : cb + cols;
     if (cb > 0 && cudaMemsetAsync(w.outer, 0, 4 * w.ctr_words, c.stream) != cudaSuccess)

@@ -265,7 +265,7 @@ static GroupWs carve_group_impl(void* ws, int64_t T, int64_t d, int64_t V, size_
   // counters in one region, zeroed by one memset per column sweep: group
   // barriers [2 rt] (first and redo launch), the redo list [1 + rt], then the
   // ring counters of the three launches of a sweep
-  const size_t rw = 2 * group_ring_words(T, d, V);
+  const size_t rw = group_ctr_words(T, d, V);
   w.ctr_words = static_cast<size_t>(3 * rt + 1) + 3 * rw;
   uint32_t* ctr = static_cast<uint32_t*>(c.take(4ull * w.ctr_words));
   w.outer = ctr;

@@ -1,5 +1,7 @@
-"""olive_token_loss_fwd_bwd (CUDA: forward and backward of Eq. (osd-ce) in one
-pass over the logits) against the oracle's token_logprob and token_loss_bwd."""
+"""olive_token_loss_fwd_bwd (CUDA: forward and backward of Eq. (osd-ce), G
+formed and consumed on chip) and olive_token_loss_fwd_bwd_slab (the same step
+through an HBM slab of G) against the oracle's token_logprob and
+token_loss_bwd."""
 
 
 import numpy as np
@@ -15,14 +17,19 @@ from tests.parity import (FULL_SIZE_ROWS, assert_close_grad, assert_close_logp, 
 pytestmark = pytest.mark.gpu
 
 
-def _gpu(b, h, W, inv_tau=1.0, reduction="sum", grad_loss=1.0, grad_dtype=torch.bfloat16):
+FORMS = ["onchip", "slab"]
+
+
+def _gpu(b, h, W, inv_tau=1.0, reduction="sum", grad_loss=1.0, grad_dtype=torch.bfloat16,
+         form="onchip", n_rows=None):
     g = gpu_pack(b)
     hc, Wc = h.cuda(), W.cuda()
     st = g["dev_status"]
     gl = torch.tensor([grad_loss], dtype=torch.float32, device="cuda")
-    logp, lse, loss, dh, dw = B.olive_token_loss_fwd_bwd(hc, Wc, g["targets"], g["rows"], g["n_rows"],
+    nr = g["n_rows"] if n_rows is None else torch.tensor([n_rows], dtype=torch.int32, device="cuda")
+    logp, lse, loss, dh, dw = B.olive_token_loss_fwd_bwd(hc, Wc, g["targets"], g["rows"], nr,
                                                          gl, inv_tau, reduction, grad_dtype,
-                                                         dev_status=st)
+                                                         dev_status=st, slab=form == "slab")
     torch.cuda.synchronize()
     assert B.status_bits(st) == []
     return (logp.cpu().numpy(), lse.cpu().numpy(), float(loss.item()), dh.float().cpu().numpy(),
@@ -46,11 +53,13 @@ def _full_check(b, h, W, **kw):
     return logp, dh, dw
 
 
-def test_tiny_workload_full():
+@pytest.mark.parametrize("form", FORMS)
+def test_tiny_workload_full(form):
     b = synth.make_batch("tiny")
-    _full_check(b, synth.make_hidden("tiny", b.T), synth.make_weight("tiny"))
+    _full_check(b, synth.make_hidden("tiny", b.T), synth.make_weight("tiny"), form=form)
 
 
+@pytest.mark.parametrize("form", FORMS)
 @pytest.mark.parametrize("S,V,d,kw", [
     (3, 4097, 64, dict()),
     (5, 300, 72, dict(inv_tau=0.7, reduction="mean", grad_loss=2.5)),
@@ -59,25 +68,27 @@ def test_tiny_workload_full():
     (4, 700, 320, dict(inv_tau=1.2)),  # d = 320: a partial 256-wide output tile
     (7, 13, 24, dict()),               # V below one 8-wide vector group
 ])
-def test_random_shapes(S, V, d, kw):
+def test_random_shapes(S, V, d, kw, form):
     b, h, W = synth.random_case(S * 17 + V, S, V, d, max_prefix=30, max_cont=80, std_w=0.08)
-    _full_check(b, h, W, **kw)
+    _full_check(b, h, W, form=form, **kw)
 
 
-def test_single_entry_vocabulary():
+@pytest.mark.parametrize("form", FORMS)
+def test_single_entry_vocabulary(form):
     rng = np.random.default_rng(4)
     b = synth.batch_from_lengths(rng, [3, 5], [7, 4], 1)
     h = synth.normal_bf16(rng, (b.T, 64), 1.0)
     W = synth.normal_bf16(rng, (1, 64), 0.3)
-    logp, _, loss, dh, dw = _gpu(b, h, W, grad_dtype=torch.float32)
+    logp, _, loss, dh, dw = _gpu(b, h, W, grad_dtype=torch.float32, form=form)
     # log p = 0 and G = p - 1 = 0 in real arithmetic; fp32 leaves a few ulp
     assert np.abs(logp).max() <= 1e-6 and abs(loss) <= 1e-5
     assert np.abs(dh).max() <= 1e-5 and np.abs(dw).max() <= 1e-5
 
 
-def test_matches_the_two_call_path():
+@pytest.mark.parametrize("form", FORMS)
+def test_matches_the_two_call_path(form):
     b, h, W = synth.random_case(77, 6, 3001, 128, max_prefix=40, max_cont=200, std_w=0.1)
-    logp, dh, dw = _full_check(b, h, W, grad_dtype=torch.float32)
+    logp, dh, dw = _full_check(b, h, W, grad_dtype=torch.float32, form=form)
     g = gpu_pack(b)
     hc, Wc = h.cuda(), W.cuda()
     l2, lse2, _ = B.olive_token_logprob_fwd(hc, Wc, g["targets"], g["rows"], g["n_rows"])
@@ -91,28 +102,43 @@ def test_matches_the_two_call_path():
 
 @pytest.mark.parametrize("slab_rows,grad_dtype", [(256, torch.float32), (384, torch.bfloat16)])
 def test_several_slabs(slab_rows, grad_dtype, monkeypatch):
-    """A lowered slab cap splits ~2.3k masked rows into many slabs: dW
-    accumulates across them (fp32 accumulator for a bf16 output)."""
+    """The slab form with a lowered slab cap splits ~2.3k masked rows into many
+    slabs: dW accumulates across them (fp32 accumulator for a bf16 output)."""
     monkeypatch.setenv("OLIVE_SLAB_ROWS", str(slab_rows))
     rng = np.random.default_rng(slab_rows)
     b = synth.batch_from_lengths(rng, [5, 40, 1], [900, 700, 750], 2000)
     h = synth.normal_bf16(rng, (b.T, 64), 1.0)
     W = synth.normal_bf16(rng, (2000, 64), 0.1)
     assert b.n_mask > 6 * slab_rows
+    _full_check(b, h, W, reduction="mean", grad_dtype=grad_dtype, form="slab")
+
+
+@pytest.mark.parametrize("grad_dtype", [torch.float32, torch.bfloat16])
+def test_many_outer_tiles(grad_dtype):
+    """~2.3k masked rows, d = 4096, V = 2000 on the on-chip form: groups of 16
+    CTAs, 19 row tiles (pass A) and 16 vocabulary tiles (pass B) over 9
+    groups, so groups run several outer tiles in both passes, the exchange
+    ring wraps many times and the last vocabulary tile is partial."""
+    rng = np.random.default_rng(991)
+    b = synth.batch_from_lengths(rng, [5, 40, 1], [900, 700, 750], 2000)
+    h = synth.rms_hidden_bf16(rng, (b.T, 4096))
+    W = synth.normal_bf16(rng, (2000, 4096), 0.03)
     _full_check(b, h, W, reduction="mean", grad_dtype=grad_dtype)
 
 
-def test_empty_mask():
+@pytest.mark.parametrize("form", FORMS)
+def test_empty_mask(form):
     rng = np.random.default_rng(22)
     b = synth.batch_from_lengths(rng, [9, 4], [0, 0], 300)
     h = synth.normal_bf16(rng, (b.T, 64), 1.0)
     W = synth.normal_bf16(rng, (300, 64), 0.1)
-    logp, _, loss, dh, dw = _gpu(b, h, W, reduction="mean")
+    logp, _, loss, dh, dw = _gpu(b, h, W, reduction="mean", form=form)
     assert loss == 0.0 and not logp.any() and not dh.any() and not dw.any()
 
 
+@pytest.mark.parametrize("form", FORMS)
 @pytest.mark.parametrize("spike", [0.2, 0.5])
-def test_rows_far_above_their_first_tile(spike):
+def test_rows_far_above_their_first_tile(spike, form):
     """Each row's stored e' = 2^(x - R) is relative to the maximum R over the
     row's first 256 vocabulary entries.  Here one id far down the vocabulary
     (1000) has a logit 31-39 nats (spike 0.2: e' up to ~2^57, the scaled form)
@@ -131,10 +157,11 @@ def test_rows_far_above_their_first_tile(spike):
     z = oracle.logits(to_f64(h), to_f64(W), 1.0)
     gap = (z.max(axis=1) - z[:, :256].max(axis=1))[::2]
     assert gap.min() > (25 if spike < 0.3 else 75)
-    _full_check(b, h, W, grad_dtype=torch.float32)
+    _full_check(b, h, W, grad_dtype=torch.float32, form=form)
 
 
-def test_confident_rows_keep_their_accuracy():
+@pytest.mark.parametrize("form", FORMS)
+def test_confident_rows_keep_their_accuracy(form):
     """Targets equal to a dominant logit (p_y close to 1): G_y = g (p_y - 1) is
     small and formed from the fp32 target logit (a bf16-rounded p_y would be
     off by up to 2^-9 p_y), so each such row's dH keeps the gradient tolerance
@@ -148,7 +175,7 @@ def test_confident_rows_keep_their_accuracy():
     cont = np.argmax(z[P - 1:P + C - 1], axis=1)          # the target of row P-1+i is cont[i]
     b = synth.Batch(rng.integers(0, V, size=P).astype(np.int32), np.array([0, P], np.int32),
                     cont.astype(np.int32), np.array([0, C], np.int32), V)
-    logp, dh, _ = _full_check(b, h, W, grad_dtype=torch.float32)
+    logp, dh, _ = _full_check(b, h, W, grad_dtype=torch.float32, form=form)
     o = oracle_pack(b)
     rdh, _ = oracle.token_loss_bwd(to_f64(h), to_f64(W), o["targets"], o["rows"])
     conf = [t for t in o["rows"] if -0.3 < logp[t] < -1e-2]
@@ -184,8 +211,9 @@ def test_medium_vocab_sampled():
 @pytest.mark.slow
 def test_fwdbwd_workload_sampled():
     """8 x 4096 tokens, d = 4096, V = 151936 (the timed step's configuration):
-    log-probs, lse and dH on 2048 sampled masked rows, dW through the
-    vocabulary-sum property, dH = 0 off the mask, loss = -sum logp."""
+    log-probs, lse and dH on 2048 sampled masked rows, dW on 40 vocabulary
+    rows against the oracle and through the vocabulary-sum property, dH = 0
+    off the mask, loss = -sum logp."""
     b = synth.make_batch("fwdbwd")
     h = synth.make_hidden("fwdbwd", b.T)
     W = synth.make_weight("fwdbwd")
@@ -200,9 +228,58 @@ def test_fwdbwd_workload_sampled():
     assert rel_frob(dh[rows], ref) <= 1e-2
     off = np.setdiff1d(np.arange(b.T), o["rows"])
     assert not dh[off].any()
+    # dW on 40 vocabulary rows (16 of them targets of sampled rows, the first
+    # and the last id) against the oracle, which forms every masked row's
+    # softmax for them (about 2e13 fp64 flops)
+    V = W.shape[0]
+    rng = np.random.default_rng(8)
+    vocab = np.unique(np.concatenate([o["targets"][rows[:16]], [0, V - 1],
+                                      rng.integers(0, V, size=22)]))
+    refw = oracle.token_loss_bwd_vocab(hf, Wf, o["targets"], o["rows"], vocab)
+    assert rel_frob(dw[vocab], refw) <= 1e-2
     # sum over the vocabulary of dW is sum_r G[r, :] . hc[r] with sum_v G[r, v] = 0
     assert np.abs(dw.astype(np.float64).sum(axis=0)).max() <= 2e-2 * np.abs(dw).sum(axis=0).max()
     assert np.isclose(loss, -logp[o["rows"]].astype(np.float64).sum(), rtol=1e-5)
+
+
+@pytest.mark.slow
+def test_varlen_rows_dw():
+    """The variable-length batch (~528k packed tokens) with N_mask lowered to
+    its first 4096 masked rows (spread over its first sequences): every
+    output of the on-chip step against the oracle, dW on 40 vocabulary rows
+    (targets among them) and dH, log-probs, lse on every one of those rows."""
+    b = synth.make_batch("varlen")
+    h = synth.make_hidden("varlen", b.T)
+    W = synth.make_weight("varlen")
+    n = 4096
+    g = gpu_pack(b)
+    st = g["dev_status"]
+    gl = torch.ones(1, dtype=torch.float32, device="cuda")
+    nr = torch.tensor([n], dtype=torch.int32, device="cuda")
+    logp, lse, loss, dh, dw = B.olive_token_loss_fwd_bwd(h.cuda(), W.cuda(), g["targets"], g["rows"],
+                                                         nr, gl, 1.0, "mean", dev_status=st)
+    torch.cuda.synchronize()
+    assert B.status_bits(st) == []
+    o = oracle_pack(b)
+    rows = o["rows"][:n]
+    sub = torch.from_numpy(rows).cuda()
+    hs = to_f32(h[torch.from_numpy(rows)])
+    ts = o["targets"][rows]
+    local = np.arange(n)
+    Wf = to_f32(W)
+    rl, rs, rloss = oracle.token_logprob(hs, Wf, ts, local, reduction="mean")
+    assert_close_logp(logp[sub].cpu().numpy(), rl)
+    assert_close_logp(lse[sub].cpu().numpy(), rs, "lse")
+    assert_close_loss(float(loss.item()), rloss)
+    ref = oracle.token_loss_bwd_rows(hs, Wf, ts, local, reduction="mean")
+    assert rel_frob(dh[sub].float().cpu().numpy(), ref) <= 1e-2
+    V = W.shape[0]
+    vocab = np.unique(np.concatenate([ts[:20], [0, V - 1], np.random.default_rng(9).integers(0, V, 18)]))
+    refw = oracle.token_loss_bwd_vocab(hs, Wf, ts, local, vocab, reduction="mean")
+    got = dw[torch.from_numpy(vocab).cuda()].float().cpu().numpy()
+    assert rel_frob(got, refw) <= 1e-2
+    rest = torch.from_numpy(o["rows"][n::101]).cuda()
+    assert not dh[rest].any().item()
 
 
 def test_runs_are_bitwise_reproducible():

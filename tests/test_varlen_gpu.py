@@ -2,10 +2,12 @@
 cut at U[10%,90%] of each length (~557k packed tokens, ~278k masked rows),
 d = 4096, V = 151936: splice/pack -> forward -> backward on the GPU, with the
 bf16 inputs drawn by synth; log-probs, lse and dH checked against the oracle
-on 2048 sampled masked rows, the rest by properties that hold at any size.
-The masked rows span many G slabs, so dW goes through the fp32 accumulator.
-The single-pass call (olive_token_loss_fwd_bwd) runs on the same batch and
-must agree."""
+on 2048 sampled masked rows, the rest by properties that hold at any size
+(test_fwd_bwd_gpu.py checks dW on this batch's first 4096 masked rows
+against the oracle).  The one-call step (olive_token_loss_fwd_bwd, G on chip)
+and the slab form (olive_token_loss_fwd_bwd_slab: 15 slabs of 18304 rows, dW
+through the fp32 accumulator) run on the same batch and must agree with the
+two calls."""
 
 import math
 
@@ -64,14 +66,18 @@ def test_varlen_end_to_end():
     off[o["rows"]] = False
     off_idx = torch.from_numpy(np.nonzero(off)[0][::97]).cuda()
     assert not dh[off_idx].any().item()
-    # the single-pass call (15 slabs of 18304 rows here) against the two calls above
-    logp2, lse2, loss2, dh2, dw2 = B.olive_token_loss_fwd_bwd(h.cuda(), Wc, g["targets"], g["rows"],
-                                                              g["n_rows"], gl, reduction="mean",
-                                                              dev_status=st)
-    torch.cuda.synchronize()
-    assert B.status_bits(st) == []
-    assert np.abs(logp2.cpu().numpy()[o["rows"]] - logp[o["rows"]]).max() <= 2e-4
-    assert abs(float(loss2.item()) - float(loss.item())) <= 1e-5 * abs(float(loss.item()))
-    assert rel_frob(dh2[sub].float().cpu().numpy(), ref) <= 1e-2
-    assert (dh2.float() - dh.float()).norm().item() <= 5e-3 * dh.float().norm().item()
-    assert (dw2.float() - dw.float()).norm().item() <= 5e-3 * dw.float().norm().item()
+    # the one-call step and the slab form against the two calls above
+    hd = h.cuda()
+    for slab in (False, True):
+        logp2, lse2, loss2, dh2, dw2 = B.olive_token_loss_fwd_bwd(hd, Wc, g["targets"], g["rows"],
+                                                                  g["n_rows"], gl, reduction="mean",
+                                                                  dev_status=st, slab=slab)
+        torch.cuda.synchronize()
+        assert B.status_bits(st) == []
+        assert np.abs(logp2.cpu().numpy()[o["rows"]] - logp[o["rows"]]).max() <= 2e-4
+        assert abs(float(loss2.item()) - float(loss.item())) <= 1e-5 * abs(float(loss.item()))
+        assert rel_frob(dh2[sub].float().cpu().numpy(), ref) <= 1e-2
+        assert (dh2.float() - dh.float()).norm().item() <= 5e-3 * dh.float().norm().item()
+        assert (dw2.float() - dw.float()).norm().item() <= 5e-3 * dw.float().norm().item()
+        del logp2, lse2, loss2, dh2, dw2
+        torch.cuda.empty_cache()
