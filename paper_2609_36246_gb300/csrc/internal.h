@@ -41,6 +41,9 @@ bool set_smem_once(const void* func, int smem, int device, std::atomic<int>* don
 // bytes) with 128-byte swizzle and the given box.  Returns false on failure.
 bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
                     uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer);
+// The same without swizzling (a box lands in shared memory row after row).
+bool encode_bf16_2d_plain(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+                          uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer);
 
 // Rows of the G slab used by the backward passes for vocabulary size V.
 int64_t slab_rows(int64_t Tpad, int64_t V);

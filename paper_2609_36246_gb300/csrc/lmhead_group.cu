@@ -70,9 +70,9 @@ constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kBM = 128;
 constexpr int kBK = 64;
 constexpr int kZN = 256;             // logit tile 128 x 256
-constexpr int kStages = 4;
-constexpr int kSA = kBM * kBK * 2;   // A operand of a stage: 128 x 64 bf16
-constexpr int kSB = kZN * kBK * 2;   // B operand: 256 x 64 (Z job) or 64 x <= 256 (accumulation)
+constexpr int kStages = 6;
+constexpr int kSA = kBM * kBK * 2;   // A operand of a stage: this CTA's 128 rows x 64
+constexpr int kSB = kBM * kBK * 2;   // B operand: this CTA's half of N (<= 128) x 64
 constexpr int kStageBytes = kSA + kSB;
 constexpr int kXSlice = kSA;         // one 128 x 64 K-slice of an exchange tile
 constexpr int kXTile = 4 * kXSlice;  // 128 x 256 bf16 (64 KB)
@@ -95,10 +95,12 @@ constexpr uint32_t kPaceDone = 0x40000000u;
 
 enum GMode : int { GM_REF = 0, GM_A = 1, GM_B = 2 };
 
-// GM_REF / GM_A: za = hc {64 x 128}, zb = W {64 x 256}, xb = W {64 x 64}
-// GM_B:          za = W {64 x 128},  zb = hc {64 x 256}, xb = hc {64 x 64}
+// GM_REF / GM_A: za = hc {64 x 128}, zb = W {64 x 128}, xb = W {64 x 64}
+// GM_B:          za = W {64 x 128},  zb = hc {64 x 128}, xb = hc {64 x 64}
+// xa: the ring, [slices x 128 rows] of 64 bf16, unswizzled {64 x 128} boxes
+// (a slice is stored already swizzled, so the copy is linear)
 struct GroupMaps {
-  CUtensorMap za, zb, xb;
+  CUtensorMap za, zb, xb, xa;
 };
 
 struct GroupParams {
@@ -142,6 +144,8 @@ struct GroupParams {
 // per-CTA schedule, the same in every CTA of a group
 struct GSched {
   int n;      // masked rows
+  int rank;   // 0: the pair's even CTA (issues the MMAs), 1: its peer
+  int ph;     // outer index standing for "no outer tile" (past the last)
   int no;     // outer tiles in all
   int ni;     // inner tiles per outer tile
   int nk;     // 64-wide K steps of a Z job
@@ -149,36 +153,51 @@ struct GSched {
   int myo;    // outer tiles of this group
   int E;      // exchange tiles of this group
   int c0, cw; // output columns of this member
-  int nbox;   // 64-column boxes of the accumulation's B operand
+  int nbox;   // 64-column boxes of this CTA's half of the accumulation's B
   int nacc;   // N of the accumulation MMA (cw rounded up to 16)
+  int b0;     // first column of this CTA's half of B
   int kcount; // inner extent: V (pass A) or n (pass B)
   float coef;
 };
 
+// CTAs come in pairs (clusters of 2): pair-group pg of g pairs runs groups
+// 2 pg (even CTAs) and 2 pg + 1 (odd CTAs) in lockstep, pair m being member m
+// of both; the two groups walk the same inner tiles at the same time, so
+// each pair's MMAs share the B operand (W or hc tiles), half from each CTA.
 __device__ GSched make_gsched(const GroupParams& p) {
   GSched s;
   s.n = read_n_rows(p.n_rows, p.T, p.dev_status);
+  s.rank = static_cast<int>(cluster_rank());
   const int rt = (s.n + kBM - 1) / kBM;
   if (p.mode == GM_B) {
     s.no = (p.V + kBM - 1) / kBM;
+    s.ph = s.no;
     s.ni = (s.n + kZN - 1) / kZN;
     s.kcount = s.n;
   } else {
     s.no = (p.mode == GM_A && p.redo) ? static_cast<int>(min(p.redo_list[0], static_cast<uint32_t>(rt))) : rt;
+    s.ph = rt;
     s.ni = p.mode == GM_REF ? 1 : (p.V + kZN - 1) / kZN;
     s.kcount = p.V;
   }
   s.nk = (p.d + kBK - 1) / kBK;
-  s.q = blockIdx.x / p.g;
-  s.m = blockIdx.x % p.g;
-  s.myo = s.q < s.no ? (s.no - s.q + p.ngroups - 1) / p.ngroups : 0;
+  const int pair = blockIdx.x >> 1;
+  s.m = pair % p.g;
+  const int pg = pair / p.g;
+  s.q = 2 * pg + s.rank;
+  // both groups of a pair-group run as many outer tiles as the even one
+  // (which has at least as many); the odd one's extra tile, if any, is a
+  // phantom whose rows are invalid
+  const int qe = 2 * pg;
+  s.myo = qe < s.no ? (s.no - qe + p.ngroups - 1) / p.ngroups : 0;
   s.E = s.myo * s.ni;
   s.c0 = p.c_base + s.m * p.chunk;
   s.cw = min(p.chunk, p.c_end - s.c0);
   if (s.cw < 0) s.cw = 0;
-  s.nbox = (s.cw + 63) / 64;
   s.nacc = (s.cw + 15) / 16 * 16;
   if (s.nacc < 16) s.nacc = 16;
+  s.b0 = s.c0 + s.rank * (s.nacc / 2);
+  s.nbox = (s.nacc / 2 + 63) / 64;
   s.coef = 0.f;
   if (p.grad_loss) {
     float gl = *p.grad_loss;
@@ -188,9 +207,13 @@ __device__ GSched make_gsched(const GroupParams& p) {
   return s;
 }
 
-// global index of the group's i-th outer tile
+// global index of the group's i-th outer tile (s.ph for a phantom)
+__device__ __forceinline__ bool phantom(const GroupParams& p, const GSched& s, int i) {
+  return s.q + i * p.ngroups >= s.no;
+}
 __device__ __forceinline__ int outer_of(const GroupParams& p, const GSched& s, int i) {
   const int k = s.q + i * p.ngroups;
+  if (k >= s.no) return s.ph;
   return (p.mode == GM_A && p.redo) ? static_cast<int>(p.redo_list[1 + k]) : k;
 }
 __device__ __forceinline__ int kvalid_of(const GSched& s, int k) {
@@ -328,6 +351,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (base - raw);
 
+  // the same layout in both CTAs of a pair: the MMA reads both at these offsets
   const uint32_t stages = base;
   const uint32_t bar0 = base + kStages * kStageBytes;
   auto full_bar = [&](int st) { return bar0 + 8u * st; };
@@ -347,16 +371,17 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
 
   if (threadIdx.x == 0) {
     for (int st = 0; st < kStages; ++st) {
-      mbar_init(full_bar(st), 1);
-      mbar_init(empty_bar(st), 1);
+      mbar_init(full_bar(st), 1);   // the even CTA's producer (both CTAs' bytes)
+      mbar_init(empty_bar(st), 1);  // the even CTA's MMA commit (multicast)
     }
     mbar_init(zfull, 1);
-    mbar_init(zempty, kEpi);
+    mbar_init(zempty, 8);           // the four epilogue warps of both CTAs
     mbar_init(ofull, 1);
-    mbar_init(oempty, kEpi);
+    mbar_init(oempty, 8);
     mbar_init(drain, 1);
     *abort_flag = 0;
     *copied = 0;
@@ -367,13 +392,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     tma_prefetch_desc(&maps.za);
     tma_prefetch_desc(&maps.zb);
     tma_prefetch_desc(&maps.xb);
+    tma_prefetch_desc(&maps.xa);
   }
   if (warp == kMmaWarp) {
-    tmem_alloc(smem_u32(tmem_slot), 512);
-    tmem_relinquish();
+    tmem_alloc_pair(smem_u32(tmem_slot), 512);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
-  __syncthreads();
+  // barriers of both CTAs initialised and TMEM allocated before any CTA
+  // touches its peer's
+  cluster_sync_all();
   tc_fence_after();
 
   const uint32_t tmem_base = *tmem_slot;
@@ -383,16 +411,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   const bool consume = p.mode != GM_REF;
   const int nr = (s.E + g - 1) / g;  // rounds
   const size_t ring0 = static_cast<size_t>(s.q) * p.R;
-  uint8_t* ring_bytes = reinterpret_cast<uint8_t*>(p.ring);
 
   if (warp == kProducerWarp) {
-    // lane 0 issues every copy; the whole warp checks the `ready` flags of a
-    // round's g exchange tiles at once (one L2 round trip per round instead
-    // of one blocking acquire per tile, which left the stage ring empty)
+    // lane 0 issues every copy (this CTA's 128 rows of A and its half of B;
+    // completion counted on the even CTA's full barrier, whose producer
+    // announces both CTAs' bytes: the odd CTA's copies may land first, the
+    // transaction count then dips below zero within the phase, which mbarriers
+    // allow; no phase can mix with the next, since a CTA refills a stage only
+    // after the MMAs that read it have committed); the whole warp checks the
+    // `ready` flags of a round's g exchange tiles at once
     int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
-    const bool paced = consume && p.ngroups > 1;
+    const bool paced = consume && p.ngroups > 2;
     for (int r = 0; ok && r <= nr; ++r) {
       const int j = r * g + s.m;
       if (paced && r < nr) {
@@ -407,10 +438,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int ks = 0; ks < s.nk; ++ks) {
             if (!mbar_wait(empty_bar(stage), phase ^ 1u, ctl)) { ok = false; break; }
             const uint32_t sA = stages + stage * kStageBytes;
-            const uint32_t fb = full_bar(stage);
-            mbar_arrive_expect_tx(fb, kStageBytes);
-            tma_load_2d(sA, &maps.za, fb, ks * kBK, o * kBM);
-            tma_load_2d(sA + kSA, &maps.zb, fb, ks * kBK, k * kZN);
+            const uint32_t fb = map_shared(full_bar(stage), 0);
+            if (rank == 0) mbar_arrive_expect_tx(full_bar(stage), 2 * kStageBytes);
+            tma_load_2d_pair(sA, &maps.za, fb, ks * kBK, o * kBM);
+            tma_load_2d_pair(sA + kSA, &maps.zb, fb, ks * kBK, k * kZN + static_cast<int>(rank) * kBM);
             if (++stage == kStages) { stage = 0; phase ^= 1u; }
           }
         }
@@ -427,15 +458,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int slot = e % p.R;
           const int k = e % s.ni;
           const int nsl = slices_of(s, k);
-          const uint8_t* img = ring_bytes + (ring0 + slot) * static_cast<size_t>(kXTile);
           for (int sl = 0; sl < nsl; ++sl) {
             if (!mbar_wait(empty_bar(stage), phase ^ 1u, ctl)) { ok = false; break; }
             const uint32_t sA = stages + stage * kStageBytes;
-            const uint32_t fb = full_bar(stage);
-            mbar_arrive_expect_tx(fb, kXSlice + s.nbox * 8192);
-            bulk_load(sA, img + sl * kXSlice, kXSlice, fb);
+            const uint32_t fb = map_shared(full_bar(stage), 0);
+            if (rank == 0) mbar_arrive_expect_tx(full_bar(stage), 2 * (kXSlice + s.nbox * 8192));
+            tma_load_2d_pair(sA, &maps.xa, fb, 0, static_cast<int>(((ring0 + slot) * 4 + sl) * kBM));
             for (int b = 0; b < s.nbox; ++b)
-              tma_load_2d(sA + kSA + b * 8192, &maps.xb, fb, s.c0 + 64 * b, k * kZN + sl * kBK);
+              tma_load_2d_pair(sA + kSA + b * 8192, &maps.xb, fb, s.b0 + 64 * b, k * kZN + sl * kBK);
             if (++stage == kStages) { stage = 0; phase ^= 1u; }
           }
         }
@@ -450,13 +480,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncwarp();
   } else if (warp == kSignalWarp) {
-    // for every exchange tile, in order, once the MMA warp has seen all its
-    // slices land: one release increment of the slot's `cons` count
+    // for every exchange tile, in order, once the pair's MMA thread has seen
+    // all its slices land: one release increment of the slot's `cons` count
     if (lane == 0 && consume) {
       uint32_t sent = 0;
       const uint32_t total = static_cast<uint32_t>(s.E);
-      const uint64_t t0 = global_timer_ns();
-      uint64_t last = t0;
+      uint64_t last = global_timer_ns();
       while (sent < total) {
         const uint32_t c = *copied;
         if (c > sent) {
@@ -474,11 +503,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncwarp();
   } else if (warp == kMmaWarp) {
-    if (lane == 0) {
+    // the even CTA's lane 0 issues the pair's MMAs (M = 256: 128 rows in each
+    // CTA's TMEM); the odd CTA's MMA warp only holds its TMEM allocation
+    if (lane == 0 && rank == 0) {
       const uint32_t zacc = tmem_base;
       const uint32_t oacc = tmem_base + 256;
-      const uint32_t idz = idesc_bf16(kBM, kZN, false, false);
-      const uint32_t idx = idesc_bf16(kBM, s.nacc, false, true);
+      const uint32_t idz = idesc_bf16(2 * kBM, kZN, false, false);
+      const uint32_t idx = idesc_bf16(2 * kBM, s.nacc, false, true);
+      const uint32_t copied_peer = map_shared(smem_u32(const_cast<uint32_t*>(copied)), 1);
       int stage = 0;
       uint32_t phase = 0, zph = 0, oph = 0;
       bool ok = true;
@@ -494,13 +526,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t sB = sA + kSA;
 #pragma unroll
             for (int kk = 0; kk < kBK / 16; ++kk)
-              umma_bf16(zacc, sdesc_sw128(sA + kk * 32, 16, 1024), sdesc_sw128(sB + kk * 32, 16, 1024),
-                        idz, (ks > 0 || kk > 0) ? 1u : 0u);
-            umma_commit(empty_bar(stage));
+              umma_bf16_pair(zacc, sdesc_sw128(sA + kk * 32, 16, 1024), sdesc_sw128(sB + kk * 32, 16, 1024),
+                             idz, (ks > 0 || kk > 0) ? 1u : 0u);
+            umma_commit_pair(empty_bar(stage));
             if (++stage == kStages) { stage = 0; phase ^= 1u; }
           }
           if (!ok) break;
-          umma_commit(zfull);
+          umma_commit_pair(zfull);
           zph ^= 1u;
         }
         if (!consume || r == 0) continue;
@@ -519,26 +551,27 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t sB = sA + kSA;
 #pragma unroll
             for (int kk = 0; kk < kBK / 16; ++kk)
-              umma_bf16(oacc, sdesc_sw128(sA + kk * 32, 16, 1024),
-                        sdesc_sw128(sB + kk * 2048, 8192, 1024), idx,
-                        (k > 0 || sl > 0 || kk > 0) ? 1u : 0u);
-            umma_commit(empty_bar(stage));
+              umma_bf16_pair(oacc, sdesc_sw128(sA + kk * 32, 16, 1024),
+                             sdesc_sw128(sB + kk * 2048, 8192, 1024), idx,
+                             (k > 0 || sl > 0 || kk > 0) ? 1u : 0u);
+            umma_commit_pair(empty_bar(stage));
             if (++stage == kStages) { stage = 0; phase ^= 1u; }
           }
           if (!ok) break;
-          // every slice of tile e has landed in shared memory: the signal
-          // warp tells the group (its slot may be rewritten once all members
-          // have said so)
+          // every slice of tile e has landed in both CTAs: their signal warps
+          // tell the two groups (a slot may be rewritten once all of its
+          // group's members have said so)
           *copied = static_cast<uint32_t>(e + 1);
+          st_shared_cluster(copied_peer, static_cast<uint32_t>(e + 1));
           if (k == s.ni - 1) {
-            umma_commit(ofull);
+            umma_commit_pair(ofull);
             oph ^= 1u;
           }
         }
       }
       // arrives once every MMA issued above has completed (bounded wait that
       // ignores the abort flag: it only waits for work already in flight)
-      umma_commit(drain);
+      umma_commit_pair(drain);
       volatile int keep_waiting = 0;
       const uint64_t floor_ns = 200ull * 1000 * 1000;
       const WaitCtl own{&keep_waiting, p.wait_limit_ns > floor_ns ? p.wait_limit_ns : floor_ns};
@@ -549,6 +582,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     // epilogue warps 0..3: thread = accumulator row = TMEM lane
     const int row = warp * 32 + lane;
     const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(warp * 32) << 16);
+    uint8_t* ring_bytes = reinterpret_cast<uint8_t*>(p.ring);
+    // the even CTA's MMA thread waits until both CTAs' epilogues are done with
+    // an accumulator: one arrival per epilogue warp on its barriers
+    const uint32_t zempty_lead = map_shared(zempty, 0);
+    const uint32_t oempty_lead = map_shared(oempty, 0);
     const uint32_t zaddr = lane_addr;
     const uint32_t oaddr = lane_addr + 256;
     uint32_t zph = 0, oph = 0;
@@ -670,7 +708,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         tc_fence_before();
-        mbar_arrive(zempty);
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(zempty_lead);
         if (p.mode == GM_REF) {
           if (o * kBM + row < s.n) p.rref[o * kBM + row] = run_m;
         } else {
@@ -710,7 +749,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                           min(32, s.cw - c), ov);
           }
           tc_fence_before();
-          mbar_arrive(oempty);
+          __syncwarp();
+          if (lane == 0) mbar_arrive_cluster(oempty_lead);
           continue;
         }
         // pass A: merge the members' partials, then dH
@@ -722,12 +762,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           p.part_s[static_cast<size_t>(s.m) * Tpad + rc] = 0.f;
           p.part_m[static_cast<size_t>(s.m) * Tpad + rc] = -INFINITY;
         }
-        __threadfence();
-        named_bar_sync(1, kEpi);
-        if (threadIdx.x == 0) red_release_add(p.outer_ctr + o, 1u);
-        const bool seen =
-            threadIdx.x == 0 ? wait_counter(p.outer_ctr + o, static_cast<uint32_t>(g), ctl) : true;
-        if (!named_bar_and(1, kEpi, seen)) { ok = false; break; }
+        if (!phantom(p, s, i)) {
+          __threadfence();
+          named_bar_sync(1, kEpi);
+          if (threadIdx.x == 0) red_release_add(p.outer_ctr + o, 1u);
+          const bool seen =
+              threadIdx.x == 0 ? wait_counter(p.outer_ctr + o, static_cast<uint32_t>(g), ctl) : true;
+          if (!named_bar_and(1, kEpi, seen)) { ok = false; break; }
+        }
         if (!named_bar_and(1, kEpi, mbar_wait(ofull, oph, ctl))) { ok = false; break; }
         oph ^= 1u;
         tc_fence_after();
@@ -802,17 +844,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         tc_fence_before();
-        mbar_arrive(oempty);
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(oempty_lead);
       }
     }
   }
 
   tc_fence_before();
-  __syncthreads();
+  // the pair's MMAs (all complete: the even CTA waited for them) and every
+  // access to the peer's barriers are over before either CTA frees its TMEM
+  cluster_sync_all();
   if (threadIdx.x == 0 && *abort_flag) atomicOr(p.dev_status, kStatusTimeoutBit);
   if (warp == kMmaWarp) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, 512);
+    tmem_dealloc_pair(tmem_base, 512);
   }
 }
 
@@ -821,37 +866,59 @@ static_assert(kGroupSmem <= 227 * 1024, "shared memory budget");
 
 int ring_slots_for(int g) { return 3 * g > 4 ? 3 * g : 4; }
 
-// groups of ceil(cols / 256) members, as many as `sms` SMs hold
+// fewest members a group of `cols` output columns can have, and the most the
+// shape search below may pick
+int g_min_for(int cols) { return cols > kZN ? (cols + kZN - 1) / kZN : 1; }
+int g_hi_for(int cols) { return g_min_for(cols) + g_min_for(cols) / 4 + 1; }
+
+// Groups of g members, run as pair-groups of 2 g CTAs.  g is the member count
+// between ceil(cols / 256) and ~1.25 times that which puts the most CTAs to
+// work (d = 4096 at 152 SMs: g = 19, four pair-groups fill all 152), the
+// smaller g on ties; members hold ceil(cols / g) columns rounded up to 16.
 struct GroupShape {
   int g, chunk, ngroups, R;
 };
 
 GroupShape group_shape(int cols, int sms) {
-  GroupShape gs;
-  gs.g = (cols + kZN - 1) / kZN;
-  if (gs.g < 1) gs.g = 1;
+  GroupShape gs{0, 0, 0, 0};
+  int best_used = 0;
+  for (int g = g_min_for(cols); g <= g_hi_for(cols); ++g) {
+    const int used = 2 * g * (sms / (2 * g));
+    if (used > best_used) {
+      best_used = used;
+      gs.g = g;
+    }
+  }
+  if (gs.g == 0) return gs;
   gs.chunk = ((cols + gs.g - 1) / gs.g + 15) / 16 * 16;
-  gs.ngroups = sms / gs.g;
+  gs.ngroups = 2 * (sms / (2 * gs.g));
   gs.R = ring_slots_for(gs.g);
   return gs;
 }
 
+// output columns one sweep covers: the widest whose fewest members still
+// form one pair-group
+int sweep_cols_for(int sms) { return (sms / 2) * kZN; }
+
 }  // namespace
 
-// widest group a launch forms (ring and counters are sized for it)
+// the widest group a launch may form for width d (ring and partials are
+// sized for it)
 int group_g_max(int64_t d) {
-  const int64_t cols = d < static_cast<int64_t>(kGroupMaxSms) * kZN ? d : static_cast<int64_t>(kGroupMaxSms) * kZN;
-  return static_cast<int>((cols + kZN - 1) / kZN);
+  const int64_t cap = static_cast<int64_t>(sweep_cols_for(kGroupMaxSms));
+  return g_hi_for(static_cast<int>(d < cap ? d : cap));
 }
 
 int ring_slots(int g) { return ring_slots_for(g); }
 
-// groups a launch forms at most: as many as the SMs hold, and no more than
-// the outer tiles of either pass (row tiles of T rows, vocabulary tiles)
+// groups a launch forms at most (an even number): as many as the SMs hold,
+// and no more than the outer tiles of either pass (row tiles of T rows,
+// vocabulary tiles) rounded up to a pair
 int group_count_max(int64_t T, int64_t d, int64_t V) {
-  const int g = group_g_max(d);
-  const int64_t outer = std::max(ceil_div(T, kBM), ceil_div(V, kBM));
-  return static_cast<int>(std::min<int64_t>(kGroupMaxSms / g, std::max<int64_t>(outer, 1)));
+  const int64_t cap = static_cast<int64_t>(sweep_cols_for(kGroupMaxSms));
+  const int gmin = g_min_for(static_cast<int>(d < cap ? d : cap));
+  const int64_t outer = std::max<int64_t>(std::max(ceil_div(T, kBM), ceil_div(V, kBM)), 2);
+  return static_cast<int>(std::min<int64_t>(2 * (kGroupMaxSms / (2 * gmin)), (outer + 1) / 2 * 2));
 }
 
 size_t group_ring_words(int64_t T, int64_t d, int64_t V) {
@@ -865,7 +932,7 @@ size_t group_ctr_words(int64_t T, int64_t d, int64_t V) {
   return 2 * group_ring_words(T, d, V) + static_cast<size_t>(group_count_max(T, d, V));
 }
 
-int group_sweep_cols(int sms) { return (sms < kGroupMaxSms ? sms : kGroupMaxSms) * kZN; }
+int group_sweep_cols(int sms) { return sweep_cols_for(sms < kGroupMaxSms ? sms : kGroupMaxSms); }
 
 olive_status launch_group(const Ctx& c, int mode, const void* hc, const void* W, int32_t T,
                           int32_t d, int32_t V, const GroupArgs& a, int c_base, int c_end,
@@ -876,12 +943,12 @@ olive_status launch_group(const Ctx& c, int mode, const void* hc, const void* W,
   if (mode == GM_REF) {
     gs.g = 1;
     gs.chunk = kZN;
-    gs.ngroups = sms;
+    gs.ngroups = sms / 2 * 2;
     gs.R = 1;
   } else {
     gs = group_shape(c_end - c_base, sms);
     gs.ngroups = std::min(gs.ngroups, group_count_max(T, d, V));
-    if (gs.ngroups < 1) return OLIVE_ERR_SHAPE;
+    if (gs.ngroups < 2 || gs.g * gs.ngroups > sms) return OLIVE_ERR_SHAPE;
   }
   GroupMaps maps;
   const bool rowsA = mode != GM_B;
@@ -889,9 +956,12 @@ olive_status launch_group(const Ctx& c, int mode, const void* hc, const void* W,
   const void* zbBase = rowsA ? W : hc;
   const uint64_t zaRows = rowsA ? Tpad : V;
   const uint64_t zbRows = rowsA ? V : Tpad;
+  // the ring viewed as rows of 64 bf16 (one 128-byte row of a slice image)
+  const uint64_t ring_rows = group_ring_bytes(T, d, V) / 128;
   if (!encode_bf16_2d(&maps.za, zaBase, d, zaRows, 2ull * d, 64, 128) ||
-      !encode_bf16_2d(&maps.zb, zbBase, d, zbRows, 2ull * d, 64, 256) ||
-      !encode_bf16_2d(&maps.xb, zbBase, d, zbRows, 2ull * d, 64, 64))
+      !encode_bf16_2d(&maps.zb, zbBase, d, zbRows, 2ull * d, 64, 128) ||
+      !encode_bf16_2d(&maps.xb, zbBase, d, zbRows, 2ull * d, 64, 64) ||
+      !encode_bf16_2d_plain(&maps.xa, a.ring, 64, ring_rows, 128, 64, 128))
     return OLIVE_ERR_CUDA;
 
   GroupParams p = {};
@@ -945,12 +1015,17 @@ olive_status launch_group(const Ctx& c, int mode, const void* hc, const void* W,
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = kGroupSmem;
   cfg.stream = c.stream;
-  // members of a group wait on one another: every CTA must be resident
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeCooperative;
-  attr[0].val.cooperative = 1;
+  // clusters of two CTAs (the MMA pairs); members of a group wait on one
+  // another, so every CTA must be resident: a cooperative launch
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeCooperative;
+  attr[1].val.cooperative = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = mode == GM_REF ? 0 : 1;
+  cfg.numAttrs = mode == GM_REF ? 1 : 2;
   if (cudaLaunchKernelEx(&cfg, lmhead_group_kernel, maps, p) != cudaSuccess) {
     cudaGetLastError();
     return OLIVE_ERR_CUDA;

@@ -74,8 +74,9 @@ bool set_smem_once(const void* func, int smem, int device, std::atomic<int>* don
   return true;
 }
 
-bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
-                    uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
+static bool encode_bf16_2d_swz(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+                               uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer,
+                               CUtensorMapSwizzle swz) {
   auto fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {inner, outer};
@@ -83,10 +84,21 @@ bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t
   cuuint32_t box[2] = {box_inner, box_outer};
   cuuint32_t estr[2] = {1, 1};
   const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
-                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+
+bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+                    uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
+  return encode_bf16_2d_swz(map, base, inner, outer, row_bytes, box_inner, box_outer,
+                            CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
+bool encode_bf16_2d_plain(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+                          uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
+  return encode_bf16_2d_swz(map, base, inner, outer, row_bytes, box_inner, box_outer,
+                            CU_TENSOR_MAP_SWIZZLE_NONE);
 }
 
 int64_t slab_rows(int64_t Tpad, int64_t V) {
