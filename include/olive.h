@@ -35,9 +35,20 @@
  *
  * Conventions shared by every call
  *   - Every pointer argument is a DEVICE pointer unless stated otherwise.  The
- *     caller owns every buffer; the library allocates no device memory and
- *     keeps no state between calls.  Scratch memory comes from the caller's
- *     `workspace` (size from olive_workspace_size, 256-byte aligned).
+ *     caller owns every buffer; no call allocates device memory.  Scratch
+ *     memory comes from the caller's `workspace` (size from
+ *     olive_workspace_size, 256-byte aligned).  Three things outlive a call:
+ *     the OLIVE_NOALLOC_SCRATCH_BYTES array that olive_token_logprob_fwd_noalloc
+ *     uses (compiled into the library, held by every GPU that loads it); the
+ *     per-device kernel attributes (shared-memory limits), set on the first
+ *     call on each device so that later calls issue no attribute call and can
+ *     be captured in a CUDA graph; and three environment variables:
+ *     OLIVE_WAIT_LIMIT_MS (wall-clock limit of every internal wait, default
+ *     1000; on expiry the call sets OLIVE_ERR_TIMEOUT) and OLIVE_SLAB_ROWS
+ *     (lowers the slab of the slab forms, see olive_slab_rows), both read at
+ *     each call, and OLIVE_NONCOOPERATIVE=1, read on first use (launches the
+ *     on-chip training step without the cooperative attribute, for profilers
+ *     that cannot replay cooperative cluster launches).
  *   - `stream` is a cudaStream_t (NULL = legacy default stream).  All calls
  *     are asynchronous on it; none synchronises the host.
  *   - The returned olive_status covers what the host can check before any
@@ -93,6 +104,17 @@ enum { OLIVE_OP_LOGPROB_FWD = 0, OLIVE_OP_LOSS_BWD = 1, OLIVE_OP_DIVERGENCE = 2,
        OLIVE_OP_TOPK_FWD = 3, OLIVE_OP_SPLICE_MASKED = 4, OLIVE_OP_TOPK_KL_BWD = 5,
        OLIVE_OP_LOSS_FWD_BWD = 6, OLIVE_OP_OPD_STATS = 7, OLIVE_OP_TOPK_KL_FWD_BWD = 8,
        OLIVE_OP_LOSS_FWD_BWD_SLAB = 9 };
+
+/*
+ * Rows of the G slab that the slab forms (olive_token_loss_fwd_bwd_slab,
+ * olive_topk_kl_bwd, olive_topk_kl_fwd_bwd, and the divergence gradient of
+ * olive_token_divergence) hold at a time for T packed rows and V vocabulary
+ * entries: about 5.6 GB of bf16 G in whole 128-row tiles, at most 32768 rows
+ * and at most T rounded up to 128, lowered by OLIVE_SLAB_ROWS (a multiple of
+ * 128).  A call on more masked rows runs ceil(N_mask / rows) slabs.  Returns 0
+ * for T < 1 or V < 1.  The paper has no counterpart.
+ */
+OLIVE_API int32_t olive_slab_rows(int32_t T, int32_t V);
 
 /* ABI version of the loaded library (OLIVE_ABI_VERSION). */
 OLIVE_API int olive_abi_version(void);

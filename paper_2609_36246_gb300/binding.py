@@ -56,6 +56,8 @@ def lib() -> ctypes.CDLL:
     L = ctypes.CDLL(LIB_PATH)
     L.olive_abi_version.restype = ctypes.c_int
     L.olive_abi_version.argtypes = []
+    L.olive_slab_rows.restype = _I
+    L.olive_slab_rows.argtypes = [_I, _I]
     L.olive_status_string.restype = ctypes.c_char_p
     L.olive_status_string.argtypes = [ctypes.c_int]
     L.olive_workspace_size.restype = _S
@@ -152,18 +154,10 @@ def olive_workspace_size(op: str, T: int, d: int, V: int, d_t: int = 0, grad: bo
     return int(lib().olive_workspace_size(OP[op], T, d, d_t, V, int(grad), DTYPE[grad_dtype]))
 
 
-def slab_rows_for(T: int, V: int) -> int:
-    """Rows of one G slab for a call with T packed rows and V vocabulary
-    entries: the library's rule (about 5.6 GB of bf16 G, whole 128-row tiles,
-    at most 32768 rows and at most T rounded up to 128, lowered by
-    OLIVE_SLAB_ROWS).  Used to count the launches of a call."""
-    vpad = (V + 7) // 8 * 8
-    tc = max(128, 5_600_000_000 // (2 * vpad) // 128 * 128)
-    tc = min(tc, 32768)
-    cap = int(os.environ.get("OLIVE_SLAB_ROWS", "0") or 0)
-    if cap >= 128 and cap % 128 == 0 and cap < tc:
-        tc = cap
-    return min(tc, (T + 127) // 128 * 128)
+def olive_slab_rows(T: int, V: int) -> int:
+    """Rows of one G slab of the slab forms for T packed rows and V vocabulary
+    entries (the library's rule, OLIVE_SLAB_ROWS included)."""
+    return int(lib().olive_slab_rows(T, V))
 
 
 def workspace(nbytes: int, device=None) -> torch.Tensor:

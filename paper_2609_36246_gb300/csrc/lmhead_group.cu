@@ -7,7 +7,7 @@
 //   dW = G^T . hc    reduces over the masked rows (K = N_mask)
 // Either output tile is [128, d] fp32 for a 128-row M tile: 2 MB at d = 4096,
 // eight SMs' worth of tensor memory, so one SM cannot hold it.  The CTAs are
-// therefore split into GROUPS of g = ceil(d / 256) members.  Member m owns
+// therefore split into GROUPS of g >= ceil(d / 256) members.  Member m owns
 // the output columns [c0, c0 + cw) of d (cw <= 256) and keeps their 128 x cw
 // fp32 accumulator in TMEM for a whole OUTER tile, while the members take
 // turns computing the 128 x 256 logit tiles (Z jobs, K = d) that every member
@@ -15,9 +15,11 @@
 // tile and stores it in its group's ring of R slots of 64 KB; every member
 // bulk-copies each exchange tile, 64 K-columns at a time, into shared memory
 // as the A operand of its accumulating MMA.  The ring has a fixed size (R
-// slots per group, a few tens of MB in all, which stays in the L2), each slot
-// is rewritten once all g members have read it, and no slot outlives R
+// slots per group, a few tens of MB in all, independent of T and V), each
+// slot is rewritten once all g members have read it, and no slot outlives R
 // exchange tiles: the logits and G are never stored as a [rows, V] array.
+// (The ring is read from the L2; its lines are written back to DRAM when the
+// L2 evicts them, about one write of each tile, the size of the exchange.)
 //
 //   Pass A (outer = 128 masked rows, inner = 256-column vocabulary tile):
 //     exchange tile P'[r, v] = 2^(x - R_r), x = z log2(e), R_r a per-row
@@ -42,22 +44,40 @@
 // accumulation), so the training step executes 4 GEMM units of 2 N_mask d V
 // flops for the 3 it counts.
 //
+// CTA pairs: the kernel runs as clusters of two CTAs.  Pair m of pair-group
+// pg is member m of group 2 pg (its even CTA) and of group 2 pg + 1 (its odd
+// CTA); the two groups walk the same inner tiles at the same time, so every
+// MMA is a tcgen05.mma.cta_group::2 issued by the even CTA (M = 256: each CTA
+// holds 128 rows of A -- its own hc, W or exchange rows -- and half of B's N
+// columns, and receives its 128 accumulator rows in its own TMEM).  Each CTA
+// loads 32 KB per 64-deep K step instead of 48 KB, and six stages fit.  The
+// group size g is chosen between ceil(d / 256) and ~1.25 times that to fill
+// the SMs with pair-groups of 2 g CTAs (d = 4096 on 152 SMs: g = 19, members
+// of 224 columns, four pair-groups).  When the even group has one more outer
+// tile than the odd one, the odd CTAs run a phantom tile whose rows are
+// invalid and never stored.
+//
 // Schedule inside a group (every member derives it from N_mask on the
 // device): the exchange tiles of the group's outer tiles form one sequence
 // e = 0 .. E-1 (e = i ni + k for the group's i-th outer tile and inner tile
 // k), cut into rounds of g tiles; tile e is computed by member e mod g and
-// lives in ring slot e mod R.  Each member's tensor pipe runs, per round r:
-// its Z job of round r, then the accumulation of all g tiles of round r - 1,
-// so the epilogue of a Z tile (and the other members' epilogues) overlaps the
-// accumulation MMAs, and a single 256-column Z accumulator suffices next to
-// the 256-column output accumulator (512 TMEM columns).  Waits between
-// members go through global release/acquire counters: a slot's `ready` count
-// (tile written) and `cons` count (tile copied by all g members).  Every
-// dependency points to a tile with a smaller index (a slot is rewritten R >=
-// 2g tiles after its previous use), the launch is cooperative (all CTAs
-// resident), and every wait is bounded (OLIVE_ERR_TIMEOUT on expiry).
+// lives in ring slot e mod R (R = 3 g).  Each pair's tensor pipe runs, per
+// round r: its Z job of round r, then the accumulation of all g tiles of
+// round r - 1, so the epilogue of a Z tile (and the other members'
+// epilogues) overlaps the accumulation MMAs, and a single 256-column Z
+// accumulator suffices next to the (<= 256)-column output accumulator (512
+// TMEM columns).  Waits between members go through global release/acquire
+// counters: a slot's `ready` count (tile written) and `cons` count (tile
+// copied by all g members); the producer warp checks a whole round's ready
+// flags at once and a signal warp posts the cons counts.  Every dependency
+// points to a tile of an earlier round, the launch is cooperative (all CTAs
+// resident), and every wait is bounded (OLIVE_ERR_TIMEOUT on expiry).  A
+// pacing hint keeps the groups within a round of one another, so the inner
+// operand stream (W in pass A, hc in pass B) is fetched from DRAM once for
+// all groups.
 #include <algorithm>
 #include <cmath>
+#include <cstdlib>
 
 #include "sched.cuh"
 #include "sm103.cuh"
@@ -1016,7 +1036,15 @@ olive_status launch_group(const Ctx& c, int mode, const void* hc, const void* W,
   cfg.dynamicSmemBytes = kGroupSmem;
   cfg.stream = c.stream;
   // clusters of two CTAs (the MMA pairs); members of a group wait on one
-  // another, so every CTA must be resident: a cooperative launch
+  // another, so every CTA must be resident: a cooperative launch.
+  // OLIVE_NONCOOPERATIVE=1 drops the cooperative attribute (for profilers
+  // that cannot replay cooperative cluster launches; the grid never exceeds
+  // one CTA per SM, so it is still resident whenever the GPU runs nothing
+  // else, and a wait that outlasts the limit reports OLIVE_ERR_TIMEOUT).
+  static const bool cooperative = [] {
+    const char* e = std::getenv("OLIVE_NONCOOPERATIVE");
+    return !(e && e[0] == '1');
+  }();
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
@@ -1025,7 +1053,7 @@ olive_status launch_group(const Ctx& c, int mode, const void* hc, const void* W,
   attr[1].id = cudaLaunchAttributeCooperative;
   attr[1].val.cooperative = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = mode == GM_REF ? 1 : 2;
+  cfg.numAttrs = (mode == GM_REF || !cooperative) ? 1 : 2;
   if (cudaLaunchKernelEx(&cfg, lmhead_group_kernel, maps, p) != cudaSuccess) {
     cudaGetLastError();
     return OLIVE_ERR_CUDA;

@@ -349,6 +349,11 @@ extern "C" {
 
 int olive_abi_version(void) { return OLIVE_ABI_VERSION; }
 
+int32_t olive_slab_rows(int32_t T, int32_t V) {
+  if (T < 1 || V < 1) return 0;
+  return static_cast<int32_t>(slab_rows(align_up(static_cast<size_t>(T), kRowAlign), V));
+}
+
 const char* olive_status_string(olive_status s) {
   switch (s) {
     case OLIVE_OK: return "ok";

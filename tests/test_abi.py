@@ -63,6 +63,22 @@ def test_workspace_sizes(L):
     assert L.olive_workspace_size(7, T, d, 0, V, 1, 0) == 0
 
 
+def test_slab_rows_rule(L, monkeypatch):
+    """The slab forms' row rule through the ABI: ~5.6 GB of bf16 G in whole
+    128-row tiles, at most 32768 rows and T rounded up to 128, lowered (never
+    raised) by OLIVE_SLAB_ROWS."""
+    V = 151936
+    tc = B.olive_slab_rows(32768, V)
+    assert tc % 128 == 0 and 2 * tc * V <= 5.6e9 < 2 * (tc + 128) * V
+    assert B.olive_slab_rows(100, V) == 128 and B.olive_slab_rows(300, 4096) == 384
+    assert B.olive_slab_rows(10**6, 100) == 32768
+    assert B.olive_slab_rows(0, V) == 0 and B.olive_slab_rows(5, 0) == 0
+    monkeypatch.setenv("OLIVE_SLAB_ROWS", "256")
+    assert B.olive_slab_rows(32768, V) == 256
+    monkeypatch.setenv("OLIVE_SLAB_ROWS", "1000000")
+    assert B.olive_slab_rows(32768, V) == tc
+
+
 def _fake(n=1 << 20):
     # host buffer used only for its (16-byte aligned) address: validation
     # never dereferences it
