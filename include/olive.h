@@ -94,7 +94,9 @@ typedef enum {
   OLIVE_ERR_TIMEOUT = 6,           /* (device) an internal wait ran out       */
   OLIVE_ERR_UNSUPPORTED_DEVICE = 7,/* current device is not sm_103           */
   OLIVE_ERR_CUDA = 8,              /* a CUDA runtime/driver call failed       */
-  OLIVE_ERR_WORKSPACE = 9          /* workspace null, misaligned or too small */
+  OLIVE_ERR_WORKSPACE = 9,         /* workspace null, misaligned or too small */
+  OLIVE_ERR_BOUNDS = 10            /* (device, OLIVE_DEBUG builds only) an index
+                                      check failed; the access was skipped      */
 } olive_status;
 
 enum { OLIVE_REDUCE_SUM = 0, OLIVE_REDUCE_MEAN = 1 };

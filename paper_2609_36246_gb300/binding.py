@@ -23,6 +23,7 @@ STATUS_NAMES = {
     0: "OLIVE_OK", 1: "OLIVE_ERR_INVALID_ARG", 2: "OLIVE_ERR_SHAPE", 3: "OLIVE_ERR_ALIGNMENT",
     4: "OLIVE_ERR_TOKEN_RANGE", 5: "OLIVE_ERR_OFFSETS", 6: "OLIVE_ERR_TIMEOUT",
     7: "OLIVE_ERR_UNSUPPORTED_DEVICE", 8: "OLIVE_ERR_CUDA", 9: "OLIVE_ERR_WORKSPACE",
+    10: "OLIVE_ERR_BOUNDS",
 }
 REDUCE = {"sum": 0, "mean": 1}
 DIRECTION = {"reverse": 0, "forward": 1}
@@ -53,7 +54,20 @@ def lib() -> ctypes.CDLL:
     if not os.path.exists(LIB_PATH):
         raise OliveError(8, f"libolive.so not found at {LIB_PATH}; build it with "
                             "paper_2609_36246_gb300.build.build()")
-    L = ctypes.CDLL(LIB_PATH)
+    _lib = _configure(ctypes.CDLL(LIB_PATH))
+    return _lib
+
+
+def use_library(path: str) -> ctypes.CDLL:
+    """Makes every call of this module go through the library at `path`
+    (e.g. the OLIVE_DEBUG build, paper_2609_36246_gb300.build.build(debug=True))
+    and returns it; use_library(LIB_PATH) goes back to the release build."""
+    global _lib
+    _lib = _configure(ctypes.CDLL(path))
+    return _lib
+
+
+def _configure(L: ctypes.CDLL) -> ctypes.CDLL:
     L.olive_abi_version.restype = ctypes.c_int
     L.olive_abi_version.argtypes = []
     L.olive_slab_rows.restype = _I
@@ -102,7 +116,6 @@ def lib() -> ctypes.CDLL:
     L.olive_token_logprob_fwd_noalloc.restype = ctypes.c_int
     L.olive_token_logprob_fwd_noalloc.argtypes = [_P, _P, _P, _P, _P, _I, _I, _I, _F, ctypes.c_int,
                                                   _P, _P, _P, _P, _P]
-    _lib = L
     return L
 
 
@@ -138,7 +151,7 @@ def new_status(device=None) -> torch.Tensor:
 def status_bits(dev_status: torch.Tensor) -> list[str]:
     """Names of the error bits set in a device status word (synchronises)."""
     v = int(dev_status.item())
-    return [STATUS_NAMES[c] for c in range(1, 10) if v & (1 << c)]
+    return [STATUS_NAMES[c] for c in range(1, 11) if v & (1 << c)]
 
 
 def olive_abi_version() -> int:

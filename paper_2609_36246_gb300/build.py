@@ -3,7 +3,10 @@
 Every ``csrc/*.cu`` file is compiled in parallel with nvcc and linked into
 ``paper_2609_36246_gb300/libolive.so`` next to this file.  Objects go to
 ``paper_2609_36246_gb300/_build/`` (git-ignored).  A source or header newer
-than the library triggers a rebuild.
+than the library triggers a rebuild.  ``build(debug=True)`` makes
+``libolive_debug.so`` (objects in ``_build_debug/``) with -DOLIVE_DEBUG: the
+kernels check indices and copy coordinates on the device and report a failed
+check as OLIVE_ERR_BOUNDS instead of making the access.
 """
 
 from __future__ import annotations
@@ -19,6 +22,8 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libolive.so")
+BUILD_DEBUG = os.path.join(HERE, "_build_debug")
+LIB_DEBUG = os.path.join(HERE, "libolive_debug.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + [
@@ -43,23 +48,28 @@ def _deps():
         glob.glob(os.path.join(CSRC, "*.h"))) + [os.path.join(ROOT, "include", "olive.h"), __file__]
 
 
-def up_to_date() -> bool:
-    if not os.path.exists(LIB):
+def up_to_date(lib: str = LIB) -> bool:
+    if not os.path.exists(lib):
         return False
-    t = os.path.getmtime(LIB)
+    t = os.path.getmtime(lib)
     return all(os.path.getmtime(p) <= t for p in _deps())
 
 
-def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
-    """Compiles and links libolive.so; returns its path."""
-    if not force and up_to_date():
-        return LIB
+def build(force: bool = False, verbose: bool = False, extra_flags=(), debug: bool = False) -> str:
+    """Compiles and links libolive.so (libolive_debug.so with debug=True);
+    returns its path."""
+    lib_out = LIB_DEBUG if debug else LIB
+    build_dir = BUILD_DEBUG if debug else BUILD
+    if debug:
+        extra_flags = (*extra_flags, "-DOLIVE_DEBUG")
+    if not force and up_to_date(lib_out):
+        return lib_out
     nvcc = nvcc_path()
-    os.makedirs(BUILD, exist_ok=True)
+    os.makedirs(build_dir, exist_ok=True)
     srcs = _sources()
 
     def compile_one(src):
-        obj = os.path.join(BUILD, os.path.basename(src)[:-3] + ".o")
+        obj = os.path.join(build_dir, os.path.basename(src)[:-3] + ".o")
         cmd = [nvcc, *NVCC_FLAGS, *extra_flags, "-c", src, "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
@@ -70,7 +80,7 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
 
     with ThreadPoolExecutor(max_workers=min(8, len(srcs))) as ex:
         objs = list(ex.map(compile_one, srcs))
-    tmp = LIB + ".tmp"
+    tmp = lib_out + ".tmp"
     cmd = [nvcc, *ARCH, "-shared", "-cudart", "shared", "-o", tmp, *objs, "-lcuda"]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
@@ -80,8 +90,8 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"link failed:\n{r.stderr}")
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, lib_out)
+    return lib_out
 
 
 if __name__ == "__main__":

@@ -159,6 +159,8 @@ struct GroupParams {
   uint32_t* pace;           // [ngroups] rounds each group has begun (a pacing hint)
   void* out;                // GM_A: d_hidden [T, d]; GM_B: d_W [V, d]
   int32_t out_dtype;
+  int64_t ring_tiles;       // exchange tiles the ring holds (debug checks)
+  int32_t part_groups;      // rows of part_s / part_m (debug checks)
 };
 
 // per-CTA schedule, the same in every CTA of a group
@@ -460,8 +462,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t sA = stages + stage * kStageBytes;
             const uint32_t fb = map_shared(full_bar(stage), 0);
             if (rank == 0) mbar_arrive_expect_tx(full_bar(stage), 2 * kStageBytes);
-            tma_load_2d_pair(sA, &maps.za, fb, ks * kBK, o * kBM);
-            tma_load_2d_pair(sA + kSA, &maps.zb, fb, ks * kBK, k * kZN + static_cast<int>(rank) * kBM);
+            // (a skipped copy leaves its stage short: the MMA's wait then runs
+            // out and the call reports OLIVE_ERR_TIMEOUT as well)
+            if (OLIVE_DCHECK(p.dev_status, o >= 0 && o <= s.ph && k >= 0 && k < s.ni)) {
+              tma_load_2d_pair(sA, &maps.za, fb, ks * kBK, o * kBM);
+              tma_load_2d_pair(sA + kSA, &maps.zb, fb, ks * kBK, k * kZN + static_cast<int>(rank) * kBM);
+            }
             if (++stage == kStages) { stage = 0; phase ^= 1u; }
           }
         }
@@ -483,9 +489,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t sA = stages + stage * kStageBytes;
             const uint32_t fb = map_shared(full_bar(stage), 0);
             if (rank == 0) mbar_arrive_expect_tx(full_bar(stage), 2 * (kXSlice + s.nbox * 8192));
-            tma_load_2d_pair(sA, &maps.xa, fb, 0, static_cast<int>(((ring0 + slot) * 4 + sl) * kBM));
-            for (int b = 0; b < s.nbox; ++b)
-              tma_load_2d_pair(sA + kSA + b * 8192, &maps.xb, fb, s.b0 + 64 * b, k * kZN + sl * kBK);
+            // TMA x coordinates must be 16-byte aligned (8 bf16)
+            if (OLIVE_DCHECK(p.dev_status, static_cast<int64_t>(ring0 + slot) < p.ring_tiles &&
+                                               s.b0 % 8 == 0 && s.b0 >= 0 && s.b0 < p.d + 64)) {
+              tma_load_2d_pair(sA, &maps.xa, fb, 0, static_cast<int>(((ring0 + slot) * 4 + sl) * kBM));
+              for (int b = 0; b < s.nbox; ++b)
+                tma_load_2d_pair(sA + kSA + b * 8192, &maps.xb, fb, s.b0 + 64 * b, k * kZN + sl * kBK);
+            }
             if (++stage == kStages) { stage = 0; phase ^= 1u; }
           }
         }
@@ -670,6 +680,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         zph ^= 1u;
         tc_fence_after();
         uint8_t* img = ring_bytes + (ring0 + slot) * static_cast<size_t>(kXTile);
+        if (!OLIVE_DCHECK(p.dev_status, !consume || static_cast<int64_t>(ring0 + slot) < p.ring_tiles))
+          img = nullptr;
         if (p.mode == GM_B) {
           const int v = o * kBM + row;
 #pragma unroll 1
@@ -686,7 +698,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               const float pm = meta_y[col] == v ? expm1f(xl * kLn2) : fast_exp2(xl);
               gv[c] = col < kv ? s.coef * pm : 0.f;
             }
-            store_img32(img, row, h, gv);
+            if (img) store_img32(img, row, h, gv);
           }
         } else {
           if (o != cur_o) {
@@ -724,7 +736,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                   p.pyb[o * kBM + row] = __bfloat162float(__float2bfloat16_rn(pv[c]));
                 }
             }
-            if (p.mode == GM_A) store_img32(img, row, h, pv);
+            if (p.mode == GM_A && img) store_img32(img, row, h, pv);
           }
         }
         tc_fence_before();
@@ -733,7 +745,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (p.mode == GM_REF) {
           if (o * kBM + row < s.n) p.rref[o * kBM + row] = run_m;
         } else {
-          if (p.mode == GM_A && ra.valid) {
+          if (p.mode == GM_A && ra.valid &&
+              OLIVE_DCHECK(p.dev_status, s.m < p.part_groups && o * kBM + row < static_cast<int>(Tpad))) {
             p.part_s[static_cast<size_t>(s.m) * Tpad + o * kBM + row] = run_s;
             p.part_m[static_cast<size_t>(s.m) * Tpad + o * kBM + row] = run_m;
           }
@@ -764,7 +777,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             float ov[32];
 #pragma unroll
             for (int q = 0; q < 32; ++q) ov[q] = __uint_as_float(a[q]);
-            if (v < p.V)
+            if (v < p.V && OLIVE_DCHECK(p.dev_status, v >= 0 && s.c0 + c + min(32, s.cw - c) <= p.d))
               store_out32(p.out, static_cast<size_t>(v) * p.d + s.c0 + c, p.out_dtype,
                           min(32, s.cw - c), ov);
           }
@@ -782,7 +795,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           p.part_s[static_cast<size_t>(s.m) * Tpad + rc] = 0.f;
           p.part_m[static_cast<size_t>(s.m) * Tpad + rc] = -INFINITY;
         }
-        if (!phantom(p, s, i)) {
+        if (!phantom(p, s, i) && OLIVE_DCHECK(p.dev_status, o >= 0 && o * kBM < static_cast<int>(Tpad))) {
           __threadfence();
           named_bar_sync(1, kEpi);
           if (threadIdx.x == 0) red_release_add(p.outer_ctr + o, 1u);
@@ -859,7 +872,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     s.coef * fmaf(scale, __uint_as_float(a[8 * q + 2 * u + 1]), corr * wf.y);
               }
             }
-            if (rw.valid)
+            if (rw.valid && OLIVE_DCHECK(p.dev_status, rw.t >= 0 && rw.t < p.T && s.c0 + c + nv <= p.d))
               store_out32(p.out, static_cast<size_t>(rw.t) * p.d + s.c0 + c, p.out_dtype, nv, dv);
           }
         }
@@ -1026,6 +1039,8 @@ olive_status launch_group(const Ctx& c, int mode, const void* hc, const void* W,
   p.pace = ring_ctr ? ring_ctr + 2 * static_cast<size_t>(gs.ngroups) * gs.R : nullptr;
   p.out = mode == GM_B ? a.d_W : a.d_hidden;
   p.out_dtype = a.out_dtype;
+  p.ring_tiles = static_cast<int64_t>(group_ring_words(T, d, V));
+  p.part_groups = group_g_max(d);
 
   static std::atomic<int> done[kMaxDevices];
   if (!set_smem_once(reinterpret_cast<const void*>(lmhead_group_kernel), kGroupSmem, c.device, done))

@@ -366,6 +366,7 @@ const char* olive_status_string(olive_status s) {
     case OLIVE_ERR_UNSUPPORTED_DEVICE: return "device is not compute capability 10.3";
     case OLIVE_ERR_CUDA: return "CUDA call failed";
     case OLIVE_ERR_WORKSPACE: return "workspace null, misaligned or too small";
+    case OLIVE_ERR_BOUNDS: return "a device index check failed (OLIVE_DEBUG build)";
   }
   return "unknown status";
 }

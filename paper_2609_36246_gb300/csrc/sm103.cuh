@@ -13,6 +13,18 @@
 
 namespace olive {
 
+// ------------------------------------------------------------ debug checks ---
+// Builds with -DOLIVE_DEBUG check indices and copy coordinates on the device:
+// a failed check ORs (1 << 10) (OLIVE_ERR_BOUNDS) into the call's status word
+// and evaluates to false, so the caller skips the access it guards; nothing
+// traps.  Release builds compile every check to `true`.
+#ifdef OLIVE_DEBUG
+#define OLIVE_DCHECK(status, cond) \
+  ((cond) ? true : (atomicOr((status), 1 << 10), false))
+#else
+#define OLIVE_DCHECK(status, cond) true
+#endif
+
 // ---------------------------------------------------------------- basics ---
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
