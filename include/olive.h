@@ -42,13 +42,12 @@
  *     uses (compiled into the library, held by every GPU that loads it); the
  *     per-device kernel attributes (shared-memory limits), set on the first
  *     call on each device so that later calls issue no attribute call and can
- *     be captured in a CUDA graph; and three environment variables:
+ *     be captured in a CUDA graph (the on-chip training step also checks
+ *     there, once, that the device holds its whole grid of CTA pairs at
+ *     once); and two environment variables, read at each call:
  *     OLIVE_WAIT_LIMIT_MS (wall-clock limit of every internal wait, default
  *     1000; on expiry the call sets OLIVE_ERR_TIMEOUT) and OLIVE_SLAB_ROWS
- *     (lowers the slab of the slab forms, see olive_slab_rows), both read at
- *     each call, and OLIVE_NONCOOPERATIVE=1, read on first use (launches the
- *     on-chip training step without the cooperative attribute, for profilers
- *     that cannot replay cooperative cluster launches).
+ *     (lowers the slab of the slab forms, see olive_slab_rows).
  *   - `stream` is a cudaStream_t (NULL = legacy default stream).  All calls
  *     are asynchronous on it; none synchronises the host.
  *   - The returned olive_status covers what the host can check before any
@@ -109,8 +108,8 @@ enum { OLIVE_OP_LOGPROB_FWD = 0, OLIVE_OP_LOSS_BWD = 1, OLIVE_OP_DIVERGENCE = 2,
 
 /*
  * Rows of the G slab that the slab forms (olive_token_loss_fwd_bwd_slab,
- * olive_topk_kl_bwd, olive_topk_kl_fwd_bwd, and the divergence gradient of
- * olive_token_divergence) hold at a time for T packed rows and V vocabulary
+ * olive_topk_kl_bwd, olive_topk_kl_fwd_bwd) hold at a time for T packed rows
+ * and V vocabulary
  * entries: about 5.6 GB of bf16 G in whole 128-row tiles, at most 32768 rows
  * and at most T rounded up to 128, lowered by OLIVE_SLAB_ROWS (a multiple of
  * 128).  A call on more masked rows runs ceil(N_mask / rows) slabs.  Returns 0
@@ -479,6 +478,10 @@ OLIVE_API olive_status olive_scale(const void* x, void* y, size_t n, int dtype,
  *   reverse: d_h_s[t] = g_t inv_tau sum_v p_s (log p_s - log p_t - kl[t]) W_s[v]
  *   forward: d_h_s[t] = g_t inv_tau sum_v (p_s - p_t) W_s[v]
  * (0 on rows not in `rows`; the teacher receives no gradient).
+ * With the gradient the call makes two sweeps over the vocabulary: the first
+ * gives kl[t] and both log-sum-exps, the second recomputes both heads' logits
+ * tile by tile and contracts G against W_s on chip (G is never written to
+ * device memory); its counters and exchange ring are in the workspace.
  */
 OLIVE_API olive_status olive_token_divergence(const void* h_s, const void* W_s, int32_t d_s,
                                     const void* h_t, const void* W_t, int32_t d_t,

@@ -48,12 +48,6 @@ bool encode_bf16_2d_plain(CUtensorMap* map, const void* base, uint64_t inner, ui
 // Rows of the G slab used by the backward passes for vocabulary size V.
 int64_t slab_rows(int64_t Tpad, int64_t V);
 inline int64_t vpad(int64_t V) { return align_up(static_cast<size_t>(V), 8); }
-// Slab rows of the forward-KL gradient, whose fp32 slab holds pairs: half of
-// tc in whole 128-row tiles, at least one tile.
-inline int64_t kl_pair_rows(int64_t tc) {
-  const int64_t h = tc / 2 / kRowAlign * kRowAlign;
-  return h > kRowAlign ? h : kRowAlign;
-}
 
 // ---- workspace carving (sizes in bytes; every region 256-byte aligned) ----
 struct FwdWs {
@@ -122,11 +116,14 @@ FbWs carve_fb(void* ws, int64_t T, int64_t d, int64_t V, int grad_dtype);
 struct KlWs {
   void* hcs;      // bf16 [Tpad, d_s]
   void* hct;      // bf16 [Tpad, d_t]
-  float* part;    // [5, kSvMax, Tpad] (value only)
-  void* g;        // bf16 [Tc, Vpad]: e_s, then G (gradient only)
-  float* s2;      // fp32 [Tc, Vpad]: second slab (gradient only)
-  float* part5;   // [5, Tc, ceil(V/128)] per-half-tile partials (gradient only)
-  int64_t tc;
+  float* part;    // [5, kSvMax, Tpad] value-sweep partials
+  // gradient only: both heads' lse per compact row (p the primary head), the
+  // exchange ring of the on-chip gradient pass and its counters
+  float* lse_p;   // [Tpad]
+  float* lse_q;   // [Tpad]
+  void* ring;     // group_ring_bytes(T, d_s, V)
+  uint32_t* ctr;  // ctr_words words
+  size_t ctr_words;
 };
 size_t kl_ws_bytes(int64_t T, int64_t ds, int64_t dt, int64_t V, int grad);
 KlWs carve_kl(void* ws, int64_t T, int64_t ds, int64_t dt, int64_t V, int grad);
@@ -175,11 +172,27 @@ struct GroupArgs {
   void* d_hidden;
   void* d_W;
   int out_dtype;
+  // mode 3 (divergence gradient) only
+  const void* hc2;      // teacher rows, bf16 [Tpad, d2]
+  const void* W2;       // teacher head, bf16 [V, d2]
+  int d2, reverse;
+  const float *lse_sc, *lse_tc, *kl, *grad_kl;
 };
-// mode 0: reference maxima, 1: pass A (lse, logp, dH), 2: pass B (dW)
+// mode 0: reference maxima, 1: pass A (lse, logp, dH), 2: pass B (dW),
+// 3: divergence gradient (d_hidden = G . W with G from both heads)
 olive_status launch_group(const Ctx& c, int mode, const void* hc, const void* W, int32_t T,
                           int32_t d, int32_t V, const GroupArgs& a, int c_base, int c_end,
                           uint32_t* ring_ctr);
+// The divergence gradient on chip: d_h_s = G . W_s with G from both heads'
+// logits (recomputed tile by tile by groups of CTA pairs, 128-wide vocabulary
+// tiles) and the value sweep's kl, lse_s, lse_t; ctr (ctr_words) is zeroed here.
+olive_status launch_kl_group_grad(const Ctx& c, const void* hcs, const void* hct, const void* W_s,
+                                  int32_t d_s, const void* W_t, int32_t d_t, const int32_t* rows,
+                                  const int32_t* n_rows, int32_t T, int32_t V, float inv_tau,
+                                  int reverse, const float* kl, const float* lse_s,
+                                  const float* lse_t, const float* grad_kl, void* d_h_s,
+                                  int grad_dtype, void* ring, uint32_t* ctr, size_t ctr_words,
+                                  int32_t* dev_status);
 // The whole step: forward + backward when lse_given is null (logp, lse, loss
 // written), else the backward of that forward.
 olive_status launch_loss_group(const Ctx& c, const void* hidden, const void* W,
@@ -307,14 +320,5 @@ olive_status launch_topk_kl_fwd_bwd(const Ctx& c, const void* h_s, const void* W
                                     int32_t* s_ids, float* s_logp, float* t_logp_s,
                                     float* kl_topk, float* overlap, void* d_h_s, void* d_W_s,
                                     int grad_dtype, void* ws, int32_t* dev_status);
-
-// Divergence forward + d_h_s in one pass over the logits (fused kernel,
-// per slab: KLZ tiles, conv_kl_kernel, DH tiles); writes kl[t] too.
-olive_status launch_kl_fwd_bwd(const Ctx& c, const void* hcs, const void* hct, const void* W_s,
-                               int32_t d_s, const void* W_t, int32_t d_t, const int32_t* rows,
-                               const int32_t* n_rows, int32_t T, int32_t V, float inv_tau,
-                               int reverse, const float* grad_kl, float* kl, void* g, float* s2,
-                               float* part5, int64_t tc, void* d_h_s, int grad_dtype,
-                               int32_t* dev_status);
 
 }  // namespace olive

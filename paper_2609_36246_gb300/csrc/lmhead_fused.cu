@@ -1,16 +1,15 @@
-// lmhead_fused.cu -- the LM-head losses' backward passes, and their single-pass
-// forward + backward forms, in one persistent tcgen05 kernel
-// (lmhead_fused_kernel) with a static tile schedule.
+// lmhead_fused.cu -- the slab forms of the LM-head losses' backward passes and
+// of their single-pass forward + backward, in one persistent tcgen05 kernel
+// (lmhead_fused_kernel) with a static tile schedule: the cross-entropy step
+// through an HBM slab of G (olive_token_loss_fwd_bwd_slab) and the top-K KL
+// calls (olive_topk_kl_bwd, olive_topk_kl_fwd_bwd).  The on-chip forms are in
+// lmhead_group.cu.
 //
 // Cross-entropy (Eq. (osd-ce), Section 3.1; the sampled sequences are fixed,
 // so only hidden and W get gradients).  With p = softmax(z) from the
 // forward's lse and G[r, v] = g inv_tau (p[r, v] - [v == y_r]):
 //   dH = G . W        (M = rows, N = d, K = V)
 //   dW = G^T . hc     (M = V,    N = d, K = rows)
-// Divergence (OPD's per-token KL, Section 1): G = g_t inv_tau p_s
-// (log p_s - log p_t - KL_t) (reverse) or g_t inv_tau (p_s - p_t) (forward),
-// and dH_s = G . W_s; it always runs in the single-pass form below (KLZ
-// tiles, conv_kl_kernel, DH tiles).
 // Top-K truncated reverse KL (OPD's top-16 approximation as read here, the
 // student's top-K set S held fixed): with l = log p_s, q = log p_t at the ids
 // of S, P_S = sum_S p_s and KL_K the forward value,
@@ -57,15 +56,7 @@
 // exceeds R by more than kRefMax keeps its own maximum as reference, and its
 // row is rewritten in full relative to lse2 by ref_fix_kernel (lam = g
 // inv_tau).  The launches are stream ordered, so these phases need no tile
-// counters.  The divergence gradient
-// uses the same phases with KLZ tiles (two products per tile, student and
-// teacher, in the two 256-column halves of one TMEM accumulator) and five
-// per-tile partials, from which conv_kl_kernel forms KL and G.  Reverse KL:
-// e_s = 2^(x_s - m_s) in bf16 in the G slab and x_s - x_t in an fp32 slab
-// (G is proportional to p_s, so a bf16 p_s only adds G's own rounding).
-// Forward KL: G = p_s - p_t cancels where the models agree, so both local
-// logits x_s - m_s and x_t - m_t stay fp32 (pairs, in half as many slab rows
-// so the workspace is the same).
+// counters.
 #include <climits>
 #include <cmath>
 
@@ -80,9 +71,8 @@ constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kBN = 256;
 constexpr int kStages = 4;
 // Eight epilogue warps: the two warps of a TMEM lane quadrant (warp % 4) take
-// the two 128-column halves (part = warp / 4) of every tile, which halves the
-// epilogue of the tile kinds whose accumulator cannot be double-buffered
-// (KLZ).  Warp 8 is the producer, warp 9 the MMA issuer.
+// the two 128-column halves (part = warp / 4) of every tile.  Warp 8 is the
+// producer, warp 9 the MMA issuer.
 constexpr int kFEpiWarps = 8;
 constexpr int kFEpi = 32 * kFEpiWarps;
 constexpr int kFProducer = kFEpiWarps;
@@ -90,7 +80,7 @@ constexpr int kFMma = kFEpiWarps + 1;
 constexpr int kFThreads = 32 * (kFEpiWarps + 2);
 constexpr int kHalf = kBN / 2;
 
-enum Kind : int { K_NONE = -1, K_GRAD = 0, K_KLZ = 1, K_DH = 2, K_DW = 3, K_ZSAVE = 4, K_ZREF = 5 };
+enum Kind : int { K_NONE = -1, K_GRAD = 0, K_DH = 2, K_DW = 3, K_ZSAVE = 4, K_ZREF = 5 };
 // phases: one launch of every tile kind with dependency waits, or one slab's
 // forward (ZSAVE) tiles, or one slab's DH and DW tiles, or the first vocabulary
 // tile of every row tile of one slab (the rows' reference maxima)
@@ -108,8 +98,6 @@ constexpr float kOwnShift = 110.f;
 
 // CE maps: 0 hc K-major 64x128, 1 W K-major 64x256, 2 G K-major 64x128,
 //          3 W MN-major 64x64, 4 G MN-major 64x64, 5 hc MN-major 64x64
-// KL maps: 0 hs K-major 64x128, 1 W_s K-major 64x256, 2 G K-major 64x128,
-//          3 W_s MN-major 64x64, 4 ht K-major 64x128, 5 W_t K-major 64x256
 struct FusedMaps {
   CUtensorMap m[6];
 };
@@ -136,12 +124,7 @@ struct FusedParams {
   const float* lam;          // CE single pass: [tc] dH row scale (null: none)
   float* part_tm;            // PH_Z: [tc, vh] true half-tile maximum (base 2), when kept
   int32_t dw_coef;           // 1: DW tiles scale by g inv_tau (/ N_mask), the CE single pass
-  float* s2;                 // KLZ: fp32 slab, [tc, ldg] (reverse) or [tc / 2, 2 ldg] (forward)
-  float* part5;              // KLZ: [5][tc][vh] m_s, s_s, m_t, s_t, A per (row, half-tile)
-  int64_t plane5;            // tc * vh
-  int32_t kl;                // 0: cross-entropy, 1: divergence
-  int32_t reverse;           // KL direction
-  int32_t T, d, d2, V, reduction, out_dtype, group_rows;
+  int32_t T, d, V, reduction, out_dtype, group_rows;
   int32_t tc_max;            // rows of the G buffer (multiple of 128)
   int32_t max_slabs, max_rt; // counter array dimensions
   int64_t ldg;               // G row stride in elements
@@ -183,7 +166,7 @@ __device__ Plan make_plan(const FusedParams& p) {
   pl.ntd = (p.d + kBN - 1) / kBN;
   pl.mtv = (p.V + kBM - 1) / kBM;
   pl.coef = 0.f;
-  if (!p.kl && p.sp_k == 0 && (p.phase == PH_ALL || p.dw_coef) && p.grad_loss) {
+  if (p.sp_k == 0 && (p.phase == PH_ALL || p.dw_coef) && p.grad_loss) {
     float g = *p.grad_loss;
     if (p.reduction == OLIVE_REDUCE_MEAN && pl.n > 0) g = g / static_cast<float>(pl.n);
     pl.coef = g * p.inv_tau;
@@ -197,8 +180,8 @@ __device__ __forceinline__ int slab_in(const Plan& pl, int s) {
 }
 __device__ __forceinline__ int units_grad(const Plan& pl, int mt) { return mt * pl.vt; }
 __device__ __forceinline__ int units_dh(const Plan& pl, int mt) { return mt * pl.ntd; }
-__device__ __forceinline__ int units_dw(const FusedParams& p, const Plan& pl, int s, int in_s) {
-  return (!p.kl && (s == 0 || in_s > 0)) ? pl.mtv * pl.ntd : 0;
+__device__ __forceinline__ int units_dw(const Plan& pl, int s, int in_s) {
+  return (s == 0 || in_s > 0) ? pl.mtv * pl.ntd : 0;
 }
 
 // slabs a launch covers
@@ -217,7 +200,7 @@ __device__ int total_units(const FusedParams& p, const Plan& pl) {
       continue;
     }
     if (p.phase != PH_DHDW) t += units_grad(pl, mt);
-    if (p.phase != PH_Z) t += units_dh(pl, mt) + units_dw(p, pl, s, in_s);
+    if (p.phase != PH_Z) t += units_dh(pl, mt) + units_dw(pl, s, in_s);
   }
   return t;
 }
@@ -246,7 +229,7 @@ __device__ Unit decode(const FusedParams& p, const Plan& pl, int u) {
     if (u < ug) {
       const Raster r{mt, pl.vt, p.group_rows};
       r.tile(u, x.i, x.j);
-      x.kind = p.phase == PH_Z ? (p.kl ? K_KLZ : K_ZSAVE) : K_GRAD;
+      x.kind = p.phase == PH_Z ? K_ZSAVE : K_GRAD;
       return x;
     }
     u -= ug;
@@ -259,7 +242,7 @@ __device__ Unit decode(const FusedParams& p, const Plan& pl, int u) {
       return x;
     }
     u -= uh;
-    const int uw = units_dw(p, pl, s, in_s);
+    const int uw = units_dw(pl, s, in_s);
     if (u < uw) {
       x.i = u / pl.ntd;
       x.j = u % pl.ntd;
@@ -271,20 +254,15 @@ __device__ Unit decode(const FusedParams& p, const Plan& pl, int u) {
   return x;
 }
 
-// K steps of each product of a unit
-__device__ __forceinline__ void unit_ksteps(const FusedParams& p, const Unit& x, int& nk, int& nk2) {
-  nk2 = 0;
+// K steps of a unit's product
+__device__ __forceinline__ int unit_ksteps(const FusedParams& p, const Unit& x) {
   switch (x.kind) {
     case K_GRAD:
     case K_ZSAVE:
-    case K_ZREF: nk = (p.d + kBK - 1) / kBK; break;
-    case K_KLZ:
-      nk = (p.d + kBK - 1) / kBK;
-      nk2 = (p.d2 + kBK - 1) / kBK;
-      break;
-    case K_DH: nk = (p.V + kBK - 1) / kBK; break;
-    case K_DW: nk = (x.in_s + kBK - 1) / kBK; break;
-    default: nk = 0;
+    case K_ZREF: return (p.d + kBK - 1) / kBK;
+    case K_DH: return (p.V + kBK - 1) / kBK;
+    case K_DW: return (x.in_s + kBK - 1) / kBK;
+    default: return 0;
   }
 }
 
@@ -377,99 +355,6 @@ __device__ void epi_grad(const FusedParams& p, const Plan& pl, const Unit& x, in
       const int u = p.sp_ids[o + k];
       if (u >= h0 && u < h1) grow[u] = __float2bfloat16_rn(p.sp_val[o + k]);
     }
-  }
-}
-
-// divergence forward tile: student (columns [0, 256)) and teacher (columns
-// [256, 512)) logits of one 128 x 256 tile; per row the tile maxima m_s, m_t,
-// sums s_s, s_t of 2^(x - m), A = sum e_p (x_p - x_q) in the primary
-// distribution's scale (p = student for the reverse KL, teacher for the
-// forward KL), e_s in bf16 into the G slab and the fp32 second slab
-__device__ void epi_klz(const FusedParams& p, const Plan& pl, const Unit& x, int row, int part,
-                        uint32_t taddr) {
-  const int r_local = x.i * kBM + row;
-  bool valid = r_local < x.in_s;
-  if (valid) {
-    const int t = p.rows[x.row0 + r_local];
-    valid = t >= 0 && t < p.T;
-  }
-  const int n0 = x.j * kBN;
-  float ms = -INFINITY, mt = -INFINITY;
-#pragma unroll 1
-  for (int c = part * kHalf; c < (part + 1) * kHalf; c += 32) {
-    const int col0 = n0 + c;
-    if (col0 >= p.V) break;
-    uint32_t a[32], b[32];
-    tmem_ld_32x32b_x32(taddr + c, a);
-    tmem_ld_32x32b_x32(taddr + kBN + c, b);
-    tmem_ld_wait();
-    const int nv = p.V - col0;
-#pragma unroll
-    for (int k = 0; k < 32; ++k) {
-      if (k < nv) {
-        ms = fmaxf(ms, __uint_as_float(a[k]) * p.scale2);
-        mt = fmaxf(mt, __uint_as_float(b[k]) * p.scale2);
-      }
-    }
-  }
-  __nv_bfloat16* grow = p.g + static_cast<size_t>(r_local) * p.ldg;
-  float* srow = p.s2 + static_cast<size_t>(r_local) * p.ldg * (p.reverse ? 1 : 2);
-  float ss = 0.f, st = 0.f, A = 0.f;
-#pragma unroll 1
-  for (int c = part * kHalf; c < (part + 1) * kHalf; c += 32) {
-    const int col0 = n0 + c;
-    if (col0 >= p.V) break;
-    uint32_t a[32], b[32];
-    tmem_ld_32x32b_x32(taddr + c, a);
-    tmem_ld_32x32b_x32(taddr + kBN + c, b);
-    tmem_ld_wait();
-    const int nv = p.V - col0;
-    float e[32];
-#pragma unroll
-    for (int k = 0; k < 32; ++k) {
-      const bool ok = valid && k < nv;
-      const float xs = __uint_as_float(a[k]) * p.scale2;
-      const float xt = __uint_as_float(b[k]) * p.scale2;
-      const float es = ok ? fast_exp2(xs - ms) : 0.f;
-      const float et = ok ? fast_exp2(xt - mt) : 0.f;
-      ss += es;
-      st += et;
-      A += p.reverse ? es * (xs - xt) : et * (xt - xs);
-      e[k] = es;
-    }
-    if (p.reverse) {
-      store_row32(grow, col0, OLIVE_DTYPE_BF16, nv, e);
-#pragma unroll
-      for (int k = 0; k < 32; ++k) {
-        const bool ok = valid && k < nv;
-        e[k] = ok ? (__uint_as_float(a[k]) - __uint_as_float(b[k])) * p.scale2 : 0.f;
-      }
-      store_row32(srow, col0, OLIVE_DTYPE_F32, nv, e);
-    } else {
-      // (x_s - m_s, x_t - m_t) pairs, 16 columns per 32-value store
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        float f[32];
-#pragma unroll
-        for (int k = 0; k < 16; ++k) {
-          const int kk = 16 * h + k;
-          const bool ok = valid && kk < nv;
-          f[2 * k] = ok ? __uint_as_float(a[kk]) * p.scale2 - ms : 0.f;
-          f[2 * k + 1] = ok ? __uint_as_float(b[kk]) * p.scale2 - mt : 0.f;
-        }
-        const int nvh = nv - 16 * h;
-        if (nvh > 0) store_row32(srow, 2 * static_cast<size_t>(col0 + 16 * h), OLIVE_DTYPE_F32,
-                                 2 * (nvh < 16 ? nvh : 16), f);
-      }
-    }
-  }
-  if (valid && n0 + part * kHalf < p.V) {  // a half past V has no partial slot
-    const size_t o = static_cast<size_t>(r_local) * pl.vh + 2 * x.j + part;
-    p.part5[o] = ms;
-    p.part5[p.plane5 + o] = ss;
-    p.part5[2 * p.plane5 + o] = mt;
-    p.part5[3 * p.plane5 + o] = st;
-    p.part5[4 * p.plane5 + o] = A;
   }
 }
 
@@ -696,10 +581,9 @@ __global__ void __launch_bounds__(kFThreads, 1)
 
   const uint32_t tmem_base = *tmem_slot;
   const Plan pl = *plan_smem;
-  // cross-entropy: two 256-column accumulators (the epilogue of one tile
-  // overlaps the next tile's MMAs); divergence: one 512-column accumulator
-  // holding the student and teacher products of a 128 x 256 tile
-  const int nbufs = p.kl ? 1 : 2;
+  // two 256-column accumulators: the epilogue of one tile overlaps the next
+  // tile's MMAs
+  constexpr int nbufs = 2;
   const WaitCtl ctl{abort_flag, p.wait_limit_ns};
 
   const int total = total_units(p, pl);
@@ -719,7 +603,7 @@ __global__ void __launch_bounds__(kFThreads, 1)
           const int pin = slab_in(pl, x.s - 1);
           const int pmt = (pin + 127) / 128;
           dep = wait_counter(ctr_dhdw(p, x.s - 1),
-                             units_dh(pl, pmt) + units_dw(p, pl, x.s - 1, pin), ctl);
+                             units_dh(pl, pmt) + units_dw(pl, x.s - 1, pin), ctl);
         } else if (x.kind == K_DH) {
           dep = wait_counter(ctr_row(p, x.s, x.i), pl.vt, ctl);
         } else if (x.kind == K_DW) {
@@ -727,9 +611,8 @@ __global__ void __launch_bounds__(kFThreads, 1)
         }
         if (!dep) { ok = false; break; }
         fence_proxy_async_global();
-        int nk, nk2;
-        unit_ksteps(p, x, nk, nk2);
-        for (int k = 0; k < nk + nk2; ++k) {
+        const int nk = unit_ksteps(p, x);
+        for (int k = 0; k < nk; ++k) {
           if (!mbar_wait(empty_bar(stage), phase ^ 1u, ctl)) { ok = false; break; }
           const uint32_t sA = ring + stage * L::STAGE_BYTES;
           const uint32_t sB = sA + L::A_BYTES;
@@ -742,13 +625,6 @@ __global__ void __launch_bounds__(kFThreads, 1)
               tma_load_2d(sA, &maps.m[0], fb, k * kBK, x.row0 + x.i * kBM);
               tma_load_2d(sB, &maps.m[1], fb, k * kBK, x.j * kBN);
               break;
-            case K_KLZ: {
-              const bool second = k >= nk;
-              const int kk = (second ? k - nk : k) * kBK;
-              tma_load_2d(sA, &maps.m[second ? 4 : 0], fb, kk, x.row0 + x.i * kBM);
-              tma_load_2d(sB, &maps.m[second ? 5 : 1], fb, kk, x.j * kBN);
-              break;
-            }
             case K_DH:
               tma_load_2d(sA, &maps.m[2], fb, k * kBK, x.i * kBM);
 #pragma unroll
@@ -779,12 +655,10 @@ __global__ void __launch_bounds__(kFThreads, 1)
       bool ok = true;
       for (int u = blockIdx.x; ok && u < total; u += gridDim.x) {
         const Unit x = decode(p, pl, u);
-        int nk, nk2;
-        unit_ksteps(p, x, nk, nk2);
+        const int nk = unit_ksteps(p, x);
         uint32_t idesc;
         bool a_mn = false, b_mn = false;
         switch (x.kind) {
-          case K_KLZ: idesc = idesc_bf16(kBM, kBN, false, false); break;
           case K_DH: idesc = idesc_bf16(kBM, kBN, false, true); b_mn = true; break;
           case K_DW: idesc = idesc_bf16(kBM, kBN, true, true); a_mn = b_mn = true; break;
           default: idesc = idesc_bf16(kBM, kBN, false, false); break;
@@ -792,12 +666,9 @@ __global__ void __launch_bounds__(kFThreads, 1)
         if (!mbar_wait(tempty_bar(buf), aphase ^ 1u, ctl)) { ok = false; break; }
         tc_fence_after();
         const uint32_t acc = tmem_base + static_cast<uint32_t>(buf * kBN);
-        for (int k = 0; k < nk + nk2; ++k) {
+        for (int k = 0; k < nk; ++k) {
           if (!mbar_wait(full_bar(stage), phase, ctl)) { ok = false; break; }
           tc_fence_after();
-          const bool second = k >= nk;
-          const uint32_t dt = second ? acc + kBN : acc;
-          const int kl = second ? k - nk : k;
           const uint32_t sA = ring + stage * L::STAGE_BYTES;
           const uint32_t sB = sA + L::A_BYTES;
 #pragma unroll
@@ -806,7 +677,7 @@ __global__ void __launch_bounds__(kFThreads, 1)
                                      : sdesc_sw128(sA + kk * 32, 16, 1024);
             const uint64_t bd = b_mn ? sdesc_sw128(sB + kk * 2048, 8192, 1024)
                                      : sdesc_sw128(sB + kk * 32, 16, 1024);
-            umma_bf16(dt, ad, bd, idesc, (kl > 0 || kk > 0) ? 1u : 0u);
+            umma_bf16(acc, ad, bd, idesc, (k > 0 || kk > 0) ? 1u : 0u);
           }
           umma_commit(empty_bar(stage));
           if (++stage == kStages) { stage = 0; phase ^= 1u; }
@@ -833,8 +704,7 @@ __global__ void __launch_bounds__(kFThreads, 1)
     // epilogue threads always leave the loop together
     for (int u = blockIdx.x; u < total; u += gridDim.x) {
       const Unit x = decode(p, pl, u);
-      int nk, nk2;
-      unit_ksteps(p, x, nk, nk2);
+      const int nk = unit_ksteps(p, x);
       if (!named_bar_and(1, kFEpi, mbar_wait(tfull_bar(buf), aphase, ctl))) break;
       tc_fence_after();
       __syncwarp();
@@ -847,7 +717,6 @@ __global__ void __launch_bounds__(kFThreads, 1)
       }
       switch (x.kind) {
         case K_GRAD: epi_grad(p, pl, x, row, part, taddr); break;
-        case K_KLZ: epi_klz(p, pl, x, row, part, taddr); break;
         case K_ZSAVE: epi_zsave(p, pl, x, row, part, taddr); break;
         case K_ZREF: epi_zref(p, x, row, part, taddr); break;
         case K_DH: epi_dh(p, x, row, part, taddr); break;
@@ -997,148 +866,6 @@ __global__ void __launch_bounds__(256)
         h2[e] = __floats2bfloat162_rn(u.x * sr, u.y * sr);
       }
       hrow[c] = v;
-    }
-  }
-}
-
-// (max, sum, A) triples: A is scaled like the sum
-__device__ __forceinline__ void lse_merge3(float& m, float& s, float& a, float m2, float s2,
-                                           float a2) {
-  if (m2 == -INFINITY) return;
-  if (m == -INFINITY) {
-    m = m2;
-    s = s2;
-    a = a2;
-    return;
-  }
-  const float mn = fmaxf(m, m2);
-  const float f1 = fast_exp2(m - mn), f2 = fast_exp2(m2 - mn);
-  s = s * f1 + s2 * f2;
-  a = a * f1 + a2 * f2;
-  m = mn;
-}
-
-// One warp per masked row of the slab: merges the KLZ partials into lse_s,
-// lse_t and KL = ln2 A / s_p - lse_p + lse_q (p the primary distribution),
-// writes kl[t], then writes the row of G into the G slab:
-//   reverse: G = coef p_s (ln2 (x_s - x_t) - (lse_s - lse_t) - KL), with
-//            p_s = e_s 2^(m_s - lse2_s) from the slab's own e_s
-//   forward: G = coef (p_s - p_t), both from the fp32 (x - m) pairs
-// with coef = grad_kl[t] inv_tau.
-__global__ void __launch_bounds__(256)
-    conv_kl_kernel(const int32_t* __restrict__ n_rows, const int32_t* __restrict__ rows, int T,
-                   int V, int tc, int slab, int vh, int64_t ldg, float inv_tau, int reverse,
-                   const float* __restrict__ grad_kl, const float* __restrict__ part5,
-                   int64_t plane5, const float* __restrict__ s2, __nv_bfloat16* g,
-                   float* __restrict__ kl) {
-  const int n = read_n_rows(n_rows, T, nullptr);
-  const SlabPlan sp(n, tc);
-  if (slab >= sp.n_slabs) return;
-  const int in_s = sp.rows_in(n, slab);
-  const int row0 = slab * sp.rps;
-  const int lane = threadIdx.x & 31;
-  const int warps = (gridDim.x * blockDim.x) >> 5;
-  const int nvec = (V + 7) / 8;
-  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < in_s; r += warps) {
-    const int t = rows[row0 + r];
-    if (t < 0 || t >= T) continue;  // reported by the gather; the G row is zero
-    const float* pms = part5 + static_cast<size_t>(r) * vh;
-    const float* pss = pms + plane5;
-    const float* pmt = pms + 2 * plane5;
-    const float* pst = pms + 3 * plane5;
-    const float* pa = pms + 4 * plane5;
-    float mp = -INFINITY, sp_ = 0.f, A = 0.f, mq = -INFINITY, sq = 0.f;
-    for (int j = lane; j < vh; j += 32) {
-      if (reverse) {
-        lse_merge3(mp, sp_, A, pms[j], pss[j], pa[j]);
-        lse_merge(mq, sq, pmt[j], pst[j]);
-      } else {
-        lse_merge3(mp, sp_, A, pmt[j], pst[j], pa[j]);
-        lse_merge(mq, sq, pms[j], pss[j]);
-      }
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float m2 = __shfl_xor_sync(0xffffffffu, mp, o);
-      const float s2v = __shfl_xor_sync(0xffffffffu, sp_, o);
-      const float a2 = __shfl_xor_sync(0xffffffffu, A, o);
-      lse_merge3(mp, sp_, A, m2, s2v, a2);
-      const float mq2 = __shfl_xor_sync(0xffffffffu, mq, o);
-      const float sq2 = __shfl_xor_sync(0xffffffffu, sq, o);
-      lse_merge(mq, sq, mq2, sq2);
-    }
-    const float lse2_p = mp + log2f(sp_);
-    const float lse2_q = mq + log2f(sq);
-    const float k = kLn2 * (A / sp_) - (lse2_p - lse2_q) * kLn2;
-    const float lse2_s = reverse ? lse2_p : lse2_q;
-    const float lse2_t = reverse ? lse2_q : lse2_p;
-    if (lane == 0) kl[t] = k;
-    const float coef = grad_kl[t] * inv_tau;
-    const float c0 = (lse2_s - lse2_t) * kLn2 + k;
-    uint4* grow = reinterpret_cast<uint4*>(g + static_cast<size_t>(r) * ldg);
-    if (reverse) {
-      const float4* srow = reinterpret_cast<const float4*>(s2 + static_cast<size_t>(r) * ldg);
-#pragma unroll 1
-      for (int base = 0; base < nvec; base += 64) {
-        uint4 v[2];
-        float4 dl[2][2];
-#pragma unroll
-        for (int q = 0; q < 2; ++q) {
-          const int idx = base + 32 * q + lane;
-          if (idx < nvec) {
-            v[q] = grow[idx];
-            dl[q][0] = srow[2 * idx];
-            dl[q][1] = srow[2 * idx + 1];
-          }
-        }
-#pragma unroll
-        for (int q = 0; q < 2; ++q) {
-          const int idx = base + 32 * q + lane;
-          if (idx >= nvec) continue;
-          const float scs = coef * fast_exp2(pms[idx >> 4] - lse2_s);  // 16 vectors per half tile
-          const float dd[8] = {dl[q][0].x, dl[q][0].y, dl[q][0].z, dl[q][0].w,
-                               dl[q][1].x, dl[q][1].y, dl[q][1].z, dl[q][1].w};
-          __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&v[q]);
-          const int col = idx * 8;
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float2 u = __bfloat1622float2(h2[e]);
-            float a = scs * u.x * (kLn2 * dd[2 * e] - c0);
-            float b = scs * u.y * (kLn2 * dd[2 * e + 1] - c0);
-            if (col + 2 * e >= V) a = 0.f;
-            if (col + 2 * e + 1 >= V) b = 0.f;
-            h2[e] = __floats2bfloat162_rn(a, b);
-          }
-          grow[idx] = v[q];
-        }
-      }
-    } else {
-      const float4* srow = reinterpret_cast<const float4*>(s2 + static_cast<size_t>(r) * 2 * ldg);
-#pragma unroll 1
-      for (int base = 0; base < nvec; base += 32) {
-        const int idx = base + lane;
-        if (idx >= nvec) continue;
-        float4 pr[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) pr[q] = srow[4 * idx + q];
-        const int j = idx >> 4;  // 16 vectors per half tile
-        const float os = pms[j] - lse2_s;
-        const float ot = pmt[j] - lse2_t;
-        const float xy[16] = {pr[0].x, pr[0].y, pr[0].z, pr[0].w, pr[1].x, pr[1].y, pr[1].z, pr[1].w,
-                              pr[2].x, pr[2].y, pr[2].z, pr[2].w, pr[3].x, pr[3].y, pr[3].z, pr[3].w};
-        uint4 out;
-        __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&out);
-        const int col = idx * 8;
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          float a = coef * (fast_exp2(xy[4 * e] + os) - fast_exp2(xy[4 * e + 1] + ot));
-          float b = coef * (fast_exp2(xy[4 * e + 2] + os) - fast_exp2(xy[4 * e + 3] + ot));
-          if (col + 2 * e >= V) a = 0.f;
-          if (col + 2 * e + 1 >= V) b = 0.f;
-          h2[e] = __floats2bfloat162_rn(a, b);
-        }
-        grow[idx] = out;
-      }
     }
   }
 }
@@ -1596,9 +1323,7 @@ olive_status launch_loss_bwd(const Ctx& c, const void* hidden, const void* W,
     p.sp_ids = sg->ids;
     p.sp_k = sg->K;
   }
-  p.kl = 0;
   p.d = d;
-  p.d2 = 0;
   p.reduction = reduction;
   p.out_dtype = grad_dtype;
   p.tc_max = static_cast<int32_t>(w.tc);
@@ -1643,7 +1368,6 @@ olive_status launch_loss_fwd_bwd(const Ctx& c, const void* hidden, const void* W
 
   FusedParams p = base_params(c, rows, n_rows, T, V, inv_tau, dev_status);
   p.targets = targets;
-  p.kl = 0;
   p.d = d;
   p.reduction = reduction;
   p.out_dtype = grad_dtype;
@@ -1682,59 +1406,6 @@ olive_status launch_loss_fwd_bwd(const Ctx& c, const void* hidden, const void* W
     if ((st = launch_lmhead_fused(c, maps, p)) != OLIVE_OK) return st;
   }
   return launch_loss_reduce(c, n_rows, T, w.nll, reduction, loss);
-}
-
-olive_status launch_kl_fwd_bwd(const Ctx& c, const void* hcs, const void* hct, const void* W_s,
-                               int32_t d_s, const void* W_t, int32_t d_t, const int32_t* rows,
-                               const int32_t* n_rows, int32_t T, int32_t V, float inv_tau,
-                               int reverse, const float* grad_kl, float* kl, void* g, float* s2,
-                               float* part5, int64_t tc, void* d_h_s, int grad_dtype,
-                               int32_t* dev_status) {
-  const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
-  const int64_t ldg = vpad(V);
-  const int vh = static_cast<int>(ceil_div(V, kHalf));
-  FusedMaps maps;
-  if (!encode_bf16_2d(&maps.m[0], hcs, d_s, Tpad, 2ull * d_s, 64, 128) ||
-      !encode_bf16_2d(&maps.m[1], W_s, d_s, V, 2ull * d_s, 64, 256) ||
-      !encode_bf16_2d(&maps.m[2], g, V, tc, 2ull * ldg, 64, 128) ||
-      !encode_bf16_2d(&maps.m[3], W_s, d_s, V, 2ull * d_s, 64, 64) ||
-      !encode_bf16_2d(&maps.m[4], hct, d_t, Tpad, 2ull * d_t, 64, 128) ||
-      !encode_bf16_2d(&maps.m[5], W_t, d_t, V, 2ull * d_t, 64, 256))
-    return OLIVE_ERR_CUDA;
-  FusedParams p = base_params(c, rows, n_rows, T, V, inv_tau, dev_status);
-  p.kl = 1;
-  p.reverse = reverse;
-  p.d = d_s;
-  p.d2 = d_t;
-  p.out_dtype = grad_dtype;
-  // the forward direction's fp32 pairs take twice the bytes per row: half the rows per slab
-  if (!reverse) tc = kl_pair_rows(tc);
-  p.tc_max = static_cast<int32_t>(tc);
-  const int64_t max_slabs = ceil_div(Tpad, tc);
-  p.max_slabs = static_cast<int32_t>(max_slabs + 1);
-  p.max_rt = static_cast<int32_t>(tc / kRowAlign);
-  p.ldg = ldg;
-  p.g = static_cast<__nv_bfloat16*>(g);
-  p.dh_out = d_h_s;
-  p.s2 = s2;
-  p.part5 = part5;
-  p.plane5 = tc * vh;
-  int conv_blocks = static_cast<int>(ceil_div(tc, 8));
-  if (conv_blocks > c.num_sms * 16) conv_blocks = c.num_sms * 16;
-  olive_status st;
-  for (int s = 0; s < max_slabs; ++s) {
-    p.slab = s;
-    p.phase = PH_Z;
-    if ((st = launch_lmhead_fused(c, maps, p)) != OLIVE_OK) return st;
-    conv_kl_kernel<<<conv_blocks, 256, 0, c.stream>>>(n_rows, rows, T, V, static_cast<int>(tc), s,
-                                                      vh, ldg, inv_tau, reverse, grad_kl, part5,
-                                                      p.plane5, s2,
-                                                      static_cast<__nv_bfloat16*>(g), kl);
-    if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;
-    p.phase = PH_DHDW;
-    if ((st = launch_lmhead_fused(c, maps, p)) != OLIVE_OK) return st;
-  }
-  return OLIVE_OK;
 }
 
 olive_status launch_topk_kl_fwd_bwd(const Ctx& c, const void* h_s, const void* W_s, int32_t d_s,
@@ -1776,7 +1447,6 @@ olive_status launch_topk_kl_fwd_bwd(const Ctx& c, const void* h_s, const void* W
 
   FusedParams p = base_params(c, rows, n_rows, T, V, inv_tau, dev_status);
   p.targets = nullptr;  // the forward tiles keep e and the partials only
-  p.kl = 0;
   p.d = d_s;
   p.reduction = OLIVE_REDUCE_SUM;
   p.out_dtype = grad_dtype;

@@ -114,14 +114,16 @@ constexpr int kPaceLag = 1;
 constexpr uint64_t kPaceLimitNs = 2000000;
 constexpr uint32_t kPaceDone = 0x40000000u;
 
-enum GMode : int { GM_REF = 0, GM_A = 1, GM_B = 2 };
+enum GMode : int { GM_REF = 0, GM_A = 1, GM_B = 2, GM_KL = 3 };
 
 // GM_REF / GM_A: za = hc {64 x 128}, zb = W {64 x 128}, xb = W {64 x 64}
 // GM_B:          za = W {64 x 128},  zb = hc {64 x 128}, xb = hc {64 x 64}
 // xa: the ring, [slices x 128 rows] of 64 bf16, unswizzled {64 x 128} boxes
 // (a slice is stored already swizzled, so the copy is linear)
+// GM_KL:         za = hc_s {64 x 128}, zb = W_s {64 x 64}, za2 = hc_t {64 x 128},
+//                zb2 = W_t {64 x 64}, xb = W_s {64 x 64} (128-wide vocabulary tiles)
 struct GroupMaps {
-  CUtensorMap za, zb, xb, xa;
+  CUtensorMap za, zb, xb, xa, za2, zb2;
 };
 
 struct GroupParams {
@@ -162,6 +164,15 @@ struct GroupParams {
   int32_t out_dtype;
   int64_t ring_tiles;       // exchange tiles the ring holds (debug checks)
   int32_t part_groups;      // rows of part_s / part_m (debug checks)
+  int32_t zn;               // width of an inner vocabulary tile: 256 (CE), 128 (GM_KL)
+  // GM_KL (divergence gradient): per compact row the lse of both heads from the
+  // value sweep, per packed row the KL and the weights g_t
+  int32_t d2;               // teacher width
+  int32_t reverse;          // KL direction
+  const float* lse_sc;      // [Tpad] student lse (natural)
+  const float* lse_tc;      // [Tpad] teacher lse (natural)
+  const float* kl;          // [T]
+  const float* grad_kl;     // [T]
 };
 
 // per-CTA schedule, the same in every CTA of a group
@@ -180,6 +191,8 @@ struct GSched {
   int nacc;   // N of the accumulation MMA (cw rounded up to 16)
   int b0;     // first column of this CTA's half of B
   int kcount; // inner extent: V (pass A) or n (pass B)
+  int zn;     // inner tile width
+  int nk2;    // 64-wide K steps of a Z job's second product (GM_KL: the teacher)
   float coef;
 };
 
@@ -200,10 +213,12 @@ __device__ GSched make_gsched(const GroupParams& p) {
   } else {
     s.no = (p.mode == GM_A && p.redo) ? static_cast<int>(min(p.redo_list[0], static_cast<uint32_t>(rt))) : rt;
     s.ph = rt;
-    s.ni = p.mode == GM_REF ? 1 : (p.V + kZN - 1) / kZN;
+    s.ni = p.mode == GM_REF ? 1 : (p.V + p.zn - 1) / p.zn;
     s.kcount = p.V;
   }
+  s.zn = p.zn;
   s.nk = (p.d + kBK - 1) / kBK;
+  s.nk2 = p.mode == GM_KL ? (p.d2 + kBK - 1) / kBK : 0;
   const int pair = blockIdx.x >> 1;
   s.m = pair % p.g;
   const int pg = pair / p.g;
@@ -240,7 +255,7 @@ __device__ __forceinline__ int outer_of(const GroupParams& p, const GSched& s, i
   return (p.mode == GM_A && p.redo) ? static_cast<int>(p.redo_list[1 + k]) : k;
 }
 __device__ __forceinline__ int kvalid_of(const GSched& s, int k) {
-  return min(kZN, s.kcount - k * kZN);
+  return min(s.zn, s.kcount - k * s.zn);
 }
 // 64-wide K slices of inner tile k that hold valid columns
 __device__ __forceinline__ int slices_of(const GSched& s, int k) {
@@ -463,17 +478,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
           const int o = outer_of(p, s, j / s.ni);
           const int k = j % s.ni;
-          for (int ks = 0; ks < s.nk; ++ks) {
+          // K steps [0, nk): the (first) product, za x zb; [nk, nk + nk2):
+          // GM_KL's teacher product, za2 x zb2; B rows of this CTA's half of
+          // the zn-wide vocabulary (or row) tile
+          const int half = s.zn / 2;
+          const uint32_t zbytes = 2 * (kSA + half * kBK * 2);
+          for (int ks = 0; ks < s.nk + s.nk2; ++ks) {
             if (!mbar_wait(empty_bar(stage), phase ^ 1u, ctl)) { ok = false; break; }
             const uint32_t sA = stages + stage * kStageBytes;
             const uint32_t fb = map_shared(full_bar(stage), 0);
-            if (rank == 0) mbar_arrive_expect_tx(full_bar(stage), 2 * kStageBytes);
+            if (rank == 0) mbar_arrive_expect_tx(full_bar(stage), zbytes);
+            const bool second = ks >= s.nk;
+            const int kx = (second ? ks - s.nk : ks) * kBK;
             // (a skipped copy leaves its stage short: the MMA's wait then runs
             // out and the call reports OLIVE_ERR_TIMEOUT as well)
             if (OLIVE_DCHECK(p.dev_status, o >= 0 && o <= s.ph && k >= 0 && k < s.ni)) {
-              tma_load_2d_pair(sA, &maps.za, fb, ks * kBK, o * kBM);
-              tma_load_2d_pair_hint(sA + kSA, &maps.zb, fb, ks * kBK, k * kZN + static_cast<int>(rank) * kBM,
-                                    keep);
+              tma_load_2d_pair(sA, second ? &maps.za2 : &maps.za, fb, kx, o * kBM);
+              tma_load_2d_pair_hint(sA + kSA, second ? &maps.zb2 : &maps.zb, fb, kx,
+                                    k * s.zn + static_cast<int>(rank) * half, keep);
             }
             if (++stage == kStages) { stage = 0; phase ^= 1u; }
           }
@@ -501,7 +523,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                                s.b0 % 8 == 0 && s.b0 >= 0 && s.b0 < p.d + 64)) {
               tma_load_2d_pair(sA, &maps.xa, fb, 0, static_cast<int>(((ring0 + slot) * 4 + sl) * kBM));
               for (int b = 0; b < s.nbox; ++b)
-                tma_load_2d_pair(sA + kSA + b * 8192, &maps.xb, fb, s.b0 + 64 * b, k * kZN + sl * kBK);
+                tma_load_2d_pair(sA + kSA + b * 8192, &maps.xb, fb, s.b0 + 64 * b, k * s.zn + sl * kBK);
             }
             if (++stage == kStages) { stage = 0; phase ^= 1u; }
           }
@@ -545,7 +567,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0 && rank == 0) {
       const uint32_t zacc = tmem_base;
       const uint32_t oacc = tmem_base + 256;
-      const uint32_t idz = idesc_bf16(2 * kBM, kZN, false, false);
+      const uint32_t idz = idesc_bf16(2 * kBM, s.zn, false, false);
       const uint32_t idx = idesc_bf16(2 * kBM, s.nacc, false, true);
       const uint32_t copied_peer = map_shared(smem_u32(const_cast<uint32_t*>(copied)), 1);
       int stage = 0;
@@ -556,15 +578,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (r < nr && j < s.E) {
           if (!mbar_wait(zempty, zph ^ 1u, ctl)) { ok = false; break; }
           tc_fence_after();
-          for (int ks = 0; ks < s.nk; ++ks) {
+          for (int ks = 0; ks < s.nk + s.nk2; ++ks) {
             if (!mbar_wait(full_bar(stage), phase, ctl)) { ok = false; break; }
             tc_fence_after();
             const uint32_t sA = stages + stage * kStageBytes;
             const uint32_t sB = sA + kSA;
+            // GM_KL: the teacher's product goes to the next zn columns
+            const bool second = ks >= s.nk;
+            const uint32_t dz = second ? zacc + static_cast<uint32_t>(s.zn) : zacc;
+            const int kl = second ? ks - s.nk : ks;
 #pragma unroll
             for (int kk = 0; kk < kBK / 16; ++kk)
-              umma_bf16_pair(zacc, sdesc_sw128(sA + kk * 32, 16, 1024), sdesc_sw128(sB + kk * 32, 16, 1024),
-                             idz, (ks > 0 || kk > 0) ? 1u : 0u);
+              umma_bf16_pair(dz, sdesc_sw128(sA + kk * 32, 16, 1024), sdesc_sw128(sB + kk * 32, 16, 1024),
+                             idz, (kl > 0 || kk > 0) ? 1u : 0u);
             umma_commit_pair(empty_bar(stage));
             if (++stage == kStages) { stage = 0; phase ^= 1u; }
           }
@@ -707,6 +733,45 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             if (img) store_img32(img, row, h, gv);
           }
+        } else if (p.mode == GM_KL) {
+          // G of the divergence for this 128 x 128 tile from both heads'
+          // fp32 logits (zn columns each) and the row's lse of each head and
+          // KL from the value sweep: reverse g inv_tau p_s (log p_s - log p_t
+          // - KL), forward g inv_tau (p_s - p_t)
+          const int rc = o * kBM + row;
+          bool valid = false;
+          float ls0 = 0.f, lt0 = 0.f, klv = 0.f, cf = 0.f;
+          if (rc < s.n) {
+            const int t = p.rows[rc];
+            if (t >= 0 && t < p.T) {
+              valid = true;
+              ls0 = p.lse_sc[rc];
+              lt0 = p.lse_tc[rc];
+              klv = p.kl[t];
+              cf = p.grad_kl[t] * p.inv_tau;
+            }
+          }
+#pragma unroll 1
+          for (int h = 0; h < hend; ++h) {
+            uint32_t a[32], b[32];
+            tmem_ld_32x32b_x32(zaddr + h * 32, a);
+            tmem_ld_32x32b_x32(zaddr + static_cast<uint32_t>(s.zn) + h * 32, b);
+            tmem_ld_wait();
+            float gv[32];
+            // log p_s - log p_t as (z_s - z_t) - (lse_s - lse_t): a teacher
+            // shifted by a constant per row cancels before the large terms meet
+            const float dl = ls0 - lt0;
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+              const float zs = __uint_as_float(a[c]) * p.inv_tau;
+              const float zt = __uint_as_float(b[c]) * p.inv_tau;
+              const float ps = fast_exp2((zs - ls0) * kLog2e);
+              const float gg = p.reverse ? cf * ps * (((zs - zt) - dl) - klv)
+                                         : cf * (ps - fast_exp2((zt - lt0) * kLog2e));
+              gv[c] = (valid && h * 32 + c < kv) ? gg : 0.f;
+            }
+            if (img) store_img32(img, row, h, gv);
+          }
         } else {
           if (o != cur_o) {
             cur_o = o;
@@ -714,7 +779,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             run_s = 0.f;
             run_m = -INFINITY;
           }
-          const int v0 = k * kZN;
+          const int v0 = k * s.zn;
 #pragma unroll 1
           for (int h = 0; h < hend; ++h) {
             uint32_t a[32];
@@ -787,6 +852,30 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (v < p.V && OLIVE_DCHECK(p.dev_status, v >= 0 && s.c0 + c + min(32, s.cw - c) <= p.d))
               store_out32(p.out, static_cast<size_t>(v) * p.d + s.c0 + c, p.out_dtype,
                           min(32, s.cw - c), ov);
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_cluster(oempty_lead);
+          continue;
+        }
+        if (p.mode == GM_KL) {
+          // the divergence gradient: G carried g inv_tau, so d_h_s is the sum
+          if (!named_bar_and(1, kEpi, mbar_wait(ofull, oph, ctl))) { ok = false; break; }
+          oph ^= 1u;
+          tc_fence_after();
+          const int rc = o * kBM + row;
+          const int t = rc < s.n ? p.rows[rc] : -1;
+#pragma unroll 1
+          for (int c = 0; c < s.cw; c += 32) {
+            uint32_t a[32];
+            tmem_ld_32x32b_x32(oaddr + c, a);
+            tmem_ld_wait();
+            float ov[32];
+#pragma unroll
+            for (int q = 0; q < 32; ++q) ov[q] = __uint_as_float(a[q]);
+            const int nv = min(32, s.cw - c);
+            if (t >= 0 && t < p.T && OLIVE_DCHECK(p.dev_status, s.c0 + c + nv <= p.d))
+              store_out32(p.out, static_cast<size_t>(t) * p.d + s.c0 + c, p.out_dtype, nv, ov);
           }
           tc_fence_before();
           __syncwarp();
@@ -998,11 +1087,23 @@ olive_status launch_group(const Ctx& c, int mode, const void* hc, const void* W,
   const uint64_t zbRows = rowsA ? V : Tpad;
   // the ring viewed as rows of 64 bf16 (one 128-byte row of a slice image)
   const uint64_t ring_rows = group_ring_bytes(T, d, V) / 128;
+  // inner tiles of 256 vocabulary entries (rows in pass B), 128 for the
+  // divergence, whose Z jobs hold both heads' logits in the Z accumulator;
+  // each CTA of a pair loads half of them as its B rows
+  const int zn = mode == GM_KL ? 128 : kZN;
   if (!encode_bf16_2d(&maps.za, zaBase, d, zaRows, 2ull * d, 64, 128) ||
-      !encode_bf16_2d(&maps.zb, zbBase, d, zbRows, 2ull * d, 64, 128) ||
+      !encode_bf16_2d(&maps.zb, zbBase, d, zbRows, 2ull * d, 64, zn / 2) ||
       !encode_bf16_2d(&maps.xb, zbBase, d, zbRows, 2ull * d, 64, 64) ||
       !encode_bf16_2d_plain(&maps.xa, a.ring, 64, ring_rows, 128, 64, 128))
     return OLIVE_ERR_CUDA;
+  if (mode == GM_KL) {
+    if (!encode_bf16_2d(&maps.za2, a.hc2, a.d2, Tpad, 2ull * a.d2, 64, 128) ||
+        !encode_bf16_2d(&maps.zb2, a.W2, a.d2, V, 2ull * a.d2, 64, zn / 2))
+      return OLIVE_ERR_CUDA;
+  } else {
+    maps.za2 = maps.za;
+    maps.zb2 = maps.zb;
+  }
 
   GroupParams p = {};
   p.dev_status = a.dev_status;
@@ -1044,10 +1145,17 @@ olive_status launch_group(const Ctx& c, int mode, const void* hc, const void* W,
   p.ready = ring_ctr;
   p.cons = ring_ctr ? ring_ctr + static_cast<size_t>(gs.ngroups) * gs.R : nullptr;
   p.pace = ring_ctr ? ring_ctr + 2 * static_cast<size_t>(gs.ngroups) * gs.R : nullptr;
-  p.out = mode == GM_B ? a.d_W : a.d_hidden;
+  p.out = mode == GM_B ? a.d_W : a.d_hidden;  // GM_KL: d_h_s
   p.out_dtype = a.out_dtype;
   p.ring_tiles = static_cast<int64_t>(group_ring_words(T, d, V));
   p.part_groups = group_g_max(d);
+  p.zn = zn;
+  p.d2 = a.d2;
+  p.reverse = a.reverse;
+  p.lse_sc = a.lse_sc;
+  p.lse_tc = a.lse_tc;
+  p.kl = a.kl;
+  p.grad_kl = a.grad_kl;
 
   static std::atomic<int> done[kMaxDevices];
   if (!set_smem_once(reinterpret_cast<const void*>(lmhead_group_kernel), kGroupSmem, c.device, done))
@@ -1144,7 +1252,7 @@ olive_status launch_loss_group(const Ctx& c, const void* hidden, const void* W,
   if (fwd && (st = launch_group(c, GM_REF, w.hc, W, T, d, V, a, 0, d, nullptr)) != OLIVE_OK)
     return st;
   // one sweep of both passes per range of output columns the SMs can hold
-  // (every d up to 38912 at 152 SMs takes one)
+  // (every d up to 19456 at 152 SMs takes one)
   const int cols = group_sweep_cols(c.num_sms);
   const size_t rw = group_ctr_words(T, d, V);
   for (int cb = 0; cb < d; cb += cols) {
@@ -1165,6 +1273,45 @@ olive_status launch_loss_group(const Ctx& c, const void* hidden, const void* W,
       return st;
   }
   return fwd ? launch_loss_reduce(c, n_rows, T, w.nll, reduction, loss) : OLIVE_OK;
+}
+
+}  // namespace olive
+
+namespace olive {
+
+olive_status launch_kl_group_grad(const Ctx& c, const void* hcs, const void* hct, const void* W_s,
+                                  int32_t d_s, const void* W_t, int32_t d_t, const int32_t* rows,
+                                  const int32_t* n_rows, int32_t T, int32_t V, float inv_tau,
+                                  int reverse, const float* kl, const float* lse_s,
+                                  const float* lse_t, const float* grad_kl, void* d_h_s,
+                                  int grad_dtype, void* ring, uint32_t* ctr, size_t ctr_words,
+                                  int32_t* dev_status) {
+  const int64_t rt = align_up(static_cast<size_t>(T), kRowAlign) / kRowAlign;
+  GroupArgs a = {};
+  a.dev_status = dev_status;
+  a.n_rows = n_rows;
+  a.rows = rows;
+  a.inv_tau = inv_tau;
+  a.ring = ring;
+  a.d_hidden = d_h_s;
+  a.out_dtype = grad_dtype;
+  a.hc2 = hct;
+  a.W2 = W_t;
+  a.d2 = d_t;
+  a.reverse = reverse;
+  a.lse_sc = lse_s;
+  a.lse_tc = lse_t;
+  a.kl = kl;
+  a.grad_kl = grad_kl;
+  uint32_t* ring_ctr = ctr + 3 * rt + 1;
+  const int cols = group_sweep_cols(c.num_sms);
+  for (int cb = 0; cb < d_s; cb += cols) {
+    const int ce = d_s - cb < cols ? d_s : cb + cols;
+    if (cudaMemsetAsync(ctr, 0, 4 * ctr_words, c.stream) != cudaSuccess) return OLIVE_ERR_CUDA;
+    const olive_status st = launch_group(c, GM_KL, hcs, W_s, T, d_s, V, a, cb, ce, ring_ctr);
+    if (st != OLIVE_OK) return st;
+  }
+  return OLIVE_OK;
 }
 
 }  // namespace olive

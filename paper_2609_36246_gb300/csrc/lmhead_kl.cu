@@ -190,9 +190,12 @@ struct KlFwdKern {
   };
 };
 
+// kl[t] per masked row; with lse_p / lse_q non-null also both heads' lse per
+// compact row (p the primary head: the student for the reverse KL)
 __global__ void kl_finalize_kernel(const int32_t* __restrict__ n_rows, const int32_t* __restrict__ rows,
                                    int T, int vt, int ctas, int ld,
-                                   const float* __restrict__ part, float* __restrict__ kl) {
+                                   const float* __restrict__ part, float* __restrict__ kl,
+                                   float* __restrict__ lse_p_out, float* __restrict__ lse_q_out) {
   __shared__ int sh_sv;
   const int n = read_n_rows(n_rows, T, nullptr);
   if (threadIdx.x == 0) sh_sv = choose_split(n, vt, ctas).sv;
@@ -218,6 +221,10 @@ __global__ void kl_finalize_kernel(const int32_t* __restrict__ n_rows, const int
     const float k = kLn2 * (A / Sp) - lse_p + lse_q;
     const int t = rows[r];
     if (t >= 0 && t < T) kl[t] = k;
+    if (lse_p_out) {
+      lse_p_out[r] = lse_p;
+      lse_q_out[r] = lse_q;
+    }
   }
 }
 
@@ -248,16 +255,6 @@ olive_status launch_divergence(const Ctx& c, const void* h_s, const void* W_s, i
   if ((st = launch_gather_rows(c, h_t, rows, n_rows, T, d_t, w.hct, dev_status)) != OLIVE_OK) return st;
   if (cudaMemsetAsync(kl, 0, sizeof(float) * T, c.stream) != cudaSuccess) return OLIVE_ERR_CUDA;
 
-  if (grad) {
-    // value and gradient in one pass over the logits
-    const size_t elt = grad_dtype == OLIVE_DTYPE_BF16 ? 2 : 4;
-    if (cudaMemsetAsync(d_h_s, 0, elt * T * static_cast<size_t>(d_s), c.stream) != cudaSuccess)
-      return OLIVE_ERR_CUDA;
-    return launch_kl_fwd_bwd(c, w.hcs, w.hct, W_s, d_s, W_t, d_t, rows, n_rows, T, V, inv_tau,
-                             reverse, grad_kl, kl, w.g, w.s2, w.part5, w.tc, d_h_s, grad_dtype,
-                             dev_status);
-  }
-
   CUtensorMap mHs, mWs, mHt, mWt;
   if (!encode_bf16_2d(&mHs, w.hcs, d_s, Tpad, 2ull * d_s, 64, 128)) return OLIVE_ERR_CUDA;
   if (!encode_bf16_2d(&mWs, W_s, d_s, V, 2ull * d_s, 64, KlFwdKern::kBN)) return OLIVE_ERR_CUDA;
@@ -282,9 +279,19 @@ olive_status launch_divergence(const Ctx& c, const void* h_s, const void* W_s, i
 
   const int vt = (V + KlFwdKern::kBN - 1) / KlFwdKern::kBN;
   kl_finalize_kernel<<<c.num_sms * 4, 256, 0, c.stream>>>(n_rows, rows, T, vt, c.num_sms, p.ld,
-                                                           w.part, kl);
+                                                           w.part, kl, grad ? w.lse_p : nullptr,
+                                                           grad ? w.lse_q : nullptr);
   if (cudaGetLastError() != cudaSuccess) return OLIVE_ERR_CUDA;
-  return OLIVE_OK;
+  if (!grad) return OLIVE_OK;
+  // the gradient: G formed from both heads' logits, recomputed tile by tile
+  // and exchanged on chip (lmhead_group.cu); the student's lse is the
+  // primary head's for the reverse KL, the other one's for the forward KL
+  const size_t elt = grad_dtype == OLIVE_DTYPE_BF16 ? 2 : 4;
+  if (cudaMemsetAsync(d_h_s, 0, elt * T * static_cast<size_t>(d_s), c.stream) != cudaSuccess)
+    return OLIVE_ERR_CUDA;
+  return launch_kl_group_grad(c, w.hcs, w.hct, W_s, d_s, W_t, d_t, rows, n_rows, T, V, inv_tau,
+                              reverse, kl, reverse ? w.lse_p : w.lse_q, reverse ? w.lse_q : w.lse_p,
+                              grad_kl, d_h_s, grad_dtype, w.ring, w.ctr, w.ctr_words, dev_status);
 }
 
 }  // namespace olive

@@ -298,21 +298,20 @@ GroupWs carve_group(void* ws, int64_t T, int64_t d, int64_t V) {
 static KlWs carve_kl_impl(void* ws, int64_t T, int64_t ds, int64_t dt, int64_t V, int grad,
                           size_t* total) {
   const int64_t Tpad = align_up(static_cast<size_t>(T), kRowAlign);
+  const int64_t rt = Tpad / kRowAlign;
   Carver c{static_cast<char*>(ws)};
-  KlWs w;
-  w.tc = slab_rows(Tpad, V);
+  KlWs w = {};
   w.hcs = c.take(2ull * Tpad * ds);
   w.hct = c.take(2ull * Tpad * dt);
-  w.part = w.s2 = w.part5 = nullptr;
-  w.g = nullptr;
+  w.part = static_cast<float*>(c.take(4ull * 5 * kSvMax * Tpad));
   if (grad) {
-    w.g = c.take(2ull * w.tc * vpad(V));
-    // reverse: [tc, Vpad] floats; forward: [kl_pair_rows(tc), 2 Vpad] floats
-    const int64_t rows2 = std::max<int64_t>(w.tc, 2 * kl_pair_rows(w.tc));
-    w.s2 = static_cast<float*>(c.take(4ull * rows2 * vpad(V)));
-    w.part5 = static_cast<float*>(c.take(4ull * 5 * w.tc * ceil_div(V, 128)));
-  } else {
-    w.part = static_cast<float*>(c.take(4ull * 5 * kSvMax * Tpad));
+    w.lse_p = static_cast<float*>(c.take(4ull * Tpad));
+    w.lse_q = static_cast<float*>(c.take(4ull * Tpad));
+    w.ring = c.take(group_ring_bytes(T, ds, V));
+    // the same counter layout as the training step's (group barriers and
+    // redo list unused here), so every sweep's launch has its ring counters
+    w.ctr_words = static_cast<size_t>(3 * rt + 1) + 3 * group_ctr_words(T, ds, V);
+    w.ctr = static_cast<uint32_t*>(c.take(4ull * w.ctr_words));
   }
   if (total) *total = c.off;
   return w;

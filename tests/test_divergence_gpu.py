@@ -90,12 +90,18 @@ def test_kl_workload_sampled_rows():
 
 
 @pytest.mark.parametrize("direction", ["reverse", "forward"])
-def test_several_slabs(direction, monkeypatch):
-    """A lowered slab cap cuts ~1.3k rows into six slabs of the single-pass
-    value + gradient."""
-    monkeypatch.setenv("OLIVE_SLAB_ROWS", "256")
-    hs, Ws, ht, Wt, rows, gk = _case(8, 2000, 64, 96, 1500)
-    assert len(rows) > 5 * 256
+def test_many_outer_tiles(direction):
+    """~1.3k masked rows, d_s = 4096: groups of ~16 CTAs that each run several
+    row tiles, so the exchange ring wraps many times; the last row tile and
+    the last vocabulary tile are partial."""
+    rng = np.random.default_rng(8)
+    T, ds, dt, V = 2000, 4096, 96, 1500
+    hs = synth.rms_hidden_bf16(rng, (T, ds))
+    Ws = synth.normal_bf16(rng, (V, ds), 0.02)
+    ht = synth.normal_bf16(rng, (T, dt), 1.0)
+    Wt = synth.normal_bf16(rng, (V, dt), 0.1)
+    rows = np.sort(rng.choice(T, size=T * 2 // 3, replace=False)).astype(np.int32)
+    gk = rng.uniform(0.5, 1.5, size=T).astype(np.float32)
     kl, dhs = _gpu(hs, Ws, ht, Wt, rows, gk, direction, grad_dtype=torch.bfloat16)
     rkl, rdhs = oracle.token_divergence(to_f64(hs), to_f64(Ws), to_f64(ht), to_f64(Wt), rows,
                                         1.0, direction, grad_kl=gk.astype(np.float64))
@@ -103,9 +109,29 @@ def test_several_slabs(direction, monkeypatch):
     assert_close_grad(dhs, rdhs, "dH_s")
 
 
+def test_two_column_sweeps():
+    """d_s one 64-column tail wider than one sweep of the on-chip gradient:
+    the group pass runs twice over the same logits."""
+    rng = np.random.default_rng(18)
+    sms = min(torch.cuda.get_device_properties(0).multi_processor_count, 192)
+    T, ds, dt, V = 300, sms // 2 * 256 + 64, 64, 700
+    hs = synth.rms_hidden_bf16(rng, (T, ds))
+    Ws = synth.normal_bf16(rng, (V, ds), 0.01)
+    ht = synth.normal_bf16(rng, (T, dt), 1.0)
+    Wt = synth.normal_bf16(rng, (V, dt), 0.3)
+    rows = np.arange(0, T, 2, dtype=np.int32)
+    gk = rng.uniform(0.5, 1.5, size=T).astype(np.float32)
+    for direction in ("reverse", "forward"):
+        kl, dhs = _gpu(hs, Ws, ht, Wt, rows, gk, direction)
+        rkl, rdhs = oracle.token_divergence(to_f64(hs), to_f64(Ws), to_f64(ht), to_f64(Wt), rows,
+                                            1.0, direction, grad_kl=gk.astype(np.float64))
+        assert_close_logp(kl, rkl, "kl")
+        assert_close_grad(dhs, rdhs, "dH_s")
+
+
 def test_value_with_and_without_gradient_agree():
-    """The value-only sweep and the single-pass value + gradient compute KL
-    from the same logits with different tilings of the partials."""
+    """KL from the value-only call and from the call with the gradient (whose
+    first sweep is the same value sweep) agree."""
     hs, Ws, ht, Wt, rows, gk = _case(9, 400, 128, 64, 3001)
     for direction in ("reverse", "forward"):
         k1, _ = _gpu(hs, Ws, ht, Wt, rows, None, direction)
@@ -136,8 +162,8 @@ def test_teacher_shifted_by_a_constant_per_row():
 
 @pytest.mark.parametrize("direction", ["reverse", "forward"])
 def test_single_row_tile(direction):
-    """T <= 128: one slab of one row tile (the forward direction's pair slab
-    is then larger than half of it)."""
+    """T <= 128: one row tile, so all but one group of the gradient pass have
+    no tile of their own."""
     hs, Ws, ht, Wt, rows, gk = _case(12, 100, 64, 64, 777)
     kl, dhs = _gpu(hs, Ws, ht, Wt, rows, gk, direction)
     rkl, rdhs = oracle.token_divergence(to_f64(hs), to_f64(Ws), to_f64(ht), to_f64(Wt), rows,

@@ -126,6 +126,26 @@ def test_many_outer_tiles(grad_dtype):
     _full_check(b, h, W, reduction="mean", grad_dtype=grad_dtype)
 
 
+def _two_sweep_width():
+    """A width one 64-column tail past what one sweep of the on-chip form
+    covers on this device (128 pairs of CTAs at most, 256 columns per member
+    of a group spanning all of them)."""
+    sms = min(torch.cuda.get_device_properties(0).multi_processor_count, 192)
+    return sms // 2 * 256 + 64
+
+
+def test_two_column_sweeps():
+    """d wider than one sweep: the on-chip form runs passes A and B twice, the
+    second sweep over the last 64 output columns with groups of one member,
+    with the forward outputs written by the first sweep only."""
+    rng = np.random.default_rng(19)
+    d = _two_sweep_width()
+    b = synth.batch_from_lengths(rng, [7, 30], [90, 120], 600)
+    h = synth.rms_hidden_bf16(rng, (b.T, d))
+    W = synth.normal_bf16(rng, (600, d), 0.01)
+    _full_check(b, h, W, reduction="mean", grad_dtype=torch.float32)
+
+
 @pytest.mark.parametrize("form", FORMS)
 def test_empty_mask(form):
     rng = np.random.default_rng(22)
