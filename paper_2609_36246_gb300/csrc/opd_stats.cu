@@ -12,17 +12,21 @@
 //   kl_topk[t]       sum_j p_s(v_j) (log p_s(v_j) - log p_t(v_j)), the top-K
 //                    truncated reverse KL
 // Every 128 x 256 tile runs the student and teacher products into the two
-// halves of one 512-column TMEM accumulator (as the divergence forward); each
-// epilogue thread owns a row and keeps, in base-2 units x = z inv_tau log2 e,
-// the online (m_s, s_s, E_s = sum e_s x_s, m_t, s_t, A) and two 16-entry top
-// lists of raw logits (the student's carries the teacher logit of each entry).
+// halves of one 512-column TMEM accumulator (as the divergence forward), so
+// the epilogue cannot overlap the next tile's MMAs; eight epilogue warps
+// shorten it: the two warps of a TMEM lane quadrant take the two 128-column
+// halves of every tile.  Each epilogue thread owns a (row, half) and keeps, in
+// base-2 units x = z inv_tau log2 e, the online (m_s, s_s, E_s = sum e_s x_s,
+// m_t, s_t, A) and two 16-entry top lists of raw logits (the student's carries
+// the teacher logit of each entry).
 // Per 32-column chunk each thread first marks, in a 32-bit mask per list, the
 // columns that beat the list's last entry (after the first tiles of a segment
 // few do), then walks the mask in a rolled loop: the value is picked from the
 // chunk's registers by a 5-level select tree and the insertion network runs
 // once per candidate, so the network exists in one copy (a copy per column
-// overflows the instruction cache).  Per-segment partials are merged by
-// opd_finalize_kernel.
+// overflows the instruction cache).  Each half writes its own partial, as
+// segment 2 sg + half of the row's vocabulary segment sg (so a row tile has at
+// most kSvMax / 2 segments); opd_finalize_kernel merges them.
 #include <climits>
 #include <cmath>
 
@@ -57,8 +61,9 @@ struct OpdKern {
   static constexpr bool kDual = true;
   static constexpr int kStages = 4;
   static constexpr int kAccBufs = 1;
-  static constexpr int kEpiWarps = 4;
+  static constexpr int kEpiWarps = 8;
   static constexpr int kEpiSmem = 0;
+  static constexpr int kSvCap = kSvMax / 2;  // segments per row tile (x 2 halves)
 
   struct Params {
     int32_t* dev_status;
@@ -79,7 +84,8 @@ struct OpdKern {
   };
   static __device__ Sched make_sched(const Params& p) {
     Sched s;
-    s.sp = choose_split(read_n_rows(p.n_rows, p.T, p.dev_status), (p.V + kBN - 1) / kBN, p.ctas);
+    s.sp = choose_split(read_n_rows(p.n_rows, p.T, p.dev_status), (p.V + kBN - 1) / kBN, p.ctas,
+                        kSvCap);
     return s;
   }
   static __device__ int num_units(const Params&, const Sched& s) { return s.sp.units; }
@@ -106,12 +112,12 @@ struct OpdKern {
   }
 
   struct Epi {
-    int r, sg;
+    int r, sg, half;
     float ms, ss, es, mt, st, A;
     float sv[kTopMax], sx[kTopMax], tv[kTopMax];
     int si[kTopMax], ti[kTopMax];
 
-    __device__ void init(uint8_t*, int) {}
+    __device__ void init(uint8_t*, int prt) { half = prt; }
     __device__ void begin(const Params& p, const Sched& s, int u, int row) {
       int i;
       unit_pos(p, s, u, i, sg);
@@ -187,7 +193,7 @@ struct OpdKern {
 
     __device__ void tile(const Params& p, const Sched&, int, int, const TileC& tc, uint32_t taddr) {
 #pragma unroll 1
-      for (int c = 0; c < kBN; c += 32) {
+      for (int c = half * (kBN / 2); c < (half + 1) * (kBN / 2); c += 32) {
         const int col0 = tc.n0 + c;
         if (col0 >= p.V) break;
         uint32_t a[32], b[32];
@@ -201,7 +207,7 @@ struct OpdKern {
     __device__ void end(const Params& p, const Sched& s, int) {
       if (r >= s.sp.n) return;
       const size_t plane = static_cast<size_t>(kSvMax) * p.ld;
-      const size_t o = static_cast<size_t>(sg) * p.ld + r;
+      const size_t o = static_cast<size_t>(2 * sg + half) * p.ld + r;
       p.part[0 * plane + o] = ms;
       p.part[1 * plane + o] = ss;
       p.part[2 * plane + o] = es;
@@ -241,9 +247,9 @@ __global__ void opd_finalize_kernel(const int32_t* __restrict__ n_rows,
                                     const int32_t* __restrict__ part_ti, OpdOut out) {
   __shared__ int sh_sv;
   const int n = read_n_rows(n_rows, T, nullptr);
-  if (threadIdx.x == 0) sh_sv = choose_split(n, vt, ctas).sv;
+  if (threadIdx.x == 0) sh_sv = 2 * choose_split(n, vt, ctas, OpdKern::kSvCap).sv;
   __syncthreads();
-  const int nsv = sh_sv;
+  const int nsv = sh_sv;  // two halves per vocabulary segment
   const size_t plane = static_cast<size_t>(kSvMax) * ld;
   for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < n; r += gridDim.x * blockDim.x) {
     const int t = rows[r];

@@ -25,14 +25,14 @@ struct Split {
   int units; // rt * sv
 };
 
-__host__ __device__ inline Split choose_split(int n, int vt, int ctas) {
+__host__ __device__ inline Split choose_split(int n, int vt, int ctas, int sv_cap = kSvMax) {
   Split s;
   s.n = n;
   s.rt = (n + 127) / 128;
   s.vt = vt;
   int best_sv = 1;
   long long best_cost = -1;
-  const int max_sv = vt < kSvMax ? vt : kSvMax;
+  const int max_sv = vt < sv_cap ? vt : sv_cap;
   for (int sv = 1; sv <= max_sv; ++sv) {
     const int seg = (vt + sv - 1) / sv;
     const int sv_eff = (vt + seg - 1) / seg;
