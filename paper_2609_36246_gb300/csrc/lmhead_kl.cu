@@ -14,11 +14,11 @@
 // so that KL = ln2 * A / s_p - lse_p + lse_q.  Per-segment partials are
 // merged by the finalize kernel.
 //
-// With a gradient request the value and
+// With a gradient request the value sweep runs first, then
 //   reverse: G = g_t inv_tau p_s (log p_s - log p_t - KL_t)
 //   forward: G = g_t inv_tau (p_s - p_t),   d_h_s = G . W_s
-// come from one pass over the logits in the fused kernel of lmhead_fused.cu
-// (the forward tiles keep what G needs in the slab; nothing is recomputed).
+// comes from one pass of the group kernel (lmhead_group.cu), which recomputes
+// both heads' logits tile by tile and contracts G with W_s on chip.
 #include <cmath>
 
 #include "gemm_core.cuh"
