@@ -73,3 +73,31 @@ def test_redo_rows_and_empty_mask(debug_lib):
     _check(b, h.to(torch.bfloat16), W.to(torch.bfloat16))
     e = synth.batch_from_lengths(rng, [9, 4], [0, 0], 300)
     _check(e, synth.normal_bf16(rng, (e.T, 64), 1.0), synth.normal_bf16(rng, (300, 64), 0.1))
+
+
+@pytest.mark.parametrize("direction", ["reverse", "forward"])
+@pytest.mark.parametrize("T,ds,dt,V", [(300, 4096, 72, 700), (150, 2056, 64, 13)])
+def test_divergence_gradient_edges(debug_lib, direction, T, ds, dt, V):
+    """The divergence's on-chip gradient pass (both heads' logits per
+    128-column tile, G formed in the epilogue): a partial last vocabulary tile,
+    V below one tile, a member chunk cut short by d_s; no check fires and KL
+    and d/dh_s match the oracle."""
+    rng = np.random.default_rng(T + V)
+    hs = synth.rms_hidden_bf16(rng, (T, ds))
+    Ws = synth.normal_bf16(rng, (V, ds), 0.02)
+    ht = synth.normal_bf16(rng, (T, dt), 1.0)
+    Wt = synth.normal_bf16(rng, (V, dt), 0.2)
+    rows = np.sort(rng.choice(T, size=T * 2 // 3, replace=False)).astype(np.int32)
+    gk = rng.uniform(0.5, 1.5, size=T).astype(np.float32)
+    st = B.new_status()
+    kl, dhs = B.olive_token_divergence(hs.cuda(), Ws.cuda(), ht.cuda(), Wt.cuda(),
+                                       torch.from_numpy(rows).cuda(),
+                                       torch.tensor([len(rows)], dtype=torch.int32, device="cuda"),
+                                       1.0, direction, torch.from_numpy(gk).cuda(), torch.float32,
+                                       dev_status=st)
+    torch.cuda.synchronize()
+    assert B.status_bits(st) == []
+    rkl, rdhs = oracle.token_divergence(to_f64(hs), to_f64(Ws), to_f64(ht), to_f64(Wt), rows, 1.0,
+                                        direction, grad_kl=gk.astype(np.float64))
+    assert_close_logp(kl.cpu().numpy(), rkl, "kl")
+    assert_close_grad(dhs.cpu().numpy(), rdhs, "dH_s")
