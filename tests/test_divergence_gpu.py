@@ -218,3 +218,25 @@ def test_kl_medium_sampled_rows():
     kl0, none = _gpu(hs, Ws, ht, Wt, rows, None, "reverse")
     assert none is None
     assert np.abs(kl0 - kl).max() <= 1e-4
+
+
+def test_empty_mask_with_gradient():
+    """No masked rows: every launch has no tile to run, KL and d/dh_s are 0."""
+    rng = np.random.default_rng(21)
+    T, ds, dt, V = 200, 128, 64, 1000
+    hs = synth.normal_bf16(rng, (T, ds), 1.0)
+    Ws = synth.normal_bf16(rng, (V, ds), 0.1)
+    ht = synth.normal_bf16(rng, (T, dt), 1.0)
+    Wt = synth.normal_bf16(rng, (V, dt), 0.1)
+    rows = np.zeros(0, dtype=np.int32)
+    gk = np.ones(T, dtype=np.float32)
+    for direction in ("reverse", "forward"):
+        r = torch.zeros(1, dtype=torch.int32, device="cuda")
+        n = torch.zeros(1, dtype=torch.int32, device="cuda")
+        st = B.new_status()
+        kl, dhs = B.olive_token_divergence(hs.cuda(), Ws.cuda(), ht.cuda(), Wt.cuda(), r, n, 1.0,
+                                           direction, torch.from_numpy(gk).cuda(), torch.float32,
+                                           dev_status=st)
+        torch.cuda.synchronize()
+        assert B.status_bits(st) == []
+        assert not kl.any() and not dhs.any()

@@ -124,3 +124,16 @@ def test_fwdbwd_workload_sampled():
     assert not dh[off].any()
     colsum = np.abs(dw.astype(np.float64).sum(axis=0)).max()
     assert colsum <= 1e-2 * np.abs(dw).sum(axis=0).max()
+
+
+def test_two_column_sweeps():
+    """d one 64-column tail wider than one sweep of the on-chip backward (the
+    lse given): passes A and B run twice, the second time over the last 64
+    columns with groups of one member."""
+    rng = np.random.default_rng(23)
+    sms = min(torch.cuda.get_device_properties(0).multi_processor_count, 192)
+    d = sms // 2 * 256 + 64
+    b = synth.batch_from_lengths(rng, [11, 25], [70, 140], 500)
+    h = synth.rms_hidden_bf16(rng, (b.T, d))
+    W = synth.normal_bf16(rng, (500, d), 0.01)
+    _full_check(b, h, W, reduction="mean", grad_dtype=torch.float32)
