@@ -685,9 +685,9 @@ def measure_varlen(dev, burst: float, steps: int = 2):
 
 
 def kernel_rev(source: str = "lmhead_fused.cu") -> str:
-    """Content hash of one kernel's translation unit and the headers it
-    includes (followed transitively), which ties a stored ncu traffic figure
-    to the code that produced it."""
+    """Hash of one kernel's translation unit and the headers it includes
+    (followed transitively), comments and blank lines left out, which ties a
+    stored ncu traffic figure to the code that produced it."""
     import hashlib
     import re as _re
     csrc = os.path.join(ROOT, "paper_2609_36246_gb300", "csrc")
@@ -702,8 +702,11 @@ def kernel_rev(source: str = "lmhead_fused.cu") -> str:
                 todo.append(os.path.normpath(os.path.join(os.path.dirname(path), inc)))
     hsh = hashlib.sha256()
     for path in sorted(seen):
-        with open(path, "rb") as f:
-            hsh.update(f.read())
+        with open(path) as f:
+            text = f.read()
+        text = _re.sub(r"/\*.*?\*/", "", text, flags=_re.S)
+        code = [ln.split("//")[0].rstrip() for ln in text.splitlines()]
+        hsh.update("\n".join(ln for ln in code if ln).encode())
     return hsh.hexdigest()[:16]
 
 

@@ -40,6 +40,15 @@
 //     row); member m accumulates dW[v, chunk] = G^T . hc[:, chunk] and stores
 //     it when the outer tile ends (every dW element has one owner: no atomics).
 //
+//   Divergence mode (GM_KL: the gradient of OPD's per-token KL, Section 1,
+//   after the value sweep of lmhead_kl.cu has given KL and both heads' lse):
+//     the pass A layout with two products per Z job, the student's (K = d_s)
+//     and the teacher's (K = d_t) logits of a 128-column vocabulary tile in
+//     the two halves of the 256-column Z accumulator; the epilogue forms the
+//     exact G (reverse: g inv_tau p_s ((z_s - z_t) - (lse_s - lse_t) - KL),
+//     forward: g inv_tau (p_s - p_t)) and the members accumulate
+//     d_h_s = G . W_s.
+//
 // Each pass executes two products per logit (the Z tile and its share of the
 // accumulation), so the training step executes 4 GEMM units of 2 N_mask d V
 // flops for the 3 it counts.
@@ -73,9 +82,10 @@
 // points to a tile of an earlier round, every CTA is resident at once (the
 // grid is one CTA per SM; the host checks that the GPU holds all its
 // clusters), and every wait is bounded (OLIVE_ERR_TIMEOUT on expiry).  A
-// pacing hint keeps the groups within a round of one another, so the inner
-// operand stream (W in pass A, hc in pass B) is fetched from DRAM once for
-// all groups.
+// pacing hint keeps the groups within a round of one another, so that one
+// DRAM fetch of an inner operand tile (W in pass A, hc in pass B) can serve
+// every group from the L2 (how often it does depends on what else the L2
+// holds: the call reads the streamed operand several times over).
 #include <algorithm>
 #include <atomic>
 #include <cmath>
