@@ -9,6 +9,14 @@
  *                            and continuation ids), runs olive_splice_pack on
  *                            the current CUDA device and prints n_rows, rows,
  *                            targets and the loss mask
+ *   olive_c_check step IN OUT
+ *                            one training step: reads a batch, the hidden
+ *                            rows and W (bf16 bit patterns) from IN, runs
+ *                            olive_splice_pack and olive_token_loss_fwd_bwd
+ *                            (fp32 gradients, a workspace sized by
+ *                            olive_workspace_size) and writes the status
+ *                            word, logp [T], lse [T], the loss, d_hidden
+ *                            [T, d] and d_W [V, d] to OUT
  */
 #include <stdio.h>
 #include <stdlib.h>
@@ -110,7 +118,96 @@ static int splice(void) {
   return 0;
 }
 
+static int read_exact(FILE* f, void* dst, size_t bytes) {
+  return fread(dst, 1, bytes, f) == bytes ? 0 : 1;
+}
+
+/* IN: int32 S, V, T, d; int32 prefix_off[S+1], cont_off[S+1]; int32
+   prefix_ids, cont_ids; uint16 hidden[T*d], W[V*d] (bf16 bits). */
+static int step(const char* in_path, const char* out_path) {
+  FILE* f = fopen(in_path, "rb");
+  if (!f) return 3;
+  int32_t hdr[4];
+  if (read_exact(f, hdr, sizeof hdr)) return 3;
+  const int S = hdr[0], V = hdr[1], T = hdr[2], d = hdr[3];
+  int32_t* poff = (int32_t*)malloc(4 * (size_t)(S + 1));
+  int32_t* coff = (int32_t*)malloc(4 * (size_t)(S + 1));
+  if (read_exact(f, poff, 4 * (size_t)(S + 1)) || read_exact(f, coff, 4 * (size_t)(S + 1))) return 3;
+  int32_t* pids = (int32_t*)malloc(4 * (size_t)(poff[S] + 1));
+  int32_t* cids = (int32_t*)malloc(4 * (size_t)(coff[S] + 1));
+  if (read_exact(f, pids, 4 * (size_t)poff[S]) || read_exact(f, cids, 4 * (size_t)coff[S])) return 3;
+  const size_t hb = 2 * (size_t)T * d, wb = 2 * (size_t)V * d;
+  void* h_hidden = malloc(hb);
+  void* h_W = malloc(wb);
+  if (read_exact(f, h_hidden, hb) || read_exact(f, h_W, wb)) return 3;
+  fclose(f);
+
+  int32_t *ids, *targets, *cu, *cut, *rows, *n_rows, *st;
+  uint8_t* mask;
+  float *logp, *lse, *loss, *gl, *dh, *dw;
+  void* ws;
+  cudaMalloc((void**)&ids, 4 * (size_t)T);
+  cudaMalloc((void**)&targets, 4 * (size_t)T);
+  cudaMalloc((void**)&mask, (size_t)T);
+  cudaMalloc((void**)&cu, 4 * (size_t)(S + 1));
+  cudaMalloc((void**)&cut, 4 * (size_t)S);
+  cudaMalloc((void**)&rows, 4 * (size_t)T);
+  cudaMalloc((void**)&n_rows, 4);
+  cudaMalloc((void**)&st, 4);
+  cudaMemset(st, 0, 4);
+  cudaMalloc((void**)&logp, 4 * (size_t)T);
+  cudaMalloc((void**)&lse, 4 * (size_t)T);
+  cudaMalloc((void**)&loss, 4);
+  cudaMalloc((void**)&dh, 4 * (size_t)T * d);
+  cudaMalloc((void**)&dw, 4 * (size_t)V * d);
+  const float one = 1.0f;
+  gl = (float*)dev_copy(&one, 4);
+  const size_t ws_bytes = olive_workspace_size(OLIVE_OP_LOSS_FWD_BWD, T, d, 0, V, 1, OLIVE_DTYPE_F32);
+  if (ws_bytes == 0 || cudaMalloc(&ws, ws_bytes) != cudaSuccess) return 4;
+  void* d_hidden = dev_copy(h_hidden, hb);
+  void* d_W = dev_copy(h_W, wb);
+
+  olive_status s = olive_splice_pack(dev_copy(pids, 4 * (size_t)poff[S]), dev_copy(poff, 4 * (size_t)(S + 1)),
+                                     dev_copy(cids, 4 * (size_t)coff[S]), dev_copy(coff, 4 * (size_t)(S + 1)),
+                                     S, V, T, ids, targets, mask, cu, cut, rows, n_rows, st, NULL);
+  if (s != OLIVE_OK) {
+    fprintf(stderr, "olive_splice_pack: %s\n", olive_status_string(s));
+    return 5;
+  }
+  s = olive_token_loss_fwd_bwd(d_hidden, d_W, targets, rows, n_rows, T, d, V, 1.0f, OLIVE_REDUCE_SUM, gl,
+                               logp, lse, loss, dh, dw, OLIVE_DTYPE_F32, ws, ws_bytes, st, NULL);
+  if (s != OLIVE_OK) {
+    fprintf(stderr, "olive_token_loss_fwd_bwd: %s\n", olive_status_string(s));
+    return 5;
+  }
+  if (cudaDeviceSynchronize() != cudaSuccess) return 4;
+
+  int32_t dst = 0;
+  float h_loss = 0.f;
+  float* h_logp = (float*)malloc(4 * (size_t)T);
+  float* h_lse = (float*)malloc(4 * (size_t)T);
+  float* h_dh = (float*)malloc(4 * (size_t)T * d);
+  float* h_dw = (float*)malloc(4 * (size_t)V * d);
+  cudaMemcpy(&dst, st, 4, cudaMemcpyDeviceToHost);
+  cudaMemcpy(&h_loss, loss, 4, cudaMemcpyDeviceToHost);
+  cudaMemcpy(h_logp, logp, 4 * (size_t)T, cudaMemcpyDeviceToHost);
+  cudaMemcpy(h_lse, lse, 4 * (size_t)T, cudaMemcpyDeviceToHost);
+  cudaMemcpy(h_dh, dh, 4 * (size_t)T * d, cudaMemcpyDeviceToHost);
+  if (cudaMemcpy(h_dw, dw, 4 * (size_t)V * d, cudaMemcpyDeviceToHost) != cudaSuccess) return 4;
+  FILE* o = fopen(out_path, "wb");
+  if (!o) return 3;
+  fwrite(&dst, 4, 1, o);
+  fwrite(h_logp, 4, (size_t)T, o);
+  fwrite(h_lse, 4, (size_t)T, o);
+  fwrite(&h_loss, 4, 1, o);
+  fwrite(h_dh, 4, (size_t)T * d, o);
+  fwrite(h_dw, 4, (size_t)V * d, o);
+  fclose(o);
+  return 0;
+}
+
 int main(int argc, char** argv) {
   if (argc > 1 && strcmp(argv[1], "splice") == 0) return splice();
+  if (argc > 3 && strcmp(argv[1], "step") == 0) return step(argv[2], argv[3]);
   return host_checks();
 }
