@@ -240,3 +240,23 @@ def test_empty_mask_with_gradient():
         torch.cuda.synchronize()
         assert B.status_bits(st) == []
         assert not kl.any() and not dhs.any()
+
+
+@pytest.mark.parametrize("direction", ["reverse", "forward"])
+def test_wide_heads(direction):
+    """Both heads 4096 wide: long Z jobs (K = 8192 over the two products),
+    members' d_s chunks of 224 with a 64-wide last one, a partial last
+    vocabulary tile and a phantom row tile."""
+    rng = np.random.default_rng(33)
+    T, ds, dt, V = 300, 4096, 4096, 3000
+    hs = synth.rms_hidden_bf16(rng, (T, ds))
+    Ws = synth.normal_bf16(rng, (V, ds), 0.02)
+    ht = synth.rms_hidden_bf16(rng, (T, dt))
+    Wt = synth.normal_bf16(rng, (V, dt), 0.02)
+    rows = np.sort(rng.choice(T, size=T * 2 // 3, replace=False)).astype(np.int32)
+    gk = rng.uniform(0.5, 1.5, size=T).astype(np.float32)
+    kl, dhs = _gpu(hs, Ws, ht, Wt, rows, gk, direction)
+    rkl, rdhs = oracle.token_divergence(to_f64(hs), to_f64(Ws), to_f64(ht), to_f64(Wt), rows, 1.0,
+                                        direction, grad_kl=gk.astype(np.float64))
+    assert_close_logp(kl, rkl, "kl")
+    assert_close_grad(dhs, rdhs, "dH_s")
